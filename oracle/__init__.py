@@ -1,0 +1,212 @@
+"""CPU oracle for the trie automaton: brute force, from the paper's definitions.
+
+TEST INFRASTRUCTURE ONLY. Only ``tests/``, ``__graft_entry__.smoke()`` and the
+bench's CPU-baseline leg may import this package. It shares no code with the
+CUDA path and imports nothing from it.
+
+The arithmetic lives in ``oracle.c`` (a plain C library, each function citing
+the passage it follows); this module loads it with ctypes and adds the decode
+loop (Eq. 1: mask, greedy choice, state advance), which only calls those
+functions in order.
+
+Pins (``tests/test_oracle_pins.py``): the worked example of App. G.1 and the
+Fig. 2 example (``tests/golden/``), exhaustive comparison with the prefix-set
+enumeration of the App. G.5 proof on small random sets, and the invariants of
+Sec. 4.2 / App. G.5 (tokenization paths allowed, leaves admit only EOS,
+prefix closure, padding bits zero, ...).
+"""
+from __future__ import annotations
+
+import contextlib
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+DEAD = -1
+FINISHED = -2
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile oracle.c into liboracle.so (gcc, OpenMP) if it is missing or stale."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-std=c99",
+                               "-o", tmp, _SRC])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def load_library(path: str):
+    """Load one build of oracle.c and declare its signatures."""
+    lib = ctypes.CDLL(path)
+    P, I32, I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+    lib.oracle_trie_build.restype = P
+    lib.oracle_trie_build.argtypes = [P, P, I32]
+    lib.oracle_trie_free.argtypes = [P]
+    lib.oracle_trie_num_nodes.restype = I32
+    lib.oracle_trie_num_nodes.argtypes = [P]
+    lib.oracle_trie_num_chars.restype = I64
+    lib.oracle_trie_num_chars.argtypes = [P]
+    lib.oracle_trie_child.restype = I32
+    lib.oracle_trie_child.argtypes = [P, I32, I32]
+    lib.oracle_trie_info.argtypes = [P, P, P, P, P]
+    lib.oracle_mask_rows.argtypes = [P, P, P, I32, P, I64, P, I32]
+    lib.oracle_advance.restype = I64
+    lib.oracle_advance.argtypes = [P, P, P, I32, P, P, I64]
+    lib.oracle_apply.argtypes = [P, P, P, I32, P, I32, P, I64]
+    lib.oracle_argmax.argtypes = [P, I32, I64, I32, P]
+    return lib
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = load_library(build())
+    return _lib
+
+
+@contextlib.contextmanager
+def use_library(path: str):
+    """Route oracle calls to another build of oracle.c (the mutation tests plant
+    mistakes in a copy of the source and check that the pins catch them)."""
+    global _lib
+    _load()
+    old = _lib
+    _lib = load_library(path)
+    try:
+        yield
+    finally:
+        _lib = old
+
+
+def _p(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def n_words(V: int) -> int:
+    return (V + 31) // 32
+
+
+class Trie:
+    """Byte trie of a string set, node ids in breadth-first / ascending-byte order."""
+
+    def __init__(self, set_bytes: np.ndarray, set_offsets: np.ndarray):
+        self._lib = _load()
+        self._b = np.ascontiguousarray(set_bytes, dtype=np.uint8)
+        self._o = np.ascontiguousarray(set_offsets, dtype=np.int64)
+        if self._b.size == 0:
+            self._b = np.zeros(1, dtype=np.uint8)
+        h = self._lib.oracle_trie_build(_p(self._b), _p(self._o), len(self._o) - 1)
+        if not h:
+            raise MemoryError("oracle_trie_build failed")
+        self._h = ctypes.c_void_p(h)
+        self.num_nodes = self._lib.oracle_trie_num_nodes(self._h)
+        self.num_chars = self._lib.oracle_trie_num_chars(self._h)
+        n = self.num_nodes
+        self.parent = np.empty(n, np.int32)
+        self.label = np.empty(n, np.uint8)
+        self.terminal = np.empty(n, np.uint8)
+        self.depth = np.empty(n, np.int32)
+        self._lib.oracle_trie_info(self._h, _p(self.parent), _p(self.label), _p(self.terminal),
+                                   _p(self.depth))
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h:
+            self._lib.oracle_trie_free(h)
+            self._h = None
+
+    def child(self, node: int, byte: int) -> int:
+        return self._lib.oracle_trie_child(self._h, node, byte)
+
+    def prefix(self, node: int) -> bytes:
+        out = bytearray()
+        while node > 0:
+            out.append(int(self.label[node]))
+            node = int(self.parent[node])
+        return bytes(reversed(out))
+
+
+class Vocab:
+    def __init__(self, vocab_bytes: np.ndarray, vocab_offsets: np.ndarray):
+        self.b = np.ascontiguousarray(vocab_bytes, dtype=np.uint8)
+        if self.b.size == 0:
+            self.b = np.zeros(1, dtype=np.uint8)
+        self.o = np.ascontiguousarray(vocab_offsets, dtype=np.int64)
+        self.V = len(self.o) - 1
+        self.eos = self.V - 1
+
+
+def mask_rows(t: Trie, voc: Vocab, rows, nthreads: int = 1) -> np.ndarray:
+    """uint32[len(rows), ceil(V/32)] mask rows (App. G.5 proof conditions, EOS at terminals)."""
+    rows = np.ascontiguousarray(rows, dtype=np.int32)
+    out = np.zeros((rows.size, n_words(voc.V)), dtype=np.uint32)
+    t._lib.oracle_mask_rows(t._h, _p(voc.b), _p(voc.o), voc.V, _p(rows), rows.size, _p(out),
+                            nthreads)
+    return out
+
+
+def mask_all(t: Trie, voc: Vocab, nthreads: int = 1) -> np.ndarray:
+    return mask_rows(t, voc, np.arange(t.num_nodes, dtype=np.int32), nthreads)
+
+
+def advance(t: Trie, voc: Vocab, states: np.ndarray, tokens: np.ndarray) -> tuple[np.ndarray, int]:
+    """(next states, number of new DEAD moves) for one batch of tokens."""
+    s = np.ascontiguousarray(states, dtype=np.int32).copy()
+    tk = np.ascontiguousarray(tokens, dtype=np.int32)
+    err = t._lib.oracle_advance(t._h, _p(voc.b), _p(voc.o), voc.V, _p(s), _p(tk), s.size)
+    return s, int(err)
+
+
+def _bits(logits: np.ndarray) -> tuple[np.ndarray, int]:
+    if logits.dtype == np.uint32:
+        return np.ascontiguousarray(logits), 0
+    if logits.dtype == np.uint16:
+        return np.ascontiguousarray(logits), 1
+    raise TypeError("pass logits as raw bits: uint32 (fp32) or uint16 (bf16)")
+
+
+def apply(t: Trie, voc: Vocab, logits_bits: np.ndarray, states: np.ndarray) -> np.ndarray:
+    """Masked copy of [B, V] raw-bit logits (uint32 = fp32, uint16 = bf16)."""
+    x, dt = _bits(logits_bits)
+    x = x.copy()
+    st = np.ascontiguousarray(states, dtype=np.int32)
+    t._lib.oracle_apply(t._h, _p(voc.b), _p(voc.o), voc.V, _p(x), dt, _p(st), st.size)
+    return x
+
+
+def argmax(logits_bits: np.ndarray) -> np.ndarray:
+    x, dt = _bits(logits_bits)
+    B, V = x.shape
+    out = np.empty(B, np.int32)
+    _load().oracle_argmax(_p(x), dt, B, V, _p(out))
+    return out
+
+
+def decode(t: Trie, voc: Vocab, logits_per_step, states0: np.ndarray):
+    """Greedy constrained decode (Eq. 1 with greedy choice): per step mask -> argmax -> advance.
+
+    ``logits_per_step`` yields [B, V] raw-bit arrays. Returns per-step lists of
+    (masked logits, tokens, states after the step) and the total error count.
+    """
+    states = np.ascontiguousarray(states0, dtype=np.int32).copy()
+    masked, toks, sts = [], [], []
+    errors = 0
+    for lg in logits_per_step:
+        m = apply(t, voc, lg, states)
+        tk = argmax(m)
+        states, e = advance(t, voc, states, tk)
+        errors += e
+        masked.append(m)
+        toks.append(tk)
+        sts.append(states.copy())
+    return masked, toks, sts, errors

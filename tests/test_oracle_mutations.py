@@ -1,0 +1,76 @@
+"""Plant plausible mistakes in a copy of the oracle and check the pins catch each.
+
+Every mutant is a textual edit of oracle/oracle.c, compiled into a temporary
+directory (CPU only). A mutant that passes all pins would mean the pins cannot
+tell that mistake from the correct oracle.
+"""
+from __future__ import annotations
+
+import os
+import subprocess
+
+import pytest
+
+import oracle
+from pins import (check_advance, check_apply, check_argmax, check_chain, check_golden,
+                  check_masks, check_numbering, random_case)
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "oracle.c")
+
+MUTANTS = {
+    "overshoot_allowed": ("        if (x < 0) return -1;\n    }\n    return x;",
+                          "        if (x < 0) return n;\n    }\n    return x;"),
+    "empty_token_allowed": ("if (e <= a) return -1;", "if (e <= a) return n;"),
+    "eos_ignores_terminal": ("if (!node || t->terminal[n]) row", "if (!node) row"),
+    "eos_everywhere": ("if (!node || t->terminal[n]) row", "if (1) row"),
+    "bit_index_off_by_one": ("if (walk(t, n, vb, vo, v) >= 0) row[v / 32] |= 1u << (v % 32);",
+                             "if (walk(t, n, vb, vo, v) >= 0) row[v / 32] |= 1u << ((v + 1) % 32);"),
+    "last_token_skipped": ("for (int32_t v = 0; v < eos; v++)", "for (int32_t v = 0; v < eos - 1; v++)"),
+    "siblings_descending": ("        for (int b = 0; b < 256; b++)\n            if (ch[(int64_t)x * 256 + b] >= 0) order",
+                            "        for (int b = 255; b >= 0; b--)\n            if (ch[(int64_t)x * 256 + b] >= 0) order"),
+    "depth_first_numbering": ("int32_t x = order[head++];", "int32_t x = order[--tail]; head++;"),
+    "finished_eos_dies": ("nxt = (v == eos) ? ORACLE_FINISHED : ORACLE_DEAD;",
+                          "nxt = ORACLE_DEAD;"),
+    "eos_finishes_anywhere": ("nxt = t->terminal[s] ? ORACLE_FINISHED : ORACLE_DEAD;",
+                              "nxt = ORACLE_FINISHED;"),
+    "dead_moves_not_counted": ("if (nxt == ORACLE_DEAD) errors++;", "if (0) errors++;"),
+    "bf16_neg_inf_wrong": ("= 0xFF80u;", "= 0x7F80u;"),
+    "f32_neg_inf_wrong": ("= 0xFF800000u;", "= 0xFF000000u;"),
+    "argmax_last_tie": ("if (v == 0 || x > bv)", "if (v == 0 || x >= bv)"),
+    "terminal_not_marked_for_prefix_values": ("        term[x] = 1;\n", "        if (x > 0 || offsets[i+1] > offsets[i]) term[x] = 1;\n        if (ch[x * 256 + 0] >= 0) term[x] = 0;\n"),
+}
+
+
+def _all_pins():
+    check_golden("appG1_worked_example.json")
+    check_golden("fig2_alignment.json")
+    check_argmax(7)
+    check_chain(b"medical_billing")
+    check_chain(bytes([0, 255, 0, 255, 7]))
+    for seed in range(40):
+        strings, toks = random_case(1000 + seed)
+        check_numbering(strings)
+        check_masks(strings, toks)
+        check_advance(strings, toks, seed)
+        check_apply(strings, toks, seed)
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_planted_mistake(oracle_lib, tmp_path, name):
+    src = open(SRC).read()
+    old, new = MUTANTS[name]
+    assert src.count(old) == 1, f"mutation site for {name} not unique / not found"
+    path = tmp_path / "mut.c"
+    path.write_text(src.replace(old, new))
+    lib = tmp_path / "libmut.so"
+    subprocess.check_call(["gcc", "-O1", "-shared", "-fPIC", "-std=c99", "-o", str(lib), str(path)])
+    with oracle.use_library(str(lib)):
+        with pytest.raises(AssertionError):
+            _all_pins()
+
+
+def test_unmutated_copy_passes(oracle_lib, tmp_path):
+    lib = tmp_path / "libsame.so"
+    subprocess.check_call(["gcc", "-O1", "-shared", "-fPIC", "-std=c99", "-o", str(lib), SRC])
+    with oracle.use_library(str(lib)):
+        _all_pins()
