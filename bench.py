@@ -1,0 +1,468 @@
+#!/usr/bin/env python
+"""Benchmark of the trie-automaton hot path on GB300.
+
+One step = one schema through the whole path: mask compile for every trie
+node (k_mask_fill + k_mask_patch) and then the batched decode loop, each
+decode step being mask application (k_apply_vec), a greedy argmax and the
+state advance (k_advance). The workload is K = 10,000 ICD-style codes with a
+152,064-token byte vocabulary, batch 256, 16 decode steps, bf16 logits.
+
+value     (node, token) pairs per second, N * V per step over the device time
+          of the step, inputs resident in HBM (one CUDA graph per step).
+e2e       the same pairs/s through the C ABI from host buffers: the trie
+          built from host strings, logits copied from pinned host memory each
+          decode step, the sampled tokens read back each decode step.
+roofline  the dominant kernel of the step (mask application), algorithmic
+          bytes per launch over its CUDA-event duration inside the timed
+          replay; roofline_compile gives the same for the mask compile.
+
+`--impl reference` times the CPU oracle (plain C, OpenMP) on the same
+workload instead. With torchrun (N > 1) every rank runs its own replica
+(weak scaling; the path needs no exchange between GPUs).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "mask-compile ms & (node,token) pairs/s; batch-256 mask-apply GB/s vs HBM peak"
+UNIT = "pairs/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=1000)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    p.add_argument("--config", type=int, default=3, choices=[1, 2, 3, 4])
+    p.add_argument("--e2e-steps", type=int, default=10)
+    p.add_argument("--cpu-seconds", type=float, default=10.0,
+                   help="time budget of the CPU-oracle baseline sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-graph", action="store_true", help="replay the step eagerly instead of as a CUDA graph")
+    return p.parse_args()
+
+
+def peaks() -> tuple[float, str]:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    with open(os.path.join(ROOT, "paper_2608_12574_gb300", "csrc", "kernels.cu"), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def ncu_traffic(kernel: str, workload: str) -> float | None:
+    """DRAM bytes per launch recorded by ncu for this kernel source, else None."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    h = kernel_source_hash()
+    for line in open(path):
+        parts = line.split()
+        if len(parts) == 4 and parts[0] == kernel and parts[1] == workload and parts[2] == h:
+            return float(parts[3])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.proc = None
+        self.uuid = uuid
+
+    def __enter__(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100"]
+        if self.uuid:
+            cmd += ["-i", self.uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        time.sleep(0.2)
+        self.out = ""
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self) -> dict:
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (getattr(self, "out", "") or "").splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                smax.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- oracle arm
+
+class OracleSample:
+    """A proportional slice of one step for the CPU oracle: a fraction f of the
+    trie's mask rows (seeded sample, root included) and of the batch rows of
+    the decode loop. value = f * N * V pairs over the slice's wall time."""
+
+    def __init__(self, w, nthreads: int):
+        import numpy as np
+        import oracle
+        oracle.build()
+        self.w, self.nthreads = w, nthreads
+        self.trie = oracle.Trie(w.set_bytes, w.set_offsets)
+        self.voc = oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+        self.N = self.trie.num_nodes
+        rng = np.random.default_rng(12345)
+        self.order = np.concatenate([[0], 1 + rng.permutation(self.N - 1)]).astype(np.int32)
+        self.bits = cpu_logits_bits(w)
+        self.set_frac(0.01)
+
+    def set_frac(self, f: float):
+        import math
+        self.f = min(1.0, max(f, 1.0 / self.N))
+        self.rows = self.order[: max(1, int(math.ceil(self.f * self.N)))]
+        self.b = max(1, int(round(self.f * self.w.batch)))
+
+    def step(self) -> float:
+        import numpy as np
+        import oracle
+        t0 = time.perf_counter()
+        oracle.mask_rows(self.trie, self.voc, self.rows, nthreads=self.nthreads)
+        oracle.decode(self.trie, self.voc, [lb[: self.b] for lb in self.bits], np.zeros(self.b, np.int32))
+        return time.perf_counter() - t0
+
+    def calibrate(self, target_s: float):
+        t = self.step()
+        self.set_frac(self.f * target_s / max(t, 1e-4))
+
+
+def cpu_logits_bits(w):
+    import numpy as np
+    import torch
+    from paper_2608_12574_gb300 import workloads as W
+    out = []
+    for s in range(w.steps):
+        x = W.logits(w, s, device="cpu")
+        out.append(x.view(torch.int16).numpy().view(np.uint16) if w.dtype == "bf16"
+                   else x.view(torch.int32).numpy().view(np.uint32))
+    return out
+
+
+def cpu_baseline(w, target_step_s: float, steps: int, warmup: int) -> dict:
+    """Time the oracle as it stands on this host's cores (bounded sample)."""
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
+    smp = OracleSample(w, cores)
+    smp.calibrate(target_step_s)
+    for _ in range(warmup):
+        smp.step()
+    times = [smp.step() for _ in range(steps)]
+    per_step = sum(times) / len(times)
+    cpu_model = ""
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part")):
+                cpu_model = line.split(":", 1)[1].strip()
+                break
+    except OSError:
+        pass
+    return {"value": smp.f * smp.N * w.V / per_step, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "steps": len(times), "s_per_step": per_step, "cpu": cpu_model, "N_nodes": smp.N,
+            "sample": f"{len(times)} steps, each a {smp.f:.4f} slice of one {w.name} step: "
+                      f"{len(smp.rows)} of {smp.N} mask rows x {w.V} tokens (brute-force walks, "
+                      f"OpenMP over rows) and the {w.steps}-step decode loop on {smp.b} of "
+                      f"{w.batch} batch rows"}
+
+
+def run_reference(args, w):
+    steps, warmup = max(1, args.steps), max(0, args.warmup)
+    target = min(2.0, 150.0 / (steps + warmup + 1))
+    cb = cpu_baseline(w, target, steps, warmup)
+    line = {"metric": METRIC, "value": cb["value"], "unit": UNIT, "n_gpus": args.gpus, "steps": cb["steps"],
+            "warmup": warmup, "ms_per_step": cb["s_per_step"] * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "u32 mask / " + w.dtype, "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": w.name, "K": w.K, "V": w.V, "batch": w.batch, "decode_steps": w.steps,
+                       "N_nodes": cb["N_nodes"]},
+            "cpu_baseline": cb,
+            "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+# --------------------------------------------------------------------------- GPU arm
+
+def run_gpu(args, w, rank: int, world: int, dist):
+    import numpy as np
+    import torch
+    from paper_2608_12574_gb300 import triemask as T
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(dev)
+    V, B, S = w.V, w.batch, w.steps
+    Wd = T.mask_words(V)
+    elt = 2 if w.dtype == "bf16" else 4
+    hbm, peak_kind = peaks()
+
+    # ---- setup (untimed): trie, cold compile (vocab pack + uploads), logits in HBM
+    t0 = time.perf_counter()
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    host_build_ms = (time.perf_counter() - t0) * 1e3
+    N = h.num_nodes
+    mask = T.alloc_mask(h, V, dev)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+    stream.synchronize()
+    cold_compile_ms = (time.perf_counter() - t0) * 1e3
+    with torch.cuda.stream(stream):
+        logits = [W_logits(w, s, dev) for s in range(S)]
+        states0 = torch.zeros(B, dtype=torch.int32, device=dev)
+        states = torch.zeros(B, dtype=torch.int32, device=dev)
+        tok64 = torch.zeros(B, dtype=torch.int64, device=dev)
+        tok = torch.zeros(B, dtype=torch.int32, device=dev)
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream.synchronize()
+
+    ext = {"external": True}
+    try:
+        torch.cuda.Event(enable_timing=True, **ext)
+    except TypeError:
+        ext = {}
+    n_ev = 2 + 2 * S + 2 * S
+    evs = [torch.cuda.Event(enable_timing=True, **ext) for _ in range(n_ev)]
+
+    def step(timed_events: bool):
+        e = iter(evs)
+        if timed_events:
+            next(e).record(stream)
+        T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+        if timed_events:
+            next(e).record(stream)
+        states.copy_(states0)
+        for t in range(S):
+            if timed_events:
+                next(e).record(stream)
+            T.trie_apply_mask(h, logits[t], states, stream)
+            if timed_events:
+                next(e).record(stream)
+            torch.argmax(logits[t], dim=1, out=tok64)
+            tok.copy_(tok64)
+            if timed_events:
+                next(e).record(stream)
+            T.trie_advance(h, states, tok, err, stream)
+            if timed_events:
+                next(e).record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(args.warmup, 3)):
+            step(False)
+    stream.synchronize()
+
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step(bool(ext))
+        with torch.cuda.stream(stream):
+            for _ in range(max(args.warmup, 3)):
+                graph.replay()
+        stream.synchronize()
+
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(uuid) as clk:
+        with torch.cuda.stream(stream):
+            t_start.record(stream)
+            for _ in range(args.steps):
+                if graph is not None:
+                    graph.replay()
+                else:
+                    step(False)
+            t_end.record(stream)
+        torch.cuda.synchronize()
+    ms = t_start.elapsed_time(t_end)
+    if dist is not None:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_per_step = ms / args.steps
+
+    # per-kernel durations: events inside the last graph replay of the timed
+    # region when the graph carries them, else one instrumented eager step
+    timing_src = "last replay of the timed region (event nodes in the graph)"
+    if graph is None or not ext:
+        with torch.cuda.stream(stream):
+            step(True)
+        stream.synchronize()
+        timing_src = "one eager step after the timed region"
+    d = [evs[i].elapsed_time(evs[i + 1]) for i in range(0, n_ev, 2)]
+    compile_ms = d[0]
+    apply_ms = [d[1 + 2 * t] for t in range(S)]
+    advance_ms = [d[2 + 2 * t] for t in range(S)]
+    apply_avg = sum(apply_ms) / S
+    apply_bytes = B * V * elt + B * Wd * 4 + B * 4
+    compile_bytes = N * Wd * 4
+    apply_gbs = apply_bytes / (apply_avg * 1e-3) / 1e9
+    compile_gbs = compile_bytes / (compile_ms * 1e-3) / 1e9
+
+    # ---- e2e: host strings -> trie_build -> compile -> decode with H2D logits, D2H tokens
+    host_logits = [lg.cpu().pin_memory() for lg in logits]
+    host_tok = torch.zeros((S, B), dtype=torch.int32).pin_memory()
+    dlog = torch.empty_like(logits[0])
+    e2e_mask = torch.empty_like(mask)
+    h2d = int(w.set_bytes.nbytes + w.set_offsets.nbytes + sum(x.numel() * x.element_size() for x in host_logits))
+    d2h = S * B * 4
+
+    def e2e_step():
+        hh = T.trie_build(w.set_bytes, w.set_offsets)
+        T.trie_compile_masks(hh, w.vocab_bytes, w.vocab_offsets, V, e2e_mask, stream)
+        states.zero_()
+        for t in range(S):
+            dlog.copy_(host_logits[t], non_blocking=True)
+            T.trie_apply_mask(hh, dlog, states, stream)
+            torch.argmax(dlog, dim=1, out=tok64)
+            tok.copy_(tok64)
+            T.trie_advance(hh, states, tok, err, stream)
+            host_tok[t].copy_(tok, non_blocking=True)
+        stream.synchronize()
+        hh.destroy()
+
+    with torch.cuda.stream(stream):
+        e2e_step()
+        if dist is not None:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+    if dist is not None:
+        tt = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_s = float(tt.item())
+
+    if rank != 0:
+        return
+    traffic = ncu_traffic("k_apply_vec", w.name)
+    traffic_c = ncu_traffic("k_mask_fill", w.name)
+    line = {
+        "metric": METRIC,
+        "value": world * N * V / (ms_per_step * 1e-3),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "u32 mask / " + w.dtype,
+        "data": "synthetic",
+        "impl": "gb300",
+        "config": {"workload": w.name, "K": w.K, "V": V, "batch": B, "decode_steps": S, "N_nodes": N,
+                   "N_chars": h.num_chars, "r": round(N / max(1, h.num_chars), 4),
+                   "parallelism": f"replicas x{world}",
+                   "l2": f"inputs larger than L2: logits {S * B * V * elt / 1e9:.2f} GB, "
+                         f"mask {compile_bytes / 1e9:.2f} GB",
+                   "graph": graph is not None},
+        "roofline": {"bound": "hbm", "achieved": apply_gbs, "peak": hbm, "unit": "GB/s",
+                     "frac": apply_gbs / hbm, "traffic": traffic, "kernel": "k_apply_vec",
+                     "bytes_per_launch": apply_bytes, "us_per_launch": apply_avg * 1e3,
+                     "peak_kind": peak_kind, "timing": timing_src},
+        "roofline_compile": {"bound": "hbm", "achieved": compile_gbs, "peak": hbm, "unit": "GB/s",
+                             "frac": compile_gbs / hbm, "traffic": traffic_c,
+                             "kernel": "k_mask_fill + k_mask_patch", "bytes_per_launch": compile_bytes,
+                             "ms": compile_ms, "pairs_per_s": N * V / (compile_ms * 1e-3),
+                             "peak_kind": peak_kind},
+        "breakdown": {"compile_ms": compile_ms, "apply_us_avg": apply_avg * 1e3,
+                      "advance_us_avg": sum(advance_ms) / S * 1e3, "host_trie_build_ms": host_build_ms,
+                      "cold_compile_ms": cold_compile_ms,
+                      "apply_gbs_conventional_rw": (2 * B * V * elt + B * Wd * 4) / (apply_avg * 1e-3) / 1e9},
+        "e2e": {"value": world * N * V / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3},
+        "gpu_launches": args.steps * (2 + 2 * S),
+        "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds / 5, 5, 1)
+    print(json.dumps(line))
+
+
+def W_logits(w, s, dev):
+    from paper_2608_12574_gb300 import workloads as W
+    return W.logits(w, s, device=str(dev))
+
+
+def main():
+    args = parse_args()
+    from paper_2608_12574_gb300 import workloads as W
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    w = W.config(args.config)
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args, w)
+        return
+    from paper_2608_12574_gb300 import _build
+    if rank == 0:
+        _build.build()
+    dist = None
+    if world > 1:
+        import torch
+        import torch.distributed as dist_
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist_.init_process_group("nccl")
+        dist = dist_
+        dist.barrier()
+    run_gpu(args, w, rank, world, dist)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

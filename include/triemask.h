@@ -1,0 +1,181 @@
+/*
+ * triemask.h -- C ABI of libtriemask.so: GB300 (sm_103a) trie-automaton token
+ * masks for constrained decoding over a finite string set.
+ *
+ * Method: Xu & Bouyarmane, "Trie Automata for Constrained Decoding over Large
+ * Finite Sets". Given an enum set E = {e_1..e_K} of byte strings and a byte
+ * vocabulary of V tokens, the library
+ *   1. builds the byte trie of E on the host (Sec. 4.1; App. G.1 Step 1),
+ *   2. computes valid[n] for every trie node n as a dense bitmask
+ *      [num_nodes, ceil(V/32)] uint32 on the GPU (Sec. 4.1-4.2; App. G.1
+ *      Steps 3-4; App. G.5 proof conditions (i)+(ii); EOS handling per App.
+ *      G.5 "EOS token handling"),
+ *   3. advances a batch of decode states by their sampled tokens,
+ *      s' = delta*(s, bytes(token)) (Sec. 2, Eq. 1),
+ *   4. writes -inf into the logits of every token not in valid[s]
+ *      (Sec. 4.2 last paragraph; App. H.3 "bitmask application").
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * Strings and tokens are raw bytes (every byte 0x00-0xFF is legal), passed
+ * as a concatenated byte array plus int64 offsets[count+1]; string i is
+ * bytes[offsets[i] : offsets[i+1]]. Host pointers are read during the call
+ * only; the library keeps its own copies.
+ *
+ * Node ids: breadth-first from the root, siblings by ascending byte, root 0.
+ * Equivalently, the distinct prefixes of E sorted by (length, bytes).
+ * A forest (trie_build_many) concatenates the tries of its sets in order;
+ * states are then global node ids and trie_root() gives each set's root.
+ *
+ * Token V-1 is EOS: its bytes are ignored. It is allowed at node n iff some
+ * e_i ends at n. Any other token with no bytes is never allowed.
+ *
+ * Mask layout: row n is W = ceil(V/32) uint32 words; token v is bit (v % 32)
+ * of word v / 32 (LSB first); bits >= V are zero.
+ *
+ * States: a node id, TRIE_STATE_FINISHED (EOS was taken at a terminal node)
+ * or TRIE_STATE_DEAD (a move the trie does not allow). FINISHED and DEAD
+ * rows allow only EOS.
+ *
+ * Errors: every call returns TRIE_OK (0) or a negative code and never
+ * aborts; trie_last_error() gives a message for the calling thread. Argument
+ * checks are synchronous. Kernel launch failures return TRIE_ECUDA; faults
+ * inside an asynchronous kernel surface on a later CUDA call or sync.
+ * Kernels never trap.
+ *
+ * Ownership: the library owns the trie (host and device copies) and the
+ * packed vocabularies (device). The caller owns every device buffer it
+ * passes (mask, states, tokens, logits, error counter). The mask passed to
+ * trie_compile_masks must stay allocated and unchanged while the handle is
+ * used by trie_apply_mask (the handle keeps a non-owning pointer to it).
+ *
+ * Streams: device work is enqueued on the given stream (0 = legacy default)
+ * and is asynchronous with respect to the host. Concurrent trie_advance /
+ * trie_apply_mask calls on one handle are safe (they only read the trie and
+ * the mask); trie_compile_masks and trie_destroy must not race with other
+ * calls on the same handle.
+ */
+#ifndef TRIEMASK_H
+#define TRIEMASK_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct trie_s *trie_t; /* opaque; owned by the library */
+
+enum {
+    TRIE_OK = 0,
+    TRIE_EINVAL = -1, /* bad argument (null pointer, bad offsets, size out of range) */
+    TRIE_ENOMEM = -2, /* host or device allocation failed */
+    TRIE_ECUDA = -3,  /* a CUDA runtime call failed */
+    TRIE_ESTATE = -4  /* call out of order (e.g. apply before compile) */
+};
+
+enum { TRIE_DTYPE_F32 = 0, TRIE_DTYPE_BF16 = 1 };
+
+#define TRIE_STATE_DEAD (-1)
+#define TRIE_STATE_FINISHED (-2)
+
+/* Build the byte trie of K strings (Sec. 4.1: insert each value character by
+ * character, merging shared prefixes; App. G.1 Step 1). Host only: no device
+ * memory is touched until the first device call on the handle.
+ *   bytes    host, offsets[K] bytes (may be NULL when that is 0)
+ *   offsets  host int64[K+1], non-decreasing, offsets[0] >= 0
+ *   K        >= 0; K = 0 gives a lone root
+ *   out      receives the handle (release with trie_destroy)
+ * Duplicate strings collapse; the empty string marks the root terminal.
+ * Returns TRIE_EINVAL on bad offsets or K < 0, TRIE_ENOMEM on allocation
+ * failure or more than 2^31-1 nodes. */
+int trie_build(const uint8_t *bytes, const int64_t *offsets, int32_t K, trie_t *out);
+
+/* Build one forest of M independent tries (per-request sets). Set i holds the
+ * strings set_offsets[i] .. set_offsets[i+1]-1 of the string list given by
+ * (bytes, offsets). Node ids of set i start at trie_root(h, i).
+ *   set_offsets  host int32[M+1], non-decreasing, set_offsets[0] = 0
+ *   M            >= 1
+ * Sets are built on host threads in parallel. Errors as trie_build. */
+int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
+                    int32_t M, trie_t *out);
+
+/* Number of nodes (the mask has this many rows); -1 for a NULL handle. */
+int32_t trie_num_nodes(trie_t h);
+
+/* Root node id of set i (0 for a single trie); -1 if i is out of range. */
+int32_t trie_root(trie_t h, int32_t i);
+
+/* Number of sets in the handle (1 for trie_build). */
+int32_t trie_num_sets(trie_t h);
+
+/* Trie statistics: total bytes of the distinct strings (N_chars of Sec. 4.1)
+ * and the deepest node's depth. */
+int64_t trie_num_chars(trie_t h);
+int32_t trie_max_depth(trie_t h);
+
+/* Copy the host CSR out (for inspection and tests). Each pointer may be NULL.
+ *   parent       int32[N]   parent id, -1 for a root
+ *   label        uint8[N]   byte on the edge into the node (0 for a root)
+ *   terminal     uint8[N]   1 where some string of the node's set ends
+ *   first_child  int32[N]   id of the first child (children are contiguous
+ *                           and sorted by byte); -1 for a leaf */
+int trie_get_csr(trie_t h, int32_t *parent, uint8_t *label, uint8_t *terminal,
+                 int32_t *first_child);
+
+/* Compute valid[n] for every node n of the handle into a dense bitmask
+ * (Sec. 4.2: the per-node valid sets, here for all nodes at once; App. G.1
+ * Steps 3-4).
+ *   vocab_bytes, vocab_offsets  host; V tokens, token V-1 is EOS
+ *   V        2 <= V <= 2^31-32; every token at most 65535 bytes
+ *   d_mask   device, caller-allocated, num_nodes * ceil(V/32) uint32,
+ *            16-byte aligned for the vector path (any 4-byte alignment works)
+ *   stream   CUDA stream for the kernels
+ * The vocabulary is packed and uploaded on its first use on the current
+ * device (the per-tokenizer step the paper caches, Sec. 4.2) and reused by
+ * later calls with byte-identical vocab arrays. The first device call on a
+ * handle also uploads the trie. d_mask is written asynchronously on stream;
+ * the handle records (d_mask, V, vocabulary) for trie_advance and
+ * trie_apply_mask. Errors: TRIE_EINVAL (bad sizes or pointers), TRIE_ENOMEM,
+ * TRIE_ECUDA. */
+int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets,
+                       int32_t V, uint32_t *d_mask, cudaStream_t stream);
+
+/* Advance B decode states in place by one token each: s' = delta*(s, bytes(t))
+ * (Sec. 2, Eq. 1; the paper's stateless character walk).
+ *   d_states  device int32[B], in/out
+ *   d_tokens  device int32[B]
+ *   d_err     device int32 counter or NULL; incremented once for every state
+ *             that moves into DEAD from a state other than DEAD
+ * Rules: a token whose bytes walk from node s inside the trie -> the end node;
+ * EOS at a terminal node -> FINISHED; FINISHED + EOS -> FINISHED; DEAD stays
+ * DEAD; every other move (including a token id outside [0, V) or a state
+ * that is not a node) -> DEAD. Needs a prior trie_compile_masks on the handle
+ * (for its vocabulary), else TRIE_ESTATE. B = 0 is a no-op. */
+int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B,
+                 int32_t *d_err, cudaStream_t stream);
+
+/* Mask a batch of logits in place (Sec. 4.2; App. H.3): logits[b][v] becomes
+ * -inf (fp32 0xFF800000, bf16 0xFF80) where bit v of the row of d_states[b]
+ * is clear; allowed entries keep their bits exactly.
+ *   d_logits  device [B, V] contiguous, dtype TRIE_DTYPE_F32 or _BF16
+ *   d_states  device int32[B]; FINISHED, DEAD and ids that are not nodes use
+ *             the row {EOS}
+ *   V         must equal the V of the last trie_compile_masks on the handle
+ * Uses the mask recorded by the last trie_compile_masks (TRIE_ESTATE if
+ * none). B = 0 is a no-op. */
+int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B,
+                    int32_t V, cudaStream_t stream);
+
+/* Release the handle, its host arrays and its device copy of the trie.
+ * Synchronises the device first if device memory is held. NULL is a no-op. */
+int trie_destroy(trie_t h);
+
+/* Message of the last error on the calling thread ("" if none). */
+const char *trie_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TRIEMASK_H */

@@ -1,0 +1,372 @@
+// C ABI of libtriemask (declared in include/triemask.h): argument checks,
+// handle and device-memory management, the per-device vocabulary cache, and
+// the kernel launches.
+#include <stdint.h>
+#include <string.h>
+
+#include <algorithm>
+#include <memory>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "../../include/triemask.h"
+#include "tm_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int code, const std::string &msg) {
+    g_last_error = msg;
+    return code;
+}
+
+int fail_cuda(cudaError_t e, const char *what) {
+    return fail(TRIE_ECUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+// Restores the caller's current device on scope exit.
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+int num_sms(int dev) {
+    static std::mutex mu;
+    static std::vector<int> cache;
+    std::lock_guard<std::mutex> lk(mu);
+    if (int(cache.size()) <= dev) cache.resize(size_t(dev) + 1, 0);
+    if (!cache[size_t(dev)]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+        cache[size_t(dev)] = n;
+    }
+    return cache[size_t(dev)];
+}
+
+// Carves 256-byte aligned sub-arrays out of one device allocation.
+struct Layout {
+    size_t total = 0;
+    size_t add(size_t bytes) {
+        size_t off = total;
+        total += (bytes + 255) / 256 * 256;
+        return off;
+    }
+};
+
+std::mutex g_vocab_mu;
+// Most recent last. Never destroyed, so no device memory is freed during
+// static destruction at process exit (the CUDA runtime may be gone by then).
+std::vector<std::shared_ptr<tmk::DevVocab>> &g_vocabs = *new std::vector<std::shared_ptr<tmk::DevVocab>>();
+constexpr size_t kVocabCacheSize = 4;
+
+int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
+              std::shared_ptr<tmk::DevVocab> *out) {
+    const int64_t b0 = vo[0], b1 = vo[V];
+    if (b0 < 0 || b1 < b0) return fail(TRIE_EINVAL, "vocab offsets must be non-negative and non-decreasing");
+    const size_t nbytes = size_t(b1 - b0);
+    if (nbytes && !vb) return fail(TRIE_EINVAL, "vocab_bytes is NULL");
+    std::lock_guard<std::mutex> lk(g_vocab_mu);
+    for (size_t i = 0; i < g_vocabs.size(); i++) {
+        auto &c = g_vocabs[i];
+        if (c->device == dev && c->V == V && c->src_bytes.size() == nbytes &&
+            memcmp(c->src_offsets.data(), vo, sizeof(int64_t) * (size_t(V) + 1)) == 0 &&
+            (nbytes == 0 || memcmp(c->src_bytes.data(), vb + b0, nbytes) == 0)) {
+            *out = c;
+            std::rotate(g_vocabs.begin() + long(i), g_vocabs.begin() + long(i) + 1, g_vocabs.end());
+            return TRIE_OK;
+        }
+    }
+    tmk::HostVocab hv;
+    std::string err;
+    try {
+        err = tmk::pack_vocab(vb, vo, V, &hv);
+    } catch (const std::bad_alloc &) {
+        return fail(TRIE_ENOMEM, "host allocation failed while packing the vocabulary");
+    }
+    if (!err.empty()) return fail(TRIE_EINVAL, err);
+    auto dv = std::make_shared<tmk::DevVocab>();
+    dv->device = dev;
+    dv->V = V;
+    dv->max_len = hv.max_len;
+    dv->ht_mask = hv.ht_mask;
+    Layout L;
+    const size_t o_off = L.add(sizeof(uint32_t) * hv.tok_off.size());
+    const size_t o_len = L.add(sizeof(uint16_t) * hv.tok_len.size());
+    const size_t o_blob = L.add(hv.blob.size());
+    const size_t o_key = L.add(sizeof(uint64_t) * hv.ht_key.size());
+    const size_t o_val = L.add(sizeof(int32_t) * hv.ht_val.size());
+    cudaError_t e = cudaMalloc(&dv->base, L.total);
+    if (e != cudaSuccess) {
+        dv->base = nullptr;
+        cudaGetLastError();
+        return fail(TRIE_ENOMEM, std::string("cudaMalloc for the vocabulary: ") + cudaGetErrorString(e));
+    }
+    char *base = static_cast<char *>(dv->base);
+    struct Up { size_t off; const void *src; size_t n; } ups[] = {
+        {o_off, hv.tok_off.data(), sizeof(uint32_t) * hv.tok_off.size()},
+        {o_len, hv.tok_len.data(), sizeof(uint16_t) * hv.tok_len.size()},
+        {o_blob, hv.blob.data(), hv.blob.size()},
+        {o_key, hv.ht_key.data(), sizeof(uint64_t) * hv.ht_key.size()},
+        {o_val, hv.ht_val.data(), sizeof(int32_t) * hv.ht_val.size()},
+    };
+    for (const Up &u : ups) {
+        e = cudaMemcpy(base + u.off, u.src, u.n, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return fail_cuda(e, "uploading the vocabulary");
+    }
+    dv->tok_off = reinterpret_cast<const uint32_t *>(base + o_off);
+    dv->tok_len = reinterpret_cast<const uint16_t *>(base + o_len);
+    dv->blob = reinterpret_cast<const uint8_t *>(base + o_blob);
+    dv->ht_key = reinterpret_cast<const uint64_t *>(base + o_key);
+    dv->ht_val = reinterpret_cast<const int32_t *>(base + o_val);
+    try {
+        dv->src_offsets.assign(vo, vo + V + 1);
+        dv->src_bytes.assign(vb ? vb + b0 : nullptr, vb ? vb + b1 : nullptr);
+    } catch (const std::bad_alloc &) {
+        return fail(TRIE_ENOMEM, "host allocation failed while caching the vocabulary");
+    }
+    g_vocabs.push_back(dv);
+    if (g_vocabs.size() > kVocabCacheSize) g_vocabs.erase(g_vocabs.begin());
+    *out = dv;
+    return TRIE_OK;
+}
+
+// Uploads the trie on first use; the handle is bound to that device.
+int ensure_device_trie(trie_t h, int dev) {
+    std::lock_guard<std::mutex> lk(h->mu);
+    if (h->dev.base) {
+        if (h->dev.device != dev)
+            return fail(TRIE_EINVAL, "handle was uploaded to device " + std::to_string(h->dev.device) +
+                                         ", called on device " + std::to_string(dev));
+        return TRIE_OK;
+    }
+    const tmk::HostTrie &t = h->host;
+    const size_t n = size_t(t.n);
+    Layout L;
+    const size_t o_par = L.add(sizeof(int32_t) * n);
+    const size_t o_lab = L.add(n);
+    const size_t o_term = L.add(n);
+    const size_t o_fc = L.add(sizeof(int32_t) * n);
+    const size_t o_bits = L.add(sizeof(uint32_t) * 8 * n);
+    void *base = nullptr;
+    cudaError_t e = cudaMalloc(&base, L.total);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(TRIE_ENOMEM, std::string("cudaMalloc for the trie: ") + cudaGetErrorString(e));
+    }
+    char *b = static_cast<char *>(base);
+    struct Up { size_t off; const void *src; size_t n; } ups[] = {
+        {o_par, t.parent.data(), sizeof(int32_t) * n},
+        {o_lab, t.label.data(), n},
+        {o_term, t.terminal.data(), n},
+        {o_fc, t.first_child.data(), sizeof(int32_t) * n},
+        {o_bits, t.child_bits.data(), sizeof(uint32_t) * 8 * n},
+    };
+    for (const Up &u : ups) {
+        e = cudaMemcpy(b + u.off, u.src, u.n, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) {
+            cudaFree(base);
+            return fail_cuda(e, "uploading the trie");
+        }
+    }
+    h->dev.device = dev;
+    h->dev.base = base;
+    h->dev.parent = reinterpret_cast<const int32_t *>(b + o_par);
+    h->dev.label = reinterpret_cast<const uint8_t *>(b + o_lab);
+    h->dev.terminal = reinterpret_cast<const uint8_t *>(b + o_term);
+    h->dev.first_child = reinterpret_cast<const int32_t *>(b + o_fc);
+    h->dev.child_bits = reinterpret_cast<const uint32_t *>(b + o_bits);
+    return TRIE_OK;
+}
+
+int current_device(int *dev) {
+    cudaError_t e = cudaGetDevice(dev);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail_cuda(e, "cudaGetDevice");
+    }
+    return TRIE_OK;
+}
+
+int finish_build(std::string err, trie_s *h, trie_t *out) {
+    if (!err.empty()) {
+        delete h;
+        return fail(err.find("exceed") != std::string::npos ? TRIE_ENOMEM : TRIE_EINVAL, err);
+    }
+    *out = h;
+    return TRIE_OK;
+}
+
+}  // namespace
+
+tmk::DevVocab::~DevVocab() {
+    if (base) {
+        DeviceGuard g(device);
+        cudaFree(base);
+    }
+}
+
+extern "C" {
+
+const char *trie_last_error(void) { return g_last_error.c_str(); }
+
+int trie_build(const uint8_t *bytes, const int64_t *offsets, int32_t K, trie_t *out) {
+    if (!out) return fail(TRIE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (K < 0) return fail(TRIE_EINVAL, "K must be >= 0");
+    if (K > 0 && !offsets) return fail(TRIE_EINVAL, "offsets is NULL");
+    if (K > 0 && offsets[K] > offsets[0] && !bytes) return fail(TRIE_EINVAL, "bytes is NULL");
+    trie_s *h = new (std::nothrow) trie_s;
+    if (!h) return fail(TRIE_ENOMEM, "host allocation failed");
+    std::string err;
+    try {
+        static const int64_t zero = 0;
+        err = tmk::build_trie(bytes, K > 0 ? offsets : &zero, 0, K, &h->host);
+    } catch (const std::bad_alloc &) {
+        delete h;
+        return fail(TRIE_ENOMEM, "host allocation failed while building the trie");
+    }
+    return finish_build(err, h, out);
+}
+
+int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
+                    int32_t M, trie_t *out) {
+    if (!out) return fail(TRIE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (M < 1) return fail(TRIE_EINVAL, "M must be >= 1");
+    if (!set_offsets) return fail(TRIE_EINVAL, "set_offsets is NULL");
+    if (set_offsets[0] != 0) return fail(TRIE_EINVAL, "set_offsets[0] must be 0");
+    for (int32_t i = 0; i < M; i++)
+        if (set_offsets[i + 1] < set_offsets[i]) return fail(TRIE_EINVAL, "set_offsets must be non-decreasing");
+    const int32_t K = set_offsets[M];
+    if (K > 0 && !offsets) return fail(TRIE_EINVAL, "offsets is NULL");
+    if (K > 0 && offsets[K] > offsets[0] && !bytes) return fail(TRIE_EINVAL, "bytes is NULL");
+    trie_s *h = new (std::nothrow) trie_s;
+    if (!h) return fail(TRIE_ENOMEM, "host allocation failed");
+    std::string err;
+    try {
+        static const int64_t zero = 0;
+        err = tmk::build_forest(bytes, K > 0 ? offsets : &zero, set_offsets, M, &h->host);
+    } catch (const std::bad_alloc &) {
+        delete h;
+        return fail(TRIE_ENOMEM, "host allocation failed while building the forest");
+    }
+    return finish_build(err, h, out);
+}
+
+int32_t trie_num_nodes(trie_t h) { return h ? h->host.n : -1; }
+
+int32_t trie_num_sets(trie_t h) { return h ? int32_t(h->host.roots.size()) : -1; }
+
+int32_t trie_root(trie_t h, int32_t i) {
+    if (!h || i < 0 || i >= int32_t(h->host.roots.size())) return -1;
+    return h->host.roots[size_t(i)];
+}
+
+int64_t trie_num_chars(trie_t h) { return h ? h->host.n_chars : -1; }
+
+int32_t trie_max_depth(trie_t h) { return h ? h->host.max_depth : -1; }
+
+int trie_get_csr(trie_t h, int32_t *parent, uint8_t *label, uint8_t *terminal, int32_t *first_child) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    const size_t n = size_t(h->host.n);
+    if (parent) memcpy(parent, h->host.parent.data(), sizeof(int32_t) * n);
+    if (label) memcpy(label, h->host.label.data(), n);
+    if (terminal) memcpy(terminal, h->host.terminal.data(), n);
+    if (first_child) memcpy(first_child, h->host.first_child.data(), sizeof(int32_t) * n);
+    return TRIE_OK;
+}
+
+int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                       uint32_t *d_mask, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    if (!d_mask) return fail(TRIE_EINVAL, "d_mask is NULL");
+    if (reinterpret_cast<uintptr_t>(d_mask) & 3u) return fail(TRIE_EINVAL, "d_mask must be 4-byte aligned");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    if ((rc = ensure_device_trie(h, dev)) != TRIE_OK) return rc;
+    const int64_t W = (int64_t(V) + 31) / 32;
+    const int32_t n = h->host.n;
+    const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
+    const int sms = num_sms(dev);
+    cudaError_t e = tmk::launch_mask_fill(d_mask, int64_t(n) * W, sms, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "mask fill launch");
+    e = tmk::launch_mask_patch(h->dev, n, *voc, lmax, d_mask, W, sms, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "mask patch launch");
+    std::lock_guard<std::mutex> lk(h->mu);
+    h->vocab = voc;
+    h->mask = d_mask;
+    h->mask_V = V;
+    return TRIE_OK;
+}
+
+int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B, int32_t *d_err,
+                 cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_states || !d_tokens)) return fail(TRIE_EINVAL, "d_states / d_tokens is NULL");
+    std::shared_ptr<tmk::DevVocab> voc;
+    {
+        std::lock_guard<std::mutex> lk(h->mu);
+        voc = h->vocab;
+    }
+    if (!voc) return fail(TRIE_ESTATE, "trie_advance before trie_compile_masks on this handle");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_advance(h->dev, h->host.n, *voc, d_states, d_tokens, B, d_err, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "advance launch");
+    return TRIE_OK;
+}
+
+int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                    cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_logits || !d_states)) return fail(TRIE_EINVAL, "d_logits / d_states is NULL");
+    uint32_t *mask;
+    int32_t mV;
+    {
+        std::lock_guard<std::mutex> lk(h->mu);
+        mask = h->mask;
+        mV = h->mask_V;
+    }
+    if (!mask) return fail(TRIE_ESTATE, "trie_apply_mask before trie_compile_masks on this handle");
+    if (V != mV) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
+    if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
+        return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_apply(d_logits, dtype, mask, d_states, B, V, h->host.n, num_sms(dev), stream);
+    if (e != cudaSuccess) return fail_cuda(e, "apply launch");
+    return TRIE_OK;
+}
+
+int trie_destroy(trie_t h) {
+    if (!h) return TRIE_OK;
+    if (h->dev.base) {
+        DeviceGuard g(h->dev.device);
+        cudaFree(h->dev.base);  // waits for work on the device that may still read it
+    }
+    delete h;
+    return TRIE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,122 @@
+// Internal structures of libtriemask shared by the host builder, the kernels
+// and the C ABI. Not part of the public interface.
+#pragma once
+
+#include <stdint.h>
+
+#include <atomic>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include <cuda_runtime_api.h>
+
+namespace tmk {
+
+// ----------------------------------------------------------------- host trie
+// Byte trie in breadth-first order, siblings by ascending byte (Sec. 4.1).
+// Children of a node are contiguous; child_bits is the 256-bit set of child
+// labels, so the child for byte c is first_child + popcount(bits below c).
+struct HostTrie {
+    int32_t n = 0;                       // nodes (all sets of a forest)
+    std::vector<int32_t> parent;         // -1 for a root
+    std::vector<uint8_t> label;          // byte on the incoming edge
+    std::vector<uint8_t> terminal;       // some string ends here
+    std::vector<int32_t> first_child;    // -1 for a leaf
+    std::vector<uint32_t> child_bits;    // [n * 8]
+    std::vector<int32_t> roots;          // root id of each set
+    int64_t n_chars = 0;                 // total bytes of the distinct strings
+    int32_t max_depth = 0;
+};
+
+// Return "" on success, else an error message. build_trie takes strings
+// first..last-1; build_forest builds set i from strings
+// set_offsets[i]..set_offsets[i+1]-1 on host threads and concatenates them.
+std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t first, int32_t last,
+                       HostTrie *out);
+std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
+                         int32_t M, HostTrie *out);
+
+// -------------------------------------------------------------- vocabulary
+// Token strings packed for 16-byte vector loads plus an open-addressing hash
+// table from (length, bytes) to token id, used to find the tokens that end
+// at a trie node.
+struct HostVocab {
+    int32_t V = 0;
+    int32_t max_len = 0;                 // longest token with bytes (EOS excluded)
+    std::vector<uint32_t> tok_off;       // [V] start of token bytes in blob (16-byte aligned)
+    std::vector<uint16_t> tok_len;       // [V] byte length; EOS and byte-less tokens: 0
+    std::vector<uint8_t> blob;           // token bytes, each token 16-byte aligned
+    std::vector<uint64_t> ht_key;        // [S] 0 = empty slot
+    std::vector<int32_t> ht_val;         // [S] token id
+    uint32_t ht_mask = 0;                // S - 1 (S a power of two)
+};
+
+std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, HostVocab *out);
+
+// Polynomial string hash used by the table: Horner over (byte + 1) with base
+// kHashBase, modulo 2^64, then mixed with the length. The kernel extends it
+// one byte to the left per trie edge it climbs.
+constexpr uint64_t kHashBase = 0x100000001B3ull;
+#if defined(__CUDACC__)
+__host__ __device__
+#endif
+inline uint64_t hash_finish(uint64_t h, uint32_t len) {
+    uint64_t z = h ^ (uint64_t(len) * 0x9E3779B97F4A7C15ull);
+    z = (z ^ (z >> 33)) * 0xFF51AFD7ED558CCDull;
+    z = (z ^ (z >> 33)) * 0xC4CEB9FE1A85EC53ull;
+    z ^= z >> 33;
+    return z | 1ull;  // 0 marks an empty slot
+}
+
+// ------------------------------------------------------------ device copies
+struct DevVocab {
+    int device = -1;
+    int32_t V = 0;
+    int32_t max_len = 0;
+    uint32_t ht_mask = 0;
+    void *base = nullptr;                // one allocation holding all arrays
+    const uint32_t *tok_off = nullptr;
+    const uint16_t *tok_len = nullptr;
+    const uint8_t *blob = nullptr;
+    const uint64_t *ht_key = nullptr;
+    const int32_t *ht_val = nullptr;
+    // host copy of the caller's arrays, to recognise the same vocabulary later
+    std::vector<uint8_t> src_bytes;
+    std::vector<int64_t> src_offsets;
+    ~DevVocab();
+};
+
+struct DevTrie {
+    int device = -1;
+    void *base = nullptr;
+    const int32_t *parent = nullptr;
+    const uint8_t *label = nullptr;
+    const uint8_t *terminal = nullptr;
+    const int32_t *first_child = nullptr;
+    const uint32_t *child_bits = nullptr;
+};
+
+}  // namespace tmk
+
+// The opaque handle of the C ABI.
+struct trie_s {
+    tmk::HostTrie host;
+    std::mutex mu;                       // guards dev / vocab / mask fields
+    tmk::DevTrie dev;
+    std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
+    uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
+    int32_t mask_V = 0;
+};
+
+namespace tmk {
+// Kernel launchers (kernels.cu). Each returns the launch's cudaError_t.
+cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaStream_t st);
+cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                              uint32_t *mask, int64_t W, int num_sms, cudaStream_t st);
+cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t *states,
+                           const int32_t *tokens, int32_t B, int32_t *err, cudaStream_t st);
+cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
+                         int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st);
+}  // namespace tmk

@@ -1,0 +1,238 @@
+"""Python binding of libtriemask.so (C ABI in include/triemask.h).
+
+Argument marshalling only: every step of the trie automaton runs in the
+library (host trie builder + sm_103a kernels). Host arrays are numpy arrays;
+device buffers are torch CUDA tensors, passed by pointer together with the
+current torch stream. There is no fallback: if the library has not been
+built, the first call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+
+TRIE_OK, TRIE_EINVAL, TRIE_ENOMEM, TRIE_ECUDA, TRIE_ESTATE = 0, -1, -2, -3, -4
+TRIE_DTYPE_F32, TRIE_DTYPE_BF16 = 0, 1
+TRIE_STATE_DEAD, TRIE_STATE_FINISHED = -1, -2
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtriemask.so")
+_lock = threading.Lock()
+_lib = None
+
+# every symbol include/triemask.h declares: (restype, argtypes)
+_P, _I32, _I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+SIGNATURES = {
+    "trie_build": (ctypes.c_int, [_P, _P, _I32, _P]),
+    "trie_build_many": (ctypes.c_int, [_P, _P, _P, _I32, _P]),
+    "trie_num_nodes": (_I32, [_P]),
+    "trie_root": (_I32, [_P, _I32]),
+    "trie_num_sets": (_I32, [_P]),
+    "trie_num_chars": (_I64, [_P]),
+    "trie_max_depth": (_I32, [_P]),
+    "trie_get_csr": (ctypes.c_int, [_P, _P, _P, _P, _P]),
+    "trie_compile_masks": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "trie_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "trie_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
+    "trie_destroy": (ctypes.c_int, [_P]),
+    "trie_last_error": (ctypes.c_char_p, []),
+}
+
+
+class TrieError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"libtriemask error {code}: {msg}")
+        self.code = code
+
+
+def load_library(path: str = LIB_PATH):
+    """Load libtriemask.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(path):
+                raise RuntimeError(f"{path} is missing: build it with "
+                                   "`python -c 'import __graft_entry__ as g; g.build()'`")
+            lib = ctypes.CDLL(path)
+            for name, (res, args) in SIGNATURES.items():
+                f = getattr(lib, name)
+                f.restype = res
+                f.argtypes = args
+            _lib = lib
+    return _lib
+
+
+def trie_last_error() -> str:
+    return load_library().trie_last_error().decode(errors="replace")
+
+
+def _check(rc: int) -> None:
+    if rc != TRIE_OK:
+        raise TrieError(rc, trie_last_error())
+
+
+def _host(a, dtype) -> np.ndarray:
+    a = np.ascontiguousarray(a, dtype=dtype)
+    return a
+
+
+def _hp(a: np.ndarray):
+    return ctypes.c_void_p(a.ctypes.data) if a.size else None
+
+
+def _stream(stream, device=None) -> ctypes.c_void_p:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream(device)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t, dtypes, name: str):
+    import torch
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype not in dtypes:
+        raise TypeError(f"{name} must have dtype in {dtypes}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class Trie:
+    """Owns one trie handle (released by trie_destroy or garbage collection)."""
+
+    def __init__(self, handle: ctypes.c_void_p):
+        self._lib = load_library()
+        self.handle = handle
+
+    @property
+    def num_nodes(self) -> int:
+        return self._lib.trie_num_nodes(self.handle)
+
+    @property
+    def num_sets(self) -> int:
+        return self._lib.trie_num_sets(self.handle)
+
+    @property
+    def num_chars(self) -> int:
+        return self._lib.trie_num_chars(self.handle)
+
+    @property
+    def max_depth(self) -> int:
+        return self._lib.trie_max_depth(self.handle)
+
+    def root(self, i: int = 0) -> int:
+        r = self._lib.trie_root(self.handle, i)
+        if r < 0:
+            raise IndexError(i)
+        return r
+
+    def roots(self) -> np.ndarray:
+        return np.array([self.root(i) for i in range(self.num_sets)], np.int32)
+
+    def csr(self) -> dict[str, np.ndarray]:
+        n = self.num_nodes
+        out = {"parent": np.empty(n, np.int32), "label": np.empty(n, np.uint8),
+               "terminal": np.empty(n, np.uint8), "first_child": np.empty(n, np.int32)}
+        _check(self._lib.trie_get_csr(self.handle, *(_hp(out[k]) for k in
+                                                     ("parent", "label", "terminal", "first_child"))))
+        return out
+
+    def destroy(self) -> None:
+        if self.handle:
+            self._lib.trie_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def mask_words(V: int) -> int:
+    return (V + 31) // 32
+
+
+def trie_build(set_bytes, set_offsets) -> Trie:
+    """Byte trie of the K strings set_bytes[set_offsets[i]:set_offsets[i+1]]."""
+    lib = load_library()
+    b = _host(set_bytes, np.uint8)
+    o = _host(set_offsets, np.int64)
+    h = ctypes.c_void_p()
+    _check(lib.trie_build(_hp(b), _hp(o), len(o) - 1, ctypes.byref(h)))
+    return Trie(h)
+
+
+def trie_build_many(set_bytes, set_offsets, set_index) -> Trie:
+    """Forest of M tries; set i owns strings set_index[i]:set_index[i+1]."""
+    lib = load_library()
+    b = _host(set_bytes, np.uint8)
+    o = _host(set_offsets, np.int64)
+    si = _host(set_index, np.int32)
+    h = ctypes.c_void_p()
+    _check(lib.trie_build_many(_hp(b), _hp(o), _hp(si), len(si) - 1, ctypes.byref(h)))
+    return Trie(h)
+
+
+def trie_num_nodes(h: Trie) -> int:
+    return h.num_nodes
+
+
+def trie_root(h: Trie, i: int = 0) -> int:
+    return h.root(i)
+
+
+def alloc_mask(h: Trie, V: int, device=None):
+    """Uninitialised [num_nodes, ceil(V/32)] int32 device tensor for trie_compile_masks."""
+    import torch
+    return torch.empty((h.num_nodes, mask_words(V)), dtype=torch.int32,
+                       device=device if device is not None else "cuda")
+
+
+def trie_compile_masks(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stream=None) -> None:
+    """Fill d_mask ([num_nodes, ceil(V/32)] int32, CUDA) with every node's valid set."""
+    import torch
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    p = _dev(d_mask, (torch.int32,), "d_mask")
+    if d_mask.numel() < h.num_nodes * mask_words(V):
+        raise ValueError("d_mask is smaller than num_nodes * ceil(V/32) words")
+    _check(h._lib.trie_compile_masks(h.handle, _hp(vb), _hp(vo), V, p,
+                                     _stream(stream, d_mask.device)))
+
+
+def trie_advance(h: Trie, d_states, d_tokens, d_err=None, stream=None) -> None:
+    """states <- delta*(states, bytes(tokens)) in place (int32 CUDA tensors of length B)."""
+    import torch
+    B = d_states.numel()
+    if d_tokens.numel() != B:
+        raise ValueError("states and tokens differ in length")
+    ps = _dev(d_states, (torch.int32,), "d_states")
+    pt = _dev(d_tokens, (torch.int32,), "d_tokens")
+    pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
+    _check(h._lib.trie_advance(h.handle, ps, pt, B, pe, _stream(stream, d_states.device)))
+
+
+def trie_apply_mask(h: Trie, d_logits, d_states, stream=None) -> None:
+    """-inf into disallowed entries of d_logits ([B, V] fp32 or bf16, CUDA), in place."""
+    import torch
+    if d_logits.dim() != 2:
+        raise ValueError("d_logits must be [B, V]")
+    B, V = d_logits.shape
+    if d_states.numel() != B:
+        raise ValueError("d_states must have B entries")
+    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
+    if dtype is None:
+        raise TypeError("d_logits must be float32 or bfloat16")
+    pl = _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits")
+    ps = _dev(d_states, (torch.int32,), "d_states")
+    _check(h._lib.trie_apply_mask(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
+
+
+def trie_destroy(h: Trie) -> None:
+    h.destroy()

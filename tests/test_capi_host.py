@@ -1,0 +1,201 @@
+"""CPU-only checks of libtriemask: exported symbols, the host trie builder and
+argument validation (no device call is made here)."""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_12574_gb300 import triemask as T
+from paper_2608_12574_gb300 import workloads as W
+from pins import prefix_ids, random_case
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "triemask.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_12574_gb300 import _build
+    _build.build()
+    return T.load_library()
+
+
+def declared_functions() -> list[str]:
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]+?\b(trie_\w+)\s*\(", src, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for f in ("trie_build", "trie_compile_masks", "trie_advance", "trie_apply_mask", "trie_destroy",
+              "trie_build_many", "trie_last_error"):
+        assert f in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    for name in names:
+        assert hasattr(lib, name), name
+        assert name in T.SIGNATURES, f"binding does not declare {name}"
+    assert sorted(T.SIGNATURES) == names
+
+
+def _csr_matches_oracle(strings):
+    sb, so = W.pack(strings)
+    h = T.trie_build(sb, so)
+    ot = oracle.Trie(sb, so)
+    c = h.csr()
+    assert h.num_nodes == ot.num_nodes
+    assert np.array_equal(c["parent"], ot.parent)
+    assert np.array_equal(c["label"], ot.label)
+    assert np.array_equal(c["terminal"], ot.terminal)
+    assert h.num_chars == ot.num_chars
+    assert h.max_depth == (int(ot.depth.max()) if ot.num_nodes else 0)
+    # first child: smallest id whose parent is the node, -1 for leaves
+    fc = np.full(ot.num_nodes, -1, np.int64)
+    for c_ in range(ot.num_nodes - 1, 0, -1):
+        fc[ot.parent[c_]] = c_
+    assert np.array_equal(c["first_child"], fc)
+    return h
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_host_builder_matches_oracle_small(lib, oracle_lib, seed):
+    strings, _ = random_case(seed)
+    _csr_matches_oracle(strings)
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 3, 4])
+def test_host_builder_matches_oracle_configs(lib, oracle_lib, cfg):
+    w = W.config(cfg)
+    _csr_matches_oracle(W.unpack(w.set_bytes, w.set_offsets))
+
+
+def test_host_builder_closed_form_ids(lib):
+    strings = [b"get_user", b"get", b"", b"\x00\xff", b"get_user", b"got"]
+    sb, so = W.pack(strings)
+    h = T.trie_build(sb, so)
+    ids, E = prefix_ids(strings)
+    c = h.csr()
+    inv = {i: p for p, i in ids.items()}
+    for i in range(h.num_nodes):
+        p = inv[i]
+        assert c["terminal"][i] == (p in E)
+        if i:
+            assert c["label"][i] == p[-1] and c["parent"][i] == ids[p[:-1]]
+
+
+def test_forest_is_concatenation(lib, oracle_lib):
+    sets = [[b"ab", b"ac"], [], [b""], [b"xyz", b"x", b"xy"], [b"ab"]]
+    flat = [s for st in sets for s in st]
+    index = np.cumsum([0] + [len(s) for s in sets]).astype(np.int32)
+    sb, so = W.pack(flat)
+    h = T.trie_build_many(sb, so, index)
+    assert h.num_sets == len(sets)
+    c = h.csr()
+    for i, st in enumerate(sets):
+        r = h.root(i)
+        ot = oracle.Trie(*W.pack(st))
+        n = ot.num_nodes
+        assert c["parent"][r] == -1
+        par = c["parent"][r:r + n].astype(np.int64)
+        par[par >= 0] -= r
+        assert np.array_equal(par, ot.parent)
+        assert np.array_equal(c["label"][r:r + n], ot.label)
+        assert np.array_equal(c["terminal"][r:r + n], ot.terminal)
+        nxt = h.root(i + 1) if i + 1 < len(sets) else h.num_nodes
+        assert nxt - r == n
+    with pytest.raises(IndexError):
+        h.root(len(sets))
+
+
+def test_forest_of_config5_prefix(lib, oracle_lib):
+    w = W.dynamic_requests(6)
+    h = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+    strings = W.unpack(w.set_bytes, w.set_offsets)
+    total = 0
+    for i in range(6):
+        st = strings[w.set_index[i]:w.set_index[i + 1]]
+        total += len(prefix_ids(st)[0])
+    assert h.num_nodes == total
+
+
+def _rc(lib, *args):
+    return lib.trie_build(*args)
+
+
+def test_build_argument_errors(lib):
+    h = ctypes.c_void_p()
+    offs = np.array([0, 3, 2], np.int64)
+    b = np.frombuffer(b"abc", np.uint8).copy()
+    assert lib.trie_build(b.ctypes.data, offs.ctypes.data, 2, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert "non-decreasing" in T.trie_last_error()
+    assert lib.trie_build(b.ctypes.data, offs.ctypes.data, -1, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert lib.trie_build(b.ctypes.data, offs.ctypes.data, 1, None) == T.TRIE_EINVAL
+    assert lib.trie_build(None, None, 1, ctypes.byref(h)) == T.TRIE_EINVAL
+    neg = np.array([-1, 2], np.int64)
+    assert lib.trie_build(b.ctypes.data, neg.ctypes.data, 1, ctypes.byref(h)) == T.TRIE_EINVAL
+    # K = 0: a lone root, offsets may be NULL
+    assert lib.trie_build(None, None, 0, ctypes.byref(h)) == T.TRIE_OK
+    assert lib.trie_num_nodes(h) == 1
+    assert lib.trie_destroy(h) == T.TRIE_OK
+
+
+def test_build_many_argument_errors(lib):
+    h = ctypes.c_void_p()
+    b = np.frombuffer(b"abcd", np.uint8).copy()
+    offs = np.array([0, 2, 4], np.int64)
+    bad_first = np.array([1, 2], np.int32)
+    bad_order = np.array([0, 2, 1], np.int32)
+    assert lib.trie_build_many(b.ctypes.data, offs.ctypes.data, bad_first.ctypes.data, 1,
+                               ctypes.byref(h)) == T.TRIE_EINVAL
+    assert lib.trie_build_many(b.ctypes.data, offs.ctypes.data, bad_order.ctypes.data, 2,
+                               ctypes.byref(h)) == T.TRIE_EINVAL
+    assert lib.trie_build_many(b.ctypes.data, offs.ctypes.data, None, 1, ctypes.byref(h)) == T.TRIE_EINVAL
+    ok = np.array([0, 2], np.int32)
+    assert lib.trie_build_many(b.ctypes.data, offs.ctypes.data, ok.ctypes.data, 0,
+                               ctypes.byref(h)) == T.TRIE_EINVAL
+
+
+def test_null_handle_queries(lib):
+    assert lib.trie_num_nodes(None) == -1
+    assert lib.trie_root(None, 0) == -1
+    assert lib.trie_destroy(None) == T.TRIE_OK
+    assert lib.trie_compile_masks(None, None, None, 10, None, None) == T.TRIE_EINVAL
+    assert lib.trie_advance(None, None, None, 1, None, None) == T.TRIE_EINVAL
+    assert lib.trie_apply_mask(None, None, 0, None, 1, 10, None) == T.TRIE_EINVAL
+
+
+def test_device_calls_checked_before_any_device_work(lib):
+    """Argument errors and call-order errors come back before the GPU is touched."""
+    sb, so = W.pack([b"ab"])
+    h = T.trie_build(sb, so)
+    L = lib
+    assert L.trie_compile_masks(h.handle, None, None, 1, None, None) == T.TRIE_EINVAL      # V < 2
+    vo = np.array([0, 1, 1], np.int64)
+    vb = np.frombuffer(b"a", np.uint8).copy()
+    assert L.trie_compile_masks(h.handle, vb.ctypes.data, vo.ctypes.data, 2, None, None) == T.TRIE_EINVAL
+    assert L.trie_compile_masks(h.handle, vb.ctypes.data, vo.ctypes.data, 2, 2, None) == T.TRIE_EINVAL  # misaligned
+    # advance / apply before compile
+    assert L.trie_advance(h.handle, 16, 16, 1, None, None) == T.TRIE_ESTATE
+    assert L.trie_apply_mask(h.handle, 16, 0, 16, 1, 2, None) == T.TRIE_ESTATE
+    assert L.trie_apply_mask(h.handle, 16, 7, 16, 1, 2, None) == T.TRIE_EINVAL           # dtype
+    assert L.trie_advance(h.handle, 16, 16, -1, None, None) == T.TRIE_EINVAL
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    import importlib
+    mod = importlib.import_module("paper_2608_12574_gb300.triemask")
+    with pytest.raises(RuntimeError, match="missing"):
+        old = mod._lib
+        mod._lib = None
+        try:
+            mod.load_library(str(tmp_path / "nope.so"))
+        finally:
+            mod._lib = old
