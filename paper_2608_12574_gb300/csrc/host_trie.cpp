@@ -206,22 +206,29 @@ std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, 
     for (int32_t v = 0; v < V; v++)
         if (out->tok_len[size_t(v)])
             memcpy(&out->blob[out->tok_off[size_t(v)]], bytes + offsets[v], out->tok_len[size_t(v)]);
+    // load factor <= 1/4; slots are probed in aligned pairs (one 16-byte load
+    // holds two keys), pair after pair, the even slot of a pair filled first
     uint64_t S = 16;
-    while (S < uint64_t(2 * n_ins)) S <<= 1;
+    while (S < uint64_t(4 * n_ins)) S <<= 1;
+    if (S > (uint64_t(1) << 31)) return "vocabulary too large for the token hash table";
     out->ht_key.assign(size_t(S), 0ull);
     out->ht_val.assign(size_t(S), -1);
     out->ht_mask = uint32_t(S - 1);
+    const uint64_t pairs_mask = S / 2 - 1;
     for (int32_t v = 0; v < V; v++) {
         uint32_t L = out->tok_len[size_t(v)];
         if (!L) continue;
         const uint8_t *p = bytes + offsets[v];
         uint64_t h = 0;
         for (uint32_t j = 0; j < L; j++) h = h * kHashBase + uint64_t(p[j]) + 1;
-        uint64_t key = hash_finish(h, L);
-        uint64_t slot = key & (S - 1);
-        while (out->ht_key[size_t(slot)]) slot = (slot + 1) & (S - 1);
-        out->ht_key[size_t(slot)] = key;
-        out->ht_val[size_t(slot)] = v;
+        const uint64_t key = hash_finish(h, L);
+        uint64_t pair = (key >> 1) & pairs_mask;
+        for (;;) {
+            size_t s0 = size_t(2 * pair);
+            if (!out->ht_key[s0]) { out->ht_key[s0] = key; out->ht_val[s0] = v; break; }
+            if (!out->ht_key[s0 + 1]) { out->ht_key[s0 + 1] = key; out->ht_val[s0 + 1] = v; break; }
+            pair = (pair + 1) & pairs_mask;
+        }
     }
     return "";
 }

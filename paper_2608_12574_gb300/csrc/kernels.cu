@@ -6,17 +6,24 @@
 //                whose bytes spell the last k edges into m (k = 1..lmax) and
 //                sets that token's bit in the row of the node k edges above m.
 //                These are exactly the Aho-Corasick outputs of Sec. 4.2 step
-//                2 ("a vocabulary token's characters end at the current trie
-//                node; that token started |token| characters earlier, at its
-//                start node", App. G.1 Step 3), found by a hash lookup per
-//                suffix instead of by failure links, so that every node is
-//                independent. Cost O(N * min(depth, l)) lookups, the paper's
-//                O(N_chars * l) traversal bound.
+//                2 (a token whose characters end at the current node is
+//                recorded at the node |token| characters earlier, App. G.1
+//                Step 3), found by one hash lookup per suffix length instead
+//                of by failure links, so every node is independent. Cost
+//                O(N * min(depth, l)) lookups, the traversal bound of Sec. 4.2.
 //  k_advance     delta*(s, bytes(token)) per request (Sec. 2, Eq. 1).
 //  k_apply_vec   -inf into the logits of disallowed tokens (Sec. 4.2; App.
-//                H.3); one warp per 1024-token segment of a row, 16-byte
-//                stores, the logits are read only where some token of the
-//                16-byte chunk is allowed.
+//                H.3): persistent warps over 1024-token segments, 16-byte
+//                stores, the logits read only in 16-byte chunks that hold an
+//                allowed token.
+//
+// Every kernel is launched with programmatic stream serialization (PDL): it
+// lets the next kernel in the stream launch at once and waits for the
+// previous kernel (griddepcontrol.wait) before it touches memory that kernel
+// may write or read. That wait is the hardware grid dependency, which always
+// resolves because the previous grid never waits on this one. The patch
+// kernel does its trie climbs and hash probes (read-only data) before the
+// wait, so they overlap the fill.
 #include <stdint.h>
 
 #include <cuda_runtime.h>
@@ -27,12 +34,38 @@ namespace tmk {
 
 namespace {
 
-constexpr int kThreads = 256;
 constexpr int32_t kDead = -1;
 constexpr int32_t kFinished = -2;
+constexpr int kMaxClimb = 16;  // suffix lengths kept in registers by the patch kernel
 
-__global__ void __launch_bounds__(kThreads) k_mask_fill(uint32_t *__restrict__ mask, int64_t n_words,
-                                                        int64_t head) {
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), int grid, int block, cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(grid));
+    cfg.blockDim = dim3(unsigned(block));
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+}
+
+// ------------------------------------------------------------------ fill
+
+constexpr int kFillThreads = 256;
+
+__global__ void __launch_bounds__(kFillThreads) k_mask_fill(uint32_t *__restrict__ mask, int64_t n_words,
+                                                            int64_t head) {
+    pdl_launch_dependents();
+    pdl_wait();  // an earlier kernel may still read the old mask
     const int64_t tid = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
     const int64_t nth = int64_t(gridDim.x) * blockDim.x;
     if (tid < head) mask[tid] = 0u;
@@ -51,59 +84,163 @@ __global__ void __launch_bounds__(kThreads) k_mask_fill(uint32_t *__restrict__ m
     if (tid < n_words - tail0) mask[tail0 + tid] = 0u;
 }
 
-// True iff the token bytes tok[0..k) equal the labels of the k edges that end
-// at node m (read bottom-up).
-__device__ __forceinline__ bool path_equals(const int32_t *__restrict__ parent,
-                                            const uint8_t *__restrict__ label, int32_t m,
-                                            const uint8_t *__restrict__ tok, int32_t k) {
-    int32_t y = m;
-    for (int32_t j = k - 1; j >= 0; j--) {
-        if (y < 0 || label[y] != tok[j]) return false;
-        y = parent[y];
-    }
-    return true;
+// ------------------------------------------------------------------ patch
+
+constexpr int kPatchThreads = 128;
+
+struct PatchArgs {
+    const int32_t *parent;
+    const uint8_t *label;
+    const uint8_t *terminal;
+    int32_t n_nodes;
+    const uint64_t *ht_key;
+    const int32_t *ht_val;
+    uint32_t pairs_mask;  // number of slot pairs - 1
+    const uint32_t *tok_off;
+    const uint16_t *tok_len;
+    const uint8_t *blob;
+    int32_t lmax;
+    uint32_t *mask;
+    int64_t W;
+    int32_t eos;
+};
+
+// Byte i of a 16-byte window packed little-endian into four words, without
+// dynamic register indexing.
+__device__ __forceinline__ uint32_t byte_at(const uint32_t (&w)[4], int32_t i) {
+    const int32_t q = i >> 2;
+    const uint32_t v = q == 0 ? w[0] : (q == 1 ? w[1] : (q == 2 ? w[2] : w[3]));
+    return (v >> ((i & 3) * 8)) & 0xFFu;
 }
 
-__global__ void __launch_bounds__(kThreads) k_mask_patch(
-    const int32_t *__restrict__ parent, const uint8_t *__restrict__ label,
-    const uint8_t *__restrict__ terminal, int32_t n_nodes, const uint64_t *__restrict__ ht_key,
-    const int32_t *__restrict__ ht_val, uint32_t ht_mask, const uint32_t *__restrict__ tok_off,
-    const uint16_t *__restrict__ tok_len, const uint8_t *__restrict__ blob, int32_t lmax,
-    uint32_t *__restrict__ mask, int64_t W, int32_t eos) {
-    const int32_t stride = gridDim.x * blockDim.x;
-    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < n_nodes; m += stride) {
-        // EOS is allowed exactly at terminal nodes (App. G.5, EOS handling)
-        if (terminal[m]) atomicOr(mask + int64_t(m) * W + (eos >> 5), 1u << (eos & 31));
-        uint64_t h = 0, pw = 1;
-        int32_t x = m;
-        for (int32_t k = 1; k <= lmax; k++) {
-            const int32_t p = parent[x];
-            if (p < 0) break;
-            h += (uint64_t(label[x]) + 1ull) * pw;  // prepend one byte to the suffix
-            pw *= kHashBase;
-            x = p;  // the suffix of length k starts at node x
-            const uint64_t key = hash_finish(h, uint32_t(k));
-            uint32_t slot = uint32_t(key) & ht_mask;
-            for (uint32_t probe = 0; probe <= ht_mask; probe++) {  // ends at an empty slot
-                const uint64_t kk = ht_key[slot];
-                if (kk == 0ull) break;
-                if (kk == key) {
-                    const int32_t t = ht_val[slot];
-                    if (int32_t(tok_len[t]) == k && path_equals(parent, label, m, blob + tok_off[t], k))
-                        atomicOr(mask + int64_t(x) * W + (t >> 5), 1u << (t & 31));
+// Calls hit(t) for every token id t stored under `key` whose bytes equal the
+// k-edge path ending at node m. lab (if not null) holds the path's labels,
+// byte i = label of the edge i levels above m; otherwise the path is walked
+// again. Probing visits aligned slot pairs.
+template <typename Hit>
+__device__ __forceinline__ void probe(const PatchArgs &a, uint64_t key, int32_t k, const uint32_t (*lab)[4],
+                                      int32_t m, Hit hit) {
+    uint32_t pair = uint32_t(key >> 1) & a.pairs_mask;
+    for (uint32_t it = 0; it <= a.pairs_mask; it++) {
+        const ulonglong2 kk = __ldg(reinterpret_cast<const ulonglong2 *>(a.ht_key) + pair);
+#pragma unroll
+        for (int q = 0; q < 2; q++) {
+            if ((q == 0 ? kk.x : kk.y) == key) {
+                const int32_t t = __ldg(a.ht_val + 2 * pair + q);
+                if (int32_t(__ldg(a.tok_len + t)) == k) {
+                    const uint8_t *tb = a.blob + __ldg(a.tok_off + t);
+                    bool eq = true;
+                    if (lab) {
+                        for (int32_t j = 0; j < k && eq; j++) eq = (uint32_t(tb[j]) == byte_at(*lab, k - 1 - j));
+                    } else {
+                        int32_t y = m;
+                        for (int32_t j = k - 1; j >= 0 && eq; j--) {
+                            eq = y >= 0 && a.label[y] == tb[j];
+                            y = a.parent[y];
+                        }
+                    }
+                    if (eq) hit(t);
                 }
-                slot = (slot + 1u) & ht_mask;
+            }
+        }
+        if (kk.y == 0ull) return;  // the pair is not full: the probe chain ends here
+        pair = (pair + 1u) & a.pairs_mask;
+    }
+}
+
+__global__ void __launch_bounds__(kPatchThreads) k_mask_patch(PatchArgs a) {
+    pdl_launch_dependents();
+    bool waited = false;
+    auto set_bit = [&](int32_t row, int32_t t) {
+        if (!waited) {
+            pdl_wait();  // the fill of this mask must be complete
+            waited = true;
+        }
+        atomicOr(a.mask + int64_t(row) * a.W + (t >> 5), 1u << (t & 31));
+    };
+    const int32_t stride = gridDim.x * blockDim.x;
+    const int32_t lim = a.lmax < kMaxClimb ? a.lmax : kMaxClimb;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        // climb: labels (packed) and start nodes of the suffixes of length 1..16
+        uint32_t lab[4] = {0u, 0u, 0u, 0u};
+        int32_t anc[kMaxClimb];
+        int32_t depth = 0;
+        int32_t x = m;
+#pragma unroll
+        for (int k = 0; k < kMaxClimb; k++) {
+            anc[k] = -1;
+            if (k < lim && x >= 0) {
+                const int32_t p = __ldg(a.parent + x);
+                if (p >= 0) {
+                    lab[k >> 2] |= uint32_t(__ldg(a.label + x)) << ((k & 3) * 8);
+                    anc[k] = p;
+                    depth = k + 1;
+                }
+                x = p;
+            }
+        }
+        if (__ldg(a.terminal + m)) set_bit(m, a.eos);  // EOS exactly at terminal nodes (App. G.5)
+        // suffix hashes (Horner over byte+1 from the suffix's first byte);
+        // the first probe of 8 suffixes is issued before any result is used
+        uint64_t h = 0, pw = 1;
+#pragma unroll
+        for (int k0 = 0; k0 < kMaxClimb; k0 += 8) {
+            if (k0 < depth) {
+                uint64_t key[8];
+                ulonglong2 first[8];
+#pragma unroll
+                for (int i = 0; i < 8; i++) {
+                    const int k = k0 + i;
+                    key[i] = 0ull;
+                    first[i] = make_ulonglong2(0ull, 0ull);
+                    if (k < depth) {
+                        h += (uint64_t(byte_at(lab, k)) + 1ull) * pw;
+                        pw *= kHashBase;
+                        key[i] = hash_finish(h, uint32_t(k + 1));
+                        first[i] = __ldg(reinterpret_cast<const ulonglong2 *>(a.ht_key) +
+                                         (uint32_t(key[i] >> 1) & a.pairs_mask));
+                    }
+                }
+#pragma unroll
+                for (int i = 0; i < 8; i++) {
+                    const int k = k0 + i;
+                    // the full probe only when the first pair holds the key or continues
+                    if (k < depth && (first[i].x == key[i] || first[i].y == key[i] || first[i].y != 0ull)) {
+                        const int32_t row = anc[k];
+                        probe(a, key[i], k + 1, &lab, m, [&](int32_t t) { set_bit(row, t); });
+                    }
+                }
+            }
+        }
+        // suffixes longer than the register window (deep tries with long tokens)
+        if (a.lmax > kMaxClimb && depth == kMaxClimb) {
+            int32_t y = anc[kMaxClimb - 1];
+            for (int32_t k = kMaxClimb + 1; k <= a.lmax; k++) {
+                const int32_t p = a.parent[y];
+                if (p < 0) break;
+                h += (uint64_t(a.label[y]) + 1ull) * pw;
+                pw *= kHashBase;
+                const int32_t row = p;
+                probe(a, hash_finish(h, uint32_t(k)), k, nullptr, m, [&](int32_t t) { set_bit(row, t); });
+                y = p;
             }
         }
     }
+    if (!waited) pdl_wait();
 }
 
-__global__ void __launch_bounds__(kThreads) k_advance(
+// ------------------------------------------------------------------ advance
+
+constexpr int kAdvanceThreads = 128;
+
+__global__ void __launch_bounds__(kAdvanceThreads) k_advance(
     const int32_t *__restrict__ first_child, const uint32_t *__restrict__ child_bits,
     const uint8_t *__restrict__ terminal, int32_t n_nodes, const uint32_t *__restrict__ tok_off,
     const uint16_t *__restrict__ tok_len, const uint8_t *__restrict__ blob, int32_t V,
     int32_t *__restrict__ states, const int32_t *__restrict__ tokens, int32_t B,
     int32_t *__restrict__ err) {
+    pdl_launch_dependents();
+    pdl_wait();  // states / tokens come from earlier kernels
     const int32_t b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b >= B) return;
     const int32_t s = states[b];
@@ -128,6 +265,7 @@ __global__ void __launch_bounds__(kThreads) k_advance(
             const uint32_t c = p[j];
             const uint4 *cb = reinterpret_cast<const uint4 *>(child_bits + int64_t(x) * 8);
             const uint4 lo = cb[0], hi = cb[1];
+            const int32_t fc = first_child[x];
             const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
             const uint32_t wi = c >> 5, bit = c & 31u;
             uint32_t below = 0, cur = 0;
@@ -140,13 +278,17 @@ __global__ void __launch_bounds__(kThreads) k_advance(
                 nxt = kDead;
                 break;
             }
-            x = first_child[x] + int32_t(below + __popc(cur & ((1u << bit) - 1u)));
+            x = fc + int32_t(below + __popc(cur & ((1u << bit) - 1u)));
             nxt = x;
         }
     }
     if (nxt == kDead && err) atomicAdd(err, 1);
     states[b] = nxt;
 }
+
+// ------------------------------------------------------------------ apply
+
+constexpr int kApplyThreads = 256;
 
 // Mask word of (state, word index w): the node's row, or {EOS} for FINISHED,
 // DEAD and ids that are not nodes.
@@ -159,58 +301,84 @@ __device__ __forceinline__ uint32_t row_word(const uint32_t *__restrict__ mask, 
 
 // kElt = 2 (bf16) or 4 (fp32). Requires V % (16 / kElt) == 0 and a 16-byte
 // aligned logits base, so that every row starts on a 16-byte boundary.
+// Work item = one 1024-token segment of one row (one mask word per lane);
+// each warp loops over items and loads the next item's mask word before it
+// stores the current one.
 template <int kElt>
-__global__ void __launch_bounds__(kThreads) k_apply_vec(uint4 *__restrict__ logits,
-                                                        const uint32_t *__restrict__ mask,
-                                                        const int32_t *__restrict__ states, int32_t B,
-                                                        int32_t V, int64_t W, int32_t n_nodes,
-                                                        int32_t segs_per_row) {
-    constexpr int kPer = 16 / kElt;             // tokens per 16-byte chunk
-    constexpr int kChunks = 1024 / kPer / 32;   // chunks per lane per segment
-    const int64_t gw = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+__global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__ logits,
+                                                             const uint32_t *__restrict__ mask,
+                                                             const int32_t *__restrict__ states, int32_t B,
+                                                             int32_t V, int64_t W, int32_t n_nodes,
+                                                             int32_t segs) {
+    constexpr int kPer = 16 / kElt;            // tokens per 16-byte chunk
+    constexpr int kChunks = 1024 / kPer / 32;  // chunks per lane per segment
+    pdl_launch_dependents();
+    pdl_wait();  // logits and states come from earlier kernels
     const int lane = threadIdx.x & 31;
-    if (gw >= int64_t(B) * segs_per_row) return;  // uniform per warp
-    const int32_t b = int32_t(gw / segs_per_row);
-    const int32_t seg = int32_t(gw % segs_per_row);
-    const int32_t s = __ldg(states + b);
+    const int32_t total = B * segs;
+    const int32_t nwarps = int32_t(gridDim.x) * (kApplyThreads / 32);
     const int32_t eos = V - 1;
-    const uint32_t word = row_word(mask, s, n_nodes, W, int64_t(seg) * 32 + lane, eos);
     const int64_t row_chunks = int64_t(V) / kPer;
-    uint4 *row = logits + int64_t(b) * row_chunks;
     const uint4 ninf = (kElt == 2) ? make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u)
                                    : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
-#pragma unroll
-    for (int j = 0; j < kChunks; j++) {
-        const int q = j * 32 + lane;                        // chunk within the segment
-        const uint32_t wv = __shfl_sync(0xffffffffu, word, (q * kPer) >> 5);
-        const uint32_t bits = (wv >> ((q * kPer) & 31)) & ((1u << kPer) - 1u);
-        const int64_t chunk = int64_t(seg) * (1024 / kPer) + q;
-        if (chunk >= row_chunks) continue;
-        if (bits == 0u) {
-            row[chunk] = ninf;
-        } else {
-            uint4 x = row[chunk];
-            uint32_t e[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-            for (int i = 0; i < 4; i++) {
-                if (kElt == 4) {
-                    if (!((bits >> i) & 1u)) e[i] = 0xFF800000u;
-                } else {
-                    if (!((bits >> (2 * i)) & 1u)) e[i] = (e[i] & 0xFFFF0000u) | 0xFF80u;
-                    if (!((bits >> (2 * i + 1)) & 1u)) e[i] = (e[i] & 0x0000FFFFu) | 0xFF800000u;
-                }
-            }
-            row[chunk] = make_uint4(e[0], e[1], e[2], e[3]);
+    int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
+    int32_t b = 0, seg = 0;
+    uint32_t word = 0;
+    if (item < total) {
+        b = item / segs;
+        seg = item - b * segs;
+        word = row_word(mask, __ldg(states + b), n_nodes, W, int64_t(seg) * 32 + lane, eos);
+    }
+    while (item < total) {  // uniform per warp
+        const int32_t nitem = item + nwarps;
+        int32_t nb = 0, nseg = 0;
+        uint32_t nword = 0;
+        if (nitem < total) {
+            nb = nitem / segs;
+            nseg = nitem - nb * segs;
+            nword = row_word(mask, __ldg(states + nb), n_nodes, W, int64_t(nseg) * 32 + lane, eos);
         }
+        uint4 *row = logits + int64_t(b) * row_chunks;
+#pragma unroll
+        for (int j = 0; j < kChunks; j++) {
+            const int q = j * 32 + lane;  // chunk within the segment
+            const uint32_t wv = __shfl_sync(0xffffffffu, word, (q * kPer) >> 5);
+            const uint32_t bits = (wv >> ((q * kPer) & 31)) & ((1u << kPer) - 1u);
+            const int64_t chunk = int64_t(seg) * (1024 / kPer) + q;
+            if (chunk >= row_chunks) continue;
+            if (bits == 0u) {
+                row[chunk] = ninf;
+            } else {
+                const uint4 x = row[chunk];
+                uint32_t e[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                for (int i = 0; i < 4; i++) {
+                    if (kElt == 4) {
+                        if (!((bits >> i) & 1u)) e[i] = 0xFF800000u;
+                    } else {
+                        if (!((bits >> (2 * i)) & 1u)) e[i] = (e[i] & 0xFFFF0000u) | 0xFF80u;
+                        if (!((bits >> (2 * i + 1)) & 1u)) e[i] = (e[i] & 0x0000FFFFu) | 0xFF800000u;
+                    }
+                }
+                row[chunk] = make_uint4(e[0], e[1], e[2], e[3]);
+            }
+        }
+        item = nitem;
+        b = nb;
+        seg = nseg;
+        word = nword;
     }
 }
 
 // Any V and alignment: one thread per logit.
 template <int kElt>
-__global__ void __launch_bounds__(kThreads) k_apply_scalar(void *__restrict__ logits,
-                                                           const uint32_t *__restrict__ mask,
-                                                           const int32_t *__restrict__ states, int32_t B,
-                                                           int32_t V, int64_t W, int32_t n_nodes) {
+__global__ void __launch_bounds__(kApplyThreads) k_apply_scalar(void *__restrict__ logits,
+                                                                const uint32_t *__restrict__ mask,
+                                                                const int32_t *__restrict__ states,
+                                                                int32_t B, int32_t V, int64_t W,
+                                                                int32_t n_nodes) {
+    pdl_launch_dependents();
+    pdl_wait();
     const int64_t total = int64_t(B) * V;
     const int32_t eos = V - 1;
     for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
@@ -237,51 +405,59 @@ cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaS
     int64_t head = int64_t(((16u - (a & 15u)) & 15u) >> 2);
     if (head > n_words) head = n_words;
     const int64_t n4 = (n_words - head) >> 2;
-    const int grid = grid_for(n4, kThreads, int64_t(num_sms) * 8);
-    k_mask_fill<<<grid, kThreads, 0, st>>>(mask, n_words, head);
-    return cudaGetLastError();
+    // 4 CTAs per SM: all resident at once, leaving room for the patch kernel
+    const int grid = grid_for(n4, kFillThreads, int64_t(num_sms) * 4);
+    return launch_pdl(k_mask_fill, grid, kFillThreads, st, mask, n_words, head);
 }
 
 cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                               uint32_t *mask, int64_t W, int num_sms, cudaStream_t st) {
-    const int grid = grid_for(n_nodes, kThreads, int64_t(num_sms) * 64);
-    k_mask_patch<<<grid, kThreads, 0, st>>>(t.parent, t.label, t.terminal, n_nodes, v.ht_key, v.ht_val,
-                                            v.ht_mask, v.tok_off, v.tok_len, v.blob, lmax, mask, W,
-                                            v.V - 1);
-    return cudaGetLastError();
+    PatchArgs a;
+    a.parent = t.parent;
+    a.label = t.label;
+    a.terminal = t.terminal;
+    a.n_nodes = n_nodes;
+    a.ht_key = v.ht_key;
+    a.ht_val = v.ht_val;
+    a.pairs_mask = v.ht_mask >> 1;
+    a.tok_off = v.tok_off;
+    a.tok_len = v.tok_len;
+    a.blob = v.blob;
+    a.lmax = lmax;
+    a.mask = mask;
+    a.W = W;
+    a.eos = v.V - 1;
+    const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 32);
+    return launch_pdl(k_mask_patch, grid, kPatchThreads, st, a);
 }
 
 cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t *states,
                            const int32_t *tokens, int32_t B, int32_t *err, cudaStream_t st) {
-    const int grid = (B + kThreads - 1) / kThreads;
-    k_advance<<<grid, kThreads, 0, st>>>(t.first_child, t.child_bits, t.terminal, n_nodes, v.tok_off,
-                                         v.tok_len, v.blob, v.V, states, tokens, B, err);
-    return cudaGetLastError();
+    const int grid = (B + kAdvanceThreads - 1) / kAdvanceThreads;
+    return launch_pdl(k_advance, grid, kAdvanceThreads, st, t.first_child, t.child_bits, t.terminal, n_nodes,
+                      v.tok_off, v.tok_len, v.blob, v.V, states, tokens, B, err);
 }
 
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
                          int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st) {
     const int64_t W = (int64_t(V) + 31) / 32;
     const int elt = dtype == 0 ? 4 : 2;
-    const bool vec = (reinterpret_cast<uintptr_t>(logits) & 15u) == 0 && (int64_t(V) * elt) % 16 == 0;
+    const int32_t segs = int32_t((W + 31) / 32);
+    const bool vec = (reinterpret_cast<uintptr_t>(logits) & 15u) == 0 && (int64_t(V) * elt) % 16 == 0 &&
+                     int64_t(B) * segs < int64_t(INT32_MAX) - int64_t(num_sms) * 64;
     if (vec) {
-        const int32_t segs = int32_t((W + 31) / 32);
-        const int64_t warps = int64_t(B) * segs;
-        const int grid = grid_for(warps * 32, kThreads, INT32_MAX);
+        const int64_t items = int64_t(B) * segs;
+        const int grid = grid_for(items, kApplyThreads / 32, int64_t(num_sms) * (2048 / kApplyThreads));
         if (elt == 2)
-            k_apply_vec<2><<<grid, kThreads, 0, st>>>(static_cast<uint4 *>(logits), mask, states, B, V, W,
-                                                      n_nodes, segs);
-        else
-            k_apply_vec<4><<<grid, kThreads, 0, st>>>(static_cast<uint4 *>(logits), mask, states, B, V, W,
-                                                      n_nodes, segs);
-    } else {
-        const int grid = grid_for(int64_t(B) * V, kThreads, int64_t(num_sms) * 16);
-        if (elt == 2)
-            k_apply_scalar<2><<<grid, kThreads, 0, st>>>(logits, mask, states, B, V, W, n_nodes);
-        else
-            k_apply_scalar<4><<<grid, kThreads, 0, st>>>(logits, mask, states, B, V, W, n_nodes);
+            return launch_pdl(k_apply_vec<2>, grid, kApplyThreads, st, static_cast<uint4 *>(logits), mask,
+                              states, B, V, W, n_nodes, segs);
+        return launch_pdl(k_apply_vec<4>, grid, kApplyThreads, st, static_cast<uint4 *>(logits), mask, states,
+                          B, V, W, n_nodes, segs);
     }
-    return cudaGetLastError();
+    const int grid = grid_for(int64_t(B) * V, kApplyThreads, int64_t(num_sms) * 16);
+    if (elt == 2)
+        return launch_pdl(k_apply_scalar<2>, grid, kApplyThreads, st, logits, mask, states, B, V, W, n_nodes);
+    return launch_pdl(k_apply_scalar<4>, grid, kApplyThreads, st, logits, mask, states, B, V, W, n_nodes);
 }
 
 }  // namespace tmk
