@@ -168,6 +168,43 @@ int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B
 int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B,
                     int32_t V, cudaStream_t stream);
 
+/* Size of the fixed device scratch used by trie_compile_masks_noalloc. */
+#define TRIE_NOALLOC_SCRATCH_BYTES (32u << 20)
+
+/* The paper has no counterpart to this entry point; it serves callers that
+ * must not have the library allocate device memory.
+ *
+ * trie_compile_masks keeps device copies of the trie and the packed
+ * vocabulary in memory it gets from cudaMalloc. Some callers cannot allow
+ * that: a serving engine that has given all free HBM to its own pool (KV
+ * cache) and forbids other allocations, a process held to a fixed device
+ * memory budget, or a latency-critical loop in which cudaMalloc / cudaFree,
+ * which may synchronise the device, must not run. This call computes the
+ * same mask as trie_compile_masks without allocating: the trie and the
+ * vocabulary are staged in a static host buffer and copied into one
+ * fixed-size device array compiled into the library
+ * (TRIE_NOALLOC_SCRATCH_BYTES = 32 MiB). Every GPU that loads that array
+ * holds it until the process exits (under CUDA's default lazy module loading,
+ * from the first call on the device).
+ *   Arguments, layout and result are those of trie_compile_masks.
+ *   The trie's node arrays (6 bytes per node) plus the packed vocabulary
+ *   (6 bytes per token, its bytes rounded up to 16 per token, and a hash
+ *   table of 12 bytes per slot, 4 slots per token with bytes) must fit in the
+ *   scratch; otherwise TRIE_EINVAL with a message, and nothing is launched.
+ *   The first call on a device looks up the device address of the scratch
+ *   (cudaGetSymbolAddress) with that device current; make that first call
+ *   before any stream capture.
+ *   All calls share the one scratch, which keeps the last call's contents
+ *   (every byte a call uses is rewritten by it). Calls whose work overlaps on
+ *   the GPU (other streams, other threads) race on it; order them, for
+ *   example on one stream.
+ *   Unlike trie_compile_masks it does not record the mask or the vocabulary
+ *   in the handle: trie_advance and trie_apply_mask keep using those of the
+ *   last trie_compile_masks.
+ *   On success nothing is allocated, on the host or on the device. */
+int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets,
+                               int32_t V, uint32_t *d_mask, cudaStream_t stream);
+
 /* Release the handle, its host arrays and its device copy of the trie.
  * Synchronises the device first if device memory is held. NULL is a no-op. */
 int trie_destroy(trie_t h);

@@ -208,6 +208,8 @@ int finish_build(std::string err, trie_s *h, trie_t *out) {
 
 }  // namespace
 
+int tmk::set_error(int code, const char *msg) { return fail(code, msg); }
+
 tmk::DevVocab::~DevVocab() {
     if (base) {
         DeviceGuard g(device);

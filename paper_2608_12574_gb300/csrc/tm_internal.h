@@ -111,6 +111,10 @@ struct trie_s {
 };
 
 namespace tmk {
+// Records msg as the calling thread's last error (trie_last_error) and
+// returns code.
+int set_error(int code, const char *msg);
+
 // Kernel launchers (kernels.cu). Each returns the launch's cudaError_t.
 cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaStream_t st);
 cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,

@@ -34,6 +34,7 @@ SIGNATURES = {
     "trie_max_depth": (_I32, [_P]),
     "trie_get_csr": (ctypes.c_int, [_P, _P, _P, _P, _P]),
     "trie_compile_masks": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "trie_compile_masks_noalloc": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
     "trie_destroy": (ctypes.c_int, [_P]),
@@ -204,6 +205,20 @@ def trie_compile_masks(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stre
         raise ValueError("d_mask is smaller than num_nodes * ceil(V/32) words")
     _check(h._lib.trie_compile_masks(h.handle, _hp(vb), _hp(vo), V, p,
                                      _stream(stream, d_mask.device)))
+
+
+def trie_compile_masks_noalloc(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stream=None) -> None:
+    """trie_compile_masks without device allocation (fixed 32 MiB library scratch)."""
+    import torch
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    p = _dev(d_mask, (torch.int32,), "d_mask")
+    if d_mask.numel() < h.num_nodes * mask_words(V):
+        raise ValueError("d_mask is smaller than num_nodes * ceil(V/32) words")
+    _check(h._lib.trie_compile_masks_noalloc(h.handle, _hp(vb), _hp(vo), V, p,
+                                             _stream(stream, d_mask.device)))
 
 
 def trie_advance(h: Trie, d_states, d_tokens, d_err=None, stream=None) -> None:
