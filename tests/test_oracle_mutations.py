@@ -1,13 +1,15 @@
 """Plant plausible mistakes in a copy of the oracle and check the pins catch each.
 
 Every mutant is a textual edit of oracle/oracle.c, compiled into a temporary
-directory (CPU only). A mutant that passes all pins would mean the pins cannot
-tell that mistake from the correct oracle.
+directory (CPU only) and checked in a child process, so that only an
+AssertionError from a pin counts as caught. A mutant that passes all pins
+would mean the pins cannot tell that mistake from the correct oracle.
 """
 from __future__ import annotations
 
 import os
 import subprocess
+import sys
 
 import pytest
 
@@ -28,7 +30,8 @@ MUTANTS = {
     "last_token_skipped": ("for (int32_t v = 0; v < eos; v++)", "for (int32_t v = 0; v < eos - 1; v++)"),
     "siblings_descending": ("        for (int b = 0; b < 256; b++)\n            if (ch[(int64_t)x * 256 + b] >= 0) order",
                             "        for (int b = 255; b >= 0; b--)\n            if (ch[(int64_t)x * 256 + b] >= 0) order"),
-    "depth_first_numbering": ("int32_t x = order[head++];", "int32_t x = order[--tail]; head++;"),
+    "insertion_order_numbering": ("for (int64_t i = 0; i < n; i++) newid[order[i]] = (int32_t)i;",
+                                  "for (int64_t i = 0; i < n; i++) { order[i] = (int32_t)i; newid[i] = (int32_t)i; }"),
     "finished_eos_dies": ("nxt = (v == eos) ? ORACLE_FINISHED : ORACLE_DEAD;",
                           "nxt = ORACLE_DEAD;"),
     "eos_finishes_anywhere": ("nxt = t->terminal[s] ? ORACLE_FINISHED : ORACLE_DEAD;",
@@ -55,22 +58,43 @@ def _all_pins():
         check_apply(strings, toks, seed)
 
 
+TESTS = os.path.dirname(os.path.abspath(__file__))
+CHILD = """
+import sys
+sys.path[:0] = [{root!r}, {tests!r}]
+import oracle, test_oracle_mutations as m
+with oracle.use_library({lib!r}):
+    try:
+        m._all_pins()
+    except AssertionError:
+        print("PIN-FAILED")
+        sys.exit(3)
+print("PINS-PASSED")
+"""
+
+
+def _run_pins_with(lib: str) -> subprocess.CompletedProcess:
+    code = CHILD.format(root=os.path.dirname(TESTS), tests=TESTS, lib=lib)
+    return subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300)
+
+
+def _compile(src_text: str, tmp_path, name: str) -> str:
+    path = tmp_path / f"{name}.c"
+    path.write_text(src_text)
+    lib = tmp_path / f"lib{name}.so"
+    subprocess.check_call(["gcc", "-O1", "-shared", "-fPIC", "-std=c99", "-o", str(lib), str(path)])
+    return str(lib)
+
+
 @pytest.mark.parametrize("name", sorted(MUTANTS))
 def test_pins_catch_planted_mistake(oracle_lib, tmp_path, name):
     src = open(SRC).read()
     old, new = MUTANTS[name]
     assert src.count(old) == 1, f"mutation site for {name} not unique / not found"
-    path = tmp_path / "mut.c"
-    path.write_text(src.replace(old, new))
-    lib = tmp_path / "libmut.so"
-    subprocess.check_call(["gcc", "-O1", "-shared", "-fPIC", "-std=c99", "-o", str(lib), str(path)])
-    with oracle.use_library(str(lib)):
-        with pytest.raises(AssertionError):
-            _all_pins()
+    r = _run_pins_with(_compile(src.replace(old, new), tmp_path, "mut"))
+    assert r.returncode == 3 and "PIN-FAILED" in r.stdout, (r.returncode, r.stdout[-500:], r.stderr[-2000:])
 
 
 def test_unmutated_copy_passes(oracle_lib, tmp_path):
-    lib = tmp_path / "libsame.so"
-    subprocess.check_call(["gcc", "-O1", "-shared", "-fPIC", "-std=c99", "-o", str(lib), SRC])
-    with oracle.use_library(str(lib)):
-        _all_pins()
+    r = _run_pins_with(_compile(open(SRC).read(), tmp_path, "same"))
+    assert r.returncode == 0 and "PINS-PASSED" in r.stdout, (r.stdout[-500:], r.stderr[-2000:])
