@@ -126,6 +126,7 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
     dv->tok_off = reinterpret_cast<const uint32_t *>(base + o_off);
     dv->tok_len = reinterpret_cast<const uint16_t *>(base + o_len);
     dv->blob = reinterpret_cast<const uint8_t *>(base + o_blob);
+    dv->blob_bytes = hv.blob.size();
     dv->ht_key = reinterpret_cast<const uint64_t *>(base + o_key);
     dv->ht_val = reinterpret_cast<const int32_t *>(base + o_val);
     try {
@@ -157,6 +158,11 @@ int ensure_device_trie(trie_t h, int dev) {
     const size_t o_term = L.add(n);
     const size_t o_fc = L.add(sizeof(int32_t) * n);
     const size_t o_bits = L.add(sizeof(uint32_t) * 8 * n);
+    const size_t o_win = L.add(sizeof(uint64_t) * 2 * n);
+    const size_t o_d8 = L.add(n);
+    const size_t o_jump = L.add(sizeof(int32_t) * 4 * n);
+    const size_t o_hits = L.add(sizeof(int2) * 8 * n);  // compile scratch (probe -> scatter)
+    const size_t o_hcnt = L.add(n);
     void *base = nullptr;
     cudaError_t e = cudaMalloc(&base, L.total);
     if (e != cudaSuccess) {
@@ -170,6 +176,9 @@ int ensure_device_trie(trie_t h, int dev) {
         {o_term, t.terminal.data(), n},
         {o_fc, t.first_child.data(), sizeof(int32_t) * n},
         {o_bits, t.child_bits.data(), sizeof(uint32_t) * 8 * n},
+        {o_win, t.window.data(), sizeof(uint64_t) * 2 * n},
+        {o_d8, t.depth8.data(), n},
+        {o_jump, t.jump.data(), sizeof(int32_t) * 4 * n},
     };
     for (const Up &u : ups) {
         e = cudaMemcpy(b + u.off, u.src, u.n, cudaMemcpyHostToDevice);
@@ -185,6 +194,11 @@ int ensure_device_trie(trie_t h, int dev) {
     h->dev.terminal = reinterpret_cast<const uint8_t *>(b + o_term);
     h->dev.first_child = reinterpret_cast<const int32_t *>(b + o_fc);
     h->dev.child_bits = reinterpret_cast<const uint32_t *>(b + o_bits);
+    h->dev.window = reinterpret_cast<const ulonglong2 *>(b + o_win);
+    h->dev.depth8 = reinterpret_cast<const uint8_t *>(b + o_d8);
+    h->dev.jump = reinterpret_cast<const int4 *>(b + o_jump);
+    h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
+    h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
     return TRIE_OK;
 }
 
@@ -304,10 +318,8 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     const int32_t n = h->host.n;
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
-    cudaError_t e = tmk::launch_mask_fill(d_mask, int64_t(n) * W, sms, stream);
-    if (e != cudaSuccess) return fail_cuda(e, "mask fill launch");
-    e = tmk::launch_mask_patch(h->dev, n, *voc, lmax, d_mask, W, sms, stream);
-    if (e != cudaSuccess) return fail_cuda(e, "mask patch launch");
+    cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "mask compile launch");
     std::lock_guard<std::mutex> lk(h->mu);
     h->vocab = voc;
     h->mask = d_mask;

@@ -42,6 +42,26 @@ inline int cmp_str(const Str &a, const Str &b) {
 
 }  // namespace
 
+// Label windows, clipped depths and ancestor jumps, in BFS order (a parent
+// always precedes its children).
+void add_compile_tables(HostTrie *t) {
+    const size_t n = size_t(t->n);
+    t->window.assign(2 * n, 0ull);
+    t->depth8.assign(n, 0);
+    t->jump.assign(4 * n, -1);
+    for (size_t i = 0; i < n; i++) {
+        const int32_t p = t->parent[i];
+        if (p < 0) continue;
+        const uint64_t lo = t->window[2 * size_t(p)], hi = t->window[2 * size_t(p) + 1];
+        t->window[2 * i] = (lo << 8) | t->label[i];
+        t->window[2 * i + 1] = (hi << 8) | (lo >> 56);
+        t->depth8[i] = uint8_t(t->depth8[size_t(p)] == 255 ? 255 : t->depth8[size_t(p)] + 1);
+        int32_t *j = &t->jump[4 * i];
+        j[0] = p;
+        for (int q = 1; q < 4; q++) j[q] = j[q - 1] < 0 ? -1 : t->jump[4 * size_t(j[q - 1]) + q - 1];
+    }
+}
+
 std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t first, int32_t last,
                        HostTrie *out) {
     const int64_t K = int64_t(last) - first;
@@ -118,6 +138,7 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
         uint8_t l = out->label[size_t(c)];
         out->child_bits[size_t(p) * 8 + (l >> 5)] |= 1u << (l & 31);
     }
+    add_compile_tables(out);
     out->roots.assign(1, 0);
     out->n_chars = n_chars;
     out->max_depth = max_depth;
@@ -156,6 +177,9 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
     out->terminal.resize(size_t(n));
     out->first_child.resize(size_t(n));
     out->child_bits.resize(size_t(n) * 8);
+    out->window.resize(size_t(n) * 2);
+    out->depth8.resize(size_t(n));
+    out->jump.resize(size_t(n) * 4);
     out->roots.resize(size_t(M));
     out->n_chars = 0;
     out->max_depth = 0;
@@ -171,6 +195,10 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
             out->terminal[g] = p.terminal[size_t(j)];
         }
         memcpy(&out->child_bits[size_t(base) * 8], p.child_bits.data(), sizeof(uint32_t) * 8 * size_t(p.n));
+        memcpy(&out->window[size_t(base) * 2], p.window.data(), sizeof(uint64_t) * 2 * size_t(p.n));
+        memcpy(&out->depth8[size_t(base)], p.depth8.data(), size_t(p.n));
+        for (size_t j = 0; j < 4 * size_t(p.n); j++)
+            out->jump[4 * size_t(base) + j] = p.jump[j] < 0 ? -1 : p.jump[j] + base;
         out->n_chars += p.n_chars;
         out->max_depth = std::max(out->max_depth, p.max_depth);
         base += p.n;

@@ -88,6 +88,32 @@ __global__ void __launch_bounds__(kFillThreads) k_mask_fill(uint32_t *__restrict
     }
 }
 
+// The fill of the probe-fill-scatter form: launched while k_mask_probe runs,
+// with evict-first stores so that the 0.4-4 GB stream does not flush the
+// tables the probe has prefetched into L2.
+// It needs no wait at entry (the probe let it launch only after every earlier
+// kernel had completed); CTA 0 waits for the probe at its end, so this grid
+// never completes before the probe and the scatter's wait covers both.
+__global__ void __launch_bounds__(kFillThreads) k_mask_fill_beside(uint32_t *__restrict__ mask, int64_t n_words,
+                                                                   int64_t head) {
+    pdl_launch_dependents();
+    uint4 *v = reinterpret_cast<uint4 *>(mask + head);
+    const int64_t n4 = (n_words - head) >> 2;
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+    const int64_t base = int64_t(blockIdx.x) * (kFillThreads * kFillVecs) + threadIdx.x;
+#pragma unroll
+    for (int j = 0; j < kFillVecs; j++) {
+        const int64_t i = base + j * kFillThreads;
+        if (i < n4) __stcs(v + i, z);  // evict-first: keep the probe's tables in L2
+    }
+    if (blockIdx.x == 0) {
+        if (threadIdx.x < head) mask[threadIdx.x] = 0u;
+        const int64_t tail0 = head + (n4 << 2);
+        if (threadIdx.x < n_words - tail0) mask[tail0 + threadIdx.x] = 0u;
+        if (threadIdx.x == 0) pdl_wait();
+    }
+}
+
 // ------------------------------------------------------------------ patch
 
 constexpr int kPatchThreads = 128;
@@ -107,7 +133,38 @@ struct PatchArgs {
     uint32_t *mask;
     int64_t W;
     int32_t eos;
+    int2 *hits;          // [n_nodes * kHitSlots] (row, token), probe-scatter form only
+    uint8_t *hit_count;  // [n_nodes]
+    const ulonglong2 *window;  // probe-scatter form: last 16 labels per node
+    const uint8_t *depth8;
+    const int4 *jump;          // ancestors 1, 2, 4, 8 levels up
 };
+constexpr int kHitSlots = 8;
+constexpr int kHitOverflow = 255;
+
+// Read-only arrays the probe reads, for a bulk L2 prefetch.
+struct Prefetch {
+    const void *ptr[10];
+    uint64_t bytes[10];
+    int count;
+};
+
+// CTA `part` of `nparts` asks the TMA unit to pull its slice of every array
+// into L2 (cp.async.bulk.prefetch: asynchronous, no completion to wait for).
+__device__ __forceinline__ void l2_prefetch_slice(const Prefetch &pf, int part, int nparts) {
+    for (int i = 0; i < pf.count; i++) {
+        const uint64_t n = pf.bytes[i] & ~uint64_t(15);
+        const uint64_t per = ((n / uint64_t(nparts)) + 15) & ~uint64_t(15);
+        const uint64_t a0 = per * uint64_t(part);
+        if (a0 >= n) continue;
+        const uint64_t len = n - a0 < per ? n - a0 : per;
+        const char *base = static_cast<const char *>(pf.ptr[i]) + a0;
+        for (uint64_t o = 0; o < len; o += 65536) {
+            const uint32_t l = uint32_t(len - o < 65536 ? len - o : 65536);
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" :: "l"(base + o), "r"(l) : "memory");
+        }
+    }
+}
 
 // Byte i of a 16-byte window packed little-endian into four words, without
 // dynamic register indexing.
@@ -152,85 +209,209 @@ __device__ __forceinline__ void probe(const PatchArgs &a, uint64_t key, int32_t 
     }
 }
 
-__global__ void __launch_bounds__(kPatchThreads) k_mask_patch(PatchArgs a) {
-    pdl_launch_dependents();
-    bool waited = false;
-    auto set_bit = [&](int32_t row, int32_t t) {
-        if (!waited) {
-            pdl_wait();  // the fill of this mask must be complete
-            waited = true;
-        }
-        atomicOr(a.mask + int64_t(row) * a.W + (t >> 5), 1u << (t & 31));
-    };
-    const int32_t stride = gridDim.x * blockDim.x;
+// Every allowed (row, token) pair whose path ends at node m: EOS at m if m is
+// terminal (App. G.5), and every token whose bytes spell the last k edges
+// into m, for the row of the node k edges above m (Sec. 4.2 step 2). Calls
+// emit(row, t) for each.
+template <typename Emit>
+__device__ __forceinline__ void node_hits(const PatchArgs &a, int32_t m, Emit emit) {
     const int32_t lim = a.lmax < kMaxClimb ? a.lmax : kMaxClimb;
-    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        // climb: labels (packed) and start nodes of the suffixes of length 1..16
-        uint32_t lab[4] = {0u, 0u, 0u, 0u};
-        int32_t anc[kMaxClimb];
-        int32_t depth = 0;
-        int32_t x = m;
+    // climb: labels (packed) and start nodes of the suffixes of length 1..16
+    uint32_t lab[4] = {0u, 0u, 0u, 0u};
+    int32_t anc[kMaxClimb];
+    int32_t depth = 0;
+    int32_t x = m;
 #pragma unroll
-        for (int k = 0; k < kMaxClimb; k++) {
-            anc[k] = -1;
-            if (k < lim && x >= 0) {
-                const int32_t p = __ldg(a.parent + x);
-                if (p >= 0) {
-                    lab[k >> 2] |= uint32_t(__ldg(a.label + x)) << ((k & 3) * 8);
-                    anc[k] = p;
-                    depth = k + 1;
-                }
-                x = p;
+    for (int k = 0; k < kMaxClimb; k++) {
+        anc[k] = -1;
+        if (k < lim && x >= 0) {
+            const int32_t p = __ldg(a.parent + x);
+            if (p >= 0) {
+                lab[k >> 2] |= uint32_t(__ldg(a.label + x)) << ((k & 3) * 8);
+                anc[k] = p;
+                depth = k + 1;
             }
+            x = p;
         }
-        if (__ldg(a.terminal + m)) set_bit(m, a.eos);  // EOS exactly at terminal nodes (App. G.5)
-        // suffix hashes (Horner over byte+1 from the suffix's first byte);
-        // the first probe of 8 suffixes is issued before any result is used
-        uint64_t h = 0, pw = 1;
+    }
+    if (__ldg(a.terminal + m)) emit(m, a.eos);
+    // suffix hashes (Horner over byte+1 from the suffix's first byte); the
+    // first probe of 8 suffixes is issued before any result is used
+    uint64_t h = 0, pw = 1;
 #pragma unroll
-        for (int k0 = 0; k0 < kMaxClimb; k0 += 8) {
-            if (k0 < depth) {
-                uint64_t key[8];
-                ulonglong2 first[8];
+    for (int k0 = 0; k0 < kMaxClimb; k0 += 8) {
+        if (k0 < depth) {
+            uint64_t key[8];
+            ulonglong2 first[8];
 #pragma unroll
-                for (int i = 0; i < 8; i++) {
-                    const int k = k0 + i;
-                    key[i] = 0ull;
-                    first[i] = make_ulonglong2(0ull, 0ull);
-                    if (k < depth) {
-                        h += (uint64_t(byte_at(lab, k)) + 1ull) * pw;
-                        pw *= kHashBase;
-                        key[i] = hash_finish(h, uint32_t(k + 1));
-                        first[i] = __ldg(reinterpret_cast<const ulonglong2 *>(a.ht_key) +
-                                         (uint32_t(key[i] >> 1) & a.pairs_mask));
-                    }
-                }
-#pragma unroll
-                for (int i = 0; i < 8; i++) {
-                    const int k = k0 + i;
-                    // the full probe only when the first pair holds the key or continues
-                    if (k < depth && (first[i].x == key[i] || first[i].y == key[i] || first[i].y != 0ull)) {
-                        const int32_t row = anc[k];
-                        probe(a, key[i], k + 1, &lab, m, [&](int32_t t) { set_bit(row, t); });
-                    }
+            for (int i = 0; i < 8; i++) {
+                const int k = k0 + i;
+                key[i] = 0ull;
+                first[i] = make_ulonglong2(0ull, 0ull);
+                if (k < depth) {
+                    h += (uint64_t(byte_at(lab, k)) + 1ull) * pw;
+                    pw *= kHashBase;
+                    key[i] = hash_finish(h, uint32_t(k + 1));
+                    first[i] = __ldg(reinterpret_cast<const ulonglong2 *>(a.ht_key) +
+                                     (uint32_t(key[i] >> 1) & a.pairs_mask));
                 }
             }
-        }
-        // suffixes longer than the register window (deep tries with long tokens)
-        if (a.lmax > kMaxClimb && depth == kMaxClimb) {
-            int32_t y = anc[kMaxClimb - 1];
-            for (int32_t k = kMaxClimb + 1; k <= a.lmax; k++) {
-                const int32_t p = a.parent[y];
-                if (p < 0) break;
-                h += (uint64_t(a.label[y]) + 1ull) * pw;
-                pw *= kHashBase;
-                const int32_t row = p;
-                probe(a, hash_finish(h, uint32_t(k)), k, nullptr, m, [&](int32_t t) { set_bit(row, t); });
-                y = p;
+#pragma unroll
+            for (int i = 0; i < 8; i++) {
+                const int k = k0 + i;
+                // the full probe only when the first pair holds the key or continues
+                if (k < depth && (first[i].x == key[i] || first[i].y == key[i] || first[i].y != 0ull)) {
+                    const int32_t row = anc[k];
+                    probe(a, key[i], k + 1, &lab, m, [&](int32_t t) { emit(row, t); });
+                }
             }
         }
     }
+    // suffixes longer than the register window (deep tries with long tokens)
+    if (a.lmax > kMaxClimb && depth == kMaxClimb) {
+        int32_t y = anc[kMaxClimb - 1];
+        for (int32_t k = kMaxClimb + 1; k <= a.lmax; k++) {
+            const int32_t p = a.parent[y];
+            if (p < 0) break;
+            h += (uint64_t(a.label[y]) + 1ull) * pw;
+            pw *= kHashBase;
+            const int32_t row = p;
+            probe(a, hash_finish(h, uint32_t(k)), k, nullptr, m, [&](int32_t t) { emit(row, t); });
+            y = p;
+        }
+    }
+}
+
+// Ancestor of m k levels up (k <= 2 * 15): at most one hop per set bit of k.
+__device__ __forceinline__ int32_t ancestor(const PatchArgs &a, int32_t m, int32_t k) {
+    int32_t y = m;
+    while (k >= 8 && y >= 0) {
+        y = __ldg(a.jump + y).w;
+        k -= 8;
+    }
+    if ((k & 4) && y >= 0) y = __ldg(a.jump + y).z;
+    if ((k & 2) && y >= 0) y = __ldg(a.jump + y).y;
+    if ((k & 1) && y >= 0) y = __ldg(a.jump + y).x;
+    return y;
+}
+
+// node_hits from the precomputed label window and ancestor jumps: one load
+// gives every suffix of length <= 16, and a hit's row costs <= 4 hops.
+template <typename Emit>
+__device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, Emit emit) {
+    const ulonglong2 win = __ldg(a.window + m);
+    const int32_t d8 = __ldg(a.depth8 + m);
+    const int32_t lim = a.lmax < kMaxClimb ? a.lmax : kMaxClimb;
+    const int32_t depth = d8 < lim ? d8 : lim;
+    const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y), uint32_t(win.y >> 32)};
+    if (__ldg(a.terminal + m)) emit(m, a.eos);
+    uint64_t h = 0, pw = 1;
+#pragma unroll
+    for (int k0 = 0; k0 < kMaxClimb; k0 += 8) {
+        if (k0 < depth) {
+            uint64_t key[8];
+            ulonglong2 first[8];
+#pragma unroll
+            for (int i = 0; i < 8; i++) {
+                const int k = k0 + i;
+                key[i] = 0ull;
+                first[i] = make_ulonglong2(0ull, 0ull);
+                if (k < depth) {
+                    h += (uint64_t(byte_at(lab, k)) + 1ull) * pw;
+                    pw *= kHashBase;
+                    key[i] = hash_finish(h, uint32_t(k + 1));
+                    first[i] = __ldg(reinterpret_cast<const ulonglong2 *>(a.ht_key) +
+                                     (uint32_t(key[i] >> 1) & a.pairs_mask));
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; i++) {
+                const int k = k0 + i;
+                if (k < depth && (first[i].x == key[i] || first[i].y == key[i] || first[i].y != 0ull)) {
+                    int32_t row = -1;  // looked up on the first hit only
+                    probe(a, key[i], k + 1, &lab, m, [&](int32_t t) {
+                        if (row < 0) row = ancestor(a, m, k + 1);
+                        emit(row, t);
+                    });
+                }
+            }
+        }
+    }
+    // suffixes longer than the window (deep tries with long tokens)
+    if (a.lmax > kMaxClimb && depth == kMaxClimb) {
+        int32_t y = ancestor(a, m, kMaxClimb);  // start of the 16-byte suffix
+        for (int32_t k = kMaxClimb + 1; k <= a.lmax; k++) {
+            const int32_t p = a.parent[y];
+            if (p < 0) break;
+            h += (uint64_t(a.label[y]) + 1ull) * pw;
+            pw *= kHashBase;
+            const int32_t row = p;
+            probe(a, hash_finish(h, uint32_t(k)), k, nullptr, m, [&](int32_t t) { emit(row, t); });
+            y = p;
+        }
+    }
+}
+
+__device__ __forceinline__ void set_mask_bit(const PatchArgs &a, int32_t row, int32_t t) {
+    atomicOr(a.mask + int64_t(row) * a.W + (t >> 5), 1u << (t & 31));
+}
+
+// Fill-then-patch form (two kernels): climbs and probes overlap the fill,
+// the bits are set once the fill has completed.
+__global__ void __launch_bounds__(kPatchThreads) k_mask_patch(PatchArgs a) {
+    pdl_launch_dependents();
+    bool waited = false;
+    const int32_t stride = gridDim.x * blockDim.x;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        node_hits(a, m, [&](int32_t row, int32_t t) {
+            if (!waited) {
+                pdl_wait();  // the fill of this mask must be complete
+                waited = true;
+            }
+            set_mask_bit(a, row, t);
+        });
+    }
     if (!waited) pdl_wait();
+}
+
+// Probe-fill-scatter form (three kernels). k_mask_probe records up to
+// kHitSlots hits per node in a buffer (count kHitOverflow: more hits, found
+// again by the scatter). It waits for all earlier work at entry, prefetches
+// its tables into L2 (its dependent loads then hit L2 while the fill
+// saturates HBM) and only then lets the fill launch, which runs beside it.
+__global__ void __launch_bounds__(kPatchThreads) k_mask_probe(PatchArgs a, Prefetch pf) {
+    pdl_wait();  // an earlier scatter may still read the hit buffer
+    if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
+    pdl_launch_dependents();
+    const int32_t stride = gridDim.x * blockDim.x;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        int32_t c = 0;
+        int2 *slot = a.hits + int64_t(m) * kHitSlots;
+        node_hits_window(a, m, [&](int32_t row, int32_t t) {
+            if (c < kHitSlots) slot[c] = make_int2(row, t);
+            c++;
+        });
+        a.hit_count[m] = uint8_t(c > kHitSlots ? kHitOverflow : c);
+    }
+}
+
+// Sets the recorded bits after the fill (which completes after the probe).
+__global__ void __launch_bounds__(kPatchThreads) k_mask_scatter(PatchArgs a) {
+    pdl_launch_dependents();
+    pdl_wait();  // fill complete, and through it the probe
+    const int32_t stride = gridDim.x * blockDim.x;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        const int32_t c = a.hit_count[m];
+        if (c == kHitOverflow) {
+            node_hits_window(a, m, [&](int32_t row, int32_t t) { set_mask_bit(a, row, t); });
+            continue;
+        }
+        const int2 *slot = a.hits + int64_t(m) * kHitSlots;
+        for (int32_t i = 0; i < c; i++) {
+            const int2 hv = slot[i];
+            set_mask_bit(a, hv.x, hv.y);
+        }
+    }
 }
 
 // ------------------------------------------------------------------ advance
@@ -393,6 +574,31 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_scalar(void *__restrict
     }
 }
 
+PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax, uint32_t *mask,
+                     int64_t W) {
+    PatchArgs a;
+    a.parent = t.parent;
+    a.label = t.label;
+    a.terminal = t.terminal;
+    a.n_nodes = n_nodes;
+    a.ht_key = v.ht_key;
+    a.ht_val = v.ht_val;
+    a.pairs_mask = v.ht_mask >> 1;
+    a.tok_off = v.tok_off;
+    a.tok_len = v.tok_len;
+    a.blob = v.blob;
+    a.lmax = lmax;
+    a.mask = mask;
+    a.W = W;
+    a.eos = v.V - 1;
+    a.hits = t.hits;
+    a.hit_count = t.hit_count;
+    a.window = t.window;
+    a.depth8 = t.depth8;
+    a.jump = t.jump;
+    return a;
+}
+
 inline int grid_for(int64_t work, int64_t per_block, int64_t cap) {
     int64_t g = (work + per_block - 1) / per_block;
     if (g < 1) g = 1;
@@ -414,23 +620,45 @@ cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaS
 
 cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                               uint32_t *mask, int64_t W, int num_sms, cudaStream_t st) {
-    PatchArgs a;
-    a.parent = t.parent;
-    a.label = t.label;
-    a.terminal = t.terminal;
-    a.n_nodes = n_nodes;
-    a.ht_key = v.ht_key;
-    a.ht_val = v.ht_val;
-    a.pairs_mask = v.ht_mask >> 1;
-    a.tok_off = v.tok_off;
-    a.tok_len = v.tok_len;
-    a.blob = v.blob;
-    a.lmax = lmax;
-    a.mask = mask;
-    a.W = W;
-    a.eos = v.V - 1;
+    PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 32);
     return launch_pdl(k_mask_patch, grid, kPatchThreads, st, a);
+}
+
+cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                                 uint32_t *mask, int64_t W, int num_sms, cudaStream_t st) {
+    PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
+    // probe grid: every CTA resident at once (so that all of them pass their
+    // entry wait and let the fill launch right away), nodes in a grid-stride loop
+    const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
+    Prefetch pf;
+    pf.count = 0;
+    auto add = [&](const void *p, uint64_t n) {
+        pf.ptr[pf.count] = p;
+        pf.bytes[pf.count] = n;
+        pf.count++;
+    };
+    const uint64_t S = uint64_t(v.ht_mask) + 1, nn = uint64_t(n_nodes), nv = uint64_t(v.V);
+    add(v.ht_key, 8 * S);
+    add(v.ht_val, 4 * S);
+    add(v.tok_len, 2 * nv);
+    add(v.tok_off, 4 * nv);
+    add(v.blob, v.blob_bytes);
+    add(t.window, 16 * nn);
+    add(t.jump, 16 * nn);
+    add(t.depth8, nn);
+    add(t.terminal, nn);
+    cudaError_t e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf);
+    if (e != cudaSuccess) return e;
+    const uintptr_t addr = reinterpret_cast<uintptr_t>(mask);
+    const int64_t n_words = int64_t(n_nodes) * W;
+    int64_t head = int64_t(((16u - (addr & 15u)) & 15u) >> 2);
+    if (head > n_words) head = n_words;
+    const int fill_grid = grid_for((n_words - head) >> 2, kFillThreads * kFillVecs, INT32_MAX);
+    e = launch_pdl(k_mask_fill_beside, fill_grid, kFillThreads, st, mask, n_words, head);
+    if (e != cudaSuccess) return e;
+    const int scatter_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
+    return launch_pdl(k_mask_scatter, scatter_grid, kPatchThreads, st, a);
 }
 
 cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t *states,

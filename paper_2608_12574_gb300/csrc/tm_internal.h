@@ -25,6 +25,12 @@ struct HostTrie {
     std::vector<uint8_t> terminal;       // some string ends here
     std::vector<int32_t> first_child;    // -1 for a leaf
     std::vector<uint32_t> child_bits;    // [n * 8]
+    // Per node, for the mask compile: the labels of the last 16 edges into it
+    // (byte i = label i levels up, 0 past the root), min(depth, 255), and the
+    // ancestors 1, 2, 4 and 8 levels up (-1 past the root).
+    std::vector<uint64_t> window;        // [n * 2] (low 8 bytes, high 8 bytes)
+    std::vector<uint8_t> depth8;         // [n]
+    std::vector<int32_t> jump;           // [n * 4]
     std::vector<int32_t> roots;          // root id of each set
     int64_t n_chars = 0;                 // total bytes of the distinct strings
     int32_t max_depth = 0;
@@ -37,6 +43,7 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
                        HostTrie *out);
 std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
                          int32_t M, HostTrie *out);
+void add_compile_tables(HostTrie *t);
 
 // -------------------------------------------------------------- vocabulary
 // Token strings packed for 16-byte vector loads plus an open-addressing hash
@@ -80,6 +87,7 @@ struct DevVocab {
     const uint32_t *tok_off = nullptr;
     const uint16_t *tok_len = nullptr;
     const uint8_t *blob = nullptr;
+    uint64_t blob_bytes = 0;
     const uint64_t *ht_key = nullptr;
     const int32_t *ht_val = nullptr;
     // host copy of the caller's arrays, to recognise the same vocabulary later
@@ -96,6 +104,11 @@ struct DevTrie {
     const uint8_t *terminal = nullptr;
     const int32_t *first_child = nullptr;
     const uint32_t *child_bits = nullptr;
+    const ulonglong2 *window = nullptr;
+    const uint8_t *depth8 = nullptr;
+    const int4 *jump = nullptr;
+    int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) per node
+    uint8_t *hit_count = nullptr;    // compile scratch: hits found per node
 };
 
 }  // namespace tmk
@@ -119,6 +132,10 @@ int set_error(int code, const char *msg);
 cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaStream_t st);
 cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                               uint32_t *mask, int64_t W, int num_sms, cudaStream_t st);
+// Probe, fill and scatter: the mask compile with the per-node searches running
+// beside the fill (needs t.hits / t.hit_count).
+cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                                 uint32_t *mask, int64_t W, int num_sms, cudaStream_t st);
 cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t *states,
                            const int32_t *tokens, int32_t B, int32_t *err, cudaStream_t st);
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,

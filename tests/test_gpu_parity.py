@@ -91,6 +91,48 @@ def test_compile_config_full(cuda, cfg):
         assert d is None, f"row {r0 + d} differs"
 
 
+@pytest.mark.parametrize("seed", range(4))
+def test_compile_long_suffixes(cuda, seed):
+    """Deep paths and tokens longer than 16 bytes (the search beyond the
+    16-label window), both compile entry points."""
+    import torch
+    r = np.random.default_rng(seed)
+    strings = W.tool_names(seed, 60, 12, lo=20, hi=48)
+    toks = [bytes([b]) for b in range(256)]
+    seen = set(toks)
+    for _ in range(3000):
+        s_ = strings[r.integers(len(strings))]
+        L = int(r.integers(2, 40))
+        a0 = int(r.integers(0, max(1, len(s_) - L + 1)))
+        t = s_[a0:a0 + L]
+        if t not in seen:
+            seen.add(t)
+            toks.append(t)
+    toks.append(b"")
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    V = len(toks)
+    h, m = _compile(cuda, sb, so, vb, vo)
+    want = oracle.mask_all(oracle.Trie(sb, so), oracle.Vocab(vb, vo), nthreads=NCPU)
+    assert max(len(t) for t in toks) > 16 and h.max_depth > 16
+    assert _first_diff(_np_u32(m), want) is None
+    m2 = torch.full_like(m, -1)
+    T.trie_compile_masks_noalloc(h, vb, vo, V, m2)
+    assert _first_diff(_np_u32(m2), want) is None
+
+
+def test_compile_many_hits_per_node(cuda):
+    """a^k for k = 1..24 are all tokens: deep nodes of a run of 'a's end more
+    than 8 allowed (row, token) pairs (the hit buffer's overflow path)."""
+    strings = [b"a" * 30, b"a" * 12 + b"b", b"ab" * 10]
+    toks = [bytes([b]) for b in range(256)] + [b"a" * k for k in range(2, 25)] + [b"ab", b"aab", b"ba" * 3, b""]
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    h, m = _compile(cuda, sb, so, vb, vo)
+    want = oracle.mask_all(oracle.Trie(sb, so), oracle.Vocab(vb, vo))
+    assert _first_diff(_np_u32(m), want) is None
+
+
 def test_compile_forest_sampled(cuda):
     """256 per-request sets (4.8M nodes, 76 GB mask): sampled rows of every set."""
     import torch
