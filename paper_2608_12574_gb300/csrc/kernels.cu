@@ -520,8 +520,10 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
         if (lane == 0) {
             const int64_t nch = (row_chunks - c0 < kSegChunks) ? row_chunks - c0 : kSegChunks;
             const uint32_t ts = static_cast<uint32_t>(__cvta_generic_to_shared(tile));
-            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
-                         :: "l"(row + c0), "r"(ts), "r"(uint32_t(nch * 16)) : "memory");
+            uint64_t policy;  // evict-first: streaming logits must not flush the trie / mask rows
+            asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
+            asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;"
+                         :: "l"(row + c0), "r"(ts), "r"(uint32_t(nch * 16)), "l"(policy) : "memory");
             asm volatile("cp.async.bulk.commit_group;" ::: "memory");
             asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");  // tile read before exit
         }
@@ -535,7 +537,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
         const int64_t chunk = c0 + q;
         if (chunk >= row_chunks) continue;
         if (bits == 0u) {
-            row[chunk] = ninf;
+            __stcs(row + chunk, ninf);
         } else {
             const uint4 x = row[chunk];
             uint32_t e[4] = {x.x, x.y, x.z, x.w};
@@ -548,7 +550,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
                     if (!((bits >> (2 * i + 1)) & 1u)) e[i] = (e[i] & 0x0000FFFFu) | 0xFF800000u;
                 }
             }
-            row[chunk] = make_uint4(e[0], e[1], e[2], e[3]);
+            __stcs(row + chunk, make_uint4(e[0], e[1], e[2], e[3]));
         }
     }
 }
