@@ -141,8 +141,10 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
     return TRIE_OK;
 }
 
-// Uploads the trie on first use; the handle is bound to that device.
-int ensure_device_trie(trie_t h, int dev) {
+// Uploads the trie on first use, ordered on `stream` (the copies read the
+// handle's own host arrays, which outlive them); the handle is bound to that
+// device.
+int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     std::lock_guard<std::mutex> lk(h->mu);
     if (h->dev.base) {
         if (h->dev.device != dev)
@@ -181,8 +183,9 @@ int ensure_device_trie(trie_t h, int dev) {
         {o_jump, t.jump.data(), sizeof(int32_t) * 4 * n},
     };
     for (const Up &u : ups) {
-        e = cudaMemcpy(b + u.off, u.src, u.n, cudaMemcpyHostToDevice);
+        e = cudaMemcpyAsync(b + u.off, u.src, u.n, cudaMemcpyHostToDevice, stream);
         if (e != cudaSuccess) {
+            cudaStreamSynchronize(stream);
             cudaFree(base);
             return fail_cuda(e, "uploading the trie");
         }
@@ -313,7 +316,7 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     std::shared_ptr<tmk::DevVocab> voc;
     if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
-    if ((rc = ensure_device_trie(h, dev)) != TRIE_OK) return rc;
+    if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
     const int64_t W = (int64_t(V) + 31) / 32;
     const int32_t n = h->host.n;
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
