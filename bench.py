@@ -429,7 +429,8 @@ def run_gpu(args, w, rank: int, world: int, dist):
     if rank != 0:
         return
     traffic = ncu_traffic("k_apply_vec", w.name)
-    traffic_c = ncu_traffic("k_mask_fill", w.name)
+    parts = [ncu_traffic(k, w.name) for k in ("k_mask_probe", "k_mask_fill_beside", "k_mask_scatter")]
+    traffic_c = None if any(p is None for p in parts) else sum(parts)
     line = {
         "metric": METRIC,
         "value": job_throughput(N * V, world, ms_per_step * 1e-3),
@@ -456,7 +457,8 @@ def run_gpu(args, w, rank: int, world: int, dist):
                      "peak_kind": peak_kind, "timing": timing_src},
         "roofline_compile": {"bound": "hbm", "achieved": compile_gbs, "peak": hbm, "unit": "GB/s",
                              "frac": compile_gbs / hbm, "traffic": traffic_c,
-                             "kernel": "k_mask_fill + k_mask_patch", "bytes_per_launch": compile_bytes,
+                             "kernel": "k_mask_probe + k_mask_fill_beside + k_mask_scatter",
+                             "bytes_per_launch": compile_bytes,
                              "ms": compile_ms, "pairs_per_s": N * V / (compile_ms * 1e-3),
                              "peak_kind": peak_kind,
                              "timing": f"CUDA events around {reps} back-to-back replays of a graph of one compile"},
