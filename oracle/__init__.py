@@ -7,7 +7,9 @@ CUDA path and imports nothing from it.
 The arithmetic lives in ``oracle.c`` (a plain C library, each function citing
 the passage it follows); this module loads it with ctypes and adds the decode
 loop (Eq. 1: mask, greedy choice, state advance), which only calls those
-functions in order.
+functions in order. ``ac.c`` adds the paper's own Aho-Corasick precomputation
+(``AhoCorasick``), used as a third check of the masks and as the stronger
+timed CPU baseline.
 
 Pins (``tests/test_oracle_pins.py``): the worked example of App. G.1 and the
 Fig. 2 example (``tests/golden/``), exhaustive comparison with the prefix-set
@@ -29,17 +31,19 @@ DEAD = -1
 FINISHED = -2
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
+_SRC_AC = os.path.join(_HERE, "ac.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
 _lock = threading.Lock()
 _lib = None
 
 
 def build(force: bool = False) -> str:
-    """Compile oracle.c into liboracle.so (gcc, OpenMP) if it is missing or stale."""
-    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+    """Compile oracle.c and ac.c into liboracle.so (gcc, OpenMP) if missing or stale."""
+    newest = max(os.path.getmtime(_SRC), os.path.getmtime(_SRC_AC))
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < newest:
         tmp = _LIB + f".{os.getpid()}.tmp"
         subprocess.check_call(["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-std=c99",
-                               "-o", tmp, _SRC])
+                               "-o", tmp, _SRC, _SRC_AC])
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -63,6 +67,14 @@ def load_library(path: str):
     lib.oracle_advance.argtypes = [P, P, P, I32, P, P, I64]
     lib.oracle_apply.argtypes = [P, P, P, I32, P, I32, P, I64]
     lib.oracle_argmax.argtypes = [P, I32, I64, I32, P]
+    if hasattr(lib, "ac_build"):
+        lib.ac_build.restype = P
+        lib.ac_build.argtypes = [P, P, I32]
+        lib.ac_free.argtypes = [P]
+        lib.ac_num_states.restype = I32
+        lib.ac_num_states.argtypes = [P]
+        lib.ac_valid_pairs.restype = I64
+        lib.ac_valid_pairs.argtypes = [P, I32, P, P, P, P, P, I64, I32]
     return lib
 
 
@@ -190,6 +202,47 @@ def argmax(logits_bits: np.ndarray) -> np.ndarray:
     out = np.empty(B, np.int32)
     _load().oracle_argmax(_p(x), dt, B, V, _p(out))
     return out
+
+
+class AhoCorasick:
+    """The paper's automaton over the vocabulary (ac.c): built once per
+    tokenizer, then run over any trie (Sec. 4.2; App. H.4 Phases 3-4)."""
+
+    def __init__(self, voc: Vocab):
+        self._lib = _load()
+        self.voc = voc
+        h = self._lib.ac_build(_p(voc.b), _p(voc.o), voc.V)
+        if not h:
+            raise MemoryError("ac_build failed")
+        self._h = ctypes.c_void_p(h)
+        self.num_states = self._lib.ac_num_states(self._h)
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h:
+            self._lib.ac_free(h)
+            self._h = None
+
+    def pairs(self, t: Trie, nthreads: int = 1) -> tuple[np.ndarray, np.ndarray]:
+        """(start node, token) of every allowed pair, EOS excluded."""
+        args = (self._h, t.num_nodes, _p(t.parent), _p(t.label), _p(t.depth))
+        n = self._lib.ac_valid_pairs(*args, None, None, 0, nthreads)
+        if n < 0:
+            raise MemoryError("ac_valid_pairs failed")
+        rows = np.empty(max(n, 1), np.int32)
+        toks = np.empty(max(n, 1), np.int32)
+        self._lib.ac_valid_pairs(*args, _p(rows), _p(toks), n, nthreads)
+        return rows[:n], toks[:n]
+
+    def mask(self, t: Trie, nthreads: int = 1) -> np.ndarray:
+        """Dense [N, ceil(V/32)] mask from the pairs, EOS at terminal nodes (App. G.5)."""
+        rows, toks = self.pairs(t, nthreads)
+        V = self.voc.V
+        m = np.zeros((t.num_nodes, n_words(V)), np.uint32)
+        np.bitwise_or.at(m, (rows, toks >> 5), (np.uint32(1) << (toks & 31).astype(np.uint32)))
+        term = np.nonzero(t.terminal)[0]
+        m[term, (V - 1) >> 5] |= np.uint32(1 << ((V - 1) & 31))
+        return m
 
 
 def decode(t: Trie, voc: Vocab, logits_per_step, states0: np.ndarray):
