@@ -168,6 +168,39 @@ int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B
 int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B,
                     int32_t V, cudaStream_t stream);
 
+/* Sparse form of the masks: for every node the ids of its allowed tokens, as
+ * the paper stores them (valid[n] as lists of 4-byte token ids, Sec. 4.2;
+ * App. H.5), computed on the GPU without the dense bitmask. At K = 10,000 and
+ * V = 152,064 the lists hold 46,899 ids (188 KB) where the bitmask takes
+ * 439 MB.
+ *   Arguments as trie_compile_masks; the lists are stored on the device by
+ *   the library, with the handle (they replace those of an earlier call).
+ *   Layout: offsets int64[num_nodes + 1] and tokens int32[offsets[N]]; the
+ *   tokens of node n are tokens[offsets[n] .. offsets[n+1]), EOS (V-1)
+ *   included where n is terminal, in no particular order.
+ *   Host-synchronous: it reads the number of entries back to size the token
+ *   buffer (one small device-to-host copy on `stream`). Records the
+ *   vocabulary for trie_advance, like trie_compile_masks.
+ *   Errors: TRIE_EINVAL, TRIE_ENOMEM, TRIE_ECUDA. */
+int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                       cudaStream_t stream);
+
+/* Number of (node, token) entries in the handle's lists; -1 before any
+ * trie_compile_lists. */
+int64_t trie_num_valid(trie_t h);
+
+/* Copy the handle's lists into caller buffers (device; each may be NULL):
+ * d_offsets int64[num_nodes + 1], d_tokens int32[trie_num_valid(h)].
+ * Asynchronous on `stream`. TRIE_ESTATE before any trie_compile_lists. */
+int trie_copy_lists(trie_t h, int64_t *d_offsets, int32_t *d_tokens, cudaStream_t stream);
+
+/* trie_apply_mask driven by the handle's valid lists instead of a bitmask
+ * (the decode-time lookup A(s_t) = valid[s_t] of Sec. 4.2, then the -inf
+ * write of App. H.3). Arguments, states and result as trie_apply_mask; V
+ * must equal the V of the last trie_compile_lists (TRIE_ESTATE if none). */
+int trie_apply_lists(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                     cudaStream_t stream);
+
 /* Size of the fixed device scratch used by trie_compile_masks_noalloc. */
 #define TRIE_NOALLOC_SCRATCH_BYTES (32u << 20)
 

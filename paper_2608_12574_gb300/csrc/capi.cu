@@ -376,11 +376,112 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
     return TRIE_OK;
 }
 
+int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                       cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
+    const int32_t n = h->host.n;
+    tmk::DevLists &L = h->lists;
+    if (!L.base) {  // per-row counters, cursors, offsets and scan scratch
+        Layout lay;
+        const size_t o_cnt = lay.add(sizeof(int32_t) * 2 * size_t(n));
+        const size_t o_off = lay.add(sizeof(int64_t) * (size_t(n) + 1));
+        const size_t o_tile = lay.add(sizeof(int64_t) * (size_t(n) / 4096 + 2));
+        const size_t o_tot = lay.add(sizeof(int64_t));
+        void *base = nullptr;
+        cudaError_t e = cudaMalloc(&base, lay.total);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(TRIE_ENOMEM, std::string("cudaMalloc for the valid lists: ") + cudaGetErrorString(e));
+        }
+        char *b = static_cast<char *>(base);
+        L.base = base;
+        L.count = reinterpret_cast<int32_t *>(b + o_cnt);
+        L.cursor = L.count + n;
+        L.off = reinterpret_cast<int64_t *>(b + o_off);
+        L.tile_sum = reinterpret_cast<int64_t *>(b + o_tile);
+        L.total = reinterpret_cast<int64_t *>(b + o_tot);
+    }
+    const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
+    const int sms = num_sms(dev);
+    int64_t total = 0;
+    cudaError_t e = tmk::launch_lists_count(h->dev, n, *voc, lmax, L, sms, stream, &total);
+    if (e != cudaSuccess) return fail_cuda(e, "valid-list count");
+    if (total > L.tok_cap) {  // grow the token buffer (by at least half)
+        const int64_t cap = std::max<int64_t>(total, L.tok_cap + L.tok_cap / 2);
+        if (L.toks) cudaFree(L.toks);
+        L.toks = nullptr;
+        L.tok_cap = 0;
+        e = cudaMalloc(reinterpret_cast<void **>(&L.toks), sizeof(int32_t) * size_t(std::max<int64_t>(cap, 1)));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            L.toks = nullptr;
+            L.n_valid = -1;
+            return fail(TRIE_ENOMEM, std::string("cudaMalloc for the valid-list tokens: ") + cudaGetErrorString(e));
+        }
+        L.tok_cap = cap;
+    }
+    e = tmk::launch_lists_scatter(h->dev, n, *voc, lmax, L, sms, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "valid-list scatter");
+    std::lock_guard<std::mutex> lk(h->mu);
+    L.n_valid = total;
+    L.V = V;
+    h->vocab = voc;
+    return TRIE_OK;
+}
+
+int64_t trie_num_valid(trie_t h) { return h ? h->lists.n_valid : -1; }
+
+int trie_copy_lists(trie_t h, int64_t *d_offsets, int32_t *d_tokens, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    const tmk::DevLists &L = h->lists;
+    if (L.n_valid < 0) return fail(TRIE_ESTATE, "trie_copy_lists before trie_compile_lists on this handle");
+    if (d_offsets) {
+        cudaError_t e = cudaMemcpyAsync(d_offsets, L.off, sizeof(int64_t) * (size_t(h->host.n) + 1),
+                                        cudaMemcpyDeviceToDevice, stream);
+        if (e != cudaSuccess) return fail_cuda(e, "copying the list offsets");
+    }
+    if (d_tokens && L.n_valid > 0) {
+        cudaError_t e = cudaMemcpyAsync(d_tokens, L.toks, sizeof(int32_t) * size_t(L.n_valid),
+                                        cudaMemcpyDeviceToDevice, stream);
+        if (e != cudaSuccess) return fail_cuda(e, "copying the list tokens");
+    }
+    return TRIE_OK;
+}
+
+int trie_apply_lists(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                     cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_logits || !d_states)) return fail(TRIE_EINVAL, "d_logits / d_states is NULL");
+    if (h->lists.n_valid < 0) return fail(TRIE_ESTATE, "trie_apply_lists before trie_compile_lists on this handle");
+    if (V != h->lists.V) return fail(TRIE_EINVAL, "V differs from the compiled lists' V");
+    if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
+        return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_apply_lists(d_logits, dtype, h->lists, d_states, B, V, h->host.n, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "apply-lists launch");
+    return TRIE_OK;
+}
+
 int trie_destroy(trie_t h) {
     if (!h) return TRIE_OK;
-    if (h->dev.base) {
+    if (h->dev.base || h->lists.base || h->lists.toks) {
         DeviceGuard g(h->dev.device);
-        cudaFree(h->dev.base);  // waits for work on the device that may still read it
+        // cudaFree waits for work on the device that may still read these
+        if (h->lists.toks) cudaFree(h->lists.toks);
+        if (h->lists.base) cudaFree(h->lists.base);
+        if (h->dev.base) cudaFree(h->dev.base);
     }
     delete h;
     return TRIE_OK;

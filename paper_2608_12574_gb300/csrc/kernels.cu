@@ -484,43 +484,39 @@ __device__ __forceinline__ uint32_t row_word(const uint32_t *__restrict__ mask, 
     return (w == (eos >> 5)) ? (1u << (eos & 31)) : 0u;
 }
 
-// kElt = 2 (bf16) or 4 (fp32). Requires V % (16 / kElt) == 0 and a 16-byte
-// aligned logits base, so that every row starts on a 16-byte boundary.
-// One warp per 1024-token segment of a row (one mask word per lane). A
-// segment without any allowed token (almost all of them) is written by one
-// TMA bulk copy (cp.async.bulk) from a -inf tile in shared memory; a segment
-// with allowed tokens is written by the lanes, 16 bytes each, reading the
-// logits only in chunks that hold an allowed token.
+// -inf pattern of 16 bytes of logits.
 template <int kElt>
-__global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__ logits,
-                                                             const uint32_t *__restrict__ mask,
-                                                             const int32_t *__restrict__ states, int32_t B,
-                                                             int32_t V, int64_t W, int32_t n_nodes,
-                                                             int32_t segs) {
+__device__ __forceinline__ uint4 ninf16() {
+    return (kElt == 2) ? make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u)
+                       : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
+}
+
+// Fills the CTA's -inf tile (one segment of logits) and makes it visible to
+// the bulk copies. Must be called by every thread of the CTA.
+template <int kElt>
+__device__ __forceinline__ void init_ninf_tile(uint4 *tile) {
+    constexpr int kSegChunks = 1024 / (16 / kElt);
+    for (int i = threadIdx.x; i < kSegChunks; i += blockDim.x) tile[i] = ninf16<kElt>();
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // tile visible to the bulk copies
+    __syncthreads();
+}
+
+// Writes one 1024-token segment of a logits row (by one warp; lane l holds
+// mask word l of the segment). A segment without an allowed token is one TMA
+// bulk copy of the -inf tile; otherwise the lanes write 16-byte chunks,
+// reading the logits only in chunks that hold an allowed token. Stores use an
+// L2 evict-first policy: the logits stream must not flush the trie tables.
+template <int kElt>
+__device__ __forceinline__ void write_segment(uint4 *__restrict__ row, int64_t c0, int64_t row_chunks,
+                                              uint32_t word, int lane, const uint4 *tile) {
     constexpr int kPer = 16 / kElt;            // tokens per 16-byte chunk
     constexpr int kChunks = 1024 / kPer / 32;  // chunks per lane per segment
     constexpr int kSegChunks = 1024 / kPer;
-    __shared__ __align__(128) uint4 tile[kSegChunks];
-    const uint4 ninf = (kElt == 2) ? make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u)
-                                   : make_uint4(0xFF800000u, 0xFF800000u, 0xFF800000u, 0xFF800000u);
-    for (int i = threadIdx.x; i < kSegChunks; i += kApplyThreads) tile[i] = ninf;
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // tile visible to the bulk copies
-    __syncthreads();
-    pdl_launch_dependents();
-    pdl_wait();  // logits and states come from earlier kernels
-    const int lane = threadIdx.x & 31;
-    const int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
-    if (item >= B * segs) return;  // uniform per warp
-    const int32_t b = item / segs, seg = item - b * segs;
-    const uint32_t word = row_word(mask, __ldg(states + b), n_nodes, W, int64_t(seg) * 32 + lane, V - 1);
-    const int64_t row_chunks = int64_t(V) / kPer;
-    uint4 *row = logits + int64_t(b) * row_chunks;
-    const int64_t c0 = int64_t(seg) * kSegChunks;
     if (!__any_sync(0xffffffffu, word != 0u)) {
         if (lane == 0) {
             const int64_t nch = (row_chunks - c0 < kSegChunks) ? row_chunks - c0 : kSegChunks;
             const uint32_t ts = static_cast<uint32_t>(__cvta_generic_to_shared(tile));
-            uint64_t policy;  // evict-first: streaming logits must not flush the trie / mask rows
+            uint64_t policy;
             asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(policy));
             asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;"
                          :: "l"(row + c0), "r"(ts), "r"(uint32_t(nch * 16)), "l"(policy) : "memory");
@@ -529,6 +525,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
         }
         return;
     }
+    const uint4 ninf = ninf16<kElt>();
 #pragma unroll
     for (int j = 0; j < kChunks; j++) {
         const int q = j * 32 + lane;  // chunk within the segment
@@ -551,6 +548,212 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
                 }
             }
             __stcs(row + chunk, make_uint4(e[0], e[1], e[2], e[3]));
+        }
+    }
+}
+
+// kElt = 2 (bf16) or 4 (fp32). Requires V % (16 / kElt) == 0 and a 16-byte
+// aligned logits base, so that every row starts on a 16-byte boundary.
+// One warp per 1024-token segment of a row (one mask word per lane).
+template <int kElt>
+__global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__ logits,
+                                                             const uint32_t *__restrict__ mask,
+                                                             const int32_t *__restrict__ states, int32_t B,
+                                                             int32_t V, int64_t W, int32_t n_nodes,
+                                                             int32_t segs) {
+    constexpr int kSegChunks = 1024 / (16 / kElt);
+    __shared__ __align__(128) uint4 tile[kSegChunks];
+    init_ninf_tile<kElt>(tile);
+    pdl_launch_dependents();
+    pdl_wait();  // logits and states come from earlier kernels
+    const int lane = threadIdx.x & 31;
+    const int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
+    if (item >= B * segs) return;  // uniform per warp
+    const int32_t b = item / segs, seg = item - b * segs;
+    const uint32_t word = row_word(mask, __ldg(states + b), n_nodes, W, int64_t(seg) * 32 + lane, V - 1);
+    const int64_t row_chunks = int64_t(V) / (16 / kElt);
+    write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
+                        tile);
+}
+
+// ---------------------------------------------------------------- valid lists
+// Sparse form of the masks (the valid[n] lists the paper stores, Sec. 4.2 and
+// App. H.5): for every node, the ids of its allowed tokens (EOS included at
+// terminal nodes) in no particular order, as CSR offsets[N+1] + tokens.
+
+// Counts the allowed tokens of every row (the start node of each hit).
+__global__ void __launch_bounds__(kPatchThreads) k_list_count(PatchArgs a, int32_t *__restrict__ row_count) {
+    pdl_launch_dependents();
+    pdl_wait();  // hits from the probe, zeroed counters
+    const int32_t stride = gridDim.x * blockDim.x;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        const int32_t c = a.hit_count[m];
+        if (c == kHitOverflow) {
+            node_hits_window(a, m, [&](int32_t row, int32_t) { atomicAdd(row_count + row, 1); });
+            continue;
+        }
+        for (int32_t i = 0; i < c; i++) atomicAdd(row_count + a.hits[int64_t(m) * kHitSlots + i].x, 1);
+    }
+}
+
+// Exclusive scan of the row counts into int64 offsets, in three passes over
+// tiles of kScanTile counts: tile sums, a scan of the tile sums by one CTA,
+// and the offsets of every row.
+constexpr int kScanThreads = 1024;
+constexpr int kScanPer = 4;
+constexpr int kScanTile = kScanThreads * kScanPer;
+
+__device__ __forceinline__ int64_t block_exclusive_scan(int64_t v, int64_t *smem_warp, int64_t *total) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    int64_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int64_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) smem_warp[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+        int64_t w = lane < int(blockDim.x >> 5) ? smem_warp[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        smem_warp[lane] = w;  // inclusive scan of the warp totals
+    }
+    __syncthreads();
+    const int64_t warp_base = wid ? smem_warp[wid - 1] : 0;
+    *total = smem_warp[(blockDim.x >> 5) - 1];
+    __syncthreads();
+    return warp_base + x - v;
+}
+
+__global__ void __launch_bounds__(kScanThreads) k_scan_tiles(const int32_t *__restrict__ cnt, int32_t n,
+                                                             int64_t *__restrict__ tile_sum) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ int64_t sw[32];
+    const int64_t base = int64_t(blockIdx.x) * kScanTile + int64_t(threadIdx.x) * kScanPer;
+    int64_t v = 0;
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++)
+        if (base + j < n) v += cnt[base + j];
+    int64_t total;
+    block_exclusive_scan(v, sw, &total);
+    if (threadIdx.x == 0) tile_sum[blockIdx.x] = total;
+}
+
+__global__ void __launch_bounds__(kScanThreads) k_scan_tile_sums(int64_t *__restrict__ tile_sum, int32_t n_tiles,
+                                                                 int64_t *__restrict__ grand_total) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ int64_t sw[32];
+    int64_t carry = 0;
+    for (int32_t t0 = 0; t0 < n_tiles; t0 += kScanThreads) {
+        const int32_t i = t0 + threadIdx.x;
+        const int64_t v = i < n_tiles ? tile_sum[i] : 0;
+        int64_t total;
+        const int64_t ex = block_exclusive_scan(v, sw, &total);
+        if (i < n_tiles) tile_sum[i] = carry + ex;
+        carry += total;
+    }
+    if (threadIdx.x == 0) *grand_total = carry;
+}
+
+__global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__restrict__ cnt, int32_t n,
+                                                            const int64_t *__restrict__ tile_off,
+                                                            const int64_t *__restrict__ grand_total,
+                                                            int64_t *__restrict__ off) {
+    pdl_launch_dependents();
+    pdl_wait();
+    __shared__ int64_t sw[32];
+    const int64_t base = int64_t(blockIdx.x) * kScanTile + int64_t(threadIdx.x) * kScanPer;
+    int64_t c[kScanPer];
+    int64_t v = 0;
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++) {
+        c[j] = base + j < n ? cnt[base + j] : 0;
+        v += c[j];
+    }
+    int64_t total;
+    int64_t run = tile_off[blockIdx.x] + block_exclusive_scan(v, sw, &total);
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++) {
+        if (base + j < n) off[base + j] = run;
+        run += c[j];
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) off[n] = *grand_total;
+}
+
+// Writes every hit into its row (positions claimed with a per-row cursor).
+__global__ void __launch_bounds__(kPatchThreads) k_list_scatter(PatchArgs a, const int64_t *__restrict__ off,
+                                                                int32_t *__restrict__ cursor,
+                                                                int32_t *__restrict__ toks) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int32_t stride = gridDim.x * blockDim.x;
+    auto put = [&](int32_t row, int32_t t) { toks[off[row] + atomicAdd(cursor + row, 1)] = t; };
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        const int32_t c = a.hit_count[m];
+        if (c == kHitOverflow) {
+            node_hits_window(a, m, put);
+            continue;
+        }
+        for (int32_t i = 0; i < c; i++) {
+            const int2 hv = a.hits[int64_t(m) * kHitSlots + i];
+            put(hv.x, hv.y);
+        }
+    }
+}
+
+// Apply from the lists: CTA (row b, part p) covers 8 segments (8,192 tokens).
+// It rebuilds their 256 mask words in shared memory from the row's list and
+// writes them like k_apply_vec (kVec) or one logit per thread (any V and
+// alignment).
+template <int kElt, bool kVec>
+__global__ void __launch_bounds__(kApplyThreads) k_apply_lists(void *__restrict__ logits,
+                                                               const int64_t *__restrict__ off,
+                                                               const int32_t *__restrict__ toks,
+                                                               const int32_t *__restrict__ states, int32_t B,
+                                                               int32_t V, int32_t n_nodes, int32_t parts) {
+    constexpr int kSegChunks = 1024 / (16 / kElt);
+    constexpr int kWords = 8 * 32;
+    __shared__ __align__(128) uint4 tile[kVec ? kSegChunks : 1];
+    __shared__ uint32_t words[kWords];
+    for (int i = threadIdx.x; i < kWords; i += kApplyThreads) words[i] = 0u;
+    if (kVec) init_ninf_tile<kElt>(tile);
+    else __syncthreads();
+    pdl_launch_dependents();
+    pdl_wait();  // logits and states come from earlier kernels
+    const int32_t b = int32_t(blockIdx.x) / parts, part = int32_t(blockIdx.x) - b * parts;
+    const int32_t s = __ldg(states + b);
+    const int32_t t0 = part * 8192, eos = V - 1;
+    if (s >= 0 && s < n_nodes) {
+        const int64_t lo = __ldg(off + s), hi = __ldg(off + s + 1);
+        for (int64_t i = lo + threadIdx.x; i < hi; i += kApplyThreads) {
+            const int32_t t = __ldg(toks + i) - t0;
+            if (t >= 0 && t < 8192) atomicOr(words + (t >> 5), 1u << (t & 31));
+        }
+    } else if (threadIdx.x == 0 && eos - t0 >= 0 && eos - t0 < 8192) {
+        words[(eos - t0) >> 5] = 1u << ((eos - t0) & 31);  // FINISHED, DEAD, not a node: {EOS}
+    }
+    __syncthreads();
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (kVec) {
+        const int64_t row_chunks = int64_t(V) / (16 / kElt);
+        const int64_t c0 = (int64_t(part) * 8 + wid) * kSegChunks;
+        if (c0 >= row_chunks) return;
+        write_segment<kElt>(static_cast<uint4 *>(logits) + int64_t(b) * row_chunks, c0, row_chunks,
+                            words[wid * 32 + lane], lane, tile);
+    } else {
+        for (int32_t j = threadIdx.x; j < 8192; j += kApplyThreads) {
+            const int32_t v = t0 + j;
+            if (v >= V) break;
+            if ((words[j >> 5] >> (j & 31)) & 1u) continue;
+            const int64_t idx = int64_t(b) * V + v;
+            if (kElt == 4) static_cast<uint32_t *>(logits)[idx] = 0xFF800000u;
+            else static_cast<uint16_t *>(logits)[idx] = 0xFF80u;
         }
     }
 }
@@ -690,6 +893,67 @@ cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const in
     if (elt == 2)
         return launch_pdl(k_apply_scalar<2>, grid, kApplyThreads, st, logits, mask, states, B, V, W, n_nodes);
     return launch_pdl(k_apply_scalar<4>, grid, kApplyThreads, st, logits, mask, states, B, V, W, n_nodes);
+}
+
+cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                               const DevLists &L, int num_sms, cudaStream_t st, int64_t *h_total) {
+    PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
+    Prefetch pf;
+    pf.count = 0;
+    const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
+    cudaError_t e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf);
+    if (e != cudaSuccess) return e;
+    // count and cursor are adjacent: zero both
+    if ((e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), 2 * int64_t(n_nodes), num_sms, st)) !=
+        cudaSuccess)
+        return e;
+    const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
+    if ((e = launch_pdl(k_list_count, grid, kPatchThreads, st, a, L.count)) != cudaSuccess) return e;
+    const int32_t n_tiles = int32_t((int64_t(n_nodes) + kScanTile - 1) / kScanTile);
+    if ((e = launch_pdl(k_scan_tiles, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count), n_nodes,
+                        L.tile_sum)) != cudaSuccess)
+        return e;
+    if ((e = launch_pdl(k_scan_tile_sums, 1, kScanThreads, st, L.tile_sum, n_tiles, L.total)) != cudaSuccess)
+        return e;
+    if ((e = launch_pdl(k_scan_rows, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count), n_nodes,
+                        static_cast<const int64_t *>(L.tile_sum), static_cast<const int64_t *>(L.total),
+                        L.off)) != cudaSuccess)
+        return e;
+    // the size decides the token buffer: read it back (the one host sync)
+    if ((e = cudaMemcpyAsync(h_total, L.total, sizeof(int64_t), cudaMemcpyDeviceToHost, st)) != cudaSuccess)
+        return e;
+    return cudaStreamSynchronize(st);
+}
+
+cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                                 const DevLists &L, int num_sms, cudaStream_t st) {
+    PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
+    const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
+    return launch_pdl(k_list_scatter, grid, kPatchThreads, st, a, static_cast<const int64_t *>(L.off), L.cursor,
+                      L.toks);
+}
+
+cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
+                               int32_t V, int32_t n_nodes, cudaStream_t st) {
+    const int elt = dtype == 0 ? 4 : 2;
+    const int32_t parts = int32_t((int64_t(V) + 8191) / 8192);
+    const bool vec = (reinterpret_cast<uintptr_t>(logits) & 15u) == 0 && (int64_t(V) * elt) % 16 == 0;
+    const int64_t grid = int64_t(B) * parts;
+    if (grid > INT32_MAX) return cudaErrorInvalidValue;
+    const int32_t *tk = L.toks;
+    const int64_t *of = L.off;
+    if (vec) {
+        if (elt == 2)
+            return launch_pdl(k_apply_lists<2, true>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
+                              n_nodes, parts);
+        return launch_pdl(k_apply_lists<4, true>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
+                          n_nodes, parts);
+    }
+    if (elt == 2)
+        return launch_pdl(k_apply_lists<2, false>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
+                          n_nodes, parts);
+    return launch_pdl(k_apply_lists<4, false>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
+                      n_nodes, parts);
 }
 
 }  // namespace tmk

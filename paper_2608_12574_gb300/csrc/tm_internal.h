@@ -111,6 +111,20 @@ struct DevTrie {
     uint8_t *hit_count = nullptr;    // compile scratch: hits found per node
 };
 
+// Device storage of the sparse valid lists of a handle (library-owned).
+struct DevLists {
+    void *base = nullptr;           // count, cursor, off, tile_sum, total
+    int32_t *count = nullptr;       // [n] allowed tokens per row (cursor follows it)
+    int32_t *cursor = nullptr;      // [n]
+    int64_t *off = nullptr;         // [n + 1]
+    int64_t *tile_sum = nullptr;    // [tiles]
+    int64_t *total = nullptr;       // [1]
+    int32_t *toks = nullptr;        // [tok_cap], separate allocation
+    int64_t tok_cap = 0;
+    int64_t n_valid = -1;           // entries of the last build, -1 before any
+    int32_t V = 0;
+};
+
 }  // namespace tmk
 
 // The opaque handle of the C ABI.
@@ -121,6 +135,7 @@ struct trie_s {
     std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
     int32_t mask_V = 0;
+    tmk::DevLists lists;                 // last compiled valid lists (library-owned)
 };
 
 namespace tmk {
@@ -140,4 +155,12 @@ cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v,
                            const int32_t *tokens, int32_t B, int32_t *err, cudaStream_t st);
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
                          int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st);
+// Valid lists: probe, per-row counts and their scan; ends by reading the
+// total into *h_total (host-synchronous). Then the scatter into L.toks.
+cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                               const DevLists &L, int num_sms, cudaStream_t st, int64_t *h_total);
+cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                                 const DevLists &L, int num_sms, cudaStream_t st);
+cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
+                               int32_t V, int32_t n_nodes, cudaStream_t st);
 }  // namespace tmk

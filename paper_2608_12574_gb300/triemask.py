@@ -35,6 +35,10 @@ SIGNATURES = {
     "trie_get_csr": (ctypes.c_int, [_P, _P, _P, _P, _P]),
     "trie_compile_masks": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_compile_masks_noalloc": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "trie_compile_lists": (ctypes.c_int, [_P, _P, _P, _I32, _P]),
+    "trie_num_valid": (_I64, [_P]),
+    "trie_copy_lists": (ctypes.c_int, [_P, _P, _P, _P]),
+    "trie_apply_lists": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
     "trie_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
     "trie_destroy": (ctypes.c_int, [_P]),
@@ -247,6 +251,52 @@ def trie_apply_mask(h: Trie, d_logits, d_states, stream=None) -> None:
     pl = _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits")
     ps = _dev(d_states, (torch.int32,), "d_states")
     _check(h._lib.trie_apply_mask(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
+
+
+def trie_compile_lists(h: Trie, vocab_bytes, vocab_offsets, V: int, stream=None, device=None) -> int:
+    """Build the handle's sparse valid lists on the GPU; returns the number of entries."""
+    import torch
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    _check(h._lib.trie_compile_lists(h.handle, _hp(vb), _hp(vo), V,
+                                     _stream(stream, device if device is not None else torch.cuda.current_device())))
+    return h._lib.trie_num_valid(h.handle)
+
+
+def trie_num_valid(h: Trie) -> int:
+    return h._lib.trie_num_valid(h.handle)
+
+
+def trie_copy_lists(h: Trie, device=None, stream=None):
+    """(offsets int64[N+1], tokens int32[n_valid]) device tensors with the handle's lists."""
+    import torch
+    n = trie_num_valid(h)
+    if n < 0:
+        raise TrieError(TRIE_ESTATE, "no valid lists on this handle")
+    dev = device if device is not None else "cuda"
+    off = torch.empty(h.num_nodes + 1, dtype=torch.int64, device=dev)
+    tok = torch.empty(max(n, 1), dtype=torch.int32, device=dev)
+    _check(h._lib.trie_copy_lists(h.handle, ctypes.c_void_p(off.data_ptr()), ctypes.c_void_p(tok.data_ptr()),
+                                  _stream(stream, off.device)))
+    return off, tok[:n]
+
+
+def trie_apply_lists(h: Trie, d_logits, d_states, stream=None) -> None:
+    """trie_apply_mask driven by the handle's valid lists."""
+    import torch
+    if d_logits.dim() != 2:
+        raise ValueError("d_logits must be [B, V]")
+    B, V = d_logits.shape
+    if d_states.numel() != B:
+        raise ValueError("d_states must have B entries")
+    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
+    if dtype is None:
+        raise TypeError("d_logits must be float32 or bfloat16")
+    pl = _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits")
+    ps = _dev(d_states, (torch.int32,), "d_states")
+    _check(h._lib.trie_apply_lists(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
 
 
 def trie_destroy(h: Trie) -> None:

@@ -1,0 +1,179 @@
+"""GPU parity of the sparse valid lists (trie_compile_lists / trie_apply_lists)
+against the CPU oracle: the (node, token) entries equal the oracle's, and the
+list-driven mask application and decode loop are bit-identical to the
+oracle's."""
+from __future__ import annotations
+
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_12574_gb300 import triemask as T
+from paper_2608_12574_gb300 import workloads as W
+from pins import random_case
+
+pytestmark = pytest.mark.gpu
+NCPU = os.cpu_count() or 1
+
+
+@pytest.fixture(scope="module")
+def cuda():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_12574_gb300 import _build
+    _build.build()
+    oracle.build()
+    return torch.device("cuda:0")
+
+
+def _bits(t):
+    import torch
+    t = t.cpu().contiguous()
+    if t.dtype == torch.float32:
+        return t.view(torch.int32).numpy().view(np.uint32)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def _gpu_pairs(h):
+    off, tok = T.trie_copy_lists(h)
+    off = off.cpu().numpy()
+    tok = tok.cpu().numpy()
+    rows = np.repeat(np.arange(len(off) - 1, dtype=np.int64), np.diff(off))
+    assert len(rows) == len(tok) == T.trie_num_valid(h)
+    return rows, tok.astype(np.int64)
+
+
+def _key(rows, toks, V):
+    return np.sort(rows.astype(np.int64) * V + toks.astype(np.int64))
+
+
+def _oracle_pairs_from_mask(m, V):
+    r, w, b = [], [], []
+    rows, words = np.nonzero(m)
+    for rr, ww in zip(rows, words):
+        x = int(m[rr, ww])
+        while x:
+            lo = x & -x
+            r.append(rr)
+            w.append(ww * 32 + lo.bit_length() - 1)
+            x ^= lo
+    return np.array(r, np.int64), np.array(w, np.int64)
+
+
+@pytest.mark.parametrize("seed", range(30))
+def test_lists_small_random(cuda, seed):
+    strings, toks = random_case(1000 + seed)
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    V = len(toks)
+    h = T.trie_build(sb, so)
+    n = T.trie_compile_lists(h, vb, vo, V)
+    want = _oracle_pairs_from_mask(oracle.mask_all(oracle.Trie(sb, so), oracle.Vocab(vb, vo)), V)
+    got = _gpu_pairs(h)
+    assert n == len(want[0])
+    assert np.array_equal(_key(*got, V), _key(*want, V))
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 3, 4])
+def test_lists_configs(cuda, cfg):
+    """Every entry of the full-size workloads against the paper-algorithm pairs
+    (oracle/ac.c, itself equal to the brute-force oracle) plus EOS at terminals."""
+    w = W.config(cfg)
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, w.V)
+    ot = oracle.Trie(w.set_bytes, w.set_offsets)
+    rows, toks = oracle.AhoCorasick(oracle.Vocab(w.vocab_bytes, w.vocab_offsets)).pairs(ot, nthreads=NCPU)
+    term = np.nonzero(ot.terminal)[0]
+    want_r = np.concatenate([rows, term]).astype(np.int64)
+    want_t = np.concatenate([toks, np.full(len(term), w.V - 1)]).astype(np.int64)
+    got = _gpu_pairs(h)
+    assert np.array_equal(_key(*got, w.V), _key(want_r, want_t, w.V))
+
+
+def test_lists_forest(cuda):
+    """The 256-request forest: every set's entries, offset by its root."""
+    w = W.config(5)
+    h = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+    T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, w.V)
+    got_r, got_t = _gpu_pairs(h)
+    got = _key(got_r, got_t, w.V)
+    ac = oracle.AhoCorasick(oracle.Vocab(w.vocab_bytes, w.vocab_offsets))
+    strings = W.unpack(w.set_bytes, w.set_offsets)
+    roots = h.roots()
+    parts_r, parts_t = [], []
+    for i in range(h.num_sets):
+        ot = oracle.Trie(*W.pack(strings[w.set_index[i]:w.set_index[i + 1]]))
+        r, t = ac.pairs(ot, nthreads=NCPU)
+        term = np.nonzero(ot.terminal)[0]
+        parts_r += [r.astype(np.int64) + roots[i], term.astype(np.int64) + roots[i]]
+        parts_t += [t.astype(np.int64), np.full(len(term), w.V - 1, np.int64)]
+    want = _key(np.concatenate(parts_r), np.concatenate(parts_t), w.V)
+    assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("V", [2, 33, 1001, 8193, 32000])
+def test_apply_lists_random_bits(cuda, dtype, V):
+    import torch
+    r = np.random.default_rng(V + 7)
+    strings = [bytes(r.integers(97, 100, r.integers(1, 6))) for _ in range(30)]
+    toks = [bytes(r.integers(97, 100, r.integers(1, 4))) for _ in range(V - 1)] + [b""]
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    h = T.trie_build(sb, so)
+    T.trie_compile_lists(h, vb, vo, V)
+    ot, ov = oracle.Trie(sb, so), oracle.Vocab(vb, vo)
+    B = 19
+    states = r.choice(np.array([-1, -2, ot.num_nodes, -9] + list(range(ot.num_nodes)) * 3, np.int32), B)
+    if dtype == "f32":
+        raw = r.integers(0, 2**32, (B, V), dtype=np.uint64).astype(np.uint32)
+        x = torch.from_numpy(raw.view(np.int32)).view(torch.float32).to(cuda)
+    else:
+        raw = r.integers(0, 2**16, (B, V), dtype=np.uint32).astype(np.uint16)
+        x = torch.from_numpy(raw.view(np.int16)).view(torch.bfloat16).to(cuda)
+    want = oracle.apply(ot, ov, raw, states)
+    T.trie_apply_lists(h, x, torch.as_tensor(states, device=cuda))
+    assert np.array_equal(_bits(x), want)
+
+
+@pytest.mark.parametrize("cfg", [1, 3])
+def test_decode_loop_lists(cuda, cfg):
+    """apply (from lists) -> greedy argmax -> advance, bit for bit at every step."""
+    import torch
+    w = W.config(cfg)
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, w.V)
+    logits = [W.logits(w, s, device="cuda") for s in range(w.steps)]
+    st = torch.zeros(w.batch, dtype=torch.int32, device=cuda)
+    err = torch.zeros(1, dtype=torch.int32, device=cuda)
+    got = []
+    for lg in logits:
+        x = lg.clone()
+        T.trie_apply_lists(h, x, st)
+        tok = torch.argmax(x, dim=1).to(torch.int32)
+        T.trie_advance(h, st, tok, err)
+        got.append((x, tok.cpu().numpy(), st.cpu().numpy().copy()))
+    ot = oracle.Trie(w.set_bytes, w.set_offsets)
+    ov = oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+    masked, toks, sts, oerr = oracle.decode(ot, ov, (_bits(lg) for lg in logits), np.zeros(w.batch, np.int32))
+    for s in range(w.steps):
+        assert np.array_equal(_bits(got[s][0]), masked[s]), s
+        assert np.array_equal(got[s][1], toks[s]), s
+        assert np.array_equal(got[s][2], sts[s]), s
+    assert int(err.item()) == oerr == 0
+
+
+def test_lists_errors(cuda):
+    import torch
+    sb, so = W.pack([b"ab"])
+    h = T.trie_build(sb, so)
+    assert T.trie_num_valid(h) == -1
+    with pytest.raises(T.TrieError):
+        T.trie_apply_lists(h, torch.zeros((1, 4), device=cuda), torch.zeros(1, dtype=torch.int32, device=cuda))
+    vb, vo = W.pack([b"a", b"b", b"ab", b""])
+    assert T.trie_compile_lists(h, vb, vo, 4) == 4   # root: a, ab; 'a': b; 'ab': EOS
+    with pytest.raises(T.TrieError):
+        T.trie_apply_lists(h, torch.zeros((1, 5), device=cuda), torch.zeros(1, dtype=torch.int32, device=cuda))
