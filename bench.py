@@ -52,6 +52,7 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=10.0,
                    help="time budget of the CPU-oracle baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-dynamic", action="store_true", help="skip the dynamic per-query-set measurement")
     p.add_argument("--no-graph", action="store_true", help="run the steps eagerly instead of as CUDA graphs")
     return p.parse_args()
 
@@ -522,10 +523,114 @@ def run_gpu(args, w, rank: int, world: int, dist):
         "gpu_launches": args.steps * (2 + 2 * S),
         "clocks": clk.summary(),
     }
+    if not args.no_dynamic:
+        del logits, mask, e2e_mask, dlogs
+        torch.cuda.empty_cache()
+        line["dynamic_sets"] = run_dynamic(dev, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds / 5, 5, 1)
         line["cpu_paper_algorithm"] = cpu_paper_algorithm(w)
     print(json.dumps(line))
+
+
+def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
+    """The dynamic per-query-set workload, end to end with logits resident:
+    256 requests, each with its own set of K ~ U[300, 2000] names from a
+    50,000-name pool; per step the 256 tries are built on the host as one
+    forest, compiled on the GPU (sparse lists; the dense forest mask is timed
+    separately) and decoded for 32 steps (apply + advance, greedy tokens
+    replayed)."""
+    import torch
+    from paper_2608_12574_gb300 import triemask as T
+    from paper_2608_12574_gb300 import workloads as W
+    w = W.config(5)
+    B, V = w.batch, w.V
+    out = {"workload": w.name, "requests": B, "V": V, "decode_steps": steps}
+    t0 = time.perf_counter()
+    h = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+    out["host_forest_build_ms"] = (time.perf_counter() - t0) * 1e3
+    N = h.num_nodes
+    out["N_nodes"] = N
+    roots = torch.as_tensor(h.roots(), device=dev)
+    with torch.cuda.stream(stream):
+        logits = [W.logits(w, t, device=str(dev)) for t in range(steps)]
+        T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
+        states = roots.clone()
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+        forced = torch.zeros((steps, B), dtype=torch.int32, device=dev)
+        for t in range(steps):
+            x = logits[t].clone()
+            T.trie_apply_lists(h, x, states, stream)
+            forced[t].copy_(torch.argmax(x, dim=1))
+            T.trie_advance(h, states, forced[t], err, stream)
+        del x
+    stream.synchronize()
+    out["dead_moves"] = int(err.item())
+    out["finished"] = int((states == T.TRIE_STATE_FINISHED).sum().item())
+
+    def decode():
+        states.copy_(roots)
+        for t in range(steps):
+            T.trie_apply_lists(h, logits[t], states, stream)
+            T.trie_advance(h, states, forced[t], err, stream)
+
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        decode()
+        with torch.cuda.graph(g, stream=stream):
+            decode()
+        g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    out["decode_ms"] = e0.elapsed_time(e1) / reps
+    lt = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            n_valid = T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
+        lt.append(time.perf_counter() - t0)
+    out["lists_compile_ms"] = min(lt) * 1e3
+    out["list_entries"] = n_valid
+    out["list_bytes"] = n_valid * 4 + (N + 1) * 8
+    # end to end per batch of requests: host forest build + list compile + decode
+    et = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        hh = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+        with torch.cuda.stream(stream):
+            T.trie_compile_lists(hh, w.vocab_bytes, w.vocab_offsets, V, stream)
+            st = torch.as_tensor(hh.roots(), device=dev)
+            for t in range(steps):
+                T.trie_apply_lists(hh, logits[t], st, stream)
+                T.trie_advance(hh, st, forced[t], err, stream)
+        stream.synchronize()
+        et.append(time.perf_counter() - t0)
+        hh.destroy()
+    out["end_to_end_ms"] = min(et) * 1e3
+    # the dense form of the same forest: a [N, ceil(V/32)] mask
+    dense_bytes = N * T.mask_words(V) * 4
+    free, _ = torch.cuda.mem_get_info(dev)
+    if dense_bytes < free * 0.8:
+        mask = T.alloc_mask(h, V, dev)
+        with torch.cuda.stream(stream):
+            T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+            e0.record(stream)
+            T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+            e1.record(stream)
+        stream.synchronize()
+        ms = e0.elapsed_time(e1)
+        out["dense_compile_ms"] = ms
+        out["dense_mask_bytes"] = dense_bytes
+        out["dense_compile_gbs"] = dense_bytes / (ms * 1e-3) / 1e9
+        del mask
+    del logits
+    torch.cuda.empty_cache()
+    h.destroy()
+    return out
 
 
 def reduce_max(x: float, dist, device) -> float:

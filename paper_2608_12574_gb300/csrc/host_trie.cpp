@@ -149,60 +149,71 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
                          int32_t M, HostTrie *out) {
     std::vector<HostTrie> parts(static_cast<size_t>(M));
     std::vector<std::string> errs(static_cast<size_t>(M));
-    std::atomic<int32_t> next(0);
     unsigned hw = std::max(1u, std::thread::hardware_concurrency());
     unsigned nth = std::min<unsigned>(hw, unsigned(M));
-    auto work = [&]() {
+    // phase 1: every set's trie on its own, in parallel
+    std::atomic<int32_t> next(0);
+    auto build = [&]() {
         for (;;) {
             int32_t i = next.fetch_add(1);
             if (i >= M) return;
-            errs[size_t(i)] = build_trie(bytes, offsets, set_offsets[i], set_offsets[i + 1],
-                                         &parts[size_t(i)]);
+            errs[size_t(i)] = build_trie(bytes, offsets, set_offsets[i], set_offsets[i + 1], &parts[size_t(i)]);
         }
     };
     std::vector<std::thread> th;
-    for (unsigned t = 1; t < nth; t++) th.emplace_back(work);
-    work();
+    for (unsigned t = 1; t < nth; t++) th.emplace_back(build);
+    build();
     for (auto &t : th) t.join();
-    int64_t total = 0;
+    th.clear();
+    int64_t total = 0, n_chars = 0;
+    int32_t max_depth = 0;
+    std::vector<int32_t> base(static_cast<size_t>(M));
     for (int32_t i = 0; i < M; i++) {
         if (!errs[size_t(i)].empty()) return "set " + std::to_string(i) + ": " + errs[size_t(i)];
+        base[size_t(i)] = int32_t(std::min<int64_t>(total, INT32_MAX));
         total += parts[size_t(i)].n;
+        n_chars += parts[size_t(i)].n_chars;
+        max_depth = std::max(max_depth, parts[size_t(i)].max_depth);
     }
     if (total > int64_t(INT32_MAX) - 2) return "forest would exceed 2^31-1 nodes";
-    const int32_t n = int32_t(total);
-    out->n = n;
-    out->parent.resize(size_t(n));
-    out->label.resize(size_t(n));
-    out->terminal.resize(size_t(n));
-    out->first_child.resize(size_t(n));
-    out->child_bits.resize(size_t(n) * 8);
-    out->window.resize(size_t(n) * 2);
-    out->depth8.resize(size_t(n));
-    out->jump.resize(size_t(n) * 4);
-    out->roots.resize(size_t(M));
-    out->n_chars = 0;
-    out->max_depth = 0;
-    int32_t base = 0;
-    for (int32_t i = 0; i < M; i++) {
-        const HostTrie &p = parts[size_t(i)];
-        out->roots[size_t(i)] = base;
-        for (int32_t j = 0; j < p.n; j++) {
-            size_t g = size_t(base) + size_t(j);
-            out->parent[g] = p.parent[size_t(j)] < 0 ? -1 : p.parent[size_t(j)] + base;
-            out->first_child[g] = p.first_child[size_t(j)] < 0 ? -1 : p.first_child[size_t(j)] + base;
-            out->label[g] = p.label[size_t(j)];
-            out->terminal[g] = p.terminal[size_t(j)];
+    const size_t n = size_t(total);
+    // phase 2: concatenate, each worker copying (and first touching) its sets
+    out->n = int32_t(n);
+    out->parent.resize(n);
+    out->label.resize(n);
+    out->terminal.resize(n);
+    out->first_child.resize(n);
+    out->child_bits.resize(n * 8);
+    out->window.resize(n * 2);
+    out->depth8.resize(n);
+    out->jump.resize(n * 4);
+    out->roots.assign(base.begin(), base.end());
+    next = 0;
+    auto concat = [&]() {
+        for (;;) {
+            int32_t i = next.fetch_add(1);
+            if (i >= M) return;
+            HostTrie &p = parts[size_t(i)];
+            const int32_t b = base[size_t(i)];
+            const size_t g = size_t(b), pn = size_t(p.n);
+            for (size_t j = 0; j < pn; j++) {
+                out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
+                out->first_child[g + j] = p.first_child[j] < 0 ? -1 : p.first_child[j] + b;
+            }
+            for (size_t j = 0; j < 4 * pn; j++) out->jump[4 * g + j] = p.jump[j] < 0 ? -1 : p.jump[j] + b;
+            memcpy(&out->label[g], p.label.data(), pn);
+            memcpy(&out->terminal[g], p.terminal.data(), pn);
+            memcpy(&out->child_bits[8 * g], p.child_bits.data(), sizeof(uint32_t) * 8 * pn);
+            memcpy(&out->window[2 * g], p.window.data(), sizeof(uint64_t) * 2 * pn);
+            memcpy(&out->depth8[g], p.depth8.data(), pn);
+            p = HostTrie();  // release the part's memory early
         }
-        memcpy(&out->child_bits[size_t(base) * 8], p.child_bits.data(), sizeof(uint32_t) * 8 * size_t(p.n));
-        memcpy(&out->window[size_t(base) * 2], p.window.data(), sizeof(uint64_t) * 2 * size_t(p.n));
-        memcpy(&out->depth8[size_t(base)], p.depth8.data(), size_t(p.n));
-        for (size_t j = 0; j < 4 * size_t(p.n); j++)
-            out->jump[4 * size_t(base) + j] = p.jump[j] < 0 ? -1 : p.jump[j] + base;
-        out->n_chars += p.n_chars;
-        out->max_depth = std::max(out->max_depth, p.max_depth);
-        base += p.n;
-    }
+    };
+    for (unsigned t = 1; t < nth; t++) th.emplace_back(concat);
+    concat();
+    for (auto &t : th) t.join();
+    out->n_chars = n_chars;
+    out->max_depth = max_depth;
     return "";
 }
 

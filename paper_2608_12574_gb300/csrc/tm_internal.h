@@ -8,11 +8,35 @@
 #include <memory>
 #include <mutex>
 #include <string>
+#include <utility>
 #include <vector>
 
 #include <cuda_runtime_api.h>
 
 namespace tmk {
+
+// std::vector allocator whose resize() leaves trivial elements uninitialised
+// (large host arrays are then first touched by the threads that fill them).
+template <class T>
+struct DefaultInitAlloc : std::allocator<T> {
+    template <class U>
+    struct rebind {
+        using other = DefaultInitAlloc<U>;
+    };
+    DefaultInitAlloc() noexcept = default;
+    template <class U>
+    DefaultInitAlloc(const DefaultInitAlloc<U> &) noexcept {}
+    template <class U>
+    void construct(U *p) noexcept {
+        ::new (static_cast<void *>(p)) U;
+    }
+    template <class U, class... Args>
+    void construct(U *p, Args &&...args) {
+        ::new (static_cast<void *>(p)) U(std::forward<Args>(args)...);
+    }
+};
+template <class T>
+using hvec = std::vector<T, DefaultInitAlloc<T>>;
 
 // ----------------------------------------------------------------- host trie
 // Byte trie in breadth-first order, siblings by ascending byte (Sec. 4.1).
@@ -20,17 +44,17 @@ namespace tmk {
 // labels, so the child for byte c is first_child + popcount(bits below c).
 struct HostTrie {
     int32_t n = 0;                       // nodes (all sets of a forest)
-    std::vector<int32_t> parent;         // -1 for a root
-    std::vector<uint8_t> label;          // byte on the incoming edge
-    std::vector<uint8_t> terminal;       // some string ends here
-    std::vector<int32_t> first_child;    // -1 for a leaf
-    std::vector<uint32_t> child_bits;    // [n * 8]
+    hvec<int32_t> parent;                // -1 for a root
+    hvec<uint8_t> label;                 // byte on the incoming edge
+    hvec<uint8_t> terminal;              // some string ends here
+    hvec<int32_t> first_child;           // -1 for a leaf
+    hvec<uint32_t> child_bits;           // [n * 8]
     // Per node, for the mask compile: the labels of the last 16 edges into it
     // (byte i = label i levels up, 0 past the root), min(depth, 255), and the
     // ancestors 1, 2, 4 and 8 levels up (-1 past the root).
-    std::vector<uint64_t> window;        // [n * 2] (low 8 bytes, high 8 bytes)
-    std::vector<uint8_t> depth8;         // [n]
-    std::vector<int32_t> jump;           // [n * 4]
+    hvec<uint64_t> window;               // [n * 2] (low 8 bytes, high 8 bytes)
+    hvec<uint8_t> depth8;                // [n]
+    hvec<int32_t> jump;                  // [n * 4]
     std::vector<int32_t> roots;          // root id of each set
     int64_t n_chars = 0;                 // total bytes of the distinct strings
     int32_t max_depth = 0;
