@@ -168,6 +168,21 @@ int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B
 int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B,
                     int32_t V, cudaStream_t stream);
 
+/* One decode step in one launch: advance the states by the tokens sampled
+ * from the previous logits, then mask the current logits by the new states
+ * (trie_advance followed by trie_apply_mask; Sec. 2 Eq. 1, Sec. 4.2, App. H.3).
+ *   d_states_in   device int32[B], the states before the move (read only)
+ *   d_tokens      device int32[B]
+ *   d_states_out  device int32[B], receives the new states; must not be
+ *                 d_states_in (TRIE_EINVAL)
+ *   d_err         as trie_advance
+ *   d_logits      device [B, V], masked in place by the rows of the new states
+ * Rules, states, dtype and V as trie_advance / trie_apply_mask; needs a prior
+ * trie_compile_masks (TRIE_ESTATE). The transitions recorded by that compile
+ * are looked up first; other moves are walked byte by byte. B = 0 is a no-op. */
+int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
+                       int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream);
+
 /* Sparse form of the masks: for every node the ids of its allowed tokens, as
  * the paper stores them (valid[n] as lists of 4-byte token ids, Sec. 4.2;
  * App. H.5), computed on the GPU without the dense bitmask. At K = 10,000 and

@@ -163,6 +163,9 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     const size_t o_win = L.add(sizeof(uint64_t) * 2 * n);
     const size_t o_d8 = L.add(n);
     const size_t o_jump = L.add(sizeof(int32_t) * 4 * n);
+    size_t trans_slots = 16;  // >= 8 per node, a power of two
+    while (trans_slots < 8 * n) trans_slots <<= 1;
+    const size_t o_trans = L.add(sizeof(ulonglong2) * trans_slots);
     const size_t o_hits = L.add(sizeof(int2) * 8 * n);  // compile scratch (probe -> scatter)
     const size_t o_hcnt = L.add(n);
     void *base = nullptr;
@@ -200,8 +203,23 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     h->dev.window = reinterpret_cast<const ulonglong2 *>(b + o_win);
     h->dev.depth8 = reinterpret_cast<const uint8_t *>(b + o_d8);
     h->dev.jump = reinterpret_cast<const int4 *>(b + o_jump);
+    h->dev.trans = reinterpret_cast<ulonglong2 *>(b + o_trans);
+    h->dev.trans_mask = uint32_t(trans_slots - 1);
     h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
     h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
+    return TRIE_OK;
+}
+
+// The transition table holds the transitions of one vocabulary: when a
+// compile uses another, clear it and let this compile's probe refill it.
+int prepare_trans(trie_t h, const tmk::DevVocab *voc, int sms, cudaStream_t stream, bool *fill) {
+    std::lock_guard<std::mutex> lk(h->mu);
+    *fill = false;
+    if (!h->dev.trans || h->trans_vocab == voc) return TRIE_OK;
+    h->trans_vocab = nullptr;
+    cudaError_t e = tmk::launch_trans_clear(h->dev, sms, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "transition table clear");
+    *fill = true;
     return TRIE_OK;
 }
 
@@ -321,9 +339,12 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     const int32_t n = h->host.n;
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
-    cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, stream);
+    bool fill_trans;
+    if ((rc = prepare_trans(h, voc.get(), sms, stream, &fill_trans)) != TRIE_OK) return rc;
+    cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, fill_trans, stream);
     if (e != cudaSuccess) return fail_cuda(e, "mask compile launch");
     std::lock_guard<std::mutex> lk(h->mu);
+    h->trans_vocab = voc.get();
     h->vocab = voc;
     h->mask = d_mask;
     h->mask_V = V;
@@ -336,17 +357,54 @@ int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B
     if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
     if (B > 0 && (!d_states || !d_tokens)) return fail(TRIE_EINVAL, "d_states / d_tokens is NULL");
     std::shared_ptr<tmk::DevVocab> voc;
+    bool use_trans;
     {
         std::lock_guard<std::mutex> lk(h->mu);
         voc = h->vocab;
+        use_trans = h->trans_vocab == voc.get();
     }
     if (!voc) return fail(TRIE_ESTATE, "trie_advance before trie_compile_masks on this handle");
     if (B == 0) return TRIE_OK;
     int dev, rc;
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
-    cudaError_t e = tmk::launch_advance(h->dev, h->host.n, *voc, d_states, d_tokens, B, d_err, stream);
+    cudaError_t e =
+        tmk::launch_advance(h->dev, h->host.n, *voc, d_states, d_states, d_tokens, B, d_err, use_trans, stream);
     if (e != cudaSuccess) return fail_cuda(e, "advance launch");
+    return TRIE_OK;
+}
+
+int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
+                       int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_states_in || !d_tokens || !d_states_out || !d_logits))
+        return fail(TRIE_EINVAL, "a device pointer is NULL");
+    if (B > 0 && d_states_in == d_states_out)
+        return fail(TRIE_EINVAL, "d_states_in and d_states_out must be different buffers");
+    std::shared_ptr<tmk::DevVocab> voc;
+    uint32_t *mask;
+    int32_t mV;
+    bool use_trans;
+    {
+        std::lock_guard<std::mutex> lk(h->mu);
+        voc = h->vocab;
+        mask = h->mask;
+        mV = h->mask_V;
+        use_trans = h->trans_vocab == voc.get();
+    }
+    if (!mask || !voc) return fail(TRIE_ESTATE, "trie_advance_apply before trie_compile_masks on this handle");
+    if (V != mV || V != voc->V) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
+    if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
+        return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_advance_apply(h->dev, h->host.n, *voc, use_trans, d_states_in, d_tokens,
+                                              d_states_out, d_err, d_logits, dtype, mask, B, num_sms(dev), stream);
+    if (e != cudaSuccess) return fail_cuda(e, "advance-apply launch");
     return TRIE_OK;
 }
 
@@ -411,7 +469,9 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
     int64_t total = 0;
-    cudaError_t e = tmk::launch_lists_count(h->dev, n, *voc, lmax, L, sms, stream, &total);
+    bool fill_trans;
+    if ((rc = prepare_trans(h, voc.get(), sms, stream, &fill_trans)) != TRIE_OK) return rc;
+    cudaError_t e = tmk::launch_lists_count(h->dev, n, *voc, lmax, L, sms, fill_trans, stream, &total);
     if (e != cudaSuccess) return fail_cuda(e, "valid-list count");
     if (total > L.tok_cap) {  // grow the token buffer (by at least half)
         const int64_t cap = std::max<int64_t>(total, L.tok_cap + L.tok_cap / 2);
@@ -432,6 +492,7 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     std::lock_guard<std::mutex> lk(h->mu);
     L.n_valid = total;
     L.V = V;
+    h->trans_vocab = voc.get();
     h->vocab = voc;
     return TRIE_OK;
 }

@@ -138,7 +138,42 @@ struct PatchArgs {
     const ulonglong2 *window;  // probe-scatter form: last 16 labels per node
     const uint8_t *depth8;
     const int4 *jump;          // ancestors 1, 2, 4, 8 levels up
+    ulonglong2 *trans;         // transition table (row, token) -> end node, or null
+    uint32_t trans_mask;       // slots - 1
+    int32_t trans_fill;        // the probe inserts every transition it finds
 };
+
+// Transition table: open addressing over 16-byte slots {key, end node};
+// key = (row << 32 | token) + 1, 0 = empty. For a fixed trie the entries
+// depend only on the vocabulary, so it is cleared and filled (by the probe)
+// only when a compile uses another vocabulary than the one it holds. An entry
+// that finds no slot within kTransProbes is left out (the advance then walks).
+constexpr int kTransProbes = 32;
+
+__device__ __forceinline__ uint64_t trans_key(int32_t row, int32_t t) {
+    return ((uint64_t(uint32_t(row)) << 32) | uint32_t(t)) + 1ull;
+}
+
+__device__ __forceinline__ uint32_t trans_slot(uint64_t key, uint32_t mask) {
+    const uint64_t z = key * 0x9E3779B97F4A7C15ull;
+    return uint32_t(z >> 32) & mask;
+}
+
+__device__ __forceinline__ void trans_insert(ulonglong2 *tab, uint32_t mask, int32_t row, int32_t t,
+                                             int32_t dest) {
+    const uint64_t key = trans_key(row, t);
+    uint32_t s = trans_slot(key, mask);
+    for (int i = 0; i < kTransProbes; i++) {
+        unsigned long long *k = reinterpret_cast<unsigned long long *>(&tab[s].x);
+        const unsigned long long old = atomicCAS(k, 0ull, key);
+        if (old == 0ull || old == key) {
+            tab[s].y = uint64_t(uint32_t(dest));
+            return;
+        }
+        s = (s + 1u) & mask;
+    }
+}
+
 constexpr int kHitSlots = 8;
 constexpr int kHitOverflow = 255;
 
@@ -379,7 +414,7 @@ __global__ void __launch_bounds__(kPatchThreads) k_mask_patch(PatchArgs a) {
 // again by the scatter). It waits for all earlier work at entry, prefetches
 // its tables into L2 (its dependent loads then hit L2 while the fill
 // saturates HBM) and only then lets the fill launch, which runs beside it.
-__global__ void __launch_bounds__(kPatchThreads) k_mask_probe(PatchArgs a, Prefetch pf) {
+__global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Prefetch pf) {
     pdl_wait();  // an earlier scatter may still read the hit buffer
     if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
     pdl_launch_dependents();
@@ -390,26 +425,28 @@ __global__ void __launch_bounds__(kPatchThreads) k_mask_probe(PatchArgs a, Prefe
         node_hits_window(a, m, [&](int32_t row, int32_t t) {
             if (c < kHitSlots) slot[c] = make_int2(row, t);
             c++;
+            if (a.trans_fill && t != a.eos) trans_insert(a.trans, a.trans_mask, row, t, m);
         });
         a.hit_count[m] = uint8_t(c > kHitSlots ? kHitOverflow : c);
     }
 }
 
 // Sets the recorded bits after the fill (which completes after the probe).
-__global__ void __launch_bounds__(kPatchThreads) k_mask_scatter(PatchArgs a) {
+__global__ void __launch_bounds__(kPatchThreads, 4) k_mask_scatter(PatchArgs a) {
     pdl_launch_dependents();
     pdl_wait();  // fill complete, and through it the probe
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        auto emit = [&](int32_t row, int32_t t) { set_mask_bit(a, row, t); };
         const int32_t c = a.hit_count[m];
         if (c == kHitOverflow) {
-            node_hits_window(a, m, [&](int32_t row, int32_t t) { set_mask_bit(a, row, t); });
+            node_hits_window(a, m, emit);
             continue;
         }
         const int2 *slot = a.hits + int64_t(m) * kHitSlots;
         for (int32_t i = 0; i < c; i++) {
             const int2 hv = slot[i];
-            set_mask_bit(a, hv.x, hv.y);
+            emit(hv.x, hv.y);
         }
     }
 }
@@ -418,57 +455,82 @@ __global__ void __launch_bounds__(kPatchThreads) k_mask_scatter(PatchArgs a) {
 
 constexpr int kAdvanceThreads = 128;
 
-__global__ void __launch_bounds__(kAdvanceThreads) k_advance(
-    const int32_t *__restrict__ first_child, const uint32_t *__restrict__ child_bits,
-    const uint8_t *__restrict__ terminal, int32_t n_nodes, const uint32_t *__restrict__ tok_off,
-    const uint16_t *__restrict__ tok_len, const uint8_t *__restrict__ blob, int32_t V,
-    int32_t *__restrict__ states, const int32_t *__restrict__ tokens, int32_t B,
-    int32_t *__restrict__ err) {
+// End node of (row, token) from the transition table; false if absent.
+__device__ __forceinline__ bool trans_lookup(const ulonglong2 *__restrict__ tab, uint32_t mask, int32_t row,
+                                             int32_t t, int32_t *dest) {
+    const uint64_t key = trans_key(row, t);
+    uint32_t s = trans_slot(key, mask);
+    for (int i = 0; i < kTransProbes; i++) {
+        const ulonglong2 e = __ldg(tab + s);
+        if (e.x == key) {
+            *dest = int32_t(uint32_t(e.y));
+            return true;
+        }
+        if (e.x == 0ull) return false;
+        s = (s + 1u) & mask;
+    }
+    return false;
+}
+
+struct AdvanceArgs {
+    const int32_t *first_child;
+    const uint32_t *child_bits;
+    const uint8_t *terminal;
+    int32_t n_nodes;
+    const uint32_t *tok_off;
+    const uint16_t *tok_len;
+    const uint8_t *blob;
+    int32_t V;
+    const ulonglong2 *trans;  // transition table of this vocabulary, or null
+    uint32_t trans_mask;
+};
+
+// delta*(s, bytes(v)) (Sec. 2, Eq. 1) with the FINISHED / DEAD rules.
+__device__ __forceinline__ int32_t advance_one(const AdvanceArgs &a, int32_t s, int32_t v) {
+    const int32_t eos = a.V - 1;
+    if (s == kDead) return kDead;
+    if (v < 0 || v >= a.V) return kDead;
+    if (s == kFinished) return (v == eos) ? kFinished : kDead;
+    if (s < 0 || s >= a.n_nodes) return kDead;
+    if (v == eos) return a.terminal[s] ? kFinished : kDead;
+    int32_t nxt;
+    if (a.trans && trans_lookup(a.trans, a.trans_mask, s, v, &nxt)) return nxt;  // recorded by the compile
+    const int32_t L = a.tok_len[v];
+    if (L <= 0) return kDead;
+    const uint8_t *p = a.blob + a.tok_off[v];
+    int32_t x = s;
+    for (int32_t j = 0; j < L; j++) {
+        const uint32_t c = p[j];
+        const uint4 *cb = reinterpret_cast<const uint4 *>(a.child_bits + int64_t(x) * 8);
+        const uint4 lo = cb[0], hi = cb[1];
+        const int32_t fc = a.first_child[x];
+        const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+        const uint32_t wi = c >> 5, bit = c & 31u;
+        uint32_t below = 0, cur = 0;
+#pragma unroll
+        for (uint32_t i = 0; i < 8; i++) {
+            below += (i < wi) ? __popc(w[i]) : 0u;
+            cur = (i == wi) ? w[i] : cur;
+        }
+        if (!((cur >> bit) & 1u)) return kDead;
+        x = fc + int32_t(below + __popc(cur & ((1u << bit) - 1u)));
+    }
+    return x;
+}
+
+// states_out[b] = delta*(states_in[b], tokens[b]); states_out may equal
+// states_in (in place). Every move into DEAD from a non-DEAD state counts.
+__global__ void __launch_bounds__(kAdvanceThreads) k_advance(AdvanceArgs a, const int32_t *states_in,
+                                                             int32_t *states_out, const int32_t *__restrict__ tokens,
+                                                             int32_t B, int32_t *__restrict__ err) {
     pdl_launch_dependents();
     pdl_wait();  // states / tokens come from earlier kernels
     const int32_t b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b >= B) return;
-    const int32_t s = states[b];
-    if (s == kDead) return;
-    const int32_t v = tokens[b];
-    const int32_t eos = V - 1;
-    int32_t nxt;
-    if (v < 0 || v >= V) {
-        nxt = kDead;
-    } else if (s == kFinished) {
-        nxt = (v == eos) ? kFinished : kDead;
-    } else if (s < 0 || s >= n_nodes) {
-        nxt = kDead;
-    } else if (v == eos) {
-        nxt = terminal[s] ? kFinished : kDead;
-    } else {
-        const int32_t L = tok_len[v];
-        const uint8_t *p = blob + tok_off[v];
-        int32_t x = s;
-        nxt = L > 0 ? s : kDead;
-        for (int32_t j = 0; j < L; j++) {
-            const uint32_t c = p[j];
-            const uint4 *cb = reinterpret_cast<const uint4 *>(child_bits + int64_t(x) * 8);
-            const uint4 lo = cb[0], hi = cb[1];
-            const int32_t fc = first_child[x];
-            const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
-            const uint32_t wi = c >> 5, bit = c & 31u;
-            uint32_t below = 0, cur = 0;
-#pragma unroll
-            for (uint32_t i = 0; i < 8; i++) {
-                below += (i < wi) ? __popc(w[i]) : 0u;
-                cur = (i == wi) ? w[i] : cur;
-            }
-            if (!((cur >> bit) & 1u)) {
-                nxt = kDead;
-                break;
-            }
-            x = fc + int32_t(below + __popc(cur & ((1u << bit) - 1u)));
-            nxt = x;
-        }
-    }
-    if (nxt == kDead && err) atomicAdd(err, 1);
-    states[b] = nxt;
+    const int32_t s = states_in[b];
+    const int32_t nxt = advance_one(a, s, tokens[b]);
+    if (nxt == kDead && s != kDead && err) atomicAdd(err, 1);
+    states_out[b] = nxt;
 }
 
 // ------------------------------------------------------------------ apply
@@ -572,6 +634,44 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
     const int32_t b = item / segs, seg = item - b * segs;
     const uint32_t word = row_word(mask, __ldg(states + b), n_nodes, W, int64_t(seg) * 32 + lane, V - 1);
     const int64_t row_chunks = int64_t(V) / (16 / kElt);
+    write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
+                        tile);
+}
+
+// Advance, then apply, in one launch (one decode step once the sampler has
+// picked tokens[b] for the previous logits): states_out[b] = delta*(states_in[b],
+// tokens[b]), and logits[b] (the next step's) are masked by the row of
+// states_out[b]. Lane 0 of every warp of row b computes the new state; the
+// warp of segment 0 stores it and counts a move into DEAD.
+template <int kElt>
+__global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs aa, uint4 *__restrict__ logits,
+                                                                     const uint32_t *__restrict__ mask,
+                                                                     const int32_t *__restrict__ states_in,
+                                                                     const int32_t *__restrict__ tokens,
+                                                                     int32_t *__restrict__ states_out,
+                                                                     int32_t *__restrict__ err, int32_t B,
+                                                                     int64_t W, int32_t segs) {
+    constexpr int kSegChunks = 1024 / (16 / kElt);
+    __shared__ __align__(128) uint4 tile[kSegChunks];
+    init_ninf_tile<kElt>(tile);
+    pdl_launch_dependents();
+    pdl_wait();  // logits, states and tokens come from earlier kernels
+    const int lane = threadIdx.x & 31;
+    const int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
+    if (item >= B * segs) return;  // uniform per warp
+    const int32_t b = item / segs, seg = item - b * segs;
+    int32_t s = 0, nxt = 0;
+    if (lane == 0) {
+        s = __ldg(states_in + b);
+        nxt = advance_one(aa, s, __ldg(tokens + b));
+    }
+    nxt = __shfl_sync(0xffffffffu, nxt, 0);
+    if (seg == 0 && lane == 0) {
+        states_out[b] = nxt;
+        if (nxt == kDead && s != kDead && err) atomicAdd(err, 1);
+    }
+    const uint32_t word = row_word(mask, nxt, aa.n_nodes, W, int64_t(seg) * 32 + lane, aa.V - 1);
+    const int64_t row_chunks = int64_t(aa.V) / (16 / kElt);
     write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
                         tile);
 }
@@ -687,14 +787,14 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__res
 }
 
 // Writes every hit into its row (positions claimed with a per-row cursor).
-__global__ void __launch_bounds__(kPatchThreads) k_list_scatter(PatchArgs a, const int64_t *__restrict__ off,
+__global__ void __launch_bounds__(kPatchThreads, 4) k_list_scatter(PatchArgs a, const int64_t *__restrict__ off,
                                                                 int32_t *__restrict__ cursor,
                                                                 int32_t *__restrict__ toks) {
     pdl_launch_dependents();
     pdl_wait();
     const int32_t stride = gridDim.x * blockDim.x;
-    auto put = [&](int32_t row, int32_t t) { toks[off[row] + atomicAdd(cursor + row, 1)] = t; };
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
+        auto put = [&](int32_t row, int32_t t) { toks[off[row] + atomicAdd(cursor + row, 1)] = t; };
         const int32_t c = a.hit_count[m];
         if (c == kHitOverflow) {
             node_hits_window(a, m, put);
@@ -801,6 +901,9 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.window = t.window;
     a.depth8 = t.depth8;
     a.jump = t.jump;
+    a.trans = t.trans;
+    a.trans_mask = t.trans_mask;
+    a.trans_fill = 0;
     return a;
 }
 
@@ -830,9 +933,14 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
     return launch_pdl(k_mask_patch, grid, kPatchThreads, st, a);
 }
 
+cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st) {
+    return launch_mask_fill(reinterpret_cast<uint32_t *>(t.trans), 4 * (int64_t(t.trans_mask) + 1), num_sms, st);
+}
+
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                                 uint32_t *mask, int64_t W, int num_sms, cudaStream_t st) {
+                                 uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
+    a.trans_fill = fill_trans && t.trans;
     // probe grid: every CTA resident at once (so that all of them pass their
     // entry wait and let the fill launch right away), nodes in a grid-stride loop
     const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
@@ -866,11 +974,51 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
     return launch_pdl(k_mask_scatter, scatter_grid, kPatchThreads, st, a);
 }
 
-cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t *states,
-                           const int32_t *tokens, int32_t B, int32_t *err, cudaStream_t st) {
+AdvanceArgs advance_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans) {
+    AdvanceArgs a;
+    a.first_child = t.first_child;
+    a.child_bits = t.child_bits;
+    a.terminal = t.terminal;
+    a.n_nodes = n_nodes;
+    a.tok_off = v.tok_off;
+    a.tok_len = v.tok_len;
+    a.blob = v.blob;
+    a.V = v.V;
+    a.trans = use_trans ? t.trans : nullptr;
+    a.trans_mask = t.trans_mask;
+    return a;
+}
+
+cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, const int32_t *states_in,
+                           int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err, bool use_trans,
+                           cudaStream_t st) {
     const int grid = (B + kAdvanceThreads - 1) / kAdvanceThreads;
-    return launch_pdl(k_advance, grid, kAdvanceThreads, st, t.first_child, t.child_bits, t.terminal, n_nodes,
-                      v.tok_off, v.tok_len, v.blob, v.V, states, tokens, B, err);
+    return launch_pdl(k_advance, grid, kAdvanceThreads, st, advance_args(t, n_nodes, v, use_trans), states_in,
+                      states_out, tokens, B, err);
+}
+
+cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
+                                 const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
+                                 int32_t *err, void *logits, int dtype, const uint32_t *mask, int32_t B,
+                                 int num_sms, cudaStream_t st) {
+    const int32_t V = v.V;
+    const int64_t W = (int64_t(V) + 31) / 32;
+    const int elt = dtype == 0 ? 4 : 2;
+    const int32_t segs = int32_t((W + 31) / 32);
+    const bool vec = (reinterpret_cast<uintptr_t>(logits) & 15u) == 0 && (int64_t(V) * elt) % 16 == 0 &&
+                     int64_t(B) * segs < int64_t(INT32_MAX);
+    if (!vec) {  // any V and alignment: the two kernels one after the other
+        cudaError_t e = launch_advance(t, n_nodes, v, states_in, states_out, tokens, B, err, use_trans, st);
+        if (e != cudaSuccess) return e;
+        return launch_apply(logits, dtype, mask, states_out, B, V, n_nodes, num_sms, st);
+    }
+    const AdvanceArgs aa = advance_args(t, n_nodes, v, use_trans);
+    const int grid = grid_for(int64_t(B) * segs, kApplyThreads / 32, INT32_MAX);
+    if (elt == 2)
+        return launch_pdl(k_advance_apply_vec<2>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
+                          states_in, tokens, states_out, err, B, W, segs);
+    return launch_pdl(k_advance_apply_vec<4>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
+                      states_in, tokens, states_out, err, B, W, segs);
 }
 
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
@@ -896,8 +1044,9 @@ cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const in
 }
 
 cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                               const DevLists &L, int num_sms, cudaStream_t st, int64_t *h_total) {
+                               const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
+    a.trans_fill = fill_trans && t.trans;
     Prefetch pf;
     pf.count = 0;
     const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
@@ -907,6 +1056,7 @@ cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab
     if ((e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), 2 * int64_t(n_nodes), num_sms, st)) !=
         cudaSuccess)
         return e;
+
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
     if ((e = launch_pdl(k_list_count, grid, kPatchThreads, st, a, L.count)) != cudaSuccess) return e;
     const int32_t n_tiles = int32_t((int64_t(n_nodes) + kScanTile - 1) / kScanTile);

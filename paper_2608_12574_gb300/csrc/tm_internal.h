@@ -131,6 +131,8 @@ struct DevTrie {
     const ulonglong2 *window = nullptr;
     const uint8_t *depth8 = nullptr;
     const int4 *jump = nullptr;
+    ulonglong2 *trans = nullptr;     // transition table {(row << 32 | token) + 1, end node}
+    uint32_t trans_mask = 0;         // slots - 1
     int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) per node
     uint8_t *hit_count = nullptr;    // compile scratch: hits found per node
 };
@@ -160,6 +162,7 @@ struct trie_s {
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
     int32_t mask_V = 0;
     tmk::DevLists lists;                 // last compiled valid lists (library-owned)
+    const tmk::DevVocab *trans_vocab = nullptr;  // vocabulary the transition table holds
 };
 
 namespace tmk {
@@ -174,15 +177,23 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
 // Probe, fill and scatter: the mask compile with the per-node searches running
 // beside the fill (needs t.hits / t.hit_count).
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                                 uint32_t *mask, int64_t W, int num_sms, cudaStream_t st);
-cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t *states,
-                           const int32_t *tokens, int32_t B, int32_t *err, cudaStream_t st);
+                                 uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st);
+// Zeroes the transition table (before it is filled for another vocabulary).
+cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st);
+cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, const int32_t *states_in,
+                           int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err, bool use_trans,
+                           cudaStream_t st);
+// Advance, then mask the next logits by the new states, in one launch.
+cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
+                                 const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
+                                 int32_t *err, void *logits, int dtype, const uint32_t *mask, int32_t B,
+                                 int num_sms, cudaStream_t st);
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
                          int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st);
 // Valid lists: probe, per-row counts and their scan; ends by reading the
 // total into *h_total (host-synchronous). Then the scatter into L.toks.
 cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                               const DevLists &L, int num_sms, cudaStream_t st, int64_t *h_total);
+                               const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total);
 cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  const DevLists &L, int num_sms, cudaStream_t st);
 cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,

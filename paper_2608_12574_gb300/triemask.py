@@ -40,6 +40,7 @@ SIGNATURES = {
     "trie_copy_lists": (ctypes.c_int, [_P, _P, _P, _P]),
     "trie_apply_lists": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
     "trie_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "trie_advance_apply": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, ctypes.c_int, _I32, _I32, _P]),
     "trie_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
     "trie_destroy": (ctypes.c_int, [_P]),
     "trie_last_error": (ctypes.c_char_p, []),
@@ -235,6 +236,26 @@ def trie_advance(h: Trie, d_states, d_tokens, d_err=None, stream=None) -> None:
     pt = _dev(d_tokens, (torch.int32,), "d_tokens")
     pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
     _check(h._lib.trie_advance(h.handle, ps, pt, B, pe, _stream(stream, d_states.device)))
+
+
+def trie_advance_apply(h: Trie, d_states_in, d_tokens, d_states_out, d_logits, d_err=None, stream=None) -> None:
+    """states_out <- delta*(states_in, tokens); then mask d_logits ([B, V]) by states_out."""
+    import torch
+    if d_logits.dim() != 2:
+        raise ValueError("d_logits must be [B, V]")
+    B, V = d_logits.shape
+    for t, name in ((d_states_in, "d_states_in"), (d_tokens, "d_tokens"), (d_states_out, "d_states_out")):
+        if t.numel() != B:
+            raise ValueError(f"{name} must have B entries")
+    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
+    if dtype is None:
+        raise TypeError("d_logits must be float32 or bfloat16")
+    pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
+    _check(h._lib.trie_advance_apply(h.handle, _dev(d_states_in, (torch.int32,), "d_states_in"),
+                                     _dev(d_tokens, (torch.int32,), "d_tokens"),
+                                     _dev(d_states_out, (torch.int32,), "d_states_out"), pe,
+                                     _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits"), dtype, B, V,
+                                     _stream(stream, d_logits.device)))
 
 
 def trie_apply_mask(h: Trie, d_logits, d_states, stream=None) -> None:
