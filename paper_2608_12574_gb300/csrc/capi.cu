@@ -127,6 +127,7 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
     dv->tok_len = reinterpret_cast<const uint16_t *>(base + o_len);
     dv->blob = reinterpret_cast<const uint8_t *>(base + o_blob);
     dv->blob_bytes = hv.blob.size();
+    dv->dup_keys = hv.dup_keys;
     dv->ht_key = reinterpret_cast<const uint64_t *>(base + o_key);
     dv->ht_val = reinterpret_cast<const int32_t *>(base + o_val);
     try {
@@ -162,7 +163,7 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     const size_t o_bits = L.add(sizeof(uint32_t) * 8 * n);
     const size_t o_win = L.add(sizeof(uint64_t) * 2 * n);
     const size_t o_d8 = L.add(n);
-    const size_t o_jump = L.add(sizeof(int32_t) * 4 * n);
+    const size_t o_anc = L.add(sizeof(int32_t) * 16 * n);
     size_t trans_slots = 16;  // >= 8 per node, a power of two
     while (trans_slots < 8 * n) trans_slots <<= 1;
     const size_t o_trans = L.add(sizeof(ulonglong2) * trans_slots);
@@ -183,7 +184,7 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
         {o_bits, t.child_bits.data(), sizeof(uint32_t) * 8 * n},
         {o_win, t.window.data(), sizeof(uint64_t) * 2 * n},
         {o_d8, t.depth8.data(), n},
-        {o_jump, t.jump.data(), sizeof(int32_t) * 4 * n},
+        {o_anc, t.anc.data(), sizeof(int32_t) * 16 * n},
     };
     for (const Up &u : ups) {
         e = cudaMemcpyAsync(b + u.off, u.src, u.n, cudaMemcpyHostToDevice, stream);
@@ -202,7 +203,7 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     h->dev.child_bits = reinterpret_cast<const uint32_t *>(b + o_bits);
     h->dev.window = reinterpret_cast<const ulonglong2 *>(b + o_win);
     h->dev.depth8 = reinterpret_cast<const uint8_t *>(b + o_d8);
-    h->dev.jump = reinterpret_cast<const int4 *>(b + o_jump);
+    h->dev.anc = reinterpret_cast<const int4 *>(b + o_anc);
     h->dev.trans = reinterpret_cast<ulonglong2 *>(b + o_trans);
     h->dev.trans_mask = uint32_t(trans_slots - 1);
     h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);

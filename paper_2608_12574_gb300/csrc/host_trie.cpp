@@ -42,13 +42,13 @@ inline int cmp_str(const Str &a, const Str &b) {
 
 }  // namespace
 
-// Label windows, clipped depths and ancestor jumps, in BFS order (a parent
-// always precedes its children).
+// Label windows, clipped depths and the 16 nearest ancestors, in BFS order
+// (a parent always precedes its children).
 void add_compile_tables(HostTrie *t) {
     const size_t n = size_t(t->n);
     t->window.assign(2 * n, 0ull);
     t->depth8.assign(n, 0);
-    t->jump.assign(4 * n, -1);
+    t->anc.assign(16 * n, -1);
     for (size_t i = 0; i < n; i++) {
         const int32_t p = t->parent[i];
         if (p < 0) continue;
@@ -56,9 +56,10 @@ void add_compile_tables(HostTrie *t) {
         t->window[2 * i] = (lo << 8) | t->label[i];
         t->window[2 * i + 1] = (hi << 8) | (lo >> 56);
         t->depth8[i] = uint8_t(t->depth8[size_t(p)] == 255 ? 255 : t->depth8[size_t(p)] + 1);
-        int32_t *j = &t->jump[4 * i];
-        j[0] = p;
-        for (int q = 1; q < 4; q++) j[q] = j[q - 1] < 0 ? -1 : t->jump[4 * size_t(j[q - 1]) + q - 1];
+        int32_t *a = &t->anc[16 * i];
+        const int32_t *ap = &t->anc[16 * size_t(p)];
+        a[0] = p;
+        for (int q = 1; q < 16; q++) a[q] = ap[q - 1];
     }
 }
 
@@ -186,7 +187,7 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
     out->child_bits.resize(n * 8);
     out->window.resize(n * 2);
     out->depth8.resize(n);
-    out->jump.resize(n * 4);
+    out->anc.resize(n * 16);
     out->roots.assign(base.begin(), base.end());
     next = 0;
     auto concat = [&]() {
@@ -200,7 +201,7 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
                 out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
                 out->first_child[g + j] = p.first_child[j] < 0 ? -1 : p.first_child[j] + b;
             }
-            for (size_t j = 0; j < 4 * pn; j++) out->jump[4 * g + j] = p.jump[j] < 0 ? -1 : p.jump[j] + b;
+            for (size_t j = 0; j < 16 * pn; j++) out->anc[16 * g + j] = p.anc[j] < 0 ? -1 : p.anc[j] + b;
             memcpy(&out->label[g], p.label.data(), pn);
             memcpy(&out->terminal[g], p.terminal.data(), pn);
             memcpy(&out->child_bits[8 * g], p.child_bits.data(), sizeof(uint32_t) * 8 * pn);
@@ -264,6 +265,8 @@ std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, 
         uint64_t pair = (key >> 1) & pairs_mask;
         for (;;) {
             size_t s0 = size_t(2 * pair);
+            // an equal key: a repeated token string, or two strings whose hashes collide
+            if (out->ht_key[s0] == key || out->ht_key[s0 + 1] == key) out->dup_keys = 1;
             if (!out->ht_key[s0]) { out->ht_key[s0] = key; out->ht_val[s0] = v; break; }
             if (!out->ht_key[s0 + 1]) { out->ht_key[s0 + 1] = key; out->ht_val[s0 + 1] = v; break; }
             pair = (pair + 1) & pairs_mask;

@@ -137,7 +137,8 @@ struct PatchArgs {
     uint8_t *hit_count;  // [n_nodes]
     const ulonglong2 *window;  // probe-scatter form: last 16 labels per node
     const uint8_t *depth8;
-    const int4 *jump;          // ancestors 1, 2, 4, 8 levels up
+    const int4 *anc;           // [n * 4]: ancestors 1..16 levels up
+    int32_t dup_keys;          // two tokens share a hash key
     ulonglong2 *trans;         // transition table (row, token) -> end node, or null
     uint32_t trans_mask;       // slots - 1
     int32_t trans_fill;        // the probe inserts every transition it finds
@@ -317,29 +318,32 @@ __device__ __forceinline__ void node_hits(const PatchArgs &a, int32_t m, Emit em
     }
 }
 
-// Ancestor of m k levels up (k <= 2 * 15): at most one hop per set bit of k.
-__device__ __forceinline__ int32_t ancestor(const PatchArgs &a, int32_t m, int32_t k) {
-    int32_t y = m;
-    while (k >= 8 && y >= 0) {
-        y = __ldg(a.jump + y).w;
-        k -= 8;
-    }
-    if ((k & 4) && y >= 0) y = __ldg(a.jump + y).z;
-    if ((k & 2) && y >= 0) y = __ldg(a.jump + y).y;
-    if ((k & 1) && y >= 0) y = __ldg(a.jump + y).x;
-    return y;
+// Element k of a register copy of 16 ancestors, without dynamic indexing.
+__device__ __forceinline__ int32_t anc_at(const int4 (&an)[4], int k) {
+    const int4 q = k < 4 ? an[0] : (k < 8 ? an[1] : (k < 12 ? an[2] : an[3]));
+    const int r = k & 3;
+    return r == 0 ? q.x : (r == 1 ? q.y : (r == 2 ? q.z : q.w));
 }
 
-// node_hits from the precomputed label window and ancestor jumps: one load
-// gives every suffix of length <= 16, and a hit's row costs <= 4 hops.
+// node_hits from the precomputed label window and ancestor table: one round
+// of loads gives every suffix of length <= 16 and every start row. The 8
+// suffixes of a batch are resolved as a wavefront: the first slot pair of all
+// 8 keys, then the token ids of the matches, their lengths and offsets, then
+// their bytes, each round issued for all candidates before any is used. A key
+// that may sit in a later pair (its first pair is full and does not hold it,
+// or some tokens share keys) takes the sequential probe.
 template <typename Emit>
 __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, Emit emit) {
     const ulonglong2 win = __ldg(a.window + m);
+    int4 an[4];
+#pragma unroll
+    for (int q = 0; q < 4; q++) an[q] = __ldg(a.anc + int64_t(m) * 4 + q);
     const int32_t d8 = __ldg(a.depth8 + m);
     const int32_t lim = a.lmax < kMaxClimb ? a.lmax : kMaxClimb;
     const int32_t depth = d8 < lim ? d8 : lim;
     const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y), uint32_t(win.y >> 32)};
     if (__ldg(a.terminal + m)) emit(m, a.eos);
+    const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
     uint64_t h = 0, pw = 1;
 #pragma unroll
     for (int k0 = 0; k0 < kMaxClimb; k0 += 8) {
@@ -348,33 +352,63 @@ __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, 
             ulonglong2 first[8];
 #pragma unroll
             for (int i = 0; i < 8; i++) {
-                const int k = k0 + i;
                 key[i] = 0ull;
                 first[i] = make_ulonglong2(0ull, 0ull);
-                if (k < depth) {
-                    h += (uint64_t(byte_at(lab, k)) + 1ull) * pw;
+                if (k0 + i < depth) {
+                    h += (uint64_t(byte_at(lab, k0 + i)) + 1ull) * pw;
                     pw *= kHashBase;
-                    key[i] = hash_finish(h, uint32_t(k + 1));
-                    first[i] = __ldg(reinterpret_cast<const ulonglong2 *>(a.ht_key) +
-                                     (uint32_t(key[i] >> 1) & a.pairs_mask));
+                    key[i] = hash_finish(h, uint32_t(k0 + i + 1));
+                    first[i] = __ldg(pairs + (uint32_t(key[i] >> 1) & a.pairs_mask));
                 }
             }
+            int32_t slot[8];  // slot of the key in its first pair, -1 none
+            uint32_t slow = 0;  // bit i: candidate i needs the sequential probe
 #pragma unroll
             for (int i = 0; i < 8; i++) {
-                const int k = k0 + i;
-                if (k < depth && (first[i].x == key[i] || first[i].y == key[i] || first[i].y != 0ull)) {
-                    int32_t row = -1;  // looked up on the first hit only
-                    probe(a, key[i], k + 1, &lab, m, [&](int32_t t) {
-                        if (row < 0) row = ancestor(a, m, k + 1);
-                        emit(row, t);
-                    });
+                const bool m0 = first[i].x == key[i], m1 = first[i].y == key[i];
+                const uint32_t pr = uint32_t(key[i] >> 1) & a.pairs_mask;
+                slot[i] = (k0 + i < depth && (m0 || m1)) ? int32_t(2 * pr + (m0 ? 0 : 1)) : -1;
+                if (k0 + i < depth && first[i].y != 0ull && (!(m0 || m1) || a.dup_keys)) {
+                    slow |= 1u << i;
+                    slot[i] = -1;
+                }
+            }
+            int32_t tid[8];
+#pragma unroll
+            for (int i = 0; i < 8; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
+            int32_t tlen[8];
+            uint32_t toff[8];
+#pragma unroll
+            for (int i = 0; i < 8; i++) {
+                tlen[i] = tid[i] >= 0 ? int32_t(__ldg(a.tok_len + tid[i])) : -1;
+                toff[i] = tid[i] >= 0 ? __ldg(a.tok_off + tid[i]) : 0u;
+            }
+            // token bytes: 16-byte aligned in the blob, which has 16 bytes of tail room
+            uint4 tb[8];
+#pragma unroll
+            for (int i = 0; i < 8; i++)
+                tb[i] = tlen[i] == k0 + i + 1 ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]))
+                                              : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int i = 0; i < 8; i++) {
+                const int k = k0 + i + 1;  // suffix length
+                if (slow & (1u << i)) {
+                    probe(a, key[i], k, &lab, m, [&](int32_t t) { emit(anc_at(an, k - 1), t); });
+                } else if (tlen[i] == k) {
+                    // token byte j must equal the label k-1-j levels above m
+                    const uint32_t tw[4] = {tb[i].x, tb[i].y, tb[i].z, tb[i].w};
+                    bool eq = true;
+#pragma unroll
+                    for (int j = 0; j < kMaxClimb; j++)
+                        if (j < k) eq = eq && byte_at(tw, j) == byte_at(lab, k - 1 - j);
+                    if (eq) emit(anc_at(an, k - 1), tid[i]);
                 }
             }
         }
     }
     // suffixes longer than the window (deep tries with long tokens)
     if (a.lmax > kMaxClimb && depth == kMaxClimb) {
-        int32_t y = ancestor(a, m, kMaxClimb);  // start of the 16-byte suffix
+        int32_t y = anc_at(an, kMaxClimb - 1);  // start of the 16-byte suffix
         for (int32_t k = kMaxClimb + 1; k <= a.lmax; k++) {
             const int32_t p = a.parent[y];
             if (p < 0) break;
@@ -682,7 +716,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
 // terminal nodes) in no particular order, as CSR offsets[N+1] + tokens.
 
 // Counts the allowed tokens of every row (the start node of each hit).
-__global__ void __launch_bounds__(kPatchThreads) k_list_count(PatchArgs a, int32_t *__restrict__ row_count) {
+__global__ void __launch_bounds__(kPatchThreads, 4) k_list_count(PatchArgs a, int32_t *__restrict__ row_count) {
     pdl_launch_dependents();
     pdl_wait();  // hits from the probe, zeroed counters
     const int32_t stride = gridDim.x * blockDim.x;
@@ -900,7 +934,8 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.hit_count = t.hit_count;
     a.window = t.window;
     a.depth8 = t.depth8;
-    a.jump = t.jump;
+    a.anc = t.anc;
+    a.dup_keys = v.dup_keys;
     a.trans = t.trans;
     a.trans_mask = t.trans_mask;
     a.trans_fill = 0;
@@ -958,7 +993,7 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
     add(v.tok_off, 4 * nv);
     add(v.blob, v.blob_bytes);
     add(t.window, 16 * nn);
-    add(t.jump, 16 * nn);
+    add(t.anc, 64 * nn);
     add(t.depth8, nn);
     add(t.terminal, nn);
     cudaError_t e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf);

@@ -51,10 +51,10 @@ struct HostTrie {
     hvec<uint32_t> child_bits;           // [n * 8]
     // Per node, for the mask compile: the labels of the last 16 edges into it
     // (byte i = label i levels up, 0 past the root), min(depth, 255), and the
-    // ancestors 1, 2, 4 and 8 levels up (-1 past the root).
+    // ancestors 1..16 levels up (entry k = k + 1 levels up, -1 past the root).
     hvec<uint64_t> window;               // [n * 2] (low 8 bytes, high 8 bytes)
     hvec<uint8_t> depth8;                // [n]
-    hvec<int32_t> jump;                  // [n * 4]
+    hvec<int32_t> anc;                   // [n * 16]
     std::vector<int32_t> roots;          // root id of each set
     int64_t n_chars = 0;                 // total bytes of the distinct strings
     int32_t max_depth = 0;
@@ -82,6 +82,7 @@ struct HostVocab {
     std::vector<uint64_t> ht_key;        // [S] 0 = empty slot
     std::vector<int32_t> ht_val;         // [S] token id
     uint32_t ht_mask = 0;                // S - 1 (S a power of two)
+    int32_t dup_keys = 0;                // two tokens share a hash key
 };
 
 std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, HostVocab *out);
@@ -112,6 +113,7 @@ struct DevVocab {
     const uint16_t *tok_len = nullptr;
     const uint8_t *blob = nullptr;
     uint64_t blob_bytes = 0;
+    int32_t dup_keys = 0;
     const uint64_t *ht_key = nullptr;
     const int32_t *ht_val = nullptr;
     // host copy of the caller's arrays, to recognise the same vocabulary later
@@ -130,7 +132,7 @@ struct DevTrie {
     const uint32_t *child_bits = nullptr;
     const ulonglong2 *window = nullptr;
     const uint8_t *depth8 = nullptr;
-    const int4 *jump = nullptr;
+    const int4 *anc = nullptr;       // [n * 4]: 16 ancestors per node
     ulonglong2 *trans = nullptr;     // transition table {(row << 32 | token) + 1, end node}
     uint32_t trans_mask = 0;         // slots - 1
     int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) per node

@@ -74,6 +74,32 @@ def test_compile_small_random_exhaustive(cuda, seed):
     assert _first_diff(got, want) is None, _first_diff(got, want)
 
 
+@pytest.mark.parametrize("seed", range(30))
+def test_compile_small_random_unique_tokens(cuda, seed):
+    """Vocabularies without repeated token strings: the per-node search then
+    accepts a key found in its first slot pair without probing further."""
+    strings, toks = random_case(3000 + seed)
+    uniq = list(dict.fromkeys(t for t in toks[:-1] if t)) + [b""]
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(uniq)
+    h, m = _compile(cuda, sb, so, vb, vo)
+    want = oracle.mask_all(oracle.Trie(sb, so), oracle.Vocab(vb, vo))
+    assert _first_diff(_np_u32(m), want) is None
+
+
+def test_compile_repeated_tokens_large_vocab(cuda):
+    """The K=100 workload's vocabulary with 2,000 of its tokens repeated at
+    the end: every copy of an allowed token must be allowed too."""
+    w = W.config(1)
+    r = np.random.default_rng(7)
+    toks = [bytes(w.vocab_bytes[w.vocab_offsets[i]:w.vocab_offsets[i + 1]]) for i in range(w.V - 1)]
+    toks += [toks[int(i)] for i in r.integers(0, len(toks), 2000)] + [b""]
+    vb, vo = W.pack(toks)
+    h, m = _compile(cuda, w.set_bytes, w.set_offsets, vb, vo)
+    want = oracle.mask_all(oracle.Trie(w.set_bytes, w.set_offsets), oracle.Vocab(vb, vo), nthreads=NCPU)
+    assert _first_diff(_np_u32(m), want) is None
+
+
 @pytest.mark.parametrize("cfg", [1, 2, 3, 4])
 def test_compile_config_full(cuda, cfg):
     """Every row of the full-size workloads, compared in row blocks."""
