@@ -162,7 +162,7 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     const size_t o_fc = L.add(sizeof(int32_t) * n);
     const size_t o_bits = L.add(sizeof(uint32_t) * 8 * n);
     const size_t o_win = L.add(sizeof(uint64_t) * 2 * n);
-    const size_t o_d8 = L.add(n);
+    const size_t o_d16 = L.add(n);
     const size_t o_anc = L.add(sizeof(int32_t) * 16 * n);
     size_t trans_slots = 16;  // >= 8 per node, a power of two
     while (trans_slots < 8 * n) trans_slots <<= 1;
@@ -182,9 +182,6 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
         {o_term, t.terminal.data(), n},
         {o_fc, t.first_child.data(), sizeof(int32_t) * n},
         {o_bits, t.child_bits.data(), sizeof(uint32_t) * 8 * n},
-        {o_win, t.window.data(), sizeof(uint64_t) * 2 * n},
-        {o_d8, t.depth8.data(), n},
-        {o_anc, t.anc.data(), sizeof(int32_t) * 16 * n},
     };
     for (const Up &u : ups) {
         e = cudaMemcpyAsync(b + u.off, u.src, u.n, cudaMemcpyHostToDevice, stream);
@@ -201,13 +198,21 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     h->dev.terminal = reinterpret_cast<const uint8_t *>(b + o_term);
     h->dev.first_child = reinterpret_cast<const int32_t *>(b + o_fc);
     h->dev.child_bits = reinterpret_cast<const uint32_t *>(b + o_bits);
-    h->dev.window = reinterpret_cast<const ulonglong2 *>(b + o_win);
-    h->dev.depth8 = reinterpret_cast<const uint8_t *>(b + o_d8);
-    h->dev.anc = reinterpret_cast<const int4 *>(b + o_anc);
+    h->dev.window = reinterpret_cast<ulonglong2 *>(b + o_win);
+    h->dev.depth16 = reinterpret_cast<uint8_t *>(b + o_d16);
+    h->dev.anc = reinterpret_cast<int4 *>(b + o_anc);
     h->dev.trans = reinterpret_cast<ulonglong2 *>(b + o_trans);
     h->dev.trans_mask = uint32_t(trans_slots - 1);
     h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
     h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
+    // the compile's per-node tables, from the uploaded parent/label arrays
+    e = tmk::launch_trie_tables(h->dev, t.n, num_sms(dev), stream);
+    if (e != cudaSuccess) {
+        cudaStreamSynchronize(stream);
+        cudaFree(base);
+        h->dev = tmk::DevTrie();
+        return fail_cuda(e, "building the trie's compile tables");
+    }
     return TRIE_OK;
 }
 

@@ -42,27 +42,6 @@ inline int cmp_str(const Str &a, const Str &b) {
 
 }  // namespace
 
-// Label windows, clipped depths and the 16 nearest ancestors, in BFS order
-// (a parent always precedes its children).
-void add_compile_tables(HostTrie *t) {
-    const size_t n = size_t(t->n);
-    t->window.assign(2 * n, 0ull);
-    t->depth8.assign(n, 0);
-    t->anc.assign(16 * n, -1);
-    for (size_t i = 0; i < n; i++) {
-        const int32_t p = t->parent[i];
-        if (p < 0) continue;
-        const uint64_t lo = t->window[2 * size_t(p)], hi = t->window[2 * size_t(p) + 1];
-        t->window[2 * i] = (lo << 8) | t->label[i];
-        t->window[2 * i + 1] = (hi << 8) | (lo >> 56);
-        t->depth8[i] = uint8_t(t->depth8[size_t(p)] == 255 ? 255 : t->depth8[size_t(p)] + 1);
-        int32_t *a = &t->anc[16 * i];
-        const int32_t *ap = &t->anc[16 * size_t(p)];
-        a[0] = p;
-        for (int q = 1; q < 16; q++) a[q] = ap[q - 1];
-    }
-}
-
 std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t first, int32_t last,
                        HostTrie *out) {
     const int64_t K = int64_t(last) - first;
@@ -139,7 +118,6 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
         uint8_t l = out->label[size_t(c)];
         out->child_bits[size_t(p) * 8 + (l >> 5)] |= 1u << (l & 31);
     }
-    add_compile_tables(out);
     out->roots.assign(1, 0);
     out->n_chars = n_chars;
     out->max_depth = max_depth;
@@ -185,9 +163,6 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
     out->terminal.resize(n);
     out->first_child.resize(n);
     out->child_bits.resize(n * 8);
-    out->window.resize(n * 2);
-    out->depth8.resize(n);
-    out->anc.resize(n * 16);
     out->roots.assign(base.begin(), base.end());
     next = 0;
     auto concat = [&]() {
@@ -201,12 +176,9 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
                 out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
                 out->first_child[g + j] = p.first_child[j] < 0 ? -1 : p.first_child[j] + b;
             }
-            for (size_t j = 0; j < 16 * pn; j++) out->anc[16 * g + j] = p.anc[j] < 0 ? -1 : p.anc[j] + b;
             memcpy(&out->label[g], p.label.data(), pn);
             memcpy(&out->terminal[g], p.terminal.data(), pn);
             memcpy(&out->child_bits[8 * g], p.child_bits.data(), sizeof(uint32_t) * 8 * pn);
-            memcpy(&out->window[2 * g], p.window.data(), sizeof(uint64_t) * 2 * pn);
-            memcpy(&out->depth8[g], p.depth8.data(), pn);
             p = HostTrie();  // release the part's memory early
         }
     };

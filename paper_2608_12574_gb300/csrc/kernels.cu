@@ -136,7 +136,7 @@ struct PatchArgs {
     int2 *hits;          // [n_nodes * kHitSlots] (row, token), probe-scatter form only
     uint8_t *hit_count;  // [n_nodes]
     const ulonglong2 *window;  // probe-scatter form: last 16 labels per node
-    const uint8_t *depth8;
+    const uint8_t *depth16;    // min(depth, 16)
     const int4 *anc;           // [n * 4]: ancestors 1..16 levels up
     int32_t dup_keys;          // two tokens share a hash key
     ulonglong2 *trans;         // transition table (row, token) -> end node, or null
@@ -318,6 +318,42 @@ __device__ __forceinline__ void node_hits(const PatchArgs &a, int32_t m, Emit em
     }
 }
 
+// Per-node tables of the probe (one thread per node, climbing at most 16
+// parents): the last 16 edge labels into m, min(depth, 16), and the 16
+// nearest ancestors. Siblings and cousins are neighbours in breadth-first
+// order, so a warp's climbs read neighbouring entries.
+constexpr int kTableThreads = 256;
+__global__ void __launch_bounds__(kTableThreads) k_trie_tables(const int32_t *__restrict__ parent,
+                                                               const uint8_t *__restrict__ label, int32_t n,
+                                                               ulonglong2 *__restrict__ window,
+                                                               uint8_t *__restrict__ depth16,
+                                                               int4 *__restrict__ anc) {
+    const int32_t stride = gridDim.x * blockDim.x;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < n; m += stride) {
+        uint64_t lo = 0, hi = 0;
+        int32_t up[kMaxClimb];
+        int32_t d = 0;
+        int32_t x = m;
+#pragma unroll
+        for (int k = 0; k < kMaxClimb; k++) {
+            const int32_t p = x >= 0 ? __ldg(parent + x) : -1;
+            up[k] = p;
+            if (p >= 0) {
+                const uint64_t b = __ldg(label + x);
+                if (k < 8) lo |= b << (8 * k);
+                else hi |= b << (8 * (k - 8));
+                d = k + 1;
+            }
+            x = p;
+        }
+        window[m] = make_ulonglong2(lo, hi);
+        depth16[m] = uint8_t(d);
+#pragma unroll
+        for (int q = 0; q < 4; q++)
+            anc[int64_t(m) * 4 + q] = make_int4(up[4 * q], up[4 * q + 1], up[4 * q + 2], up[4 * q + 3]);
+    }
+}
+
 // Element k of a register copy of 16 ancestors, without dynamic indexing.
 __device__ __forceinline__ int32_t anc_at(const int4 (&an)[4], int k) {
     const int4 q = k < 4 ? an[0] : (k < 8 ? an[1] : (k < 12 ? an[2] : an[3]));
@@ -338,9 +374,8 @@ __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, 
     int4 an[4];
 #pragma unroll
     for (int q = 0; q < 4; q++) an[q] = __ldg(a.anc + int64_t(m) * 4 + q);
-    const int32_t d8 = __ldg(a.depth8 + m);
-    const int32_t lim = a.lmax < kMaxClimb ? a.lmax : kMaxClimb;
-    const int32_t depth = d8 < lim ? d8 : lim;
+    const int32_t d16 = __ldg(a.depth16 + m);
+    const int32_t depth = a.lmax < d16 ? a.lmax : d16;
     const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y), uint32_t(win.y >> 32)};
     if (__ldg(a.terminal + m)) emit(m, a.eos);
     const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
@@ -933,7 +968,7 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.hits = t.hits;
     a.hit_count = t.hit_count;
     a.window = t.window;
-    a.depth8 = t.depth8;
+    a.depth16 = t.depth16;
     a.anc = t.anc;
     a.dup_keys = v.dup_keys;
     a.trans = t.trans;
@@ -968,6 +1003,13 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
     return launch_pdl(k_mask_patch, grid, kPatchThreads, st, a);
 }
 
+cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st) {
+    if (n_nodes <= 0) return cudaSuccess;
+    const int grid = grid_for(n_nodes, kTableThreads, int64_t(num_sms) * 8);
+    k_trie_tables<<<grid, kTableThreads, 0, st>>>(t.parent, t.label, n_nodes, t.window, t.depth16, t.anc);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st) {
     return launch_mask_fill(reinterpret_cast<uint32_t *>(t.trans), 4 * (int64_t(t.trans_mask) + 1), num_sms, st);
 }
@@ -994,7 +1036,7 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
     add(v.blob, v.blob_bytes);
     add(t.window, 16 * nn);
     add(t.anc, 64 * nn);
-    add(t.depth8, nn);
+    add(t.depth16, nn);
     add(t.terminal, nn);
     cudaError_t e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf);
     if (e != cudaSuccess) return e;

@@ -49,12 +49,6 @@ struct HostTrie {
     hvec<uint8_t> terminal;              // some string ends here
     hvec<int32_t> first_child;           // -1 for a leaf
     hvec<uint32_t> child_bits;           // [n * 8]
-    // Per node, for the mask compile: the labels of the last 16 edges into it
-    // (byte i = label i levels up, 0 past the root), min(depth, 255), and the
-    // ancestors 1..16 levels up (entry k = k + 1 levels up, -1 past the root).
-    hvec<uint64_t> window;               // [n * 2] (low 8 bytes, high 8 bytes)
-    hvec<uint8_t> depth8;                // [n]
-    hvec<int32_t> anc;                   // [n * 16]
     std::vector<int32_t> roots;          // root id of each set
     int64_t n_chars = 0;                 // total bytes of the distinct strings
     int32_t max_depth = 0;
@@ -67,7 +61,6 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
                        HostTrie *out);
 std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
                          int32_t M, HostTrie *out);
-void add_compile_tables(HostTrie *t);
 
 // -------------------------------------------------------------- vocabulary
 // Token strings packed for 16-byte vector loads plus an open-addressing hash
@@ -130,9 +123,13 @@ struct DevTrie {
     const uint8_t *terminal = nullptr;
     const int32_t *first_child = nullptr;
     const uint32_t *child_bits = nullptr;
-    const ulonglong2 *window = nullptr;
-    const uint8_t *depth8 = nullptr;
-    const int4 *anc = nullptr;       // [n * 4]: 16 ancestors per node
+    // Per node, for the mask compile, built on the device from parent/label
+    // (launch_trie_tables): the labels of the last 16 edges into it (byte i =
+    // label i levels up, 0 past the root), min(depth, 16), and the ancestors
+    // 1..16 levels up (entry k = k + 1 levels up, -1 past the root).
+    ulonglong2 *window = nullptr;    // [n]
+    uint8_t *depth16 = nullptr;      // [n]
+    int4 *anc = nullptr;             // [n * 4]
     ulonglong2 *trans = nullptr;     // transition table {(row << 32 | token) + 1, end node}
     uint32_t trans_mask = 0;         // slots - 1
     int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) per node
@@ -180,6 +177,8 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
 // beside the fill (needs t.hits / t.hit_count).
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st);
+// Fills t.window, t.depth16 and t.anc from t.parent and t.label.
+cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
 // Zeroes the transition table (before it is filled for another vocabulary).
 cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st);
 cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, const int32_t *states_in,
