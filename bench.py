@@ -424,6 +424,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
 
         run_apply_lists = capture(apply_lists_only)
         apply_lists_avg = timed(run_apply_lists, reps) / S
+        lazy = run_lazy(w, logits, forced, dev, stream, capture, timed, reps)
     timing_src = (f"CUDA events around {reps} back-to-back replays of a graph of the {S - 1} fused "
                   f"advance+apply launches of a step (over {S - 1} logits buffers, "
                   f"{(S - 1) * B * V * elt / 1e9:.2f} GB > L2), launching stream, right after the timed region")
@@ -551,6 +552,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
                          "apply_gbs": (B * V * elt + B * 4) / (apply_lists_avg * 1e-3) / 1e9,
                          "note": "valid lists as the paper stores them (Sec. 4.2); compile includes its one "
                                  "device-to-host read of the size"},
+        "lazy_rows": lazy,
         "breakdown": {"compile_ms": compile_ms, "apply_us_avg": apply_avg * 1e3,
                       "advance_us_avg": advance_avg * 1e3, "advance_apply_us_avg": fused_avg * 1e3,
                       "host_trie_build_ms": host_build_ms,
@@ -570,6 +572,49 @@ def run_gpu(args, w, rank: int, world: int, dist):
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds / 5, 5, 1)
         line["cpu_paper_algorithm"] = cpu_paper_algorithm(w)
     print(json.dumps(line))
+
+
+def run_lazy(w, logits, forced, dev, stream, capture, timed, reps: int) -> dict:
+    """The decode loop of the workload with lazy rows (App. H.5) instead of a
+    compiled mask: step 0 masked by trie_lazy_apply, steps 1.. by
+    trie_lazy_advance_apply (the same tokens as the dense loop). With no
+    cache every pass computes every row it needs; with a 4,096-row cache the
+    first pass after set-up computes them and later passes find them cached."""
+    import torch
+    from paper_2608_12574_gb300 import triemask as T
+    V, B, S = w.V, w.batch, w.steps
+    out = {"note": "rows computed on first use (App. H.5); a pass = step 0 apply + "
+                   f"{S - 1} fused advance+apply calls, 3 kernels each"}
+    sb = [torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(2)]
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    for cache in (0, 4096):
+        hl = T.trie_build(w.set_bytes, w.set_offsets)
+        T.trie_lazy_init(hl, w.vocab_bytes, w.vocab_offsets, V, cache, B)
+
+        def loop():
+            sb[0].zero_()
+            T.trie_lazy_apply(hl, logits[0], sb[0], stream)
+            cur = 0
+            for t in range(1, S):
+                T.trie_lazy_advance_apply(hl, sb[cur], forced[t - 1], sb[1 - cur], logits[t], err, stream)
+                cur = 1 - cur
+
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            loop()
+            e1.record(stream)
+        stream.synchronize()
+        cold = e0.elapsed_time(e1)
+        run = capture(loop)
+        pass_ms = timed(run, reps)
+        hits, misses = T.trie_lazy_stats(hl)
+        rows_bytes = (((cache + 7) // 8 * 8) + B) * T.mask_words(V) * 4
+        out[f"cache_{cache}"] = {"cache_rows": cache, "first_pass_ms": cold, "pass_ms": pass_ms,
+                                 "us_per_step": pass_ms * 1e3 / S, "hits": hits, "misses": misses,
+                                 "row_bytes": rows_bytes}
+        hl.destroy()
+    return out
 
 
 def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
@@ -650,6 +695,45 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
         et.append(time.perf_counter() - t0)
         hh.destroy()
     out["end_to_end_ms"] = min(et) * 1e3
+    # lazy rows (App. H.5) instead of the lists: no per-batch compile, each
+    # step computes the rows its states reach (the requests are new every
+    # batch, so no cache is kept)
+    def lazy_steps(hh, st):
+        T.trie_lazy_apply(hh, logits[0], st[0], stream)
+        for t in range(1, steps):
+            T.trie_lazy_advance_apply(hh, st[(t - 1) % 2], forced[t - 1], st[t % 2], logits[t], err, stream)
+
+    et = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        hh = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+        T.trie_lazy_init(hh, w.vocab_bytes, w.vocab_offsets, V, 0, B)
+        with torch.cuda.stream(stream):
+            st = [torch.as_tensor(hh.roots(), device=dev), torch.empty(B, dtype=torch.int32, device=dev)]
+            lazy_steps(hh, st)
+        stream.synchronize()
+        et.append(time.perf_counter() - t0)
+        hh.destroy()
+    out["lazy_end_to_end_ms"] = min(et) * 1e3
+    T.trie_lazy_init(h, w.vocab_bytes, w.vocab_offsets, V, 0, B)
+    lst = [roots.clone(), torch.empty(B, dtype=torch.int32, device=dev)]
+
+    def lazy_decode():
+        lst[0].copy_(roots)
+        lazy_steps(h, lst)
+
+    gl = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        lazy_decode()
+        with torch.cuda.graph(gl, stream=stream):
+            lazy_decode()
+        gl.replay()
+        e0.record(stream)
+        for _ in range(reps):
+            gl.replay()
+        e1.record(stream)
+    stream.synchronize()
+    out["lazy_decode_ms"] = e0.elapsed_time(e1) / reps
     # the dense form of the same forest: a [N, ceil(V/32)] mask
     dense_bytes = N * T.mask_words(V) * 4
     free, _ = torch.cuda.mem_get_info(dev)

@@ -216,6 +216,58 @@ int trie_copy_lists(trie_t h, int64_t *d_offsets, int32_t *d_tokens, cudaStream_
 int trie_apply_lists(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
                      cudaStream_t stream);
 
+/* Lazy rows (App. H.5, the memory-constrained mode: valid[n] is computed
+ * only when decoding first reaches node n, and kept in an LRU cache of
+ * bounded size). No mask of all nodes is built: each call computes the rows
+ * of the batch's states that are not cached, on the GPU, and applies them.
+ * A row is computed from the node's subtree: the strings of the paths from
+ * n down into it that are tokens (App. G.5 condition (i)), plus EOS where n
+ * is terminal; the result equals that row of trie_compile_masks.
+ *
+ * Set-up (host-synchronous; synchronises the device). Allocates, on the
+ * current device, (rounded-up cache_rows + max_batch) rows of ceil(V/32)
+ * uint32 words plus 16 bytes per trie node and 16 per batch row; replaces the
+ * cache of an earlier trie_lazy_init on the handle (starting empty).
+ *   vocab_bytes, vocab_offsets, V  as trie_compile_masks, 2 <= V <= 524,288
+ *   cache_rows  rows kept between calls (rounded up to a multiple of 8; 0 =
+ *               no cache, every row is recomputed). The cache is 8-way set
+ *               associative: a node may only use the 8 rows of its set, and
+ *               a new row replaces the least recently used of them.
+ *   max_batch   largest B of the calls below, 1 <= max_batch <= 4096
+ * Errors: TRIE_EINVAL, TRIE_ENOMEM, TRIE_ECUDA. */
+int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                   int32_t cache_rows, int32_t max_batch);
+
+/* trie_apply_mask with lazily computed rows (same arguments, states and
+ * result; V must equal trie_lazy_init's V; B <= max_batch). Rows of states
+ * that are cached are reused; the others are computed and cached, unless all
+ * 8 rows of their set are used by this same call (they are then computed for
+ * this call only). Three kernels on `stream`; no host synchronisation, no
+ * allocation. All lazy calls on one handle share its cache and scratch: they
+ * must run one after the other (one stream, or ordered by events), not
+ * concurrently. TRIE_ESTATE before trie_lazy_init. */
+int trie_lazy_apply(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                    cudaStream_t stream);
+
+/* trie_advance_apply with lazily computed rows: the states are advanced
+ * (rules of trie_advance, written to d_states_out, which must differ from
+ * d_states_in), then the logits are masked by the rows of the new states as
+ * trie_lazy_apply does. d_err as trie_advance. */
+int trie_lazy_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
+                            int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream);
+
+/* The rows themselves (for inspection and tests): d_rows device
+ * uint32[B][ceil(V/32)] receives the row of each d_states[b] (FINISHED, DEAD
+ * and non-node states: the {EOS} row), computed and cached as by
+ * trie_lazy_apply. */
+int trie_lazy_rows(trie_t h, const int32_t *d_states, int32_t B, uint32_t *d_rows, cudaStream_t stream);
+
+/* Cache counters since trie_lazy_init: batch rows whose node's row was found
+ * in the cache (hits) and batch rows whose node's row had to be computed
+ * (misses; batch rows sharing a node in one call all count, the row is
+ * computed once). Host-synchronous (synchronises the device). */
+int trie_lazy_stats(trie_t h, int64_t *hits, int64_t *misses);
+
 /* Size of the fixed device scratch used by trie_compile_masks_noalloc. */
 #define TRIE_NOALLOC_SCRATCH_BYTES (32u << 20)
 

@@ -247,6 +247,39 @@ int finish_build(std::string err, trie_s *h, trie_t *out) {
     return TRIE_OK;
 }
 
+// Shared checks and the launch of the three lazy-row calls.
+int lazy_call(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out, int32_t *d_err,
+              void *d_logits, int dtype, uint32_t *d_rows, int32_t B, int32_t V, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    const tmk::DevLazy &L = h->lazy;
+    if (!L.base) return fail(TRIE_ESTATE, "lazy call before trie_lazy_init on this handle");
+    if (B < 0 || B > L.max_batch)
+        return fail(TRIE_EINVAL, "B must be in [0, max_batch = " + std::to_string(L.max_batch) + "]");
+    if (V != L.V) return fail(TRIE_EINVAL, "V differs from the V given to trie_lazy_init");
+    if (B == 0) return TRIE_OK;
+    if (!d_states_in) return fail(TRIE_EINVAL, "d_states is NULL");
+    if (d_tokens && (!d_states_out || d_states_out == d_states_in))
+        return fail(TRIE_EINVAL, "d_states_out must be a buffer other than d_states_in");
+    if (d_logits) {
+        if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
+        if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
+            return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
+    }
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != L.device || dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    bool use_trans;
+    {
+        std::lock_guard<std::mutex> lk(h->mu);
+        use_trans = h->trans_vocab == L.vocab.get();
+    }
+    const int32_t lmax = std::min(L.vocab->max_len, h->host.max_depth);
+    cudaError_t e = tmk::launch_lazy(h->dev, h->host.n, *L.vocab, use_trans, lmax, L, d_states_in, d_tokens,
+                                     d_states_out, d_err, B, d_logits, dtype, d_rows, num_sms(dev), stream);
+    if (e != cudaSuccess) return fail_cuda(e, "lazy-row launch");
+    return TRIE_OK;
+}
+
 }  // namespace
 
 int tmk::set_error(int code, const char *msg) { return fail(code, msg); }
@@ -541,8 +574,123 @@ int trie_apply_lists(trie_t h, void *d_logits, int dtype, const int32_t *d_state
     return TRIE_OK;
 }
 
+int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                   int32_t cache_rows, int32_t max_batch) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || (int64_t(V) + 31) / 32 > tmk::kLazyMaxWords)
+        return fail(TRIE_EINVAL, "V must be in [2, " + std::to_string(tmk::kLazyMaxWords * 32) + "] for lazy rows");
+    if (cache_rows < 0) return fail(TRIE_EINVAL, "cache_rows must be >= 0");
+    if (max_batch < 1 || max_batch > tmk::kLazyMaxBatch)
+        return fail(TRIE_EINVAL, "max_batch must be in [1, " + std::to_string(tmk::kLazyMaxBatch) + "]");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    if ((rc = ensure_device_trie(h, dev, 0)) != TRIE_OK) return rc;
+    cudaError_t e = cudaDeviceSynchronize();  // earlier lazy calls may still use the old cache
+    if (e != cudaSuccess) return fail_cuda(e, "synchronising before the lazy set-up");
+    tmk::DevLazy &L = h->lazy;
+    if (L.base) cudaFree(L.base);
+    L = tmk::DevLazy();
+    const int32_t C = (cache_rows + tmk::kLazyWays - 1) / tmk::kLazyWays * tmk::kLazyWays;
+    const int64_t W = (int64_t(V) + 31) / 32;
+    const size_t n = size_t(h->host.n), mb = size_t(max_batch);
+    Layout lay;
+    const size_t o_rows = lay.add(sizeof(uint32_t) * size_t(W) * (size_t(C) + mb));
+    const size_t o_tag = lay.add(sizeof(int32_t) * size_t(C));
+    const size_t o_stamp = lay.add(sizeof(uint32_t) * size_t(C));
+    const size_t o_ctrl = lay.add(sizeof(tmk::LazyCtrl));
+    const size_t o_slot = lay.add(sizeof(int32_t) * mb);
+    const size_t o_mnode = lay.add(sizeof(int32_t) * mb);
+    const size_t o_mslot = lay.add(sizeof(int32_t) * mb);
+    const size_t o_rowu = lay.add(sizeof(int32_t) * mb);
+    const size_t o_pnode = lay.add(sizeof(int32_t) * n);
+    const size_t o_pdep = lay.add(sizeof(int32_t) * n);
+    const size_t o_psize = lay.add(sizeof(int32_t) * n);
+    const size_t o_pos = lay.add(sizeof(int32_t) * n);
+    void *base = nullptr;
+    e = cudaMalloc(&base, lay.total);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(TRIE_ENOMEM, std::string("cudaMalloc for the lazy rows: ") + cudaGetErrorString(e));
+    }
+    char *b = static_cast<char *>(base);
+    L.device = dev;
+    L.base = base;
+    L.C = C;
+    L.max_batch = max_batch;
+    L.V = V;
+    L.W = W;
+    L.rows = reinterpret_cast<uint32_t *>(b + o_rows);
+    L.tag = reinterpret_cast<int32_t *>(b + o_tag);
+    L.stamp = reinterpret_cast<uint32_t *>(b + o_stamp);
+    L.ctrl = reinterpret_cast<tmk::LazyCtrl *>(b + o_ctrl);
+    L.slot_of = reinterpret_cast<int32_t *>(b + o_slot);
+    L.miss_node = reinterpret_cast<int32_t *>(b + o_mnode);
+    L.miss_slot = reinterpret_cast<int32_t *>(b + o_mslot);
+    L.row_u = reinterpret_cast<int32_t *>(b + o_rowu);
+    L.pre_node = reinterpret_cast<int32_t *>(b + o_pnode);
+    L.pre_depth = reinterpret_cast<int32_t *>(b + o_pdep);
+    L.pre_size = reinterpret_cast<int32_t *>(b + o_psize);
+    L.pos_of = reinterpret_cast<int32_t *>(b + o_pos);
+    const tmk::LazyCtrl ctrl0 = {1u, 0, 0ull, 0ull};
+    const tmk::HostTrie &t = h->host;
+    if ((e = cudaMemset(L.tag, 0xFF, sizeof(int32_t) * size_t(C))) != cudaSuccess ||
+        (e = cudaMemset(L.stamp, 0, sizeof(uint32_t) * size_t(C))) != cudaSuccess ||
+        (e = cudaMemcpy(L.ctrl, &ctrl0, sizeof(ctrl0), cudaMemcpyHostToDevice)) != cudaSuccess ||
+        (e = cudaMemcpy(L.pre_node, t.pre_node.data(), sizeof(int32_t) * n, cudaMemcpyHostToDevice)) !=
+            cudaSuccess ||
+        (e = cudaMemcpy(L.pre_depth, t.pre_depth.data(), sizeof(int32_t) * n, cudaMemcpyHostToDevice)) !=
+            cudaSuccess ||
+        (e = cudaMemcpy(L.pre_size, t.pre_size.data(), sizeof(int32_t) * n, cudaMemcpyHostToDevice)) !=
+            cudaSuccess ||
+        (e = tmk::launch_lazy_tables(L, h->host.n, 0)) != cudaSuccess || (e = cudaDeviceSynchronize()) != cudaSuccess) {
+        cudaFree(base);
+        L = tmk::DevLazy();
+        return fail_cuda(e, "lazy-row set-up");
+    }
+    L.vocab = voc;
+    return TRIE_OK;
+}
+
+int trie_lazy_apply(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                    cudaStream_t stream) {
+    if (B > 0 && !d_logits) return fail(TRIE_EINVAL, "d_logits is NULL");
+    return lazy_call(h, d_states, nullptr, nullptr, nullptr, d_logits, dtype, nullptr, B, V, stream);
+}
+
+int trie_lazy_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
+                            int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream) {
+    if (B > 0 && (!d_tokens || !d_logits)) return fail(TRIE_EINVAL, "d_tokens / d_logits is NULL");
+    return lazy_call(h, d_states_in, d_tokens, d_states_out, d_err, d_logits, dtype, nullptr, B, V, stream);
+}
+
+int trie_lazy_rows(trie_t h, const int32_t *d_states, int32_t B, uint32_t *d_rows, cudaStream_t stream) {
+    if (B > 0 && !d_rows) return fail(TRIE_EINVAL, "d_rows is NULL");
+    const int32_t V = h ? h->lazy.V : 0;
+    return lazy_call(h, d_states, nullptr, nullptr, nullptr, nullptr, 0, d_rows, B, V, stream);
+}
+
+int trie_lazy_stats(trie_t h, int64_t *hits, int64_t *misses) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!h->lazy.base) return fail(TRIE_ESTATE, "trie_lazy_stats before trie_lazy_init on this handle");
+    DeviceGuard g(h->lazy.device);
+    tmk::LazyCtrl c;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemcpy(&c, h->lazy.ctrl, sizeof(c), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return fail_cuda(e, "reading the lazy-row counters");
+    if (hits) *hits = int64_t(c.hits);
+    if (misses) *misses = int64_t(c.misses);
+    return TRIE_OK;
+}
+
 int trie_destroy(trie_t h) {
     if (!h) return TRIE_OK;
+    if (h->lazy.base) {
+        DeviceGuard g(h->lazy.device);
+        cudaFree(h->lazy.base);
+    }
     if (h->dev.base || h->lists.base || h->lists.toks) {
         DeviceGuard g(h->dev.device);
         // cudaFree waits for work on the device that may still read these

@@ -62,7 +62,8 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
     std::sort(s.begin(), s.end(), [](const Str &a, const Str &b) { return cmp_str(a, b) < 0; });
 
     // pre-order creation
-    std::vector<int32_t> pparent(1, -1), pdepth(1, 0);
+    std::vector<int32_t> pparent(1, -1);
+    hvec<int32_t> pdepth(1, 0);
     std::vector<uint8_t> plabel(1, 0), pterm(1, 0);
     pparent.reserve(size_t(total / 2 + 16));
     std::vector<int32_t> path(1, 0);
@@ -96,8 +97,12 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
     std::vector<int32_t> level(size_t(max_depth) + 2, 0);
     for (int32_t i = 0; i < n; i++) level[size_t(pdepth[i]) + 1]++;
     for (size_t d = 1; d < level.size(); d++) level[d] += level[d - 1];
-    std::vector<int32_t> bfs(static_cast<size_t>(n));
+    hvec<int32_t> bfs(static_cast<size_t>(n));
     for (int32_t i = 0; i < n; i++) bfs[size_t(i)] = level[size_t(pdepth[i])]++;
+    // subtree sizes in pre-order (a parent precedes its descendants)
+    hvec<int32_t> psize(static_cast<size_t>(n));
+    for (int32_t i = 0; i < n; i++) psize[size_t(i)] = 1;
+    for (int32_t i = n - 1; i > 0; i--) psize[size_t(pparent[size_t(i)])] += psize[size_t(i)];
 
     out->n = n;
     out->parent.assign(size_t(n), -1);
@@ -118,6 +123,9 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
         uint8_t l = out->label[size_t(c)];
         out->child_bits[size_t(p) * 8 + (l >> 5)] |= 1u << (l & 31);
     }
+    out->pre_node = std::move(bfs);
+    out->pre_depth = std::move(pdepth);
+    out->pre_size = std::move(psize);
     out->roots.assign(1, 0);
     out->n_chars = n_chars;
     out->max_depth = max_depth;
@@ -163,6 +171,9 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
     out->terminal.resize(n);
     out->first_child.resize(n);
     out->child_bits.resize(n * 8);
+    out->pre_node.resize(n);
+    out->pre_depth.resize(n);
+    out->pre_size.resize(n);
     out->roots.assign(base.begin(), base.end());
     next = 0;
     auto concat = [&]() {
@@ -176,6 +187,9 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
                 out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
                 out->first_child[g + j] = p.first_child[j] < 0 ? -1 : p.first_child[j] + b;
             }
+            for (size_t j = 0; j < pn; j++) out->pre_node[g + j] = p.pre_node[j] + b;
+            memcpy(&out->pre_depth[g], p.pre_depth.data(), sizeof(int32_t) * pn);
+            memcpy(&out->pre_size[g], p.pre_size.data(), sizeof(int32_t) * pn);
             memcpy(&out->label[g], p.label.data(), pn);
             memcpy(&out->terminal[g], p.terminal.data(), pn);
             memcpy(&out->child_bits[8 * g], p.child_bits.data(), sizeof(uint32_t) * 8 * pn);

@@ -45,11 +45,12 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 template <typename... Params, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(Params...), int grid, int block, cudaStream_t st, Args... args) {
+cudaError_t launch_pdl_smem(void (*kernel)(Params...), int grid, int block, size_t smem, cudaStream_t st,
+                            Args... args) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned(grid));
     cfg.blockDim = dim3(unsigned(block));
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -57,6 +58,11 @@ cudaError_t launch_pdl(void (*kernel)(Params...), int grid, int block, cudaStrea
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+}
+
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), int grid, int block, cudaStream_t st, Args... args) {
+    return launch_pdl_smem(kernel, grid, block, 0, st, args...);
 }
 
 // ------------------------------------------------------------------ fill
@@ -948,6 +954,241 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_scalar(void *__restrict
     }
 }
 
+// ------------------------------------------------------------ lazy rows
+// valid[n] computed when a state first reaches n and kept in a row cache
+// (App. H.5), instead of all rows up front. A call is three kernels:
+//   k_lazy_resolve  one CTA: (advance,) then map every batch row's state to a
+//                   cache row: a hit refreshes the row's stamp; the distinct
+//                   missing nodes get the least recently used row of their
+//                   set (or a per-call row when every row of the set is in use
+//                   by this call);
+//   k_lazy_rows     one CTA per missing node s: valid[s] from s's subtree;
+//   apply (k_apply_vec on the cache rows) or k_lazy_gather.
+
+struct LazyArgs {
+    uint32_t *rows;
+    int32_t *tag;
+    uint32_t *stamp;
+    LazyCtrl *ctrl;
+    int32_t *slot_of;
+    int32_t *miss_node;
+    int32_t *miss_slot;
+    int32_t *row_u;
+    const int32_t *pre_node;
+    const int32_t *pre_depth;
+    const int32_t *pre_size;
+    const int32_t *pos_of;
+    int32_t C;        // cache rows
+    int32_t n_sets;   // C / kLazyWays
+    int32_t n_nodes;
+    int64_t W;
+    int32_t uniq;     // slots of the resolve's table of distinct missing nodes (a power of two)
+};
+
+constexpr int kResolveThreads = 1024;
+constexpr int kLazyRowThreads = 512;
+constexpr int32_t kPending = -3;
+
+__device__ __forceinline__ uint32_t mix32(uint32_t x) {
+    x ^= x >> 16;
+    x *= 0x7FEB352Du;
+    x ^= x >> 15;
+    x *= 0x846CA68Bu;
+    x ^= x >> 16;
+    return x;
+}
+
+__device__ __forceinline__ int32_t lazy_set(int32_t s, int32_t n_sets) {
+    return int32_t((uint64_t(mix32(uint32_t(s))) * uint64_t(uint32_t(n_sets))) >> 32);
+}
+
+// Cache tags and stamps are read through L2 (ld.global.cg): other threads of
+// the CTA change them with atomics during the kernel.
+template <bool kAdvance>
+__global__ void __launch_bounds__(kResolveThreads) k_lazy_resolve(LazyArgs L, AdvanceArgs aa,
+                                                                  const int32_t *states_in,
+                                                                  const int32_t *__restrict__ tokens,
+                                                                  int32_t *states_out, int32_t *__restrict__ err,
+                                                                  int32_t B) {
+    extern __shared__ int32_t sh[];  // [uniq] node keys, [uniq] their miss index
+    int32_t *keys = sh;
+    int32_t *vals = sh + L.uniq;
+    __shared__ int32_t n_u;
+    __shared__ unsigned long long n_hit, n_miss_rows;
+    for (int32_t i = threadIdx.x; i < L.uniq; i += blockDim.x) keys[i] = -1;
+    if (threadIdx.x == 0) {
+        n_u = 0;
+        n_hit = 0ull;
+        n_miss_rows = 0ull;
+    }
+    __syncthreads();
+    pdl_launch_dependents();
+    pdl_wait();  // states, tokens, cache and scratch of earlier kernels
+    const uint32_t now = __ldcg(&L.ctrl->now);
+    const uint32_t umask = uint32_t(L.uniq - 1);
+    // 1. states; cache lookups; distinct missing nodes into the table
+    for (int32_t b = threadIdx.x; b < B; b += blockDim.x) {
+        int32_t s;
+        if (kAdvance) {
+            const int32_t s0 = states_in[b];
+            s = advance_one(aa, s0, tokens[b]);
+            if (s == kDead && s0 != kDead && err) atomicAdd(err, 1);
+            states_out[b] = s;
+        } else {
+            s = states_in[b];
+        }
+        int32_t slot = -1;  // the {EOS} row
+        if (s >= 0 && s < L.n_nodes) {
+            const int32_t base = (L.n_sets > 0 ? lazy_set(s, L.n_sets) : 0) * kLazyWays;
+            int32_t hit = -1;
+            if (L.n_sets > 0) {
+#pragma unroll
+                for (int w = 0; w < kLazyWays; w++)
+                    if (__ldcg(L.tag + base + w) == s) hit = base + w;
+            }
+            if (hit >= 0) {
+                L.stamp[hit] = now;
+                slot = hit;
+                atomicAdd(&n_hit, 1ull);
+            } else {
+                uint32_t h = mix32(uint32_t(s)) & umask;
+                for (uint32_t it = 0; it <= umask; it++) {  // the table holds >= 2 B slots
+                    const int32_t k = atomicCAS(keys + h, -1, s);
+                    if (k == -1 || k == s) break;
+                    h = (h + 1u) & umask;
+                }
+                L.row_u[b] = int32_t(h);
+                slot = kPending;
+                atomicAdd(&n_miss_rows, 1ull);
+            }
+        }
+        L.slot_of[b] = slot;
+    }
+    __syncthreads();
+    // 2. number the distinct missing nodes
+    for (int32_t i = threadIdx.x; i < L.uniq; i += blockDim.x) {
+        const int32_t k = keys[i];
+        if (k >= 0) {
+            const int32_t u = atomicAdd(&n_u, 1);
+            vals[i] = u;
+            L.miss_node[u] = k;
+        }
+    }
+    __syncthreads();
+    // 3. a row for each: the least recently used row of its set that this call
+    // does not use, claimed by a compare-and-swap of its stamp
+    for (int32_t u = threadIdx.x; u < n_u; u += blockDim.x) {
+        const int32_t s = L.miss_node[u];
+        int32_t slot = L.C + u;  // per-call row
+        if (L.n_sets > 0) {
+            const int32_t base = lazy_set(s, L.n_sets) * kLazyWays;
+            for (int att = 0; att < 4 * kLazyWays; att++) {
+                int32_t best = -1;
+                uint32_t best_st = 0xFFFFFFFFu;
+#pragma unroll
+                for (int w = 0; w < kLazyWays; w++) {
+                    const uint32_t st = __ldcg(L.stamp + base + w);
+                    if (st != now && st < best_st) {
+                        best_st = st;
+                        best = w;
+                    }
+                }
+                if (best < 0) break;
+                if (atomicCAS(L.stamp + base + best, best_st, now) == best_st) {
+                    slot = base + best;
+                    L.tag[slot] = s;
+                    break;
+                }
+            }
+        }
+        L.miss_slot[u] = slot;
+    }
+    __syncthreads();
+    // 4. batch rows of missing nodes
+    for (int32_t b = threadIdx.x; b < B; b += blockDim.x)
+        if (L.slot_of[b] == kPending) L.slot_of[b] = L.miss_slot[vals[L.row_u[b]]];
+    if (threadIdx.x == 0) {
+        L.ctrl->n_miss = n_u;
+        L.ctrl->now = now + 1u;
+        L.ctrl->hits += n_hit;
+        L.ctrl->misses += n_miss_rows;
+    }
+}
+
+// valid[s] for a missing node s (App. H.5), written to its cache row. The
+// allowed tokens are the strings of the paths from s down into its subtree
+// (App. G.5 condition (i): the token's bytes walk from s inside the trie),
+// and EOS if s is terminal. The subtree is one interval of the pre-order
+// tables; a descendant d at depth j below s (1 <= j <= the longest token)
+// contributes the token, if any, whose bytes are the last j edge labels into
+// d. The row is built in shared memory, then stored.
+__global__ void __launch_bounds__(kLazyRowThreads) k_lazy_rows(LazyArgs L, PatchArgs a) {
+    extern __shared__ uint32_t bits[];
+    pdl_launch_dependents();
+    pdl_wait();  // the resolve's miss list
+    const int32_t n_miss = __ldcg(&L.ctrl->n_miss);
+    for (int32_t u = blockIdx.x; u < n_miss; u += gridDim.x) {
+        const int32_t s = L.miss_node[u];
+        const int32_t slot = L.miss_slot[u];
+        for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x) bits[i] = 0u;
+        __syncthreads();
+        if (threadIdx.x == 0 && __ldg(a.terminal + s)) atomicOr(bits + (a.eos >> 5), 1u << (a.eos & 31));
+        const int32_t pos = __ldg(L.pos_of + s);
+        const int32_t end = pos + __ldg(L.pre_size + pos);
+        const int32_t d0 = __ldg(L.pre_depth + pos);
+        for (int32_t k = pos + 1 + int32_t(threadIdx.x); k < end; k += blockDim.x) {
+            const int32_t j = __ldg(L.pre_depth + k) - d0;
+            if (j > a.lmax) continue;
+            const int32_t d = __ldg(L.pre_node + k);
+            auto hit = [&](int32_t t) { atomicOr(bits + (t >> 5), 1u << (t & 31)); };
+            uint64_t h = 0, pw = 1;
+            if (j <= kMaxClimb) {
+                const ulonglong2 win = __ldg(a.window + d);
+                const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y),
+                                         uint32_t(win.y >> 32)};
+                for (int32_t i = 0; i < j; i++) {  // byte i levels above d
+                    h += (uint64_t(byte_at(lab, i)) + 1ull) * pw;
+                    pw *= kHashBase;
+                }
+                probe(a, hash_finish(h, uint32_t(j)), j, &lab, d, hit);
+            } else {
+                int32_t y = d;
+                for (int32_t i = 0; i < j; i++) {
+                    h += (uint64_t(__ldg(a.label + y)) + 1ull) * pw;
+                    pw *= kHashBase;
+                    y = __ldg(a.parent + y);
+                }
+                probe(a, hash_finish(h, uint32_t(j)), j, nullptr, d, hit);
+            }
+        }
+        __syncthreads();
+        uint32_t *row = L.rows + int64_t(slot) * L.W;
+        for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x) row[i] = bits[i];
+        __syncthreads();  // bits are reused by the next node
+    }
+}
+
+// Copies the rows of a call out: out[b] = row of slot_of[b] ({EOS} if < 0).
+__global__ void __launch_bounds__(kApplyThreads) k_lazy_gather(const uint32_t *__restrict__ rows,
+                                                               const int32_t *__restrict__ slot_of, int32_t B,
+                                                               int64_t W, int32_t n_rows, int32_t eos,
+                                                               uint32_t *__restrict__ out) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int64_t total = int64_t(B) * W;
+    for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+         i += int64_t(gridDim.x) * blockDim.x) {
+        const int32_t b = int32_t(i / W);
+        out[i] = row_word(rows, slot_of[b], n_rows, W, i - int64_t(b) * W, eos);
+    }
+}
+
+// pos_of[pre_node[k]] = k.
+__global__ void k_lazy_tables(const int32_t *__restrict__ pre_node, int32_t n, int32_t *__restrict__ pos_of) {
+    for (int32_t k = blockIdx.x * blockDim.x + threadIdx.x; k < n; k += gridDim.x * blockDim.x)
+        pos_of[pre_node[k]] = k;
+}
+
 PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax, uint32_t *mask,
                      int64_t W) {
     PatchArgs a;
@@ -1181,6 +1422,68 @@ cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const
                           n_nodes, parts);
     return launch_pdl(k_apply_lists<4, false>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
                       n_nodes, parts);
+}
+
+cudaError_t launch_lazy_tables(const DevLazy &L, int32_t n_nodes, cudaStream_t st) {
+    // shared memory above the default 48 KB: the resolve's table of distinct
+    // nodes (<= 2 * 2 * kLazyMaxBatch int32) and the row kernel's row
+    const int uniq_max = int(2 * 2 * kLazyMaxBatch * sizeof(int32_t));
+    const int row_max = int(kLazyMaxWords * sizeof(uint32_t));
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(k_lazy_resolve<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, uniq_max)) !=
+        cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_lazy_resolve<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, uniq_max)) !=
+        cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_lazy_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, row_max)) !=
+        cudaSuccess)
+        return e;
+    if (n_nodes <= 0) return cudaSuccess;
+    const int grid = grid_for(n_nodes, 256, 4096);
+    k_lazy_tables<<<grid, 256, 0, st>>>(L.pre_node, n_nodes, L.pos_of);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans, int32_t lmax,
+                        const DevLazy &L, const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
+                        int32_t *err, int32_t B, void *logits, int dtype, uint32_t *rows_out, int num_sms,
+                        cudaStream_t st) {
+    LazyArgs la;
+    la.rows = L.rows;
+    la.tag = L.tag;
+    la.stamp = L.stamp;
+    la.ctrl = L.ctrl;
+    la.slot_of = L.slot_of;
+    la.miss_node = L.miss_node;
+    la.miss_slot = L.miss_slot;
+    la.row_u = L.row_u;
+    la.pre_node = L.pre_node;
+    la.pre_depth = L.pre_depth;
+    la.pre_size = L.pre_size;
+    la.pos_of = L.pos_of;
+    la.C = L.C;
+    la.n_sets = L.C / kLazyWays;
+    la.n_nodes = n_nodes;
+    la.W = L.W;
+    int32_t uniq = 16;
+    while (uniq < 2 * B) uniq <<= 1;
+    la.uniq = uniq;
+    const AdvanceArgs aa = advance_args(t, n_nodes, v, use_trans);
+    const size_t rsmem = size_t(2) * size_t(uniq) * sizeof(int32_t);
+    cudaError_t e = tokens ? launch_pdl_smem(k_lazy_resolve<true>, 1, kResolveThreads, rsmem, st, la, aa, states_in,
+                                             tokens, states_out, err, B)
+                           : launch_pdl_smem(k_lazy_resolve<false>, 1, kResolveThreads, rsmem, st, la, aa,
+                                             states_in, tokens, states_out, err, B);
+    if (e != cudaSuccess) return e;
+    const PatchArgs pa = patch_args(t, n_nodes, v, lmax, nullptr, L.W);
+    e = launch_pdl_smem(k_lazy_rows, B, kLazyRowThreads, size_t(L.W) * sizeof(uint32_t), st, la, pa);
+    if (e != cudaSuccess) return e;
+    const int32_t n_rows = L.C + L.max_batch;
+    if (logits) return launch_apply(logits, dtype, L.rows, L.slot_of, B, L.V, n_rows, num_sms, st);
+    const int grid = grid_for(int64_t(B) * L.W, kApplyThreads, int64_t(num_sms) * 8);
+    return launch_pdl(k_lazy_gather, grid, kApplyThreads, st, static_cast<const uint32_t *>(L.rows),
+                      static_cast<const int32_t *>(L.slot_of), B, L.W, n_rows, L.V - 1, rows_out);
 }
 
 }  // namespace tmk

@@ -49,6 +49,13 @@ struct HostTrie {
     hvec<uint8_t> terminal;              // some string ends here
     hvec<int32_t> first_child;           // -1 for a leaf
     hvec<uint32_t> child_bits;           // [n * 8]
+    // Depth-first pre-order of the same nodes (the order in which the builder
+    // creates them): position i holds node pre_node[i], at depth pre_depth[i],
+    // whose subtree is positions i .. i + pre_size[i] - 1. Used by the lazy
+    // rows, which enumerate a node's subtree as one interval.
+    hvec<int32_t> pre_node;              // [n]
+    hvec<int32_t> pre_depth;             // [n]
+    hvec<int32_t> pre_size;              // [n]
     std::vector<int32_t> roots;          // root id of each set
     int64_t n_chars = 0;                 // total bytes of the distinct strings
     int32_t max_depth = 0;
@@ -150,6 +157,42 @@ struct DevLists {
     int32_t V = 0;
 };
 
+// Lazy rows (App. H.5): valid[n] computed when a decode state first reaches
+// n, kept in a set-associative cache of rows with least-recently-used
+// replacement inside each set.
+constexpr int kLazyWays = 8;       // rows per cache set
+constexpr int kLazyMaxBatch = 4096;
+constexpr int64_t kLazyMaxWords = 16384;  // row built in shared memory (64 KB): V <= 524,288
+
+struct LazyCtrl {
+    uint32_t now;                   // call counter (stamps of rows used by this call)
+    int32_t n_miss;                 // rows computed by the current call
+    unsigned long long hits;        // batch rows whose node row was cached
+    unsigned long long misses;      // batch rows whose node row was computed
+};
+
+struct DevLazy {
+    int device = -1;
+    void *base = nullptr;
+    int32_t C = 0;                  // cache rows (a multiple of kLazyWays)
+    int32_t max_batch = 0;
+    int32_t V = 0;
+    int64_t W = 0;
+    std::shared_ptr<DevVocab> vocab;
+    uint32_t *rows = nullptr;       // [(C + max_batch) * W]: cache rows, then per-call rows
+    int32_t *tag = nullptr;         // [C] node of the row, -1 empty
+    uint32_t *stamp = nullptr;      // [C] call that last used the row (0 never)
+    LazyCtrl *ctrl = nullptr;
+    int32_t *slot_of = nullptr;     // [max_batch] row of each batch row, < 0: {EOS}
+    int32_t *miss_node = nullptr;   // [max_batch] nodes whose rows the call computes
+    int32_t *miss_slot = nullptr;   // [max_batch] where
+    int32_t *row_u = nullptr;       // [max_batch] scratch
+    int32_t *pre_node = nullptr;    // [n] pre-order tables of the trie (HostTrie)
+    int32_t *pre_depth = nullptr;   // [n]
+    int32_t *pre_size = nullptr;    // [n]
+    int32_t *pos_of = nullptr;      // [n] pre-order position of each node
+};
+
 }  // namespace tmk
 
 // The opaque handle of the C ABI.
@@ -162,6 +205,7 @@ struct trie_s {
     int32_t mask_V = 0;
     tmk::DevLists lists;                 // last compiled valid lists (library-owned)
     const tmk::DevVocab *trans_vocab = nullptr;  // vocabulary the transition table holds
+    tmk::DevLazy lazy;                   // lazy-row cache (trie_lazy_init)
 };
 
 namespace tmk {
@@ -197,6 +241,15 @@ cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab
                                const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total);
 cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  const DevLists &L, int num_sms, cudaStream_t st);
+// Lazy rows: pos_of from the pre-order tables (once, at set-up).
+cudaError_t launch_lazy_tables(const DevLazy &L, int32_t n_nodes, cudaStream_t st);
+// One lazy call: map the batch's states (after the advance when tokens is not
+// null) to cache rows, compute the missing rows, then apply them to the
+// logits (logits not null) or copy them out (rows_out not null).
+cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans, int32_t lmax,
+                        const DevLazy &L, const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
+                        int32_t *err, int32_t B, void *logits, int dtype, uint32_t *rows_out, int num_sms,
+                        cudaStream_t st);
 cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
                                int32_t V, int32_t n_nodes, cudaStream_t st);
 }  // namespace tmk

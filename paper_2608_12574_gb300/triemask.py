@@ -42,6 +42,11 @@ SIGNATURES = {
     "trie_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_advance_apply": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, ctypes.c_int, _I32, _I32, _P]),
     "trie_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
+    "trie_lazy_init": (ctypes.c_int, [_P, _P, _P, _I32, _I32, _I32]),
+    "trie_lazy_apply": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
+    "trie_lazy_advance_apply": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, ctypes.c_int, _I32, _I32, _P]),
+    "trie_lazy_rows": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
+    "trie_lazy_stats": (ctypes.c_int, [_P, _P, _P]),
     "trie_destroy": (ctypes.c_int, [_P]),
     "trie_last_error": (ctypes.c_char_p, []),
 }
@@ -318,6 +323,74 @@ def trie_apply_lists(h: Trie, d_logits, d_states, stream=None) -> None:
     pl = _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits")
     ps = _dev(d_states, (torch.int32,), "d_states")
     _check(h._lib.trie_apply_lists(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
+
+
+def trie_lazy_init(h: Trie, vocab_bytes, vocab_offsets, V: int, cache_rows: int, max_batch: int) -> None:
+    """Set up lazily computed rows with an LRU cache of cache_rows rows (current device)."""
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    _check(h._lib.trie_lazy_init(h.handle, _hp(vb), _hp(vo), V, cache_rows, max_batch))
+
+
+def _logits_dtype(d_logits) -> int:
+    import torch
+    if d_logits.dim() != 2:
+        raise ValueError("d_logits must be [B, V]")
+    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
+    if dtype is None:
+        raise TypeError("d_logits must be float32 or bfloat16")
+    return dtype
+
+
+def trie_lazy_apply(h: Trie, d_logits, d_states, stream=None) -> None:
+    """trie_apply_mask with rows computed on first use and cached."""
+    import torch
+    dtype = _logits_dtype(d_logits)
+    B, V = d_logits.shape
+    if d_states.numel() != B:
+        raise ValueError("d_states must have B entries")
+    _check(h._lib.trie_lazy_apply(h.handle, _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits"), dtype,
+                                  _dev(d_states, (torch.int32,), "d_states"), B, V,
+                                  _stream(stream, d_logits.device)))
+
+
+def trie_lazy_advance_apply(h: Trie, d_states_in, d_tokens, d_states_out, d_logits, d_err=None,
+                            stream=None) -> None:
+    """states_out <- delta*(states_in, tokens); then mask d_logits by lazily computed rows."""
+    import torch
+    dtype = _logits_dtype(d_logits)
+    B, V = d_logits.shape
+    for t, name in ((d_states_in, "d_states_in"), (d_tokens, "d_tokens"), (d_states_out, "d_states_out")):
+        if t.numel() != B:
+            raise ValueError(f"{name} must have B entries")
+    pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
+    _check(h._lib.trie_lazy_advance_apply(h.handle, _dev(d_states_in, (torch.int32,), "d_states_in"),
+                                          _dev(d_tokens, (torch.int32,), "d_tokens"),
+                                          _dev(d_states_out, (torch.int32,), "d_states_out"), pe,
+                                          _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits"), dtype, B,
+                                          V, _stream(stream, d_logits.device)))
+
+
+def trie_lazy_rows(h: Trie, d_states, V: int, out=None, stream=None):
+    """The rows ([B, ceil(V/32)] int32 CUDA tensor) of the states, computed or taken from the cache."""
+    import torch
+    B = d_states.numel()
+    if out is None:
+        out = torch.empty((B, mask_words(V)), dtype=torch.int32, device=d_states.device)
+    if out.shape != (B, mask_words(V)):
+        raise ValueError("out must be [B, ceil(V/32)]")
+    _check(h._lib.trie_lazy_rows(h.handle, _dev(d_states, (torch.int32,), "d_states"), B,
+                                 _dev(out, (torch.int32,), "out"), _stream(stream, d_states.device)))
+    return out
+
+
+def trie_lazy_stats(h: Trie) -> tuple[int, int]:
+    """(hits, misses) of the lazy-row cache since trie_lazy_init."""
+    hits, misses = ctypes.c_int64(0), ctypes.c_int64(0)
+    _check(h._lib.trie_lazy_stats(h.handle, ctypes.byref(hits), ctypes.byref(misses)))
+    return hits.value, misses.value
 
 
 def trie_destroy(h: Trie) -> None:

@@ -189,6 +189,28 @@ def test_device_calls_checked_before_any_device_work(lib):
     assert L.trie_advance(h.handle, 16, 16, -1, None, None) == T.TRIE_EINVAL
 
 
+def test_lazy_calls_checked_before_any_device_work(lib):
+    """Lazy-row calls: argument and call-order errors before the GPU is touched."""
+    sb, so = W.pack([b"ab"])
+    h = T.trie_build(sb, so)
+    L = lib
+    vo = np.array([0, 1, 1], np.int64)
+    vb = np.frombuffer(b"a", np.uint8).copy()
+    assert L.trie_lazy_apply(h.handle, 16, 0, 16, 1, 2, None) == T.TRIE_ESTATE
+    assert L.trie_lazy_advance_apply(h.handle, 16, 16, 32, None, 16, 0, 1, 2, None) == T.TRIE_ESTATE
+    assert L.trie_lazy_rows(h.handle, 16, 1, 16, None) == T.TRIE_ESTATE
+    assert L.trie_lazy_stats(h.handle, None, None) == T.TRIE_ESTATE
+    assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 1, 8, 8) == T.TRIE_EINVAL       # V < 2
+    assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 600000, 8, 8) == T.TRIE_EINVAL  # V too big
+    assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, -1, 8) == T.TRIE_EINVAL      # cache_rows
+    assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, 8, 0) == T.TRIE_EINVAL       # max_batch
+    assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, 8, 4097) == T.TRIE_EINVAL
+    assert L.trie_lazy_init(h.handle, vb.ctypes.data, None, 2, 8, 8) == T.TRIE_EINVAL
+    for f, args in (("trie_lazy_init", (None, None, 2, 8, 8)), ("trie_lazy_apply", (16, 0, 16, 1, 2, None)),
+                    ("trie_lazy_rows", (16, 1, 16, None)), ("trie_lazy_stats", (None, None))):
+        assert getattr(L, f)(None, *args) == T.TRIE_EINVAL
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     import importlib
     mod = importlib.import_module("paper_2608_12574_gb300.triemask")
