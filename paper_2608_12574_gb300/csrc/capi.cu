@@ -605,10 +605,12 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
     const size_t o_mnode = lay.add(sizeof(int32_t) * mb);
     const size_t o_mslot = lay.add(sizeof(int32_t) * mb);
     const size_t o_rowu = lay.add(sizeof(int32_t) * mb);
+    const size_t o_task = lay.add(sizeof(int4) * (mb + size_t(tmk::kLazySplitRows) * tmk::kLazyMaxParts));
     const size_t o_pnode = lay.add(sizeof(int32_t) * n);
     const size_t o_pdep = lay.add(sizeof(int32_t) * n);
     const size_t o_psize = lay.add(sizeof(int32_t) * n);
     const size_t o_pos = lay.add(sizeof(int32_t) * n);
+    const size_t o_pre = lay.add(sizeof(tmk::LazyNode) * n);
     void *base = nullptr;
     e = cudaMalloc(&base, lay.total);
     if (e != cudaSuccess) {
@@ -630,11 +632,13 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
     L.miss_node = reinterpret_cast<int32_t *>(b + o_mnode);
     L.miss_slot = reinterpret_cast<int32_t *>(b + o_mslot);
     L.row_u = reinterpret_cast<int32_t *>(b + o_rowu);
+    L.task = reinterpret_cast<int4 *>(b + o_task);
     L.pre_node = reinterpret_cast<int32_t *>(b + o_pnode);
     L.pre_depth = reinterpret_cast<int32_t *>(b + o_pdep);
     L.pre_size = reinterpret_cast<int32_t *>(b + o_psize);
     L.pos_of = reinterpret_cast<int32_t *>(b + o_pos);
-    const tmk::LazyCtrl ctrl0 = {1u, 0, 0ull, 0ull};
+    L.pre = reinterpret_cast<tmk::LazyNode *>(b + o_pre);
+    const tmk::LazyCtrl ctrl0 = {1u, 0, 0, 0, 0ull, 0ull};
     const tmk::HostTrie &t = h->host;
     if ((e = cudaMemset(L.tag, 0xFF, sizeof(int32_t) * size_t(C))) != cudaSuccess ||
         (e = cudaMemset(L.stamp, 0, sizeof(uint32_t) * size_t(C))) != cudaSuccess ||
@@ -645,7 +649,7 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
             cudaSuccess ||
         (e = cudaMemcpy(L.pre_size, t.pre_size.data(), sizeof(int32_t) * n, cudaMemcpyHostToDevice)) !=
             cudaSuccess ||
-        (e = tmk::launch_lazy_tables(L, h->host.n, 0)) != cudaSuccess || (e = cudaDeviceSynchronize()) != cudaSuccess) {
+        (e = tmk::launch_lazy_tables(h->dev, L, h->host.n, 0)) != cudaSuccess || (e = cudaDeviceSynchronize()) != cudaSuccess) {
         cudaFree(base);
         L = tmk::DevLazy();
         return fail_cuda(e, "lazy-row set-up");

@@ -360,6 +360,45 @@ __global__ void __launch_bounds__(kTableThreads) k_trie_tables(const int32_t *__
     }
 }
 
+// Slot of each key of a batch in the paired-slot table, -1 if absent, for
+// vocabularies in which no two tokens share a key (so a key is stored at
+// most once). f holds each key's first pair, already loaded. The keys of the
+// batch advance together: each round checks every pending key's current pair
+// and loads the next pair of those still pending (a full pair without the
+// key); a pair that is not full ends the chain. The table is at most a
+// quarter full, so every chain ends.
+template <int G>
+__device__ __forceinline__ void find_slots(const PatchArgs &a, const uint64_t (&key)[G], uint32_t pending,
+                                           ulonglong2 (&f)[G], int32_t (&slot)[G]) {
+    const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
+    uint32_t pr[G];
+#pragma unroll
+    for (int g = 0; g < G; g++) {
+        pr[g] = uint32_t(key[g] >> 1) & a.pairs_mask;
+        slot[g] = -1;
+    }
+    for (uint32_t it = 0; pending && it <= a.pairs_mask; it++) {
+#pragma unroll
+        for (int g = 0; g < G; g++) {
+            if (!((pending >> g) & 1u)) continue;
+            if (f[g].x == key[g]) {
+                slot[g] = int32_t(2 * pr[g]);
+                pending &= ~(1u << g);
+            } else if (f[g].y == key[g]) {
+                slot[g] = int32_t(2 * pr[g] + 1);
+                pending &= ~(1u << g);
+            } else if (f[g].y == 0ull) {
+                pending &= ~(1u << g);
+            } else {
+                pr[g] = (pr[g] + 1u) & a.pairs_mask;
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < G; g++)
+            if ((pending >> g) & 1u) f[g] = __ldg(pairs + pr[g]);
+    }
+}
+
 // Element k of a register copy of 16 ancestors, without dynamic indexing.
 __device__ __forceinline__ int32_t anc_at(const int4 (&an)[4], int k) {
     const int4 q = k < 4 ? an[0] : (k < 8 ? an[1] : (k < 12 ? an[2] : an[3]));
@@ -371,9 +410,10 @@ __device__ __forceinline__ int32_t anc_at(const int4 (&an)[4], int k) {
 // of loads gives every suffix of length <= 16 and every start row. The 8
 // suffixes of a batch are resolved as a wavefront: the first slot pair of all
 // 8 keys, then the token ids of the matches, their lengths and offsets, then
-// their bytes, each round issued for all candidates before any is used. A key
-// that may sit in a later pair (its first pair is full and does not hold it,
-// or some tokens share keys) takes the sequential probe.
+// their bytes, each round issued for all candidates before any is used; keys
+// not in their first pair follow their chains together (find_slots). In a
+// vocabulary where some tokens share a key, a key whose first pair is full
+// takes the sequential probe, which finds every token under it.
 template <typename Emit>
 __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, Emit emit) {
     const ulonglong2 win = __ldg(a.window + m);
@@ -402,16 +442,24 @@ __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, 
                     first[i] = __ldg(pairs + (uint32_t(key[i] >> 1) & a.pairs_mask));
                 }
             }
-            int32_t slot[8];  // slot of the key in its first pair, -1 none
+            int32_t slot[8];  // slot of the key, -1 none
             uint32_t slow = 0;  // bit i: candidate i needs the sequential probe
+            if (!a.dup_keys) {
+                uint32_t pending = 0;
 #pragma unroll
-            for (int i = 0; i < 8; i++) {
-                const bool m0 = first[i].x == key[i], m1 = first[i].y == key[i];
-                const uint32_t pr = uint32_t(key[i] >> 1) & a.pairs_mask;
-                slot[i] = (k0 + i < depth && (m0 || m1)) ? int32_t(2 * pr + (m0 ? 0 : 1)) : -1;
-                if (k0 + i < depth && first[i].y != 0ull && (!(m0 || m1) || a.dup_keys)) {
-                    slow |= 1u << i;
-                    slot[i] = -1;
+                for (int i = 0; i < 8; i++)
+                    if (k0 + i < depth) pending |= 1u << i;
+                find_slots<8>(a, key, pending, first, slot);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 8; i++) {
+                    const bool m0 = first[i].x == key[i], m1 = first[i].y == key[i];
+                    const uint32_t pr = uint32_t(key[i] >> 1) & a.pairs_mask;
+                    slot[i] = (k0 + i < depth && (m0 || m1)) ? int32_t(2 * pr + (m0 ? 0 : 1)) : -1;
+                    if (k0 + i < depth && first[i].y != 0ull) {
+                        slow |= 1u << i;
+                        slot[i] = -1;
+                    }
                 }
             }
             int32_t tid[8];
@@ -962,7 +1010,8 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_scalar(void *__restrict
 //                   missing nodes get the least recently used row of their
 //                   set (or a per-call row when every row of the set is in use
 //                   by this call);
-//   k_lazy_rows     one CTA per missing node s: valid[s] from s's subtree;
+//   k_lazy_rows     one CTA per task: valid[s] of a missing node s from s's
+//                   subtree, or one part of it for a large subtree;
 //   apply (k_apply_vec on the cache rows) or k_lazy_gather.
 
 struct LazyArgs {
@@ -974,10 +1023,12 @@ struct LazyArgs {
     int32_t *miss_node;
     int32_t *miss_slot;
     int32_t *row_u;
+    int4 *task;
     const int32_t *pre_node;
     const int32_t *pre_depth;
     const int32_t *pre_size;
     const int32_t *pos_of;
+    const LazyNode *pre;
     int32_t C;        // cache rows
     int32_t n_sets;   // C / kLazyWays
     int32_t n_nodes;
@@ -986,7 +1037,7 @@ struct LazyArgs {
 };
 
 constexpr int kResolveThreads = 1024;
-constexpr int kLazyRowThreads = 512;
+constexpr int kLazyRowThreads = 256;
 constexpr int32_t kPending = -3;
 
 __device__ __forceinline__ uint32_t mix32(uint32_t x) {
@@ -1013,11 +1064,14 @@ __global__ void __launch_bounds__(kResolveThreads) k_lazy_resolve(LazyArgs L, Ad
     extern __shared__ int32_t sh[];  // [uniq] node keys, [uniq] their miss index
     int32_t *keys = sh;
     int32_t *vals = sh + L.uniq;
-    __shared__ int32_t n_u;
+    __shared__ int32_t n_u, n_tasks, n_split;
+    __shared__ int32_t split_slot[kLazySplitRows];
     __shared__ unsigned long long n_hit, n_miss_rows;
     for (int32_t i = threadIdx.x; i < L.uniq; i += blockDim.x) keys[i] = -1;
     if (threadIdx.x == 0) {
         n_u = 0;
+        n_tasks = 0;
+        n_split = 0;
         n_hit = 0ull;
         n_miss_rows = 0ull;
     }
@@ -1102,13 +1156,34 @@ __global__ void __launch_bounds__(kResolveThreads) k_lazy_resolve(LazyArgs L, Ad
             }
         }
         L.miss_slot[u] = slot;
+        // CTA tasks: one, or up to kLazyMaxParts for a large subtree (for the
+        // first kLazySplitRows such rows of the call)
+        const int32_t desc = __ldg(L.pre_size + __ldg(L.pos_of + s)) - 1;
+        int32_t parts = 1;
+        if (desc > kLazyPartNodes) {
+            const int32_t i = atomicAdd(&n_split, 1);
+            if (i < kLazySplitRows) {
+                parts = (desc + kLazyPartNodes - 1) / kLazyPartNodes;
+                parts = parts < kLazyMaxParts ? parts : kLazyMaxParts;
+                split_slot[i] = slot;
+            }
+        }
+        const int32_t t0 = atomicAdd(&n_tasks, parts);
+        for (int32_t p = 0; p < parts; p++) L.task[t0 + p] = make_int4(u, p, parts, 0);
     }
     __syncthreads();
+    // rows built in parts are ORed together by atomics: zero them first
+    const int32_t n_zero = n_split < kLazySplitRows ? n_split : kLazySplitRows;
+    for (int32_t r = 0; r < n_zero; r++) {
+        uint32_t *row = L.rows + int64_t(split_slot[r]) * L.W;
+        for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x) row[i] = 0u;
+    }
     // 4. batch rows of missing nodes
     for (int32_t b = threadIdx.x; b < B; b += blockDim.x)
         if (L.slot_of[b] == kPending) L.slot_of[b] = L.miss_slot[vals[L.row_u[b]]];
     if (threadIdx.x == 0) {
         L.ctrl->n_miss = n_u;
+        L.ctrl->n_tasks = n_tasks;
         L.ctrl->now = now + 1u;
         L.ctrl->hits += n_hit;
         L.ctrl->misses += n_miss_rows;
@@ -1121,50 +1196,136 @@ __global__ void __launch_bounds__(kResolveThreads) k_lazy_resolve(LazyArgs L, Ad
 // and EOS if s is terminal. The subtree is one interval of the pre-order
 // tables; a descendant d at depth j below s (1 <= j <= the longest token)
 // contributes the token, if any, whose bytes are the last j edge labels into
-// d. The row is built in shared memory, then stored.
-__global__ void __launch_bounds__(kLazyRowThreads) k_lazy_rows(LazyArgs L, PatchArgs a) {
+// d. A CTA builds the row (or, for a subtree split into parts, the part of it
+// from its share of the interval) in shared memory, then stores it (a part
+// ORs its non-zero words into the row, which the resolve has zeroed).
+// B^j mod 2^64 by squaring.
+__device__ __forceinline__ uint64_t hash_pow(uint32_t j) {
+    uint64_t r = 1, b = kHashBase;
+    while (j) {
+        if (j & 1u) r *= b;
+        b *= b;
+        j >>= 1;
+    }
+    return r;
+}
+
+constexpr int kLazyNodesPerThread = 4;  // descendants resolved together by one thread
+
+__global__ void __launch_bounds__(kLazyRowThreads, 2) k_lazy_rows(LazyArgs L, PatchArgs a) {
     extern __shared__ uint32_t bits[];
     pdl_launch_dependents();
-    pdl_wait();  // the resolve's miss list
-    const int32_t n_miss = __ldcg(&L.ctrl->n_miss);
-    for (int32_t u = blockIdx.x; u < n_miss; u += gridDim.x) {
-        const int32_t s = L.miss_node[u];
-        const int32_t slot = L.miss_slot[u];
+    pdl_wait();  // the resolve's task list
+    const int32_t n_tasks = __ldcg(&L.ctrl->n_tasks);
+    const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
+    for (int32_t ti = blockIdx.x; ti < n_tasks; ti += gridDim.x) {
+        const int4 tk = __ldcg(L.task + ti);  // {miss, part, parts, -}
+        const int32_t s = L.miss_node[tk.x];
         for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x) bits[i] = 0u;
         __syncthreads();
-        if (threadIdx.x == 0 && __ldg(a.terminal + s)) atomicOr(bits + (a.eos >> 5), 1u << (a.eos & 31));
+        if (threadIdx.x == 0 && tk.y == 0 && __ldg(a.terminal + s)) atomicOr(bits + (a.eos >> 5), 1u << (a.eos & 31));
         const int32_t pos = __ldg(L.pos_of + s);
-        const int32_t end = pos + __ldg(L.pre_size + pos);
-        const int32_t d0 = __ldg(L.pre_depth + pos);
-        for (int32_t k = pos + 1 + int32_t(threadIdx.x); k < end; k += blockDim.x) {
-            const int32_t j = __ldg(L.pre_depth + k) - d0;
-            if (j > a.lmax) continue;
-            const int32_t d = __ldg(L.pre_node + k);
-            auto hit = [&](int32_t t) { atomicOr(bits + (t >> 5), 1u << (t & 31)); };
-            uint64_t h = 0, pw = 1;
-            if (j <= kMaxClimb) {
-                const ulonglong2 win = __ldg(a.window + d);
-                const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y),
-                                         uint32_t(win.y >> 32)};
-                for (int32_t i = 0; i < j; i++) {  // byte i levels above d
-                    h += (uint64_t(byte_at(lab, i)) + 1ull) * pw;
-                    pw *= kHashBase;
+        const int32_t desc = __ldg(L.pre_size + pos) - 1;
+        const int32_t k0 = pos + 1 + int32_t(int64_t(desc) * tk.y / tk.z);
+        const int32_t k1 = pos + 1 + int32_t(int64_t(desc) * (tk.y + 1) / tk.z);
+        const ulonglong2 *rec = reinterpret_cast<const ulonglong2 *>(L.pre);  // 2 per record
+        const ulonglong2 sh0 = __ldg(rec + 2 * int64_t(pos));
+        const uint64_t ps = sh0.x;
+        const int32_t d0 = int32_t(uint32_t(sh0.y));
+        for (int32_t kb = k0 + int32_t(threadIdx.x); kb < k1; kb += kLazyNodesPerThread * blockDim.x) {
+            int32_t d[kLazyNodesPerThread], j[kLazyNodesPerThread];
+            uint64_t pd[kLazyNodesPerThread];
+            uint32_t lab[kLazyNodesPerThread][4];
+#pragma unroll
+            for (int g = 0; g < kLazyNodesPerThread; g++) {
+                const int32_t k = kb + g * int32_t(blockDim.x);
+                ulonglong2 r0 = make_ulonglong2(0ull, 0ull), r1 = make_ulonglong2(0ull, 0ull);
+                if (k < k1) {
+                    r0 = __ldg(rec + 2 * int64_t(k));
+                    r1 = __ldg(rec + 2 * int64_t(k) + 1);
                 }
-                probe(a, hash_finish(h, uint32_t(j)), j, &lab, d, hit);
+                pd[g] = r0.x;
+                j[g] = k < k1 ? int32_t(uint32_t(r0.y)) - d0 : 0;
+                d[g] = int32_t(uint32_t(r0.y >> 32));
+                if (j[g] > a.lmax) j[g] = 0;  // no token is this long
+                lab[g][0] = uint32_t(r1.x);
+                lab[g][1] = uint32_t(r1.x >> 32);
+                lab[g][2] = uint32_t(r1.y);
+                lab[g][3] = uint32_t(r1.y >> 32);
+            }
+            uint64_t key[kLazyNodesPerThread];
+            ulonglong2 f[kLazyNodesPerThread];
+#pragma unroll
+            for (int g = 0; g < kLazyNodesPerThread; g++) {
+                key[g] = hash_finish(pd[g] - ps * hash_pow(uint32_t(j[g])), uint32_t(j[g]));
+                f[g] = j[g] > 0 ? __ldg(pairs + (uint32_t(key[g] >> 1) & a.pairs_mask)) : make_ulonglong2(0ull, 0ull);
+            }
+            // keys are resolved together (find_slots); paths longer than the
+            // label window, and full first pairs in a vocabulary where tokens
+            // share keys, take the sequential probe
+            int32_t slot[kLazyNodesPerThread];
+            uint32_t slow = 0;
+            if (!a.dup_keys) {
+                uint32_t pending = 0;
+#pragma unroll
+                for (int g = 0; g < kLazyNodesPerThread; g++) {
+                    if (j[g] > kMaxClimb) slow |= 1u << g;
+                    else if (j[g] > 0) pending |= 1u << g;
+                }
+                find_slots<kLazyNodesPerThread>(a, key, pending, f, slot);
             } else {
-                int32_t y = d;
-                for (int32_t i = 0; i < j; i++) {
-                    h += (uint64_t(__ldg(a.label + y)) + 1ull) * pw;
-                    pw *= kHashBase;
-                    y = __ldg(a.parent + y);
+#pragma unroll
+                for (int g = 0; g < kLazyNodesPerThread; g++) {
+                    const bool m0 = f[g].x == key[g], m1 = f[g].y == key[g];
+                    const uint32_t pr = uint32_t(key[g] >> 1) & a.pairs_mask;
+                    slot[g] = -1;
+                    if (j[g] > 0) {
+                        if (j[g] > kMaxClimb || f[g].y != 0ull) slow |= 1u << g;
+                        else if (m0 || m1) slot[g] = int32_t(2 * pr + (m0 ? 0 : 1));
+                    }
                 }
-                probe(a, hash_finish(h, uint32_t(j)), j, nullptr, d, hit);
+            }
+            int32_t tid[kLazyNodesPerThread];
+#pragma unroll
+            for (int g = 0; g < kLazyNodesPerThread; g++) tid[g] = slot[g] >= 0 ? __ldg(a.ht_val + slot[g]) : -1;
+            int32_t tlen[kLazyNodesPerThread];
+            uint32_t toff[kLazyNodesPerThread];
+#pragma unroll
+            for (int g = 0; g < kLazyNodesPerThread; g++) {
+                tlen[g] = tid[g] >= 0 ? int32_t(__ldg(a.tok_len + tid[g])) : -1;
+                toff[g] = tid[g] >= 0 ? __ldg(a.tok_off + tid[g]) : 0u;
+            }
+            uint4 tb[kLazyNodesPerThread];
+#pragma unroll
+            for (int g = 0; g < kLazyNodesPerThread; g++)
+                tb[g] = tlen[g] == j[g] ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[g]))
+                                        : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int g = 0; g < kLazyNodesPerThread; g++) {
+                auto hit = [&](int32_t t) { atomicOr(bits + (t >> 5), 1u << (t & 31)); };
+                if (slow & (1u << g)) {
+                    if (j[g] > kMaxClimb) probe(a, key[g], j[g], nullptr, d[g], hit);
+                    else probe(a, key[g], j[g], &lab[g], d[g], hit);
+                } else if (tid[g] >= 0 && tlen[g] == j[g]) {
+                    // token byte i must equal the label j-1-i levels above d
+                    const uint32_t tw[4] = {tb[g].x, tb[g].y, tb[g].z, tb[g].w};
+                    bool eq = true;
+#pragma unroll
+                    for (int i = 0; i < kMaxClimb; i++)
+                        if (i < j[g]) eq = eq && byte_at(tw, i) == byte_at(lab[g], j[g] - 1 - i);
+                    if (eq) hit(tid[g]);
+                }
             }
         }
         __syncthreads();
-        uint32_t *row = L.rows + int64_t(slot) * L.W;
-        for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x) row[i] = bits[i];
-        __syncthreads();  // bits are reused by the next node
+        uint32_t *row = L.rows + int64_t(L.miss_slot[tk.x]) * L.W;
+        if (tk.z == 1) {
+            for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x) row[i] = bits[i];
+        } else {
+            for (int64_t i = threadIdx.x; i < L.W; i += blockDim.x)
+                if (bits[i]) atomicOr(row + i, bits[i]);
+        }
+        __syncthreads();  // bits are reused by the next task
     }
 }
 
@@ -1183,11 +1344,33 @@ __global__ void __launch_bounds__(kApplyThreads) k_lazy_gather(const uint32_t *_
     }
 }
 
-// pos_of[pre_node[k]] = k.
-__global__ void k_lazy_tables(const int32_t *__restrict__ pre_node, int32_t n, int32_t *__restrict__ pos_of) {
-    for (int32_t k = blockIdx.x * blockDim.x + threadIdx.x; k < n; k += gridDim.x * blockDim.x)
-        pos_of[pre_node[k]] = k;
+// The pre-order records of the lazy rows: for position k, node d =
+// pre_node[k], pos_of[d] = k, d's depth and label window, and the path hash
+// of d: the Horner polynomial of the token table's hash over (label + 1) of
+// the edges from the root to d, P(d) = P(parent) * B + label(d) + 1
+// (mod 2^64), summed here by climbing to the root. The path from s down to a
+// descendant d, j edges long, then hashes to P(d) - P(s) * B^j.
+__global__ void k_lazy_tables(const int32_t *__restrict__ pre_node, const int32_t *__restrict__ pre_depth,
+                              const int32_t *__restrict__ parent, const uint8_t *__restrict__ label,
+                              const ulonglong2 *__restrict__ window, int32_t n, int32_t *__restrict__ pos_of,
+                              LazyNode *__restrict__ pre) {
+    for (int32_t k = blockIdx.x * blockDim.x + threadIdx.x; k < n; k += gridDim.x * blockDim.x) {
+        const int32_t d = pre_node[k];
+        pos_of[d] = k;
+        uint64_t h = 0, pw = 1;
+        for (int32_t y = d; __ldg(parent + y) >= 0; y = __ldg(parent + y)) {
+            h += (uint64_t(__ldg(label + y)) + 1ull) * pw;
+            pw *= kHashBase;
+        }
+        LazyNode r;
+        r.phash = h;
+        r.depth = pre_depth[k];
+        r.node = d;
+        r.window = window[d];
+        pre[k] = r;
+    }
 }
+
 
 PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax, uint32_t *mask,
                      int64_t W) {
@@ -1424,7 +1607,7 @@ cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const
                       n_nodes, parts);
 }
 
-cudaError_t launch_lazy_tables(const DevLazy &L, int32_t n_nodes, cudaStream_t st) {
+cudaError_t launch_lazy_tables(const DevTrie &t, const DevLazy &L, int32_t n_nodes, cudaStream_t st) {
     // shared memory above the default 48 KB: the resolve's table of distinct
     // nodes (<= 2 * 2 * kLazyMaxBatch int32) and the row kernel's row
     const int uniq_max = int(2 * 2 * kLazyMaxBatch * sizeof(int32_t));
@@ -1441,7 +1624,8 @@ cudaError_t launch_lazy_tables(const DevLazy &L, int32_t n_nodes, cudaStream_t s
         return e;
     if (n_nodes <= 0) return cudaSuccess;
     const int grid = grid_for(n_nodes, 256, 4096);
-    k_lazy_tables<<<grid, 256, 0, st>>>(L.pre_node, n_nodes, L.pos_of);
+    k_lazy_tables<<<grid, 256, 0, st>>>(L.pre_node, L.pre_depth, t.parent, t.label, t.window, n_nodes, L.pos_of,
+                                        L.pre);
     return cudaGetLastError();
 }
 
@@ -1458,10 +1642,12 @@ cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bo
     la.miss_node = L.miss_node;
     la.miss_slot = L.miss_slot;
     la.row_u = L.row_u;
+    la.task = L.task;
     la.pre_node = L.pre_node;
     la.pre_depth = L.pre_depth;
     la.pre_size = L.pre_size;
     la.pos_of = L.pos_of;
+    la.pre = L.pre;
     la.C = L.C;
     la.n_sets = L.C / kLazyWays;
     la.n_nodes = n_nodes;
@@ -1477,7 +1663,9 @@ cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bo
                                              states_in, tokens, states_out, err, B);
     if (e != cudaSuccess) return e;
     const PatchArgs pa = patch_args(t, n_nodes, v, lmax, nullptr, L.W);
-    e = launch_pdl_smem(k_lazy_rows, B, kLazyRowThreads, size_t(L.W) * sizeof(uint32_t), st, la, pa);
+    // tasks in a grid-stride loop over two CTAs per SM
+    const int rows_grid = grid_for(int64_t(B) + int64_t(kLazySplitRows) * kLazyMaxParts, 1, int64_t(num_sms) * 2);
+    e = launch_pdl_smem(k_lazy_rows, rows_grid, kLazyRowThreads, size_t(L.W) * sizeof(uint32_t), st, la, pa);
     if (e != cudaSuccess) return e;
     const int32_t n_rows = L.C + L.max_batch;
     if (logits) return launch_apply(logits, dtype, L.rows, L.slot_of, B, L.V, n_rows, num_sms, st);

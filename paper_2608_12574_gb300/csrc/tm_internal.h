@@ -163,12 +163,30 @@ struct DevLists {
 constexpr int kLazyWays = 8;       // rows per cache set
 constexpr int kLazyMaxBatch = 4096;
 constexpr int64_t kLazyMaxWords = 16384;  // row built in shared memory (64 KB): V <= 524,288
+// A missing row whose subtree has more than kLazyPartNodes nodes is computed
+// in parts by several CTAs (at most kLazyMaxParts per row), for at most
+// kLazySplitRows rows per call (splitting only pays while few rows are
+// missing; with many the grid is full anyway).
+constexpr int32_t kLazyPartNodes = 1024;
+constexpr int32_t kLazyMaxParts = 64;
+constexpr int32_t kLazySplitRows = 16;
 
 struct LazyCtrl {
     uint32_t now;                   // call counter (stamps of rows used by this call)
     int32_t n_miss;                 // rows computed by the current call
+    int32_t n_tasks;                // CTA tasks of the current call (parts of rows)
+    int32_t pad;
     unsigned long long hits;        // batch rows whose node row was cached
     unsigned long long misses;      // batch rows whose node row was computed
+};
+
+// One node of the depth-first pre-order, as the lazy-row kernel reads it (a
+// subtree is a contiguous run of these, 32 bytes each).
+struct LazyNode {
+    uint64_t phash;      // Horner hash of the path from the root (unfinished)
+    int32_t depth;
+    int32_t node;        // breadth-first id
+    ulonglong2 window;   // labels of the last 16 edges into the node
 };
 
 struct DevLazy {
@@ -187,10 +205,12 @@ struct DevLazy {
     int32_t *miss_node = nullptr;   // [max_batch] nodes whose rows the call computes
     int32_t *miss_slot = nullptr;   // [max_batch] where
     int32_t *row_u = nullptr;       // [max_batch] scratch
+    int4 *task = nullptr;           // [max_batch + kLazySplitRows * kLazyMaxParts] {miss, part, parts, -}
     int32_t *pre_node = nullptr;    // [n] pre-order tables of the trie (HostTrie)
     int32_t *pre_depth = nullptr;   // [n]
     int32_t *pre_size = nullptr;    // [n]
     int32_t *pos_of = nullptr;      // [n] pre-order position of each node
+    LazyNode *pre = nullptr;        // [n] by pre-order position
 };
 
 }  // namespace tmk
@@ -241,8 +261,8 @@ cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab
                                const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total);
 cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  const DevLists &L, int num_sms, cudaStream_t st);
-// Lazy rows: pos_of from the pre-order tables (once, at set-up).
-cudaError_t launch_lazy_tables(const DevLazy &L, int32_t n_nodes, cudaStream_t st);
+// Lazy rows: pos_of from the pre-order tables and the path hashes (once, at set-up).
+cudaError_t launch_lazy_tables(const DevTrie &t, const DevLazy &L, int32_t n_nodes, cudaStream_t st);
 // One lazy call: map the batch's states (after the advance when tokens is not
 // null) to cache rows, compute the missing rows, then apply them to the
 // logits (logits not null) or copy them out (rows_out not null).
