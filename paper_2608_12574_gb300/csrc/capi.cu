@@ -216,13 +216,19 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     return TRIE_OK;
 }
 
-// The transition table holds the transitions of one vocabulary: when a
-// compile uses another, clear it and let this compile's probe refill it.
-int prepare_trans(trie_t h, const tmk::DevVocab *voc, int sms, cudaStream_t stream, bool *fill) {
+// The transition table holds transitions of one vocabulary: when a compile
+// uses another, clear it and let this compile's probe refill it; when it
+// holds only the entries lazy rows added, let the compile complete it.
+int prepare_trans(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, int sms, cudaStream_t stream, bool *fill) {
     std::lock_guard<std::mutex> lk(h->mu);
     *fill = false;
-    if (!h->dev.trans || h->trans_vocab == voc) return TRIE_OK;
-    h->trans_vocab = nullptr;
+    if (!h->dev.trans) return TRIE_OK;
+    if (h->trans_vocab == voc) {
+        *fill = !h->trans_complete;
+        return TRIE_OK;
+    }
+    h->trans_vocab.reset();
+    h->trans_complete = false;
     cudaError_t e = tmk::launch_trans_clear(h->dev, sms, stream);
     if (e != cudaSuccess) return fail_cuda(e, "transition table clear");
     *fill = true;
@@ -268,13 +274,14 @@ int lazy_call(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int
     int dev, rc;
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     if (dev != L.device || dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
-    bool use_trans;
+    bool use_trans, fill_trans;
     {
         std::lock_guard<std::mutex> lk(h->mu);
-        use_trans = h->trans_vocab == L.vocab.get();
+        use_trans = h->trans_vocab == L.vocab;
+        fill_trans = use_trans && !h->trans_complete;  // record the moves the rows find
     }
     const int32_t lmax = std::min(L.vocab->max_len, h->host.max_depth);
-    cudaError_t e = tmk::launch_lazy(h->dev, h->host.n, *L.vocab, use_trans, lmax, L, d_states_in, d_tokens,
+    cudaError_t e = tmk::launch_lazy(h->dev, h->host.n, *L.vocab, use_trans, fill_trans, lmax, L, d_states_in, d_tokens,
                                      d_states_out, d_err, B, d_logits, dtype, d_rows, num_sms(dev), stream);
     if (e != cudaSuccess) return fail_cuda(e, "lazy-row launch");
     return TRIE_OK;
@@ -379,11 +386,12 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
     bool fill_trans;
-    if ((rc = prepare_trans(h, voc.get(), sms, stream, &fill_trans)) != TRIE_OK) return rc;
+    if ((rc = prepare_trans(h, voc, sms, stream, &fill_trans)) != TRIE_OK) return rc;
     cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, fill_trans, stream);
     if (e != cudaSuccess) return fail_cuda(e, "mask compile launch");
     std::lock_guard<std::mutex> lk(h->mu);
-    h->trans_vocab = voc.get();
+    h->trans_vocab = voc;
+    h->trans_complete = h->trans_complete || fill_trans;
     h->vocab = voc;
     h->mask = d_mask;
     h->mask_V = V;
@@ -400,7 +408,7 @@ int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B
     {
         std::lock_guard<std::mutex> lk(h->mu);
         voc = h->vocab;
-        use_trans = h->trans_vocab == voc.get();
+        use_trans = h->trans_vocab == voc;
     }
     if (!voc) return fail(TRIE_ESTATE, "trie_advance before trie_compile_masks on this handle");
     if (B == 0) return TRIE_OK;
@@ -431,7 +439,7 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
         voc = h->vocab;
         mask = h->mask;
         mV = h->mask_V;
-        use_trans = h->trans_vocab == voc.get();
+        use_trans = h->trans_vocab == voc;
     }
     if (!mask || !voc) return fail(TRIE_ESTATE, "trie_advance_apply before trie_compile_masks on this handle");
     if (V != mV || V != voc->V) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
@@ -509,7 +517,7 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     const int sms = num_sms(dev);
     int64_t total = 0;
     bool fill_trans;
-    if ((rc = prepare_trans(h, voc.get(), sms, stream, &fill_trans)) != TRIE_OK) return rc;
+    if ((rc = prepare_trans(h, voc, sms, stream, &fill_trans)) != TRIE_OK) return rc;
     cudaError_t e = tmk::launch_lists_count(h->dev, n, *voc, lmax, L, sms, fill_trans, stream, &total);
     if (e != cudaSuccess) return fail_cuda(e, "valid-list count");
     if (total > L.tok_cap) {  // grow the token buffer (by at least half)
@@ -531,7 +539,8 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     std::lock_guard<std::mutex> lk(h->mu);
     L.n_valid = total;
     L.V = V;
-    h->trans_vocab = voc.get();
+    h->trans_vocab = voc;
+    h->trans_complete = h->trans_complete || fill_trans;
     h->vocab = voc;
     return TRIE_OK;
 }
@@ -590,6 +599,16 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
     if ((rc = ensure_device_trie(h, dev, 0)) != TRIE_OK) return rc;
     cudaError_t e = cudaDeviceSynchronize();  // earlier lazy calls may still use the old cache
     if (e != cudaSuccess) return fail_cuda(e, "synchronising before the lazy set-up");
+    {  // the transition table takes the moves the lazy rows find for this vocabulary
+        std::lock_guard<std::mutex> lk(h->mu);
+        if (h->dev.trans && h->trans_vocab != voc) {
+            h->trans_vocab.reset();
+            h->trans_complete = false;
+            if ((e = tmk::launch_trans_clear(h->dev, num_sms(dev), 0)) != cudaSuccess)
+                return fail_cuda(e, "transition table clear");
+            h->trans_vocab = voc;
+        }
+    }
     tmk::DevLazy &L = h->lazy;
     if (L.base) cudaFree(L.base);
     L = tmk::DevLazy();

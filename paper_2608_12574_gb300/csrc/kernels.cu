@@ -1302,7 +1302,11 @@ __global__ void __launch_bounds__(kLazyRowThreads, 2) k_lazy_rows(LazyArgs L, Pa
                                         : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
             for (int g = 0; g < kLazyNodesPerThread; g++) {
-                auto hit = [&](int32_t t) { atomicOr(bits + (t >> 5), 1u << (t & 31)); };
+                // token t moves s to d: its bit, and the move for later advances
+                auto hit = [&](int32_t t) {
+                    atomicOr(bits + (t >> 5), 1u << (t & 31));
+                    if (a.trans_fill) trans_insert(a.trans, a.trans_mask, s, t, d[g]);
+                };
                 if (slow & (1u << g)) {
                     if (j[g] > kMaxClimb) probe(a, key[g], j[g], nullptr, d[g], hit);
                     else probe(a, key[g], j[g], &lab[g], d[g], hit);
@@ -1629,7 +1633,8 @@ cudaError_t launch_lazy_tables(const DevTrie &t, const DevLazy &L, int32_t n_nod
     return cudaGetLastError();
 }
 
-cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans, int32_t lmax,
+cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans, bool fill_trans,
+                        int32_t lmax,
                         const DevLazy &L, const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                         int32_t *err, int32_t B, void *logits, int dtype, uint32_t *rows_out, int num_sms,
                         cudaStream_t st) {
@@ -1662,7 +1667,8 @@ cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bo
                            : launch_pdl_smem(k_lazy_resolve<false>, 1, kResolveThreads, rsmem, st, la, aa,
                                              states_in, tokens, states_out, err, B);
     if (e != cudaSuccess) return e;
-    const PatchArgs pa = patch_args(t, n_nodes, v, lmax, nullptr, L.W);
+    PatchArgs pa = patch_args(t, n_nodes, v, lmax, nullptr, L.W);
+    pa.trans_fill = fill_trans && t.trans;
     // tasks in a grid-stride loop over two CTAs per SM
     const int rows_grid = grid_for(int64_t(B) + int64_t(kLazySplitRows) * kLazyMaxParts, 1, int64_t(num_sms) * 2);
     e = launch_pdl_smem(k_lazy_rows, rows_grid, kLazyRowThreads, size_t(L.W) * sizeof(uint32_t), st, la, pa);

@@ -224,7 +224,8 @@ struct trie_s {
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
     int32_t mask_V = 0;
     tmk::DevLists lists;                 // last compiled valid lists (library-owned)
-    const tmk::DevVocab *trans_vocab = nullptr;  // vocabulary the transition table holds
+    std::shared_ptr<tmk::DevVocab> trans_vocab;  // vocabulary the transition table holds
+    bool trans_complete = false;         // filled by a whole compile (else partly, by lazy rows)
     tmk::DevLazy lazy;                   // lazy-row cache (trie_lazy_init)
 };
 
@@ -266,7 +267,8 @@ cudaError_t launch_lazy_tables(const DevTrie &t, const DevLazy &L, int32_t n_nod
 // One lazy call: map the batch's states (after the advance when tokens is not
 // null) to cache rows, compute the missing rows, then apply them to the
 // logits (logits not null) or copy them out (rows_out not null).
-cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans, int32_t lmax,
+cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans, bool fill_trans,
+                        int32_t lmax,
                         const DevLazy &L, const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                         int32_t *err, int32_t B, void *logits, int dtype, uint32_t *rows_out, int num_sms,
                         cudaStream_t st);

@@ -291,3 +291,64 @@ def test_lazy_argument_checks(cuda):
     T.trie_lazy_apply(h, torch.zeros((0, 3), device=cuda), st[:0])
     T.trie_lazy_init(h, vb, vo, 3, cache_rows=0, max_batch=2)
     assert T.trie_lazy_stats(h) == (0, 0)
+
+
+def test_lazy_and_dense_share_the_transition_table(cuda):
+    """One handle used by lazy rows and dense compiles in turn, with two
+    vocabularies: lazy rows record the moves they find in the handle's
+    transition table, a dense compile completes or replaces it, and every
+    advance stays equal to the oracle's."""
+    import torch
+    w = W.config(1)
+    ot = oracle.Trie(w.set_bytes, w.set_offsets)
+    toks_a = W.unpack(w.vocab_bytes, w.vocab_offsets)
+    toks_b = toks_a[:-1][::-1] + [b""]                 # same strings, other ids
+    vb_b, vo_b = W.pack(toks_b)
+    ov_a = oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+    ov_b = oracle.Vocab(vb_b, vo_b)
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    r = np.random.default_rng(11)
+    B, V = 64, w.V
+    n = ot.num_nodes
+
+    def lazy_step(ov, states, tokens):
+        x = torch.zeros((B, V), device=cuda)
+        out = torch.empty(B, dtype=torch.int32, device=cuda)
+        T.trie_lazy_advance_apply(h, torch.as_tensor(states, device=cuda), torch.as_tensor(tokens, device=cuda),
+                                  out, x)
+        want, _ = oracle.advance(ot, ov, states, tokens)
+        assert np.array_equal(out.cpu().numpy(), want)
+        return want
+
+    def dense_step(ov, states, tokens):
+        st = torch.as_tensor(states, device=cuda).clone()
+        T.trie_advance(h, st, torch.as_tensor(tokens, device=cuda))
+        want, _ = oracle.advance(ot, ov, states, tokens)
+        assert np.array_equal(st.cpu().numpy(), want)
+
+    def batch():
+        states = r.integers(0, n, B).astype(np.int32)
+        # tokens that are allowed from each state half the time
+        rows = oracle.mask_rows(ot, ov_a, states)
+        toks = r.integers(0, V - 1, B).astype(np.int32)
+        for b in range(0, B, 2):
+            ids = np.nonzero(np.unpackbits(rows[b].view(np.uint8), bitorder="little")[:V])[0]
+            ids = ids[ids != V - 1]
+            if ids.size:
+                toks[b] = ids[r.integers(ids.size)]
+        return states, toks
+
+    T.trie_lazy_init(h, w.vocab_bytes, w.vocab_offsets, V, cache_rows=256, max_batch=B)
+    for _ in range(3):                                 # the lazy rows fill the table in part
+        lazy_step(ov_a, *batch())
+    m = T.alloc_mask(h, V, cuda)
+    T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, m)   # completes it
+    for _ in range(2):
+        dense_step(ov_a, *batch())
+        lazy_step(ov_a, *batch())
+    T.trie_compile_masks(h, vb_b, vo_b, V, m)          # replaces it (vocabulary b)
+    s, t = batch()
+    dense_step(ov_b, s, t)
+    lazy_step(ov_a, s, t)                              # lazy rows keep vocabulary a, walk the bytes
+    T.trie_lazy_init(h, vb_b, vo_b, V, cache_rows=256, max_batch=B)
+    lazy_step(ov_b, s, t)
