@@ -15,7 +15,10 @@ Pins (``tests/test_oracle_pins.py``): the worked example of App. G.1 and the
 Fig. 2 example (``tests/golden/``), exhaustive comparison with the prefix-set
 enumeration of the App. G.5 proof on small random sets, and the invariants of
 Sec. 4.2 / App. G.5 (tokenization paths allowed, leaves admit only EOS,
-prefix closure, padding bits zero, ...).
+prefix closure, padding bits zero, ...). ``Format`` (the character-position
+masks of App. K) is pinned in ``tests/test_fmt_oracle.py`` to the same
+prefix-set definition on the enumerated strings of small formats, to a closed
+form and to a date format worked by hand.
 """
 from __future__ import annotations
 
@@ -67,6 +70,9 @@ def load_library(path: str):
     lib.oracle_advance.argtypes = [P, P, P, I32, P, P, I64]
     lib.oracle_apply.argtypes = [P, P, P, I32, P, I32, P, I64]
     lib.oracle_argmax.argtypes = [P, I32, I64, I32, P]
+    lib.oracle_fmt_mask_rows.argtypes = [P, I32, P, P, I32, P, I64, P]
+    lib.oracle_fmt_advance.restype = I64
+    lib.oracle_fmt_advance.argtypes = [P, I32, P, P, I32, P, P, I64]
     if hasattr(lib, "ac_build"):
         lib.ac_build.restype = P
         lib.ac_build.argtypes = [P, P, I32]
@@ -263,3 +269,41 @@ def decode(t: Trie, voc: Vocab, logits_per_step, states0: np.ndarray):
         toks.append(tk)
         sts.append(states.copy())
     return masked, toks, sts, errors
+
+
+class Format:
+    """A fixed format for the character-position masks (App. K): L byte
+    classes, classes[i] a 32-byte bitmap (byte c allowed iff bit c % 8 of
+    classes[i][c // 8]). States are the positions 0..L."""
+
+    def __init__(self, classes: np.ndarray):
+        self.classes = np.ascontiguousarray(classes, dtype=np.uint8).reshape(-1, 32)
+        self.L = self.classes.shape[0]
+        self._lib = _load()
+
+    def mask_rows(self, voc: Vocab, rows) -> np.ndarray:
+        rows = np.ascontiguousarray(rows, dtype=np.int32)
+        out = np.zeros((rows.size, n_words(voc.V)), np.uint32)
+        self._lib.oracle_fmt_mask_rows(_p(self.classes), self.L, _p(voc.b), _p(voc.o), voc.V, _p(rows), rows.size,
+                                       _p(out))
+        return out
+
+    def mask_all(self, voc: Vocab) -> np.ndarray:
+        return self.mask_rows(voc, np.arange(self.L + 1, dtype=np.int32))
+
+    def advance(self, voc: Vocab, states: np.ndarray, tokens: np.ndarray) -> tuple[np.ndarray, int]:
+        s = np.array(states, dtype=np.int32, copy=True)
+        tk = np.ascontiguousarray(tokens, dtype=np.int32)
+        err = self._lib.oracle_fmt_advance(_p(self.classes), self.L, _p(voc.b), _p(voc.o), voc.V, _p(s), _p(tk),
+                                           s.size)
+        return s, int(err)
+
+    def apply(self, voc: Vocab, logits_bits: np.ndarray, states: np.ndarray) -> np.ndarray:
+        """-inf (fp32 0xFF800000 / bf16 0xFF80) where the row of the state's
+        position clears the token (Sec. 4.2 last paragraph, App. H.3)."""
+        x = np.array(logits_bits, copy=True)
+        rows = self.mask_rows(voc, states)
+        allowed = np.unpackbits(rows.view(np.uint8), axis=1, bitorder="little")[:, :voc.V].astype(bool)
+        x[~allowed] = np.uint32(0xFF800000) if x.dtype == np.uint32 else np.uint16(0xFF80)
+        return x
+

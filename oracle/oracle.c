@@ -266,3 +266,71 @@ void oracle_argmax(const void *logits, int32_t dtype, int64_t B, int32_t V, int3
         out[b] = best;
     }
 }
+
+/* ------------------------------------------------------------------------
+ * Character-position masks for fixed-format strings (App. K, "constraint-
+ * aware dispatch beyond finite sets"): a format of length L is a sequence of
+ * byte classes C_0..C_{L-1}; class i allows byte c iff bit (c % 8) of
+ * classes[32 * i + c / 8] is set. The strings of the format are the
+ * products C_0 x ... x C_{L-1}; the automaton's states are the positions
+ * 0..L (position p: p bytes written).
+ *
+ *  - valid[p]: token v (not EOS) iff 1 <= len(v) <= L - p and byte i of v is
+ *    in C_{p+i} for every i (the position-wise character check of App. K);
+ *    EOS iff p == L. Every position p < L has a continuation in the format,
+ *    so this is the same live-path condition as the trie's (App. G.5).
+ *  - advance: a valid token moves p to p + len(v); EOS at L -> FINISHED;
+ *    FINISHED + EOS -> FINISHED; DEAD stays DEAD; anything else -> DEAD (one
+ *    error per move into DEAD), as for the trie.
+ * ---------------------------------------------------------------------- */
+
+static int fmt_class_has(const uint8_t *classes, int32_t i, uint8_t c) {
+    return (classes[32 * (int64_t)i + c / 8] >> (c % 8)) & 1;
+}
+
+static int fmt_valid(const uint8_t *classes, int32_t L, const uint8_t *vb, const int64_t *vo,
+                     int32_t V, int32_t p, int32_t v) {
+    if (v == V - 1) return p == L;
+    int64_t len = vo[v + 1] - vo[v];
+    if (len < 1 || len > (int64_t)(L - p)) return 0;
+    for (int64_t i = 0; i < len; i++)
+        if (!fmt_class_has(classes, p + (int32_t)i, vb[vo[v] + i])) return 0;
+    return 1;
+}
+
+static void fmt_row(const uint8_t *classes, int32_t L, const uint8_t *vb, const int64_t *vo, int32_t V,
+                    int32_t p, uint32_t *row) {
+    int64_t W = (V + 31) / 32;
+    memset(row, 0, sizeof(uint32_t) * W);
+    if (p < 0 || p > L) {  /* FINISHED, DEAD, not a position: {EOS} */
+        row[(V - 1) / 32] |= 1u << ((V - 1) % 32);
+        return;
+    }
+    for (int32_t v = 0; v < V; v++)
+        if (fmt_valid(classes, L, vb, vo, V, p, v)) row[v / 32] |= 1u << (v % 32);
+}
+
+void oracle_fmt_mask_rows(const uint8_t *classes, int32_t L, const uint8_t *vb, const int64_t *vo,
+                          int32_t V, const int32_t *rows, int64_t nrows, uint32_t *out) {
+    int64_t W = (V + 31) / 32;
+    for (int64_t i = 0; i < nrows; i++) fmt_row(classes, L, vb, vo, V, rows[i], out + i * W);
+}
+
+int64_t oracle_fmt_advance(const uint8_t *classes, int32_t L, const uint8_t *vb, const int64_t *vo,
+                           int32_t V, int32_t *states, const int32_t *tokens, int64_t B) {
+    int64_t errors = 0;
+    int32_t eos = V - 1;
+    for (int64_t b = 0; b < B; b++) {
+        int32_t s = states[b], v = tokens[b], nxt;
+        if (s == ORACLE_DEAD) continue;
+        if (v < 0 || v >= V) nxt = ORACLE_DEAD;
+        else if (s == ORACLE_FINISHED) nxt = v == eos ? ORACLE_FINISHED : ORACLE_DEAD;
+        else if (s < 0 || s > L) nxt = ORACLE_DEAD;
+        else if (v == eos) nxt = (s == L) ? ORACLE_FINISHED : ORACLE_DEAD;
+        else nxt = fmt_valid(classes, L, vb, vo, V, s, v) ? s + (int32_t)(vo[v + 1] - vo[v]) : ORACLE_DEAD;
+        errors += nxt == ORACLE_DEAD;
+        states[b] = nxt;
+    }
+    return errors;
+}
+

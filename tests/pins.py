@@ -219,3 +219,93 @@ def check_chain(s: bytes) -> None:
     for d in range(len(s) + 1):
         got = row_ids(m[d], len(toks))
         assert got == ({s[d]} if d < len(s) else {256}), (d, got)
+
+
+# ------------------------------------------------------------ fixed formats (App. K)
+
+def fmt_case(seed: int):
+    """A small format (L <= 5, each position a class of 1-3 bytes out of a
+    few, 0x00 and 0xFF included) and a vocabulary over those bytes and others."""
+    r = random.Random(seed)
+    alpha = [0x00, 0x2D, 0x30, 0x31, 0x39, 0x61, 0xFF]
+    L = r.randint(0, 5)
+    cls = [sorted(r.sample(alpha, r.randint(1, 3))) for _ in range(L)]
+    V = r.randint(2, 200)
+    toks = []
+    for _ in range(V - 1):
+        n = r.choice([0, 1, 1, 2, 2, 3, 4, 6])
+        pool = alpha + ([r.randrange(256)] if r.random() < 0.2 else [])
+        toks.append(bytes(r.choice(pool) for _ in range(n)))
+    toks.append(b"")
+    return cls, toks
+
+
+def fmt_bitmaps(cls: list[list[int]]) -> np.ndarray:
+    out = np.zeros((len(cls), 32), np.uint8)
+    for i, c in enumerate(cls):
+        for b in c:
+            out[i, b // 8] |= 1 << (b % 8)
+    return out
+
+
+def fmt_strings(cls: list[list[int]]) -> list[bytes]:
+    """Every string of the format: the product of its classes."""
+    import itertools
+    return [bytes(t) for t in itertools.product(*cls)]
+
+
+def check_fmt_masks(cls: list[list[int]], toks: list[bytes]) -> None:
+    """Row p equals the prefix-set row (App. G.5 conditions) of every prefix
+    of length p of the format's strings: the format's language is a finite
+    set, and all its prefixes of one length share their continuations."""
+    f = oracle.Format(fmt_bitmaps(cls))
+    voc = oracle.Vocab(*W.pack(toks))
+    V = len(toks)
+    strings = fmt_strings(cls)
+    ids, E = prefix_ids(strings)
+    m = f.mask_all(voc)
+    assert m.shape == (len(cls) + 1, (V + 31) // 32)
+    for pre in ids:
+        got = row_ids(m[len(pre)], V)
+        assert got == expected_row(pre, toks, ids, E), (pre, sorted(got))
+    m2 = f.mask_rows(voc, [oracle.FINISHED, oracle.DEAD, len(cls) + 1, -7])
+    for k in range(4):
+        assert row_ids(m2[k], V) == {V - 1}
+
+
+def check_fmt_advance(cls: list[list[int]], toks: list[bytes], seed: int) -> None:
+    """Positions move like the prefix walk: p -> len(p + bytes(v))."""
+    f = oracle.Format(fmt_bitmaps(cls))
+    voc = oracle.Vocab(*W.pack(toks))
+    V, L = len(toks), len(cls)
+    ids, E = prefix_ids(fmt_strings(cls))
+    first = {}
+    for pre in sorted(ids, key=lambda x: (len(x), x)):
+        first.setdefault(len(pre), pre)
+    r = random.Random(seed)
+    B = 300
+    states = np.array([r.choice([oracle.DEAD, oracle.FINISHED, L + 1, r.randint(0, L), r.randint(0, L)])
+                       for _ in range(B)], np.int32)
+    tokens = np.array([r.choice([-1, V, V - 1, r.randrange(V), r.randrange(V)]) for _ in range(B)], np.int32)
+    got, err = f.advance(voc, states, tokens)
+    inv = {i: pre for pre, i in ids.items()}
+    want = []
+    for s, v in zip(states.tolist(), tokens.tolist()):
+        pre = first.get(s) if 0 <= s <= L else None
+        nxt = expected_next(pre, ids[pre] if pre is not None else s, v, toks, ids, E)
+        want.append(len(inv[nxt]) if nxt >= 0 else nxt)
+    assert got.tolist() == want, [(s, v, g, w) for s, v, g, w in zip(states, tokens, got, want) if g != w][:5]
+    assert err == sum(1 for s, w in zip(states, want) if w == oracle.DEAD and s != oracle.DEAD)
+
+
+def check_fmt_closed_form(L: int, toks: list[bytes]) -> None:
+    """Every class the full byte set: position p allows exactly the tokens of
+    1..L-p bytes, and EOS at p = L."""
+    f = oracle.Format(np.full((L, 32), 0xFF, np.uint8))
+    voc = oracle.Vocab(*W.pack(toks))
+    V = len(toks)
+    m = f.mask_all(voc)
+    for p in range(L + 1):
+        want = {v for v in range(V - 1) if 1 <= len(toks[v]) <= L - p} | ({V - 1} if p == L else set())
+        assert row_ids(m[p], V) == want, p
+

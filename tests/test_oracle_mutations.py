@@ -14,8 +14,9 @@ import sys
 import pytest
 
 import oracle
-from pins import (check_advance, check_apply, check_argmax, check_chain, check_golden,
-                  check_masks, check_numbering, random_case)
+from pins import (check_advance, check_apply, check_argmax, check_chain, check_fmt_advance,
+                  check_fmt_closed_form, check_fmt_masks, check_golden, check_masks, check_numbering,
+                  fmt_case, random_case)
 
 SRC = os.path.join(os.path.dirname(oracle.__file__), "oracle.c")
 
@@ -40,6 +41,12 @@ MUTANTS = {
     "bf16_neg_inf_wrong": ("= 0xFF80u;", "= 0x7F80u;"),
     "f32_neg_inf_wrong": ("= 0xFF800000u;", "= 0xFF000000u;"),
     "argmax_last_tie": ("if (v == 0 || x > bv)", "if (v == 0 || x >= bv)"),
+    "fmt_length_bound_off_by_one": ("if (len < 1 || len > (int64_t)(L - p)) return 0;",
+                                    "if (len < 1 || len > (int64_t)(L - p + 1)) return 0;"),
+    "fmt_class_of_token_position": ("if (!fmt_class_has(classes, p + (int32_t)i, vb[vo[v] + i])) return 0;",
+                                    "if (!fmt_class_has(classes, (int32_t)i, vb[vo[v] + i])) return 0;"),
+    "fmt_eos_anywhere": ("if (v == V - 1) return p == L;", "if (v == V - 1) return 1;"),
+    "fmt_advance_one_position": ("s + (int32_t)(vo[v + 1] - vo[v])", "s + 1"),
     "terminal_not_marked_for_prefix_values": ("        term[x] = 1;\n", "        if (x > 0 || offsets[i+1] > offsets[i]) term[x] = 1;\n        if (ch[x * 256 + 0] >= 0) term[x] = 0;\n"),
 }
 
@@ -56,6 +63,11 @@ def _all_pins():
         check_masks(strings, toks)
         check_advance(strings, toks, seed)
         check_apply(strings, toks, seed)
+    for seed in range(30):
+        cls, ftoks = fmt_case(7000 + seed)
+        check_fmt_masks(cls, ftoks)
+        check_fmt_advance(cls, ftoks, seed)
+    check_fmt_closed_form(5, [b"a", b"ab", b"abcdef", b"", b"xyz", b"\x00\xff", b""])
 
 
 TESTS = os.path.dirname(os.path.abspath(__file__))
