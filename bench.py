@@ -425,6 +425,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
         run_apply_lists = capture(apply_lists_only)
         apply_lists_avg = timed(run_apply_lists, reps) / S
         lazy = run_lazy(w, logits, forced, dev, stream, capture, timed, reps)
+        formats = run_formats(w, dev, stream, capture, timed, reps)
     timing_src = (f"CUDA events around {reps} back-to-back replays of a graph of the {S - 1} fused "
                   f"advance+apply launches of a step (over {S - 1} logits buffers, "
                   f"{(S - 1) * B * V * elt / 1e9:.2f} GB > L2), launching stream, right after the timed region")
@@ -553,6 +554,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
                          "note": "valid lists as the paper stores them (Sec. 4.2); compile includes its one "
                                  "device-to-host read of the size"},
         "lazy_rows": lazy,
+        "char_position_masks": formats,
         "breakdown": {"compile_ms": compile_ms, "apply_us_avg": apply_avg * 1e3,
                       "advance_us_avg": advance_avg * 1e3, "advance_apply_us_avg": fused_avg * 1e3,
                       "host_trie_build_ms": host_build_ms,
@@ -614,6 +616,31 @@ def run_lazy(w, logits, forced, dev, stream, capture, timed, reps: int) -> dict:
                                  "us_per_step": pass_ms * 1e3 / S, "hits": hits, "misses": misses,
                                  "row_bytes": rows_bytes}
         hl.destroy()
+    return out
+
+
+def run_formats(w, dev, stream, capture, timed, reps: int) -> dict:
+    """Character-position masks (App. K) of the four fixed formats of the
+    paper's comparison, compiled with the workload's vocabulary: per format
+    the mask compile (a graph of one fmt_compile_masks, CUDA events) and the
+    number of allowed (position, token) pairs."""
+    import numpy as np
+    import torch
+    from paper_2608_12574_gb300 import triemask as T
+    from paper_2608_12574_gb300 import workloads as W
+    out = {"V": w.V, "note": "App. K: one row per position of the format; compile = fmt_compile_masks"}
+    for name, pat in W.FORMATS.items():
+        f = T.fmt_build(W.format_classes(pat))
+        m = T.fmt_alloc_mask(f, w.V, dev)
+        with torch.cuda.stream(stream):
+            T.fmt_compile_masks(f, w.vocab_bytes, w.vocab_offsets, w.V, m, stream)
+        stream.synchronize()
+        run = capture(lambda: T.fmt_compile_masks(f, w.vocab_bytes, w.vocab_offsets, w.V, m, stream))
+        us = timed(run, reps) * 1e3
+        pairs = int(np.unpackbits(m.cpu().numpy().view(np.uint8)).sum())
+        out[name] = {"L": f.L, "compile_us": us, "allowed_pairs": pairs,
+                     "pairs_per_s": (f.L + 1) * w.V / (us * 1e-6)}
+        f.destroy()
     return out
 
 

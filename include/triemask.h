@@ -305,6 +305,49 @@ int trie_lazy_stats(trie_t h, int64_t *hits, int64_t *misses);
 int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets,
                                int32_t V, uint32_t *d_mask, cudaStream_t stream);
 
+/* ---- Fixed formats: character-position masks (App. K) ----
+ * A format of length L (0 <= L <= 1024) is a sequence of byte classes
+ * C_0..C_{L-1}, e.g. YYYY-MM-DD: ten positions, digits but for '-' at 4 and
+ * 7. Its strings are the products of its classes; the automaton's states are
+ * the positions 0..L (p bytes written). valid[p] holds token v (not EOS) iff
+ * 1 <= len(v) <= L - p and byte i of v lies in C_{p+i} for every i (the
+ * position-wise check of App. K), and EOS iff p = L. Masks have the trie
+ * masks' layout with L + 1 rows; states, FINISHED / DEAD and errors follow
+ * the trie calls, with positions in place of node ids. */
+typedef struct fmt_s *fmt_t; /* opaque; owned by the library */
+
+/* Build a format from L class bitmaps (host, read during the call):
+ *   classes  uint8[L * 32]; byte c is in class i iff bit (c % 8) of
+ *            classes[32 * i + c / 8] is set (may be NULL when L = 0)
+ * Host only. TRIE_EINVAL for L outside [0, 1024] or NULL pointers. */
+int fmt_build(const uint8_t *classes, int32_t L, fmt_t *out);
+
+/* L of the format; -1 for a NULL handle. */
+int32_t fmt_length(fmt_t f);
+
+/* valid[p] for every position into the caller's mask d_mask (device,
+ * (L + 1) * ceil(V/32) uint32, 4-byte aligned). Vocabulary arguments,
+ * caching and errors as trie_compile_masks; the first call uploads the
+ * format's classes to the current device. The handle records (d_mask, V,
+ * vocabulary) for fmt_advance and fmt_apply_mask. */
+int fmt_compile_masks(fmt_t f, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                      uint32_t *d_mask, cudaStream_t stream);
+
+/* Positions in place: p -> p + len(v) for an allowed token; EOS at p = L ->
+ * FINISHED; other rules and d_err as trie_advance. Needs a prior
+ * fmt_compile_masks (TRIE_ESTATE). */
+int fmt_advance(fmt_t f, int32_t *d_states, const int32_t *d_tokens, int32_t B, int32_t *d_err,
+                cudaStream_t stream);
+
+/* trie_apply_mask for a format: -inf where bit v of the row of position
+ * d_states[b] is clear (positions outside [0, L], FINISHED and DEAD use
+ * {EOS}); V must equal the compiled mask's V. */
+int fmt_apply_mask(fmt_t f, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                   cudaStream_t stream);
+
+/* Release the format and its device copy. NULL is a no-op. */
+int fmt_destroy(fmt_t f);
+
 /* Release the handle, its host arrays and its device copy of the trie.
  * Synchronises the device first if device memory is held. NULL is a no-op. */
 int trie_destroy(trie_t h);

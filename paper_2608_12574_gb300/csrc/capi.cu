@@ -708,6 +708,126 @@ int trie_lazy_stats(trie_t h, int64_t *hits, int64_t *misses) {
     return TRIE_OK;
 }
 
+int fmt_build(const uint8_t *classes, int32_t L, fmt_t *out) {
+    if (!out) return fail(TRIE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (L < 0 || L > tmk::kFmtMaxLen)
+        return fail(TRIE_EINVAL, "L must be in [0, " + std::to_string(tmk::kFmtMaxLen) + "]");
+    if (L > 0 && !classes) return fail(TRIE_EINVAL, "classes is NULL");
+    fmt_s *f = new (std::nothrow) fmt_s;
+    if (!f) return fail(TRIE_ENOMEM, "host allocation failed");
+    try {
+        f->classes.assign(size_t(L) * 8, 0u);
+    } catch (const std::bad_alloc &) {
+        delete f;
+        return fail(TRIE_ENOMEM, "host allocation failed");
+    }
+    for (int32_t i = 0; i < L; i++)
+        for (int c = 0; c < 256; c++)
+            if ((classes[32 * size_t(i) + size_t(c / 8)] >> (c % 8)) & 1)
+                f->classes[8 * size_t(i) + size_t(c / 32)] |= 1u << (c % 32);
+    f->L = L;
+    *out = f;
+    return TRIE_OK;
+}
+
+int32_t fmt_length(fmt_t f) { return f ? f->L : -1; }
+
+int fmt_compile_masks(fmt_t f, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                      uint32_t *d_mask, cudaStream_t stream) {
+    if (!f) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    if (!d_mask) return fail(TRIE_EINVAL, "d_mask is NULL");
+    if (reinterpret_cast<uintptr_t>(d_mask) & 3u) return fail(TRIE_EINVAL, "d_mask must be 4-byte aligned");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    std::lock_guard<std::mutex> lk(f->mu);
+    if (f->d_classes && f->device != dev)
+        return fail(TRIE_EINVAL, "format was uploaded to device " + std::to_string(f->device) + ", called on device " +
+                                     std::to_string(dev));
+    if (!f->d_classes) {
+        void *p = nullptr;
+        cudaError_t e = cudaMalloc(&p, sizeof(uint32_t) * std::max<size_t>(f->classes.size(), 1));
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(TRIE_ENOMEM, std::string("cudaMalloc for the format: ") + cudaGetErrorString(e));
+        }
+        if (!f->classes.empty() &&
+            (e = cudaMemcpy(p, f->classes.data(), sizeof(uint32_t) * f->classes.size(), cudaMemcpyHostToDevice)) !=
+                cudaSuccess) {
+            cudaFree(p);
+            return fail_cuda(e, "uploading the format");
+        }
+        f->d_classes = static_cast<uint32_t *>(p);
+        f->device = dev;
+    }
+    cudaError_t e = tmk::launch_fmt_compile(f->d_classes, f->L, *voc, d_mask, num_sms(dev), stream);
+    if (e != cudaSuccess) return fail_cuda(e, "format mask launch");
+    f->vocab = voc;
+    f->mask = d_mask;
+    f->mask_V = V;
+    return TRIE_OK;
+}
+
+int fmt_advance(fmt_t f, int32_t *d_states, const int32_t *d_tokens, int32_t B, int32_t *d_err,
+                cudaStream_t stream) {
+    if (!f) return fail(TRIE_EINVAL, "handle is NULL");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_states || !d_tokens)) return fail(TRIE_EINVAL, "d_states / d_tokens is NULL");
+    std::shared_ptr<tmk::DevVocab> voc;
+    {
+        std::lock_guard<std::mutex> lk(f->mu);
+        voc = f->vocab;
+    }
+    if (!voc) return fail(TRIE_ESTATE, "fmt_advance before fmt_compile_masks on this handle");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != f->device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_fmt_advance(f->d_classes, f->L, *voc, d_states, d_states, d_tokens, B, d_err, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "format advance launch");
+    return TRIE_OK;
+}
+
+int fmt_apply_mask(fmt_t f, void *d_logits, int dtype, const int32_t *d_states, int32_t B, int32_t V,
+                   cudaStream_t stream) {
+    if (!f) return fail(TRIE_EINVAL, "handle is NULL");
+    if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_logits || !d_states)) return fail(TRIE_EINVAL, "d_logits / d_states is NULL");
+    uint32_t *mask;
+    int32_t mV;
+    {
+        std::lock_guard<std::mutex> lk(f->mu);
+        mask = f->mask;
+        mV = f->mask_V;
+    }
+    if (!mask) return fail(TRIE_ESTATE, "fmt_apply_mask before fmt_compile_masks on this handle");
+    if (V != mV) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
+    if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
+        return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != f->device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_apply(d_logits, dtype, mask, d_states, B, V, f->L + 1, num_sms(dev), stream);
+    if (e != cudaSuccess) return fail_cuda(e, "format apply launch");
+    return TRIE_OK;
+}
+
+int fmt_destroy(fmt_t f) {
+    if (!f) return TRIE_OK;
+    if (f->d_classes) {
+        DeviceGuard g(f->device);
+        cudaFree(f->d_classes);  // waits for work that may still read it
+    }
+    delete f;
+    return TRIE_OK;
+}
+
 int trie_destroy(trie_t h) {
     if (!h) return TRIE_OK;
     if (h->lazy.base) {

@@ -213,7 +213,23 @@ struct DevLazy {
     LazyNode *pre = nullptr;        // [n] by pre-order position
 };
 
+// Character-position masks (App. K): formats of at most kFmtMaxLen positions
+// (their classes are staged in shared memory, 32 bytes per position).
+constexpr int32_t kFmtMaxLen = 1024;
+
 }  // namespace tmk
+
+// The opaque handle of a fixed format (fmt_* calls).
+struct fmt_s {
+    std::vector<uint32_t> classes;       // [L * 8] class bitmaps as words
+    int32_t L = 0;
+    std::mutex mu;                       // guards the fields below
+    int device = -1;
+    uint32_t *d_classes = nullptr;       // device copy (one allocation)
+    std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
+    uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
+    int32_t mask_V = 0;
+};
 
 // The opaque handle of the C ABI.
 struct trie_s {
@@ -272,6 +288,12 @@ cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bo
                         const DevLazy &L, const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                         int32_t *err, int32_t B, void *logits, int dtype, uint32_t *rows_out, int num_sms,
                         cudaStream_t st);
+// Fixed formats (fmt.cu): the dense [L + 1, ceil(V/32)] mask, and the advance.
+cudaError_t launch_fmt_compile(const uint32_t *classes, int32_t L, const DevVocab &v, uint32_t *mask, int num_sms,
+                               cudaStream_t st);
+cudaError_t launch_fmt_advance(const uint32_t *classes, int32_t L, const DevVocab &v, const int32_t *states_in,
+                               int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err,
+                               cudaStream_t st);
 cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
                                int32_t V, int32_t n_nodes, cudaStream_t st);
 }  // namespace tmk

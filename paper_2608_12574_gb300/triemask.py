@@ -47,6 +47,12 @@ SIGNATURES = {
     "trie_lazy_advance_apply": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, ctypes.c_int, _I32, _I32, _P]),
     "trie_lazy_rows": (ctypes.c_int, [_P, _P, _I32, _P, _P]),
     "trie_lazy_stats": (ctypes.c_int, [_P, _P, _P]),
+    "fmt_build": (ctypes.c_int, [_P, _I32, _P]),
+    "fmt_length": (_I32, [_P]),
+    "fmt_compile_masks": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "fmt_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "fmt_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
+    "fmt_destroy": (ctypes.c_int, [_P]),
     "trie_destroy": (ctypes.c_int, [_P]),
     "trie_last_error": (ctypes.c_char_p, []),
 }
@@ -395,3 +401,74 @@ def trie_lazy_stats(h: Trie) -> tuple[int, int]:
 
 def trie_destroy(h: Trie) -> None:
     h.destroy()
+
+
+# ------------------------------------------------------------ fixed formats
+
+class Fmt:
+    """A fixed format (character-position masks): an owned library handle."""
+
+    def __init__(self, handle: ctypes.c_void_p):
+        self.handle = handle
+        self._lib = load_library()
+        self.L = self._lib.fmt_length(handle)
+
+    def destroy(self) -> None:
+        if self.handle:
+            self._lib.fmt_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def fmt_build(classes) -> Fmt:
+    """classes: uint8 [L, 32] bitmaps (byte c allowed at position i iff bit c % 8 of classes[i, c // 8])."""
+    c = np.ascontiguousarray(classes, dtype=np.uint8).reshape(-1, 32)
+    h = ctypes.c_void_p()
+    lib = load_library()
+    _check(lib.fmt_build(_hp(c), c.shape[0], ctypes.byref(h)))
+    return Fmt(h)
+
+
+def fmt_alloc_mask(f: Fmt, V: int, device=None):
+    import torch
+    return torch.zeros((f.L + 1, mask_words(V)), dtype=torch.int32, device=device if device is not None else "cuda")
+
+
+def fmt_compile_masks(f: Fmt, vocab_bytes, vocab_offsets, V: int, d_mask, stream=None) -> None:
+    import torch
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    p = _dev(d_mask, (torch.int32,), "d_mask")
+    if d_mask.numel() < (f.L + 1) * mask_words(V):
+        raise ValueError("d_mask is smaller than (L + 1) * ceil(V/32) words")
+    _check(f._lib.fmt_compile_masks(f.handle, _hp(vb), _hp(vo), V, p, _stream(stream, d_mask.device)))
+
+
+def fmt_advance(f: Fmt, d_states, d_tokens, d_err=None, stream=None) -> None:
+    """Positions in place by one token each (int32 CUDA tensors of length B)."""
+    import torch
+    B = d_states.numel()
+    if d_tokens.numel() != B:
+        raise ValueError("states and tokens differ in length")
+    pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
+    _check(f._lib.fmt_advance(f.handle, _dev(d_states, (torch.int32,), "d_states"),
+                              _dev(d_tokens, (torch.int32,), "d_tokens"), B, pe, _stream(stream, d_states.device)))
+
+
+def fmt_apply_mask(f: Fmt, d_logits, d_states, stream=None) -> None:
+    """-inf into the logits ([B, V] fp32 or bf16) of tokens not allowed at each position."""
+    import torch
+    dtype = _logits_dtype(d_logits)
+    B, V = d_logits.shape
+    if d_states.numel() != B:
+        raise ValueError("d_states must have B entries")
+    _check(f._lib.fmt_apply_mask(f.handle, _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits"), dtype,
+                                 _dev(d_states, (torch.int32,), "d_states"), B, V, _stream(stream, d_logits.device)))
+

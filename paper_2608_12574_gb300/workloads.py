@@ -419,3 +419,27 @@ def logits(w: Workload, step: int, device: str = "cpu", batch: int | None = None
     g.manual_seed(w.logit_seed + step)
     x = torch.randn(B, w.V, generator=g, device=device, dtype=torch.float32) * w.logit_std
     return x.to(torch.bfloat16) if w.dtype == "bf16" else x
+
+
+# ------------------------------------------------------------ fixed formats
+
+# The fixed formats of App. K's comparison, as patterns: '#' a decimal digit,
+# 'x' a lowercase hexadecimal digit, 'y' one of 8 9 a b (the UUID version 4
+# variant nibble), any other character itself.
+FORMATS = {
+    "YYYY-MM-DD": "####-##-##",
+    "datetime": "####-##-##T##:##:##",
+    "datetime.ms": "####-##-##T##:##:##.###",
+    "UUID v4": "xxxxxxxx-xxxx-4xxx-yxxx-xxxxxxxxxxxx",
+}
+
+
+def format_classes(pattern: str) -> np.ndarray:
+    """uint8 [L, 32] class bitmaps of a pattern (byte c of position i: bit c % 8 of [i, c // 8])."""
+    sets = {"#": b"0123456789", "x": b"0123456789abcdef", "y": b"89ab"}
+    out = np.zeros((len(pattern), 32), np.uint8)
+    for i, ch in enumerate(pattern):
+        for c in sets.get(ch, ch.encode()):
+            out[i, c // 8] |= 1 << (c % 8)
+    return out
+

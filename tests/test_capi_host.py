@@ -28,7 +28,7 @@ def lib():
 def declared_functions() -> list[str]:
     src = open(HEADER).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]+?\b(trie_\w+)\s*\(", src, flags=re.M)))
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]+?\b((?:trie|fmt)_\w+)\s*\(", src, flags=re.M)))
 
 
 def test_header_declares_the_boundary():
@@ -209,6 +209,37 @@ def test_lazy_calls_checked_before_any_device_work(lib):
     for f, args in (("trie_lazy_init", (None, None, 2, 8, 8)), ("trie_lazy_apply", (16, 0, 16, 1, 2, None)),
                     ("trie_lazy_rows", (16, 1, 16, None)), ("trie_lazy_stats", (None, None))):
         assert getattr(L, f)(None, *args) == T.TRIE_EINVAL
+
+
+def test_fmt_calls_checked_before_any_device_work(lib):
+    """Fixed formats: argument and call-order errors before the GPU is touched."""
+    L = lib
+    h = ctypes.c_void_p()
+    cls = W.format_classes("####-##-##")
+    assert L.fmt_build(cls.ctypes.data, 1025, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert L.fmt_build(cls.ctypes.data, -1, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert L.fmt_build(None, 3, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert L.fmt_build(cls.ctypes.data, 10, None) == T.TRIE_EINVAL
+    f = T.fmt_build(cls)
+    assert f.L == 10 and L.fmt_length(None) == -1
+    assert L.fmt_advance(f.handle, 16, 16, 1, None, None) == T.TRIE_ESTATE
+    assert L.fmt_apply_mask(f.handle, 16, 0, 16, 1, 2, None) == T.TRIE_ESTATE
+    assert L.fmt_apply_mask(f.handle, 16, 9, 16, 1, 2, None) == T.TRIE_EINVAL           # dtype
+    assert L.fmt_compile_masks(f.handle, None, None, 1, None, None) == T.TRIE_EINVAL      # V < 2
+    assert L.fmt_destroy(None) == T.TRIE_OK
+    f0 = T.fmt_build(np.zeros((0, 32), np.uint8))                                        # L = 0
+    assert f0.L == 0
+
+
+def test_format_patterns():
+    """The four formats of App. K's comparison as class bitmaps."""
+    for name, pat in W.FORMATS.items():
+        c = W.format_classes(pat)
+        assert c.shape == (len(pat), 32)
+        sizes = np.unpackbits(c, axis=1).sum(axis=1)
+        for ch, n in zip(pat, sizes):
+            assert n == {"#": 10, "x": 16, "y": 4}.get(ch, 1), (name, ch)
+    assert len(W.FORMATS["UUID v4"]) == 36 and len(W.FORMATS["datetime.ms"]) == 23
 
 
 def test_binding_fails_loudly_without_library(tmp_path):
