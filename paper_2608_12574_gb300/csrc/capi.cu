@@ -180,8 +180,6 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
         {o_par, t.parent.data(), sizeof(int32_t) * n},
         {o_lab, t.label.data(), n},
         {o_term, t.terminal.data(), n},
-        {o_fc, t.first_child.data(), sizeof(int32_t) * n},
-        {o_bits, t.child_bits.data(), sizeof(uint32_t) * 8 * n},
     };
     for (const Up &u : ups) {
         e = cudaMemcpyAsync(b + u.off, u.src, u.n, cudaMemcpyHostToDevice, stream);
@@ -196,8 +194,8 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     h->dev.parent = reinterpret_cast<const int32_t *>(b + o_par);
     h->dev.label = reinterpret_cast<const uint8_t *>(b + o_lab);
     h->dev.terminal = reinterpret_cast<const uint8_t *>(b + o_term);
-    h->dev.first_child = reinterpret_cast<const int32_t *>(b + o_fc);
-    h->dev.child_bits = reinterpret_cast<const uint32_t *>(b + o_bits);
+    h->dev.first_child = reinterpret_cast<int32_t *>(b + o_fc);
+    h->dev.child_bits = reinterpret_cast<uint32_t *>(b + o_bits);
     h->dev.window = reinterpret_cast<ulonglong2 *>(b + o_win);
     h->dev.depth16 = reinterpret_cast<uint8_t *>(b + o_d16);
     h->dev.anc = reinterpret_cast<int4 *>(b + o_anc);
@@ -205,8 +203,12 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     h->dev.trans_mask = uint32_t(trans_slots - 1);
     h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
     h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
-    // the compile's per-node tables, from the uploaded parent/label arrays
-    e = tmk::launch_trie_tables(h->dev, t.n, num_sms(dev), stream);
+    // the child links and the compile's per-node tables, from the uploaded
+    // parent/label arrays
+    if ((e = cudaMemsetAsync(b + o_fc, 0xFF, sizeof(int32_t) * n, stream)) == cudaSuccess &&
+        (e = cudaMemsetAsync(b + o_bits, 0, sizeof(uint32_t) * 8 * n, stream)) == cudaSuccess &&
+        (e = tmk::launch_trie_links(h->dev, t.n, num_sms(dev), stream)) == cudaSuccess)
+        e = tmk::launch_trie_tables(h->dev, t.n, num_sms(dev), stream);
     if (e != cudaSuccess) {
         cudaStreamSynchronize(stream);
         cudaFree(base);
@@ -365,7 +367,11 @@ int trie_get_csr(trie_t h, int32_t *parent, uint8_t *label, uint8_t *terminal, i
     if (parent) memcpy(parent, h->host.parent.data(), sizeof(int32_t) * n);
     if (label) memcpy(label, h->host.label.data(), n);
     if (terminal) memcpy(terminal, h->host.terminal.data(), n);
-    if (first_child) memcpy(first_child, h->host.first_child.data(), sizeof(int32_t) * n);
+    if (first_child) {  // children are contiguous: the first is the smallest id with that parent
+        for (size_t i = 0; i < n; i++) first_child[i] = -1;
+        for (size_t c = n; c-- > 1;)
+            if (h->host.parent[c] >= 0) first_child[size_t(h->host.parent[c])] = int32_t(c);
+    }
     return TRIE_OK;
 }
 

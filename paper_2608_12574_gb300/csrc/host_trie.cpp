@@ -61,11 +61,14 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
     if (total > int64_t(INT32_MAX) - 2) return "trie would exceed 2^31-1 nodes";
     std::sort(s.begin(), s.end(), [](const Str &a, const Str &b) { return cmp_str(a, b) < 0; });
 
-    // pre-order creation
-    std::vector<int32_t> pparent(1, -1);
-    hvec<int32_t> pdepth(1, 0);
-    std::vector<uint8_t> plabel(1, 0), pterm(1, 0);
-    pparent.reserve(size_t(total / 2 + 16));
+    // pre-order creation (at most 1 + total nodes)
+    hvec<int32_t> pparent(size_t(total) + 1), pdepth(size_t(total) + 1);
+    hvec<uint8_t> plabel(size_t(total) + 1), pterm(size_t(total) + 1);
+    pparent[0] = -1;
+    pdepth[0] = 0;
+    plabel[0] = 0;
+    pterm[0] = 0;
+    int32_t n = 1;
     std::vector<int32_t> path(1, 0);
     const Str *prev = nullptr;
     int64_t n_chars = 0;
@@ -79,19 +82,19 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
         }
         if (int64_t(path.size()) < x.n + 1) path.resize(size_t(x.n + 1));
         for (int64_t d = lcp + 1; d <= x.n; d++) {
-            int32_t id = int32_t(pparent.size());
-            pparent.push_back(path[size_t(d - 1)]);
-            plabel.push_back(x.p[d - 1]);
-            pterm.push_back(0);
-            pdepth.push_back(int32_t(d));
-            path[size_t(d)] = id;
+            const size_t id = size_t(n++);
+            pparent[id] = path[size_t(d - 1)];
+            plabel[id] = x.p[d - 1];
+            pterm[id] = 0;
+            pdepth[id] = int32_t(d);
+            path[size_t(d)] = int32_t(id);
         }
         pterm[size_t(path[size_t(x.n)])] = 1;
         n_chars += x.n;
         max_depth = std::max<int32_t>(max_depth, int32_t(x.n));
         prev = &x;
     }
-    const int32_t n = int32_t(pparent.size());
+    pdepth.resize(size_t(n));
 
     // breadth-first ids: stable bucket by depth
     std::vector<int32_t> level(size_t(max_depth) + 2, 0);
@@ -105,23 +108,14 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
     for (int32_t i = n - 1; i > 0; i--) psize[size_t(pparent[size_t(i)])] += psize[size_t(i)];
 
     out->n = n;
-    out->parent.assign(size_t(n), -1);
-    out->label.assign(size_t(n), 0);
-    out->terminal.assign(size_t(n), 0);
-    out->first_child.assign(size_t(n), -1);
-    out->child_bits.assign(size_t(n) * 8, 0u);
-    for (int32_t i = 0; i < n; i++) {
+    out->parent.resize(size_t(n));
+    out->label.resize(size_t(n));
+    out->terminal.resize(size_t(n));
+    for (int32_t i = 0; i < n; i++) {  // every BFS id is written once
         int32_t b = bfs[size_t(i)];
         out->label[size_t(b)] = plabel[size_t(i)];
         out->terminal[size_t(b)] = pterm[size_t(i)];
         out->parent[size_t(b)] = pparent[size_t(i)] < 0 ? -1 : bfs[size_t(pparent[size_t(i)])];
-    }
-    // first child = smallest BFS id among the children
-    for (int32_t c = 1; c < n; c++) {
-        int32_t p = out->parent[size_t(c)];
-        if (out->first_child[size_t(p)] < 0) out->first_child[size_t(p)] = c;
-        uint8_t l = out->label[size_t(c)];
-        out->child_bits[size_t(p) * 8 + (l >> 5)] |= 1u << (l & 31);
     }
     out->pre_node = std::move(bfs);
     out->pre_depth = std::move(pdepth);
@@ -169,8 +163,6 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
     out->parent.resize(n);
     out->label.resize(n);
     out->terminal.resize(n);
-    out->first_child.resize(n);
-    out->child_bits.resize(n * 8);
     out->pre_node.resize(n);
     out->pre_depth.resize(n);
     out->pre_size.resize(n);
@@ -183,16 +175,12 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
             HostTrie &p = parts[size_t(i)];
             const int32_t b = base[size_t(i)];
             const size_t g = size_t(b), pn = size_t(p.n);
-            for (size_t j = 0; j < pn; j++) {
-                out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
-                out->first_child[g + j] = p.first_child[j] < 0 ? -1 : p.first_child[j] + b;
-            }
+            for (size_t j = 0; j < pn; j++) out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
             for (size_t j = 0; j < pn; j++) out->pre_node[g + j] = p.pre_node[j] + b;
             memcpy(&out->pre_depth[g], p.pre_depth.data(), sizeof(int32_t) * pn);
             memcpy(&out->pre_size[g], p.pre_size.data(), sizeof(int32_t) * pn);
             memcpy(&out->label[g], p.label.data(), pn);
             memcpy(&out->terminal[g], p.terminal.data(), pn);
-            memcpy(&out->child_bits[8 * g], p.child_bits.data(), sizeof(uint32_t) * 8 * pn);
             p = HostTrie();  // release the part's memory early
         }
     };

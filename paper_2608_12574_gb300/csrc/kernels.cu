@@ -324,6 +324,21 @@ __device__ __forceinline__ void node_hits(const PatchArgs &a, int32_t m, Emit em
     }
 }
 
+// Child links from parent and label (thread per node c): in breadth-first
+// order the children of a node are contiguous, so c is its parent's first
+// child iff c - 1 has another parent; every child sets its label's bit in its
+// parent's 256-bit set.
+__global__ void k_trie_links(const int32_t *__restrict__ parent, const uint8_t *__restrict__ label, int32_t n,
+                             int32_t *__restrict__ first_child, uint32_t *__restrict__ child_bits) {
+    for (int32_t c = blockIdx.x * blockDim.x + threadIdx.x; c < n; c += gridDim.x * blockDim.x) {
+        const int32_t p = parent[c];
+        if (p < 0) continue;
+        if (parent[c - 1] != p) first_child[p] = c;
+        const uint32_t l = label[c];
+        atomicOr(child_bits + int64_t(p) * 8 + (l >> 5), 1u << (l & 31u));
+    }
+}
+
 // Per-node tables of the probe (one thread per node, climbing at most 16
 // parents): the last 16 edge labels into m, min(depth, 16), and the 16
 // nearest ancestors. Siblings and cousins are neighbours in breadth-first
@@ -1429,6 +1444,13 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 32);
     return launch_pdl(k_mask_patch, grid, kPatchThreads, st, a);
+}
+
+cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st) {
+    if (n_nodes <= 0) return cudaSuccess;
+    const int grid = grid_for(n_nodes, 256, int64_t(num_sms) * 8);
+    k_trie_links<<<grid, 256, 0, st>>>(t.parent, t.label, n_nodes, t.first_child, t.child_bits);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st) {

@@ -40,15 +40,15 @@ using hvec = std::vector<T, DefaultInitAlloc<T>>;
 
 // ----------------------------------------------------------------- host trie
 // Byte trie in breadth-first order, siblings by ascending byte (Sec. 4.1).
-// Children of a node are contiguous; child_bits is the 256-bit set of child
-// labels, so the child for byte c is first_child + popcount(bits below c).
+// Children of a node are contiguous, so the device derives each node's first
+// child and the 256-bit set of its child labels from parent and label
+// (launch_trie_links); the child for byte c is then first_child +
+// popcount(bits below c).
 struct HostTrie {
     int32_t n = 0;                       // nodes (all sets of a forest)
     hvec<int32_t> parent;                // -1 for a root
     hvec<uint8_t> label;                 // byte on the incoming edge
     hvec<uint8_t> terminal;              // some string ends here
-    hvec<int32_t> first_child;           // -1 for a leaf
-    hvec<uint32_t> child_bits;           // [n * 8]
     // Depth-first pre-order of the same nodes (the order in which the builder
     // creates them): position i holds node pre_node[i], at depth pre_depth[i],
     // whose subtree is positions i .. i + pre_size[i] - 1. Used by the lazy
@@ -128,8 +128,8 @@ struct DevTrie {
     const int32_t *parent = nullptr;
     const uint8_t *label = nullptr;
     const uint8_t *terminal = nullptr;
-    const int32_t *first_child = nullptr;
-    const uint32_t *child_bits = nullptr;
+    int32_t *first_child = nullptr;      // built on the device (launch_trie_links)
+    uint32_t *child_bits = nullptr;      // [n * 8], built on the device
     // Per node, for the mask compile, built on the device from parent/label
     // (launch_trie_tables): the labels of the last 16 edges into it (byte i =
     // label i levels up, 0 past the root), min(depth, 16), and the ancestors
@@ -258,6 +258,9 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
 // beside the fill (needs t.hits / t.hit_count).
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st);
+// Fills t.first_child and t.child_bits from t.parent and t.label (which must
+// be -1 / zero on entry: the caller clears them on the same stream).
+cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
 // Fills t.window, t.depth16 and t.anc from t.parent and t.label.
 cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
 // Zeroes the transition table (before it is filled for another vocabulary).
