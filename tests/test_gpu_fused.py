@@ -151,3 +151,40 @@ def test_transitions_follow_the_vocabulary(cuda):
         st = torch.as_tensor(rows, device=cuda)
         T.trie_advance(h, st, torch.as_tensor(toks, device=cuda))
         assert np.array_equal(st.cpu().numpy(), want), k
+
+
+def test_fused_decode_loop_largest_workload_sampled(cuda):
+    """K = 74,719 codes, V = 262,144, B = 256, fp32, 16 steps, in the bench's
+    launch configuration (step 0 apply, then one advance + apply launch per
+    step): every state each step against the oracle's advance by the same
+    tokens, and on 8 sampled requests per step the masked logits and the
+    greedy token against the oracle's (the oracle would take minutes for all
+    256 x 262,144 logits of 16 steps)."""
+    import torch
+    w = W.config(4)
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    m = T.alloc_mask(h, w.V, cuda)
+    T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, w.V, m)
+    ot = oracle.Trie(w.set_bytes, w.set_offsets)
+    ov = oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+    r = np.random.default_rng(4)
+    bufs = [torch.zeros(w.batch, dtype=torch.int32, device=cuda) for _ in range(2)]
+    err = torch.zeros(1, dtype=torch.int32, device=cuda)
+    ost = np.zeros(w.batch, np.int32)
+    tok = None
+    for t in range(w.steps):
+        lg = W.logits(w, t, device="cuda")
+        x = lg.clone()
+        if t == 0:
+            T.trie_apply_mask(h, x, bufs[0])
+        else:
+            T.trie_advance_apply(h, bufs[(t - 1) % 2], tok, bufs[t % 2], x, err)
+            ost, _ = oracle.advance(ot, ov, ost, tok.cpu().numpy())
+        assert np.array_equal(bufs[t % 2].cpu().numpy(), ost), f"states differ at step {t}"
+        tok = torch.argmax(x, dim=1).to(torch.int32)
+        rows = np.sort(r.choice(w.batch, 8, replace=False))
+        raw = _bits(lg[torch.as_tensor(rows, device=cuda)])
+        want = oracle.apply(ot, ov, raw, ost[rows])
+        assert np.array_equal(_bits(x[torch.as_tensor(rows, device=cuda)]), want), f"logits differ at step {t}"
+        assert np.array_equal(tok.cpu().numpy()[rows], oracle.argmax(want)), f"tokens differ at step {t}"
+    assert int(err.item()) == 0
