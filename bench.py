@@ -208,7 +208,14 @@ def cpu_baseline(w, target_step_s: float, steps: int, warmup: int) -> dict:
                 break
     except OSError:
         pass
+    # the same oracle on one core (a smaller slice, about 2 s)
+    one = OracleSample(w, 1)
+    one.calibrate(min(2.0, target_step_s))
+    t1 = one.step()
+    single = {"value": one.f * one.N * w.V / t1, "unit": UNIT, "cores": 1, "s_per_step": t1,
+              "sample": f"{len(one.rows)} mask rows and {one.b} batch rows, one step"}
     return {"value": smp.f * smp.N * w.V / per_step, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "single_core": single,
             "steps": len(times), "s_per_step": per_step, "cpu": cpu_model, "N_nodes": smp.N,
             "sample": f"{len(times)} steps, each a {smp.f:.4f} slice of one {w.name} step: "
                       f"{len(smp.rows)} of {smp.N} mask rows x {w.V} tokens (brute-force walks, "
