@@ -167,7 +167,7 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     size_t trans_slots = 16;  // >= 8 per node, a power of two
     while (trans_slots < 8 * n) trans_slots <<= 1;
     const size_t o_trans = L.add(sizeof(ulonglong2) * trans_slots);
-    const size_t o_hits = L.add(sizeof(int2) * 8 * n);  // compile scratch (probe -> scatter)
+    const size_t o_hits = L.add(sizeof(int2) * tmk::kHitSlots * n);  // compile scratch (probe -> scatter)
     const size_t o_hcnt = L.add(n);
     void *base = nullptr;
     cudaError_t e = cudaMalloc(&base, L.total);

@@ -181,7 +181,6 @@ __device__ __forceinline__ void trans_insert(ulonglong2 *tab, uint32_t mask, int
     }
 }
 
-constexpr int kHitSlots = 8;
 constexpr int kHitOverflow = 255;
 
 // Read-only arrays the probe reads, for a bulk L2 prefetch.

@@ -122,6 +122,12 @@ struct DevVocab {
     ~DevVocab();
 };
 
+// (row, token) pairs the compile's probe records per node for the scatter; a
+// node has at most one per suffix length up to the longest token plus EOS,
+// so with tokens of up to 15 bytes no node has more (a node with more is
+// searched again by the scatter).
+constexpr int kHitSlots = 16;
+
 struct DevTrie {
     int device = -1;
     void *base = nullptr;
@@ -139,7 +145,7 @@ struct DevTrie {
     int4 *anc = nullptr;             // [n * 4]
     ulonglong2 *trans = nullptr;     // transition table {(row << 32 | token) + 1, end node}
     uint32_t trans_mask = 0;         // slots - 1
-    int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) per node
+    int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) pairs per node
     uint8_t *hit_count = nullptr;    // compile scratch: hits found per node
 };
 

@@ -149,7 +149,7 @@ def test_compile_long_suffixes(cuda, seed):
 
 def test_compile_many_hits_per_node(cuda):
     """a^k for k = 1..24 are all tokens: deep nodes of a run of 'a's end more
-    than 8 allowed (row, token) pairs (the hit buffer's overflow path)."""
+    than 16 allowed (row, token) pairs (the hit buffer's overflow path)."""
     strings = [b"a" * 30, b"a" * 12 + b"b", b"ab" * 10]
     toks = [bytes([b]) for b in range(256)] + [b"a" * k for k in range(2, 25)] + [b"ab", b"aab", b"ba" * 3, b""]
     sb, so = W.pack(strings)
