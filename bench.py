@@ -686,11 +686,13 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
     out["dead_moves"] = int(err.item())
     out["finished"] = int((states == T.TRIE_STATE_FINISHED).sum().item())
 
-    def decode():
-        states.copy_(roots)
-        for t in range(steps):
-            T.trie_apply_lists(h, logits[t], states, stream)
-            T.trie_advance(h, states, forced[t], err, stream)
+    sb = [states, torch.empty_like(states)]
+
+    def decode():  # one launch per step: apply, then advance + apply of the next step
+        sb[0].copy_(roots)
+        T.trie_apply_lists(h, logits[0], sb[0], stream)
+        for t in range(1, steps):
+            T.trie_advance_apply_lists(h, sb[(t - 1) % 2], forced[t - 1], sb[t % 2], logits[t], err, stream)
 
     g = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
@@ -721,10 +723,10 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
         hh = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
         with torch.cuda.stream(stream):
             T.trie_compile_lists(hh, w.vocab_bytes, w.vocab_offsets, V, stream)
-            st = torch.as_tensor(hh.roots(), device=dev)
-            for t in range(steps):
-                T.trie_apply_lists(hh, logits[t], st, stream)
-                T.trie_advance(hh, st, forced[t], err, stream)
+            st = [torch.as_tensor(hh.roots(), device=dev), torch.empty(B, dtype=torch.int32, device=dev)]
+            T.trie_apply_lists(hh, logits[0], st[0], stream)
+            for t in range(1, steps):
+                T.trie_advance_apply_lists(hh, st[(t - 1) % 2], forced[t - 1], st[t % 2], logits[t], err, stream)
         stream.synchronize()
         et.append(time.perf_counter() - t0)
         hh.destroy()

@@ -268,6 +268,15 @@ int trie_lazy_rows(trie_t h, const int32_t *d_states, int32_t B, uint32_t *d_row
  * computed once). Host-synchronous (synchronises the device). */
 int trie_lazy_stats(trie_t h, int64_t *hits, int64_t *misses);
 
+/* trie_advance_apply driven by the handle's valid lists: advance the states
+ * by the tokens (rules of trie_advance; d_states_out must differ from
+ * d_states_in), then mask the logits by the lists of the new states
+ * (trie_apply_lists), in one launch. V must equal the V of the last
+ * trie_compile_lists, whose vocabulary the advance uses (TRIE_ESTATE if there
+ * was none, or if a later trie_compile_masks took another vocabulary). */
+int trie_advance_apply_lists(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
+                             int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream);
+
 /* Size of the fixed device scratch used by trie_compile_masks_noalloc. */
 #define TRIE_NOALLOC_SCRATCH_BYTES (32u << 20)
 

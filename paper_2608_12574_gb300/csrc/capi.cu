@@ -714,6 +714,38 @@ int trie_lazy_stats(trie_t h, int64_t *hits, int64_t *misses) {
     return TRIE_OK;
 }
 
+int trie_advance_apply_lists(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
+                             int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
+    if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
+    if (B > 0 && (!d_states_in || !d_tokens || !d_states_out || !d_logits))
+        return fail(TRIE_EINVAL, "a device pointer is NULL");
+    if (B > 0 && d_states_in == d_states_out)
+        return fail(TRIE_EINVAL, "d_states_in and d_states_out must be different buffers");
+    if (h->lists.n_valid < 0)
+        return fail(TRIE_ESTATE, "trie_advance_apply_lists before trie_compile_lists on this handle");
+    if (V != h->lists.V) return fail(TRIE_EINVAL, "V differs from the compiled lists' V");
+    if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
+        return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
+    std::shared_ptr<tmk::DevVocab> voc;
+    bool use_trans;
+    {
+        std::lock_guard<std::mutex> lk(h->mu);
+        voc = h->vocab;
+        use_trans = h->trans_vocab == voc;
+    }
+    if (!voc || voc->V != V) return fail(TRIE_ESTATE, "the handle's vocabulary is not the lists' vocabulary");
+    if (B == 0) return TRIE_OK;
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
+    cudaError_t e = tmk::launch_advance_apply_lists(h->dev, h->host.n, *voc, use_trans, d_states_in, d_tokens,
+                                                    d_states_out, d_err, d_logits, dtype, h->lists, B, stream);
+    if (e != cudaSuccess) return fail_cuda(e, "advance-apply-lists launch");
+    return TRIE_OK;
+}
+
 int fmt_build(const uint8_t *classes, int32_t L, fmt_t *out) {
     if (!out) return fail(TRIE_EINVAL, "out is NULL");
     *out = nullptr;

@@ -947,24 +947,43 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_list_scatter(PatchArgs a, 
 // Apply from the lists: CTA (row b, part p) covers 8 segments (8,192 tokens).
 // It rebuilds their 256 mask words in shared memory from the row's list and
 // writes them like k_apply_vec (kVec) or one logit per thread (any V and
-// alignment).
-template <int kElt, bool kVec>
+// alignment). With kAdvance the row's state is first moved by its token
+// (thread 0; the CTA of part 0 stores it and counts a move into DEAD): the
+// advance of one decode step and the apply of the next in one launch.
+template <int kElt, bool kVec, bool kAdvance>
 __global__ void __launch_bounds__(kApplyThreads) k_apply_lists(void *__restrict__ logits,
                                                                const int64_t *__restrict__ off,
-                                                               const int32_t *__restrict__ toks,
-                                                               const int32_t *__restrict__ states, int32_t B,
-                                                               int32_t V, int32_t n_nodes, int32_t parts) {
+                                                               const int32_t *__restrict__ toks, AdvanceArgs aa,
+                                                               const int32_t *__restrict__ states,
+                                                               const int32_t *__restrict__ tokens,
+                                                               int32_t *__restrict__ states_out,
+                                                               int32_t *__restrict__ err, int32_t B, int32_t V,
+                                                               int32_t n_nodes, int32_t parts) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     constexpr int kWords = 8 * 32;
     __shared__ __align__(128) uint4 tile[kVec ? kSegChunks : 1];
     __shared__ uint32_t words[kWords];
+    __shared__ int32_t state;
     for (int i = threadIdx.x; i < kWords; i += kApplyThreads) words[i] = 0u;
     if (kVec) init_ninf_tile<kElt>(tile);
     else __syncthreads();
     pdl_launch_dependents();
-    pdl_wait();  // logits and states come from earlier kernels
+    pdl_wait();  // logits, states and tokens come from earlier kernels
     const int32_t b = int32_t(blockIdx.x) / parts, part = int32_t(blockIdx.x) - b * parts;
-    const int32_t s = __ldg(states + b);
+    if (threadIdx.x == 0) {
+        const int32_t s0 = __ldg(states + b);
+        int32_t s1 = s0;
+        if (kAdvance) {
+            s1 = advance_one(aa, s0, __ldg(tokens + b));
+            if (part == 0) {
+                states_out[b] = s1;
+                if (s1 == kDead && s0 != kDead && err) atomicAdd(err, 1);
+            }
+        }
+        state = s1;
+    }
+    __syncthreads();
+    const int32_t s = state;
     const int32_t t0 = part * 8192, eos = V - 1;
     if (s >= 0 && s < n_nodes) {
         const int64_t lo = __ldg(off + s), hi = __ldg(off + s + 1);
@@ -1609,8 +1628,11 @@ cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVoc
                       L.toks);
 }
 
-cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
-                               int32_t V, int32_t n_nodes, cudaStream_t st) {
+namespace {
+
+cudaError_t launch_lists(void *logits, int dtype, const DevLists &L, const AdvanceArgs *aa,
+                         const int32_t *states, const int32_t *tokens, int32_t *states_out, int32_t *err,
+                         int32_t B, int32_t V, int32_t n_nodes, cudaStream_t st) {
     const int elt = dtype == 0 ? 4 : 2;
     const int32_t parts = int32_t((int64_t(V) + 8191) / 8192);
     const bool vec = (reinterpret_cast<uintptr_t>(logits) & 15u) == 0 && (int64_t(V) * elt) % 16 == 0;
@@ -1618,18 +1640,42 @@ cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const
     if (grid > INT32_MAX) return cudaErrorInvalidValue;
     const int32_t *tk = L.toks;
     const int64_t *of = L.off;
-    if (vec) {
-        if (elt == 2)
-            return launch_pdl(k_apply_lists<2, true>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
-                              n_nodes, parts);
-        return launch_pdl(k_apply_lists<4, true>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
-                          n_nodes, parts);
+    const AdvanceArgs a = aa ? *aa : AdvanceArgs{};
+    if (aa) {
+        if (vec)
+            return elt == 2 ? launch_pdl(k_apply_lists<2, true, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                         states, tokens, states_out, err, B, V, n_nodes, parts)
+                            : launch_pdl(k_apply_lists<4, true, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                         states, tokens, states_out, err, B, V, n_nodes, parts);
+        return elt == 2 ? launch_pdl(k_apply_lists<2, false, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                     states, tokens, states_out, err, B, V, n_nodes, parts)
+                        : launch_pdl(k_apply_lists<4, false, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                     states, tokens, states_out, err, B, V, n_nodes, parts);
     }
-    if (elt == 2)
-        return launch_pdl(k_apply_lists<2, false>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
-                          n_nodes, parts);
-    return launch_pdl(k_apply_lists<4, false>, int(grid), kApplyThreads, st, logits, of, tk, states, B, V,
-                      n_nodes, parts);
+    if (vec)
+        return elt == 2 ? launch_pdl(k_apply_lists<2, true, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                     states, tokens, states_out, err, B, V, n_nodes, parts)
+                        : launch_pdl(k_apply_lists<4, true, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                     states, tokens, states_out, err, B, V, n_nodes, parts);
+    return elt == 2 ? launch_pdl(k_apply_lists<2, false, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                 states, tokens, states_out, err, B, V, n_nodes, parts)
+                    : launch_pdl(k_apply_lists<4, false, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
+                                 states, tokens, states_out, err, B, V, n_nodes, parts);
+}
+
+}  // namespace
+
+cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
+                               int32_t V, int32_t n_nodes, cudaStream_t st) {
+    return launch_lists(logits, dtype, L, nullptr, states, nullptr, nullptr, nullptr, B, V, n_nodes, st);
+}
+
+cudaError_t launch_advance_apply_lists(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
+                                       const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
+                                       int32_t *err, void *logits, int dtype, const DevLists &L, int32_t B,
+                                       cudaStream_t st) {
+    const AdvanceArgs aa = advance_args(t, n_nodes, v, use_trans);
+    return launch_lists(logits, dtype, L, &aa, states_in, tokens, states_out, err, B, v.V, n_nodes, st);
 }
 
 cudaError_t launch_lazy_tables(const DevTrie &t, const DevLazy &L, int32_t n_nodes, cudaStream_t st) {

@@ -303,6 +303,11 @@ cudaError_t launch_fmt_compile(const uint32_t *classes, int32_t L, const DevVoca
 cudaError_t launch_fmt_advance(const uint32_t *classes, int32_t L, const DevVocab &v, const int32_t *states_in,
                                int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err,
                                cudaStream_t st);
+// Advance, then apply from the lists by the new states, in one launch.
+cudaError_t launch_advance_apply_lists(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
+                                       const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
+                                       int32_t *err, void *logits, int dtype, const DevLists &L, int32_t B,
+                                       cudaStream_t st);
 cudaError_t launch_apply_lists(void *logits, int dtype, const DevLists &L, const int32_t *states, int32_t B,
                                int32_t V, int32_t n_nodes, cudaStream_t st);
 }  // namespace tmk

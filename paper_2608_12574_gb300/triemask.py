@@ -39,6 +39,7 @@ SIGNATURES = {
     "trie_num_valid": (_I64, [_P]),
     "trie_copy_lists": (ctypes.c_int, [_P, _P, _P, _P]),
     "trie_apply_lists": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
+    "trie_advance_apply_lists": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, ctypes.c_int, _I32, _I32, _P]),
     "trie_advance": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_advance_apply": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, ctypes.c_int, _I32, _I32, _P]),
     "trie_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
@@ -397,6 +398,23 @@ def trie_lazy_stats(h: Trie) -> tuple[int, int]:
     hits, misses = ctypes.c_int64(0), ctypes.c_int64(0)
     _check(h._lib.trie_lazy_stats(h.handle, ctypes.byref(hits), ctypes.byref(misses)))
     return hits.value, misses.value
+
+
+def trie_advance_apply_lists(h: Trie, d_states_in, d_tokens, d_states_out, d_logits, d_err=None,
+                             stream=None) -> None:
+    """states_out <- delta*(states_in, tokens); then mask d_logits ([B, V]) by the lists of states_out."""
+    import torch
+    dtype = _logits_dtype(d_logits)
+    B, V = d_logits.shape
+    for t, name in ((d_states_in, "d_states_in"), (d_tokens, "d_tokens"), (d_states_out, "d_states_out")):
+        if t.numel() != B:
+            raise ValueError(f"{name} must have B entries")
+    pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
+    _check(h._lib.trie_advance_apply_lists(h.handle, _dev(d_states_in, (torch.int32,), "d_states_in"),
+                                           _dev(d_tokens, (torch.int32,), "d_tokens"),
+                                           _dev(d_states_out, (torch.int32,), "d_states_out"), pe,
+                                           _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits"), dtype, B,
+                                           V, _stream(stream, d_logits.device)))
 
 
 def trie_destroy(h: Trie) -> None:

@@ -166,6 +166,73 @@ def test_decode_loop_lists(cuda, cfg):
     assert int(err.item()) == oerr == 0
 
 
+@pytest.mark.parametrize("cfg", [1, 2, 3])
+def test_decode_loop_lists_fused(cuda, cfg):
+    """trie_apply_lists for step 0, then trie_advance_apply_lists for every
+    later step (one launch each), greedy argmax in between: masked logits,
+    tokens and states bit for bit equal to the oracle's at every step."""
+    import torch
+    w = W.config(cfg)
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, w.V)
+    logits = [W.logits(w, s, device="cuda") for s in range(w.steps)]
+    bufs = [torch.zeros(w.batch, dtype=torch.int32, device=cuda) for _ in range(2)]
+    err = torch.zeros(1, dtype=torch.int32, device=cuda)
+    got = []
+    tok = None
+    for t in range(w.steps):
+        x = logits[t].clone()
+        if t == 0:
+            T.trie_apply_lists(h, x, bufs[0])
+        else:
+            T.trie_advance_apply_lists(h, bufs[(t - 1) % 2], tok, bufs[t % 2], x, err)
+        tok = torch.argmax(x, dim=1).to(torch.int32)
+        got.append((x, tok.cpu().numpy(), bufs[t % 2].cpu().numpy().copy()))
+    ot = oracle.Trie(w.set_bytes, w.set_offsets)
+    ov = oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+    masked, toks, sts, oerr = oracle.decode(ot, ov, (_bits(lg) for lg in logits), np.zeros(w.batch, np.int32))
+    for t in range(w.steps):
+        assert np.array_equal(_bits(got[t][0]), masked[t]), t
+        assert np.array_equal(got[t][1], toks[t]), t
+        if t > 0:
+            assert np.array_equal(got[t][2], sts[t - 1]), t
+    assert int(err.item()) == oerr == 0
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("V", [33, 1001, 8193])
+def test_advance_apply_lists_random(cuda, dtype, V):
+    """Random states (invalid ones included) and tokens, the scalar path for
+    V = 33 / 1001: states against the oracle's advance, logits against its
+    apply by the new states."""
+    import torch
+    r = np.random.default_rng(V + 3)
+    strings = [bytes(r.integers(97, 100, r.integers(1, 6))) for _ in range(40)]
+    toks = [bytes(r.integers(97, 100, r.integers(1, 4))) for _ in range(V - 1)] + [b""]
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    h = T.trie_build(sb, so)
+    T.trie_compile_lists(h, vb, vo, V)
+    ot, ov = oracle.Trie(sb, so), oracle.Vocab(vb, vo)
+    B = 41
+    states = r.choice(np.array([-1, -2, ot.num_nodes, -9] + list(range(ot.num_nodes)) * 3, np.int32), B)
+    tokens = r.choice(np.array([-1, V, V - 1] + list(range(V)) * 2, np.int32), B)
+    want_st, want_err = oracle.advance(ot, ov, states, tokens)
+    if dtype == "f32":
+        raw = r.integers(0, 2**32, (B, V), dtype=np.uint64).astype(np.uint32)
+        x = torch.from_numpy(raw.view(np.int32)).view(torch.float32).to(cuda)
+    else:
+        raw = r.integers(0, 2**16, (B, V), dtype=np.uint32).astype(np.uint16)
+        x = torch.from_numpy(raw.view(np.int16)).view(torch.bfloat16).to(cuda)
+    out = torch.empty(B, dtype=torch.int32, device=cuda)
+    err = torch.zeros(1, dtype=torch.int32, device=cuda)
+    T.trie_advance_apply_lists(h, torch.as_tensor(states, device=cuda), torch.as_tensor(tokens, device=cuda), out, x,
+                               err)
+    assert np.array_equal(out.cpu().numpy(), want_st)
+    assert int(err.item()) == want_err
+    assert np.array_equal(_bits(x), oracle.apply(ot, ov, raw, want_st))
+
+
 def test_lists_errors(cuda):
     import torch
     sb, so = W.pack([b"ab"])
