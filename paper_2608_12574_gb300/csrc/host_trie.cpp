@@ -13,6 +13,8 @@
 
 #include <algorithm>
 #include <atomic>
+#include <cstdlib>
+#include <mutex>
 #include <numeric>
 #include <string>
 #include <thread>
@@ -21,6 +23,56 @@
 #include "tm_internal.h"
 
 namespace tmk {
+
+namespace {
+
+struct BlockCache {
+    std::mutex mu;
+    std::vector<std::pair<size_t, void *>> free;  // (size class in bytes, block)
+    size_t held = 0;
+};
+constexpr size_t kBlockCacheMax = size_t(1) << 30;
+
+BlockCache &block_cache() {
+    static BlockCache *c = new BlockCache();  // never destroyed: blocks may be freed during exit
+    return *c;
+}
+
+size_t block_class(size_t bytes) { return (bytes + kBigBlock - 1) / kBigBlock * kBigBlock; }
+
+}  // namespace
+
+void *big_block_alloc(size_t bytes) {
+    const size_t cls = block_class(bytes);
+    BlockCache &c = block_cache();
+    {
+        std::lock_guard<std::mutex> lk(c.mu);
+        for (size_t i = 0; i < c.free.size(); i++)
+            if (c.free[i].first == cls) {
+                void *p = c.free[i].second;
+                c.free[i] = c.free.back();
+                c.free.pop_back();
+                c.held -= cls;
+                return p;
+            }
+    }
+    return std::malloc(cls);
+}
+
+void big_block_free(void *p, size_t bytes) {
+    if (!p) return;
+    const size_t cls = block_class(bytes);
+    BlockCache &c = block_cache();
+    {
+        std::lock_guard<std::mutex> lk(c.mu);
+        if (c.held + cls <= kBlockCacheMax) {
+            c.free.emplace_back(cls, p);
+            c.held += cls;
+            return;
+        }
+    }
+    std::free(p);
+}
 
 namespace {
 
@@ -42,8 +94,19 @@ inline int cmp_str(const Str &a, const Str &b) {
 
 }  // namespace
 
-std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t first, int32_t last,
-                       HostTrie *out) {
+namespace {
+
+// A set's nodes in pre-order (the order the sorted strings create them).
+struct PreTrie {
+    int32_t n = 0;
+    hvec<int32_t> pparent, pdepth;
+    hvec<uint8_t> plabel, pterm;
+    int64_t n_chars = 0;
+    int32_t max_depth = 0;
+};
+
+// Sorts strings first..last-1 and creates their nodes in pre-order.
+std::string prepare_trie(const uint8_t *bytes, const int64_t *offsets, int32_t first, int32_t last, PreTrie *out) {
     const int64_t K = int64_t(last) - first;
     std::vector<Str> s(size_t(std::max<int64_t>(K, 0)));
     int64_t total = 0;
@@ -95,57 +158,85 @@ std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t fir
         prev = &x;
     }
     pdepth.resize(size_t(n));
-
-    // breadth-first ids: stable bucket by depth
-    std::vector<int32_t> level(size_t(max_depth) + 2, 0);
-    for (int32_t i = 0; i < n; i++) level[size_t(pdepth[i]) + 1]++;
-    for (size_t d = 1; d < level.size(); d++) level[d] += level[d - 1];
-    hvec<int32_t> bfs(static_cast<size_t>(n));
-    for (int32_t i = 0; i < n; i++) bfs[size_t(i)] = level[size_t(pdepth[i])]++;
-    // subtree sizes in pre-order (a parent precedes its descendants)
-    hvec<int32_t> psize(static_cast<size_t>(n));
-    for (int32_t i = 0; i < n; i++) psize[size_t(i)] = 1;
-    for (int32_t i = n - 1; i > 0; i--) psize[size_t(pparent[size_t(i)])] += psize[size_t(i)];
-
+    out->pparent = std::move(pparent);
+    out->plabel = std::move(plabel);
+    out->pterm = std::move(pterm);
+    out->pdepth = std::move(pdepth);
     out->n = n;
-    out->parent.resize(size_t(n));
-    out->label.resize(size_t(n));
-    out->terminal.resize(size_t(n));
-    for (int32_t i = 0; i < n; i++) {  // every BFS id is written once
-        int32_t b = bfs[size_t(i)];
-        out->label[size_t(b)] = plabel[size_t(i)];
-        out->terminal[size_t(b)] = pterm[size_t(i)];
-        out->parent[size_t(b)] = pparent[size_t(i)] < 0 ? -1 : bfs[size_t(pparent[size_t(i)])];
-    }
-    out->pre_node = std::move(bfs);
-    out->pre_depth = std::move(pdepth);
-    out->pre_size = std::move(psize);
-    out->roots.assign(1, 0);
     out->n_chars = n_chars;
     out->max_depth = max_depth;
     return "";
 }
 
+// Writes a prepared set into out's arrays at node ids base .. base + n - 1:
+// breadth-first ids (the pre-order nodes stably bucketed by depth), parent /
+// label / terminal, and the pre-order tables (node, depth, subtree size).
+void emit_trie(const PreTrie &p, int32_t base, HostTrie *out) {
+    const int32_t n = p.n;
+    const size_t g = size_t(base);
+    std::vector<int32_t> level(size_t(p.max_depth) + 2, 0);
+    for (int32_t i = 0; i < n; i++) level[size_t(p.pdepth[size_t(i)]) + 1]++;
+    for (size_t d = 1; d < level.size(); d++) level[d] += level[d - 1];
+    int32_t *bfs = &out->pre_node[g];  // local BFS ids first, offset below
+    for (int32_t i = 0; i < n; i++) bfs[i] = level[size_t(p.pdepth[size_t(i)])]++;
+    int32_t *psize = &out->pre_size[g];  // subtree sizes (a parent precedes its descendants)
+    for (int32_t i = 0; i < n; i++) psize[i] = 1;
+    for (int32_t i = n - 1; i > 0; i--) psize[p.pparent[size_t(i)]] += psize[i];
+    for (int32_t i = 0; i < n; i++) {  // every BFS id is written once
+        const size_t b = g + size_t(bfs[i]);
+        out->label[b] = p.plabel[size_t(i)];
+        out->terminal[b] = p.pterm[size_t(i)];
+        out->parent[b] = p.pparent[size_t(i)] < 0 ? -1 : bfs[p.pparent[size_t(i)]] + base;
+    }
+    memcpy(&out->pre_depth[g], p.pdepth.data(), sizeof(int32_t) * size_t(n));
+    for (int32_t i = 0; i < n; i++) bfs[i] += base;
+}
+
+void alloc_out(HostTrie *out, size_t n) {
+    out->n = int32_t(n);
+    out->parent.resize(n);
+    out->label.resize(n);
+    out->terminal.resize(n);
+    out->pre_node.resize(n);
+    out->pre_depth.resize(n);
+    out->pre_size.resize(n);
+}
+
+}  // namespace
+
+std::string build_trie(const uint8_t *bytes, const int64_t *offsets, int32_t first, int32_t last,
+                       HostTrie *out) {
+    PreTrie p;
+    std::string err = prepare_trie(bytes, offsets, first, last, &p);
+    if (!err.empty()) return err;
+    alloc_out(out, size_t(p.n));
+    emit_trie(p, 0, out);
+    out->roots.assign(1, 0);
+    out->n_chars = p.n_chars;
+    out->max_depth = p.max_depth;
+    return "";
+}
+
 std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
                          int32_t M, HostTrie *out) {
-    std::vector<HostTrie> parts(static_cast<size_t>(M));
+    std::vector<PreTrie> parts(static_cast<size_t>(M));
     std::vector<std::string> errs(static_cast<size_t>(M));
     unsigned hw = std::max(1u, std::thread::hardware_concurrency());
     unsigned nth = std::min<unsigned>(hw, unsigned(M));
-    // phase 1: every set's trie on its own, in parallel
-    std::atomic<int32_t> next(0);
-    auto build = [&]() {
-        for (;;) {
-            int32_t i = next.fetch_add(1);
-            if (i >= M) return;
-            errs[size_t(i)] = build_trie(bytes, offsets, set_offsets[i], set_offsets[i + 1], &parts[size_t(i)]);
-        }
+    auto run = [&](auto &&work) {  // work(i) for every set, on nth threads
+        std::atomic<int32_t> next(0);
+        auto loop = [&]() {
+            for (int32_t i; (i = next.fetch_add(1)) < M;) work(i);
+        };
+        std::vector<std::thread> th;
+        for (unsigned t = 1; t < nth; t++) th.emplace_back(loop);
+        loop();
+        for (auto &t : th) t.join();
     };
-    std::vector<std::thread> th;
-    for (unsigned t = 1; t < nth; t++) th.emplace_back(build);
-    build();
-    for (auto &t : th) t.join();
-    th.clear();
+    // phase 1: every set sorted and laid out in pre-order, in parallel
+    run([&](int32_t i) {
+        errs[size_t(i)] = prepare_trie(bytes, offsets, set_offsets[i], set_offsets[i + 1], &parts[size_t(i)]);
+    });
     int64_t total = 0, n_chars = 0;
     int32_t max_depth = 0;
     std::vector<int32_t> base(static_cast<size_t>(M));
@@ -157,36 +248,13 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
         max_depth = std::max(max_depth, parts[size_t(i)].max_depth);
     }
     if (total > int64_t(INT32_MAX) - 2) return "forest would exceed 2^31-1 nodes";
-    const size_t n = size_t(total);
-    // phase 2: concatenate, each worker copying (and first touching) its sets
-    out->n = int32_t(n);
-    out->parent.resize(n);
-    out->label.resize(n);
-    out->terminal.resize(n);
-    out->pre_node.resize(n);
-    out->pre_depth.resize(n);
-    out->pre_size.resize(n);
+    // phase 2: every set written at its offset of the forest's arrays
+    alloc_out(out, size_t(total));
+    run([&](int32_t i) {
+        emit_trie(parts[size_t(i)], base[size_t(i)], out);
+        parts[size_t(i)] = PreTrie();  // release the set's memory early
+    });
     out->roots.assign(base.begin(), base.end());
-    next = 0;
-    auto concat = [&]() {
-        for (;;) {
-            int32_t i = next.fetch_add(1);
-            if (i >= M) return;
-            HostTrie &p = parts[size_t(i)];
-            const int32_t b = base[size_t(i)];
-            const size_t g = size_t(b), pn = size_t(p.n);
-            for (size_t j = 0; j < pn; j++) out->parent[g + j] = p.parent[j] < 0 ? -1 : p.parent[j] + b;
-            for (size_t j = 0; j < pn; j++) out->pre_node[g + j] = p.pre_node[j] + b;
-            memcpy(&out->pre_depth[g], p.pre_depth.data(), sizeof(int32_t) * pn);
-            memcpy(&out->pre_size[g], p.pre_size.data(), sizeof(int32_t) * pn);
-            memcpy(&out->label[g], p.label.data(), pn);
-            memcpy(&out->terminal[g], p.terminal.data(), pn);
-            p = HostTrie();  // release the part's memory early
-        }
-    };
-    for (unsigned t = 1; t < nth; t++) th.emplace_back(concat);
-    concat();
-    for (auto &t : th) t.join();
     out->n_chars = n_chars;
     out->max_depth = max_depth;
     return "";

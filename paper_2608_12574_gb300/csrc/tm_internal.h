@@ -6,6 +6,7 @@
 
 #include <atomic>
 #include <memory>
+#include <new>
 #include <mutex>
 #include <string>
 #include <utility>
@@ -15,8 +16,17 @@
 
 namespace tmk {
 
+// Blocks of at least 2 MB for the builder's arrays come from a process-wide
+// cache of freed blocks (whole 2 MB classes, at most 1 GB held): a server that
+// builds a new forest for every batch then reuses pages it has already
+// touched instead of faulting in fresh ones. Defined in host_trie.cpp.
+void *big_block_alloc(size_t bytes);
+void big_block_free(void *p, size_t bytes);
+constexpr size_t kBigBlock = size_t(2) << 20;
+
 // std::vector allocator whose resize() leaves trivial elements uninitialised
-// (large host arrays are then first touched by the threads that fill them).
+// (large host arrays are then first touched by the threads that fill them),
+// with large blocks from the cache above.
 template <class T>
 struct DefaultInitAlloc : std::allocator<T> {
     template <class U>
@@ -26,6 +36,18 @@ struct DefaultInitAlloc : std::allocator<T> {
     DefaultInitAlloc() noexcept = default;
     template <class U>
     DefaultInitAlloc(const DefaultInitAlloc<U> &) noexcept {}
+    T *allocate(size_t n) {
+        const size_t bytes = n * sizeof(T);
+        if (bytes < kBigBlock) return std::allocator<T>::allocate(n);
+        void *p = big_block_alloc(bytes);
+        if (!p) throw std::bad_alloc();
+        return static_cast<T *>(p);
+    }
+    void deallocate(T *p, size_t n) noexcept {
+        const size_t bytes = n * sizeof(T);
+        if (bytes < kBigBlock) std::allocator<T>::deallocate(p, n);
+        else big_block_free(p, bytes);
+    }
     template <class U>
     void construct(U *p) noexcept {
         ::new (static_cast<void *>(p)) U;
