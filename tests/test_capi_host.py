@@ -252,3 +252,37 @@ def test_binding_fails_loudly_without_library(tmp_path):
             mod.load_library(str(tmp_path / "nope.so"))
         finally:
             mod._lib = old
+
+
+def test_concurrent_builds_equal_serial(lib):
+    """Forests built from 6 threads at once (each build itself multi-threaded,
+    all sharing the builder's cache of large blocks) equal a build on its own,
+    array for array; every handle is destroyed while the others build."""
+    import threading
+    w = W.config(5)
+    so = w.set_index[:97].astype(np.int32)     # the first 96 sets of the forest workload
+    ref = T.trie_build_many(w.set_bytes, w.set_offsets, so)
+    want = ref.csr()
+    want_roots = ref.roots()
+    errors = []
+
+    def work(k):
+        try:
+            for _ in range(3):
+                h = T.trie_build_many(w.set_bytes, w.set_offsets, so)
+                got = h.csr()
+                for name, arr in want.items():
+                    if not np.array_equal(got[name], arr):
+                        errors.append((k, name))
+                if not np.array_equal(h.roots(), want_roots):
+                    errors.append((k, "roots"))
+                h.destroy()
+        except Exception as e:  # pragma: no cover - reported below
+            errors.append((k, repr(e)))
+
+    th = [threading.Thread(target=work, args=(k,)) for k in range(6)]
+    for t in th:
+        t.start()
+    for t in th:
+        t.join()
+    assert not errors, errors[:5]
