@@ -352,3 +352,28 @@ def test_lazy_and_dense_share_the_transition_table(cuda):
     lazy_step(ov_a, s, t)                              # lazy rows keep vocabulary a, walk the bytes
     T.trie_lazy_init(h, vb_b, vo_b, V, cache_rows=256, max_batch=B)
     lazy_step(ov_b, s, t)
+
+
+def test_lazy_large_batch_small_cache(cuda):
+    """3,000 batch rows (more than the resolve's 1,024 threads) over a
+    512-row cache, so that sets overflow into per-call rows and rows are
+    evicted between calls; three calls with overlapping state sets, every
+    row against the oracle."""
+    w = W.config(3)
+    h = T.trie_build(w.set_bytes, w.set_offsets)
+    ot, ov = oracle.Trie(w.set_bytes, w.set_offsets), oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+    n = ot.num_nodes
+    T.trie_lazy_init(h, w.vocab_bytes, w.vocab_offsets, w.V, cache_rows=512, max_batch=3000)
+    r = np.random.default_rng(33)
+    pool = r.choice(n, 1500, replace=False).astype(np.int32)
+    total = 0
+    for call in range(3):
+        states = r.choice(pool, 3000).astype(np.int32)
+        states[::97] = -2
+        got = _rows(cuda, h, states, w.V)
+        want = _want_rows(ot, ov, states, w.V)
+        bad = np.nonzero((got != want).any(axis=1))[0]
+        assert bad.size == 0, f"call {call}: state {states[bad[0]]} differs"
+        total += int((states >= 0).sum())
+    hits, misses = T.trie_lazy_stats(h)
+    assert hits + misses == total and hits > 0
