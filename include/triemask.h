@@ -48,6 +48,11 @@
  * passes (mask, states, tokens, logits, error counter). The mask passed to
  * trie_compile_masks must stay allocated and unchanged while the handle is
  * used by trie_apply_mask (the handle keeps a non-owning pointer to it).
+ * A handle's device memory (trie arrays, valid lists, lazy rows) and the
+ * scratch of trie_build_many_device come from a memory pool per device that
+ * the library creates on first use; up to 8 GiB of memory freed by
+ * trie_destroy stays reserved in it for later handles until the process
+ * exits, so building and destroying a handle per batch maps no new memory.
  *
  * Streams: device work is enqueued on the given stream (0 = legacy default)
  * and is asynchronous with respect to the host. Concurrent trie_advance /
@@ -100,6 +105,25 @@ int trie_build(const uint8_t *bytes, const int64_t *offsets, int32_t K, trie_t *
  * Sets are built on host threads in parallel. Errors as trie_build. */
 int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
                     int32_t M, trie_t *out);
+
+/* trie_build_many with the insertion of Sec. 4.1 (App. G.1 Step 1) run on the
+ * current device, for per-request sets that change with every batch. The
+ * handle's node numbering, terminal flags, roots and statistics equal those
+ * of trie_build_many for the same arguments.
+ *   Arguments as trie_build_many (all host, read during the call); stream is
+ *   the stream the build kernels and the copies run on.
+ * The strings are copied to the device and inserted level by level (depth
+ * d = 0, 1, ...) for all sets at once; the trie lives on the device only and
+ * is bound to the current device. Host-synchronous: returns once the forest
+ * is complete on `stream`. Calls that need the host arrays (trie_get_csr,
+ * trie_lazy_init) copy them back once. Strings longer than 1024 bytes, more
+ * than 2^24 (set, depth) pairs or more than 2^31-3 string bytes plus sets
+ * are built by trie_build_many on the host instead. Device scratch (about
+ * 20 bytes per string byte plus 90 per string) is taken with cudaMallocAsync
+ * on `stream` and released there. Errors as trie_build_many; TRIE_ECUDA if
+ * a CUDA call fails. */
+int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
+                           int32_t M, cudaStream_t stream, trie_t *out);
 
 /* Number of nodes (the mask has this many rows); -1 for a NULL handle. */
 int32_t trie_num_nodes(trie_t h);

@@ -63,6 +63,37 @@ struct Layout {
     }
 };
 
+// Per-handle device memory (the trie's arrays, the valid lists, the lazy
+// rows) and the scratch of device builds come from one memory pool per
+// device, owned by the library and kept until exit. Up to kPoolKeepBytes of
+// freed memory stays mapped for the next allocations, so a loop that builds,
+// uses and destroys a forest for every batch does not map and unmap device
+// memory each time. A freed block is reused only once its free has completed
+// on the device, so an allocation carries no stream dependency.
+constexpr uint64_t kPoolKeepBytes = uint64_t(8) << 30;
+
+int pool_alloc(int dev, size_t bytes, cudaStream_t stream, void **out, const char *what) {
+    *out = nullptr;
+    cudaMemPool_t pool = tmk::device_pool(dev);
+    if (!pool) return fail(TRIE_ECUDA, std::string("creating the device memory pool for ") + what);
+    cudaError_t e = cudaMallocFromPoolAsync(out, std::max<size_t>(bytes, 1), pool, stream);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        *out = nullptr;
+        return fail(TRIE_ENOMEM, std::string("device allocation for ") + what + ": " + cudaGetErrorString(e));
+    }
+    return TRIE_OK;
+}
+
+// Frees a pool block once no device work can still use it: waits for the
+// current device (the block's device must be current).
+void pool_free(void *p) {
+    if (!p) return;
+    cudaDeviceSynchronize();
+    cudaFreeAsync(p, 0);
+    cudaGetLastError();
+}
+
 std::mutex g_vocab_mu;
 // Most recent last. Never destroyed, so no device memory is freed during
 // static destruction at process exit (the CUDA runtime may be gone by then).
@@ -145,16 +176,8 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
 // Uploads the trie on first use, ordered on `stream` (the copies read the
 // handle's own host arrays, which outlive them); the handle is bound to that
 // device.
-int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
-    std::lock_guard<std::mutex> lk(h->mu);
-    if (h->dev.base) {
-        if (h->dev.device != dev)
-            return fail(TRIE_EINVAL, "handle was uploaded to device " + std::to_string(h->dev.device) +
-                                         ", called on device " + std::to_string(dev));
-        return TRIE_OK;
-    }
-    const tmk::HostTrie &t = h->host;
-    const size_t n = size_t(t.n);
+// Device arrays of a trie of n nodes (one allocation); nothing is uploaded.
+int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream) {
     Layout L;
     const size_t o_par = L.add(sizeof(int32_t) * n);
     const size_t o_lab = L.add(n);
@@ -170,25 +193,9 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     const size_t o_hits = L.add(sizeof(int2) * tmk::kHitSlots * n);  // compile scratch (probe -> scatter)
     const size_t o_hcnt = L.add(n);
     void *base = nullptr;
-    cudaError_t e = cudaMalloc(&base, L.total);
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        return fail(TRIE_ENOMEM, std::string("cudaMalloc for the trie: ") + cudaGetErrorString(e));
-    }
+    const int rc = pool_alloc(dev, L.total, stream, &base, "the trie");
+    if (rc != TRIE_OK) return rc;
     char *b = static_cast<char *>(base);
-    struct Up { size_t off; const void *src; size_t n; } ups[] = {
-        {o_par, t.parent.data(), sizeof(int32_t) * n},
-        {o_lab, t.label.data(), n},
-        {o_term, t.terminal.data(), n},
-    };
-    for (const Up &u : ups) {
-        e = cudaMemcpyAsync(b + u.off, u.src, u.n, cudaMemcpyHostToDevice, stream);
-        if (e != cudaSuccess) {
-            cudaStreamSynchronize(stream);
-            cudaFree(base);
-            return fail_cuda(e, "uploading the trie");
-        }
-    }
     h->dev.device = dev;
     h->dev.base = base;
     h->dev.parent = reinterpret_cast<const int32_t *>(b + o_par);
@@ -203,19 +210,52 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     h->dev.trans_mask = uint32_t(trans_slots - 1);
     h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
     h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
-    // the child links and the compile's per-node tables, from the uploaded
-    // parent/label arrays
-    if ((e = cudaMemsetAsync(b + o_fc, 0xFF, sizeof(int32_t) * n, stream)) == cudaSuccess &&
-        (e = cudaMemsetAsync(b + o_bits, 0, sizeof(uint32_t) * 8 * n, stream)) == cudaSuccess &&
-        (e = tmk::launch_trie_links(h->dev, t.n, num_sms(dev), stream)) == cudaSuccess)
-        e = tmk::launch_trie_tables(h->dev, t.n, num_sms(dev), stream);
+    return TRIE_OK;
+}
+
+// The child links and the compile's per-node tables, from the device's
+// parent / label / terminal arrays (once they are written on `stream`).
+int finish_device_trie(trie_t h, int dev, cudaStream_t stream) {
+    const size_t n = size_t(h->host.n);
+    cudaError_t e;
+    if ((e = cudaMemsetAsync(h->dev.first_child, 0xFF, sizeof(int32_t) * n, stream)) == cudaSuccess &&
+        (e = cudaMemsetAsync(h->dev.child_bits, 0, sizeof(uint32_t) * 8 * n, stream)) == cudaSuccess &&
+        (e = tmk::launch_trie_links(h->dev, h->host.n, num_sms(dev), stream)) == cudaSuccess)
+        e = tmk::launch_trie_tables(h->dev, h->host.n, num_sms(dev), stream);
     if (e != cudaSuccess) {
-        cudaStreamSynchronize(stream);
-        cudaFree(base);
+        pool_free(h->dev.base);
         h->dev = tmk::DevTrie();
         return fail_cuda(e, "building the trie's compile tables");
     }
     return TRIE_OK;
+}
+
+int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
+    std::lock_guard<std::mutex> lk(h->mu);
+    if (h->dev.base) {
+        if (h->dev.device != dev)
+            return fail(TRIE_EINVAL, "handle was uploaded to device " + std::to_string(h->dev.device) +
+                                         ", called on device " + std::to_string(dev));
+        return TRIE_OK;
+    }
+    const tmk::HostTrie &t = h->host;
+    const size_t n = size_t(t.n);
+    int rc = alloc_device_trie(h, dev, n, stream);
+    if (rc != TRIE_OK) return rc;
+    struct Up { const void *dst; const void *src; size_t n; } ups[] = {
+        {h->dev.parent, t.parent.data(), sizeof(int32_t) * n},
+        {h->dev.label, t.label.data(), n},
+        {h->dev.terminal, t.terminal.data(), n},
+    };
+    for (const Up &u : ups) {
+        cudaError_t e = cudaMemcpyAsync(const_cast<void *>(u.dst), u.src, u.n, cudaMemcpyHostToDevice, stream);
+        if (e != cudaSuccess) {
+            pool_free(h->dev.base);
+            h->dev = tmk::DevTrie();
+            return fail_cuda(e, "uploading the trie");
+        }
+    }
+    return finish_device_trie(h, dev, stream);
 }
 
 // The transition table holds transitions of one vocabulary: when a compile
@@ -293,6 +333,66 @@ int lazy_call(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int
 
 int tmk::set_error(int code, const char *msg) { return fail(code, msg); }
 
+cudaMemPool_t tmk::device_pool(int dev) {
+    static std::mutex mu;
+    static std::vector<cudaMemPool_t> &pools = *new std::vector<cudaMemPool_t>();  // never destroyed
+    std::lock_guard<std::mutex> lk(mu);
+    if (dev < 0) return nullptr;
+    if (int(pools.size()) <= dev) pools.resize(size_t(dev) + 1, nullptr);
+    if (!pools[size_t(dev)]) {
+        cudaMemPoolProps props = {};
+        props.allocType = cudaMemAllocationTypePinned;
+        props.handleTypes = cudaMemHandleTypeNone;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        cudaMemPool_t p = nullptr;
+        if (cudaMemPoolCreate(&p, &props) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        uint64_t keep = kPoolKeepBytes;
+        int no = 0;
+        if (cudaMemPoolSetAttribute(p, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess ||
+            cudaMemPoolSetAttribute(p, cudaMemPoolReuseFollowEventDependencies, &no) != cudaSuccess ||
+            cudaMemPoolSetAttribute(p, cudaMemPoolReuseAllowInternalDependencies, &no) != cudaSuccess) {
+            cudaGetLastError();
+            cudaMemPoolDestroy(p);
+            return nullptr;
+        }
+        pools[size_t(dev)] = p;
+    }
+    return pools[size_t(dev)];
+}
+
+int tmk::ensure_host_arrays(trie_s *h) {
+    std::lock_guard<std::mutex> lk(h->mu);
+    if (h->host_arrays) return TRIE_OK;
+    tmk::HostTrie &t = h->host;
+    const size_t n = size_t(t.n);
+    try {
+        t.parent.resize(n);
+        t.label.resize(n);
+        t.terminal.resize(n);
+    } catch (const std::bad_alloc &) {
+        return fail(TRIE_ENOMEM, "host allocation failed while copying the trie back");
+    }
+    DeviceGuard g(h->dev.device);
+    cudaError_t e;
+    if ((e = cudaDeviceSynchronize()) != cudaSuccess ||
+        (e = cudaMemcpy(t.parent.data(), h->dev.parent, sizeof(int32_t) * n, cudaMemcpyDeviceToHost)) !=
+            cudaSuccess ||
+        (e = cudaMemcpy(t.label.data(), h->dev.label, n, cudaMemcpyDeviceToHost)) != cudaSuccess ||
+        (e = cudaMemcpy(t.terminal.data(), h->dev.terminal, n, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return fail_cuda(e, "copying the trie back from the device");
+    try {
+        tmk::pre_order_from_parents(&t);
+    } catch (const std::bad_alloc &) {
+        return fail(TRIE_ENOMEM, "host allocation failed for the pre-order tables");
+    }
+    h->host_arrays = true;
+    return TRIE_OK;
+}
+
 tmk::DevVocab::~DevVocab() {
     if (base) {
         DeviceGuard g(device);
@@ -348,6 +448,73 @@ int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t 
     return finish_build(err, h, out);
 }
 
+int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets, int32_t M,
+                           cudaStream_t stream, trie_t *out) {
+    if (!out) return fail(TRIE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (M < 1) return fail(TRIE_EINVAL, "M must be >= 1");
+    if (!set_offsets) return fail(TRIE_EINVAL, "set_offsets is NULL");
+    if (set_offsets[0] != 0) return fail(TRIE_EINVAL, "set_offsets[0] must be 0");
+    for (int32_t i = 0; i < M; i++)
+        if (set_offsets[i + 1] < set_offsets[i]) return fail(TRIE_EINVAL, "set_offsets must be non-decreasing");
+    const int32_t K = set_offsets[M];
+    if (K > 0 && !offsets) return fail(TRIE_EINVAL, "offsets is NULL");
+    if (K > 0 && offsets[K] > offsets[0] && !bytes) return fail(TRIE_EINVAL, "bytes is NULL");
+    int64_t max_len = 0;
+    for (int32_t i = 0; i < K; i++) {
+        if (offsets[i] < 0 || offsets[i + 1] < offsets[i])
+            return fail(TRIE_EINVAL, "offsets must be non-negative and non-decreasing");
+        max_len = std::max<int64_t>(max_len, offsets[i + 1] - offsets[i]);
+    }
+    const int64_t n_bytes = K > 0 ? offsets[K] - offsets[0] : 0;
+    // long strings (a long level loop), many sets with deep strings (the
+    // per-(set, depth) tables) or more bytes than node ids: the host builder
+    if (max_len > tmk::kDeviceBuildMaxDepth || int64_t(M) * (max_len + 1) > tmk::kDeviceBuildMaxGroups ||
+        n_bytes + M > int64_t(INT32_MAX) - 2)
+        return trie_build_many(bytes, offsets, set_offsets, M, out);
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    trie_s *h = new (std::nothrow) trie_s;
+    if (!h) return fail(TRIE_ENOMEM, "host allocation failed");
+    static const int64_t zero = 0;
+    const int64_t *off = K > 0 ? offsets : &zero;
+    const int sms = num_sms(dev);
+    int32_t n = 0;
+    int64_t n_chars = 0;
+    cudaError_t e;
+    {
+        tmk::DeviceBuild db;
+        cudaMemPool_t pool = tmk::device_pool(dev);
+        e = pool ? db.levels(K > 0 ? bytes + off[0] : nullptr, off, set_offsets, M, K, n_bytes, int32_t(max_len),
+                             sms, pool, stream, &n, &h->host.roots, &n_chars)
+                 : cudaErrorMemoryAllocation;
+        if (e == cudaSuccess) {
+            h->host.n = n;
+            h->host.n_chars = n_chars;
+            h->host.max_depth = int32_t(max_len);
+            h->host_arrays = false;
+            if ((rc = alloc_device_trie(h, dev, size_t(n), stream)) != TRIE_OK) {
+                delete h;
+                return rc;
+            }
+            e = db.emit(const_cast<int32_t *>(h->dev.parent), const_cast<uint8_t *>(h->dev.label),
+                        const_cast<uint8_t *>(h->dev.terminal), sms);
+        }
+    }  // the scratch is freed on the stream after the last kernel
+    if (e == cudaSuccess && (rc = finish_device_trie(h, dev, stream)) != TRIE_OK) {
+        delete h;
+        return rc;
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) {
+        pool_free(h->dev.base);
+        delete h;
+        return fail_cuda(e, "building the forest on the device");
+    }
+    *out = h;
+    return TRIE_OK;
+}
+
 int32_t trie_num_nodes(trie_t h) { return h ? h->host.n : -1; }
 
 int32_t trie_num_sets(trie_t h) { return h ? int32_t(h->host.roots.size()) : -1; }
@@ -363,6 +530,8 @@ int32_t trie_max_depth(trie_t h) { return h ? h->host.max_depth : -1; }
 
 int trie_get_csr(trie_t h, int32_t *parent, uint8_t *label, uint8_t *terminal, int32_t *first_child) {
     if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    int rc = tmk::ensure_host_arrays(h);
+    if (rc != TRIE_OK) return rc;
     const size_t n = size_t(h->host.n);
     if (parent) memcpy(parent, h->host.parent.data(), sizeof(int32_t) * n);
     if (label) memcpy(label, h->host.label.data(), n);
@@ -506,11 +675,7 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         const size_t o_tile = lay.add(sizeof(int64_t) * (size_t(n) / 4096 + 2));
         const size_t o_tot = lay.add(sizeof(int64_t));
         void *base = nullptr;
-        cudaError_t e = cudaMalloc(&base, lay.total);
-        if (e != cudaSuccess) {
-            cudaGetLastError();
-            return fail(TRIE_ENOMEM, std::string("cudaMalloc for the valid lists: ") + cudaGetErrorString(e));
-        }
+        if ((rc = pool_alloc(dev, lay.total, stream, &base, "the valid lists")) != TRIE_OK) return rc;
         char *b = static_cast<char *>(base);
         L.base = base;
         L.count = reinterpret_cast<int32_t *>(b + o_cnt);
@@ -528,16 +693,16 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     if (e != cudaSuccess) return fail_cuda(e, "valid-list count");
     if (total > L.tok_cap) {  // grow the token buffer (by at least half)
         const int64_t cap = std::max<int64_t>(total, L.tok_cap + L.tok_cap / 2);
-        if (L.toks) cudaFree(L.toks);
+        pool_free(L.toks);  // earlier apply calls may still read it
         L.toks = nullptr;
         L.tok_cap = 0;
-        e = cudaMalloc(reinterpret_cast<void **>(&L.toks), sizeof(int32_t) * size_t(std::max<int64_t>(cap, 1)));
-        if (e != cudaSuccess) {
-            cudaGetLastError();
-            L.toks = nullptr;
+        void *toks = nullptr;
+        if ((rc = pool_alloc(dev, sizeof(int32_t) * size_t(std::max<int64_t>(cap, 1)), stream, &toks,
+                             "the valid-list tokens")) != TRIE_OK) {
             L.n_valid = -1;
-            return fail(TRIE_ENOMEM, std::string("cudaMalloc for the valid-list tokens: ") + cudaGetErrorString(e));
+            return rc;
         }
+        L.toks = static_cast<int32_t *>(toks);
         L.tok_cap = cap;
     }
     e = tmk::launch_lists_scatter(h->dev, n, *voc, lmax, L, sms, stream);
@@ -602,6 +767,7 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     std::shared_ptr<tmk::DevVocab> voc;
     if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    if ((rc = tmk::ensure_host_arrays(h)) != TRIE_OK) return rc;  // the pre-order tables
     if ((rc = ensure_device_trie(h, dev, 0)) != TRIE_OK) return rc;
     cudaError_t e = cudaDeviceSynchronize();  // earlier lazy calls may still use the old cache
     if (e != cudaSuccess) return fail_cuda(e, "synchronising before the lazy set-up");
@@ -616,7 +782,7 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
         }
     }
     tmk::DevLazy &L = h->lazy;
-    if (L.base) cudaFree(L.base);
+    pool_free(L.base);
     L = tmk::DevLazy();
     const int32_t C = (cache_rows + tmk::kLazyWays - 1) / tmk::kLazyWays * tmk::kLazyWays;
     const int64_t W = (int64_t(V) + 31) / 32;
@@ -637,11 +803,7 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
     const size_t o_pos = lay.add(sizeof(int32_t) * n);
     const size_t o_pre = lay.add(sizeof(tmk::LazyNode) * n);
     void *base = nullptr;
-    e = cudaMalloc(&base, lay.total);
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        return fail(TRIE_ENOMEM, std::string("cudaMalloc for the lazy rows: ") + cudaGetErrorString(e));
-    }
+    if ((rc = pool_alloc(dev, lay.total, 0, &base, "the lazy rows")) != TRIE_OK) return rc;
     char *b = static_cast<char *>(base);
     L.device = dev;
     L.base = base;
@@ -675,7 +837,7 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
         (e = cudaMemcpy(L.pre_size, t.pre_size.data(), sizeof(int32_t) * n, cudaMemcpyHostToDevice)) !=
             cudaSuccess ||
         (e = tmk::launch_lazy_tables(h->dev, L, h->host.n, 0)) != cudaSuccess || (e = cudaDeviceSynchronize()) != cudaSuccess) {
-        cudaFree(base);
+        pool_free(base);
         L = tmk::DevLazy();
         return fail_cuda(e, "lazy-row set-up");
     }
@@ -870,14 +1032,14 @@ int trie_destroy(trie_t h) {
     if (!h) return TRIE_OK;
     if (h->lazy.base) {
         DeviceGuard g(h->lazy.device);
-        cudaFree(h->lazy.base);
+        pool_free(h->lazy.base);
     }
     if (h->dev.base || h->lists.base || h->lists.toks) {
         DeviceGuard g(h->dev.device);
-        // cudaFree waits for work on the device that may still read these
-        if (h->lists.toks) cudaFree(h->lists.toks);
-        if (h->lists.base) cudaFree(h->lists.base);
-        if (h->dev.base) cudaFree(h->dev.base);
+        // after the work on the device that may still read these
+        pool_free(h->lists.toks);
+        pool_free(h->lists.base);
+        pool_free(h->dev.base);
     }
     delete h;
     return TRIE_OK;

@@ -1,0 +1,472 @@
+// The byte tries of a forest built on the device from the raw strings
+// (Sec. 4.1; App. G.1 Step 1), for per-request sets that change every batch.
+//
+// Level by level over depth d, for all sets at once, without sorting the
+// strings: every string of length > d ORs its byte d into the 256-bit
+// child-label set of the node it has reached (its parent at depth d); the
+// parents of a level, in order, give their children consecutive ids (first
+// child = the level's end + an exclusive scan of the sets' popcounts), and a
+// string moves to child first_child + popcount(labels below its byte). Level d
+// is thus ordered by (set, parent, byte): breadth-first with sorted siblings
+// within every set, the sets' nodes interleaved by depth. A final pass
+// renumbers every node to base(set) + (its rank within the set's own
+// breadth-first order), the layout of the host builder.
+#include <stdint.h>
+
+#include <algorithm>
+#include <vector>
+
+#include <cuda_runtime.h>
+
+#include "tm_internal.h"
+
+namespace tmk {
+
+namespace {
+
+constexpr int kBThreads = 256;
+constexpr int kScanTile = 1024;  // parents per tile of the level scan
+
+__device__ __forceinline__ void pdl_go() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_after() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... Params, typename... Args>
+cudaError_t launch(void (*kernel)(Params...), int64_t grid, int block, cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(grid < 1 ? 1 : grid));
+    cfg.blockDim = dim3(unsigned(block));
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+}
+
+// Strings: their set (from set_offsets), their node (the set's root), and the
+// roots of sets with an empty string are terminal. Level 0 = the M roots.
+__global__ void k_b_init(const int64_t *__restrict__ off, const int32_t *__restrict__ set_off, int32_t M,
+                         int32_t K, int32_t *__restrict__ str_set, int32_t *__restrict__ cur,
+                         int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
+                         uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g,
+                         int32_t *__restrict__ ls) {
+    pdl_go();
+    pdl_after();
+    const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < M) {
+        parent_g[i] = -1;
+        label_g[i] = 0;
+        set_g[i] = i;
+        depth_g[i] = 0;
+    }
+    if (i == 0) {
+        ls[0] = 0;
+        ls[1] = M;
+    }
+    if (i >= K) return;
+    int32_t lo = 0, hi = M;  // the set s with set_off[s] <= i < set_off[s + 1]
+    while (hi - lo > 1) {
+        const int32_t mid = (lo + hi) >> 1;
+        if (set_off[mid] <= i) lo = mid;
+        else hi = mid;
+    }
+    str_set[i] = lo;
+    cur[i] = lo;
+    if (off[i + 1] == off[i]) term_g[lo] = 1;  // the empty string: the root is terminal
+}
+
+// Level d, pass 1: each string of length > d sets its byte d in its parent's
+// child-label set (bits of level d: row x - ls[d]).
+__global__ void k_b_bits(const uint8_t *__restrict__ bytes, const int64_t *__restrict__ off, int32_t K, int32_t d,
+                         const int32_t *__restrict__ cur, const int32_t *__restrict__ ls,
+                         uint32_t *__restrict__ bits) {
+    pdl_go();
+    pdl_after();
+    const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= K) return;
+    const int64_t a = off[i] - off[0];
+    if (off[i + 1] - off[i] <= d) return;
+    const uint32_t b = bytes[a + d];
+    atomicOr(bits + int64_t(cur[i] - ls[d]) * 8 + (b >> 5), 1u << (b & 31u));
+}
+
+__device__ __forceinline__ int32_t row_popc(const uint32_t *bits, int64_t row) {
+    const uint4 *r = reinterpret_cast<const uint4 *>(bits + row * 8);
+    const uint4 a = r[0], b = r[1];
+    return __popc(a.x) + __popc(a.y) + __popc(a.z) + __popc(a.w) + __popc(b.x) + __popc(b.y) + __popc(b.z) +
+           __popc(b.w);
+}
+
+// Block-wide exclusive scan of one int per thread (kBThreads threads).
+__device__ __forceinline__ int32_t block_excl_scan(int32_t v, int32_t *warp_sums, int32_t *total) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    int32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) warp_sums[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+        int32_t w = lane < kBThreads / 32 ? warp_sums[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < kBThreads / 32) warp_sums[lane] = w;
+    }
+    __syncthreads();
+    const int32_t before = wid > 0 ? warp_sums[wid - 1] : 0;
+    if (total) *total = warp_sums[kBThreads / 32 - 1];
+    return before + x - v;
+}
+
+// Level d, pass 2: the children of every tile of kScanTile parents.
+__global__ void __launch_bounds__(kBThreads) k_b_tile_sums(int32_t d, const int32_t *__restrict__ ls,
+                                                           const uint32_t *__restrict__ bits,
+                                                           int32_t *__restrict__ tile_sum) {
+    __shared__ int32_t ws[kBThreads / 32];
+    pdl_go();
+    pdl_after();
+    const int32_t width = ls[d + 1] - ls[d];
+    const int32_t t0 = blockIdx.x * kScanTile;
+    if (t0 >= width) {
+        if (threadIdx.x == 0) tile_sum[blockIdx.x] = 0;
+        return;
+    }
+    int32_t s = 0;
+    for (int32_t j = threadIdx.x; j < kScanTile; j += kBThreads)
+        if (t0 + j < width) s += row_popc(bits, t0 + j);
+    int32_t tot;
+    block_excl_scan(s, ws, &tot);
+    if (threadIdx.x == 0) tile_sum[blockIdx.x] = tot;
+}
+
+// Level d, pass 3 (one CTA): exclusive scan of the tile sums; the end of level d + 1.
+__global__ void __launch_bounds__(kBThreads) k_b_tile_scan(int32_t d, int32_t n_tiles, int32_t *__restrict__ ls,
+                                                           int32_t *__restrict__ tile_sum) {
+    __shared__ int32_t ws[kBThreads / 32];
+    __shared__ int32_t carry;
+    pdl_go();
+    pdl_after();
+    if (threadIdx.x == 0) carry = 0;
+    __syncthreads();
+    for (int32_t t0 = 0; t0 < n_tiles; t0 += kBThreads) {
+        const int32_t t = t0 + threadIdx.x;
+        const int32_t v = t < n_tiles ? tile_sum[t] : 0;
+        int32_t tot;
+        const int32_t ex = block_excl_scan(v, ws, &tot);
+        if (t < n_tiles) tile_sum[t] = carry + ex;
+        __syncthreads();
+        if (threadIdx.x == 0) carry += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) ls[d + 2] = ls[d + 1] + carry;
+}
+
+// Level d, pass 4: first child of every parent of the level; also clears the
+// other bits buffer (level d - 1's rows) for level d + 1.
+__global__ void __launch_bounds__(kBThreads) k_b_first(int32_t d, const int32_t *__restrict__ ls,
+                                                       const uint32_t *__restrict__ bits,
+                                                       const int32_t *__restrict__ tile_off,
+                                                       int32_t *__restrict__ first, uint32_t *__restrict__ other) {
+    __shared__ int32_t ws[kBThreads / 32];
+    __shared__ int32_t carry;
+    pdl_go();
+    pdl_after();
+    const int32_t width = ls[d + 1] - ls[d];
+    const int32_t prev = d > 0 ? ls[d] - ls[d - 1] : 0;
+    const int32_t t0 = blockIdx.x * kScanTile;
+    for (int32_t j = threadIdx.x; j < kScanTile; j += kBThreads)
+        if (t0 + j < prev) {
+            uint4 *r = reinterpret_cast<uint4 *>(other + int64_t(t0 + j) * 8);
+            r[0] = make_uint4(0u, 0u, 0u, 0u);
+            r[1] = make_uint4(0u, 0u, 0u, 0u);
+        }
+    if (t0 >= width) return;
+    if (threadIdx.x == 0) carry = ls[d + 1] + tile_off[blockIdx.x];
+    __syncthreads();
+    for (int32_t j0 = 0; j0 < kScanTile; j0 += kBThreads) {
+        const int32_t x = t0 + j0 + threadIdx.x;
+        const int32_t c = x < width ? row_popc(bits, x) : 0;
+        int32_t tot;
+        const int32_t ex = block_excl_scan(c, ws, &tot);
+        if (x < width) first[x] = carry + ex;
+        __syncthreads();
+        if (threadIdx.x == 0) carry += tot;
+        __syncthreads();
+    }
+}
+
+// Level d, pass 5: every string of length > d moves to its child at depth
+// d + 1, writing the child's parent, label, set, depth and terminal flag
+// (all strings through a child write the same values).
+__global__ void k_b_move(const uint8_t *__restrict__ bytes, const int64_t *__restrict__ off, int32_t K, int32_t d,
+                         const int32_t *__restrict__ ls, const uint32_t *__restrict__ bits,
+                         const int32_t *__restrict__ first, const int32_t *__restrict__ str_set,
+                         int32_t *__restrict__ cur, int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
+                         uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g) {
+    pdl_go();
+    pdl_after();
+    const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= K) return;
+    const int64_t len = off[i + 1] - off[i];
+    if (len <= d) return;
+    const uint32_t b = bytes[off[i] - off[0] + d];
+    const int32_t x = cur[i];
+    const int64_t row = x - ls[d];
+    const uint32_t *r = bits + row * 8;
+    int32_t below = 0;
+#pragma unroll
+    for (int w = 0; w < 8; w++) {
+        const uint32_t v = r[w];
+        const int32_t lo = w * 32;
+        if (int32_t(b) >= lo + 32) below += __popc(v);
+        else if (int32_t(b) >= lo) below += __popc(v & ((1u << (b - lo)) - 1u));
+    }
+    const int32_t c = first[row] + below;
+    parent_g[c] = x;
+    label_g[c] = uint8_t(b);
+    set_g[c] = str_set[i];
+    depth_g[c] = d + 1;
+    if (len == d + 1) term_g[c] = 1;
+    cur[i] = c;
+}
+
+// Renumbering, pass 1: the level-order range [first, end) of every (set,
+// depth) group (level order sorts by depth, then set, so each group is one
+// run), and the characters of the distinct strings (depths of terminals).
+__global__ void k_b_count(const int32_t *__restrict__ ls, int32_t D, const int32_t *__restrict__ set_g,
+                          const int32_t *__restrict__ depth_g, const uint8_t *__restrict__ term_g,
+                          int32_t *__restrict__ first_sd, int32_t *__restrict__ end_sd,
+                          unsigned long long *__restrict__ n_chars) {
+    pdl_go();
+    pdl_after();
+    const int32_t n = ls[D + 1];
+    unsigned long long chars = 0;
+    for (int32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
+        const int32_t k = set_g[g] * (D + 1) + depth_g[g];
+        if (g == 0 || set_g[g - 1] * (D + 1) + depth_g[g - 1] != k) first_sd[k] = g;
+        if (g == n - 1 || set_g[g + 1] * (D + 1) + depth_g[g + 1] != k) end_sd[k] = g + 1;
+        if (term_g[g]) chars += unsigned(depth_g[g]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) chars += __shfl_down_sync(0xffffffffu, chars, o);
+    if ((threadIdx.x & 31) == 0 && chars) atomicAdd(n_chars, chars);
+}
+
+__device__ __forceinline__ int32_t group_size(const int32_t *first_sd, const int32_t *end_sd, int32_t k) {
+    const int32_t e = end_sd[k];
+    return e > 0 ? e - first_sd[k] : 0;  // end 0: no node of that set at that depth
+}
+
+// Renumbering, pass 2 (one CTA): the offset of every (set, depth) in the
+// final layout (set after set, each in breadth-first order), and the roots.
+__global__ void __launch_bounds__(kBThreads) k_b_offsets(int32_t M, int32_t D, const int32_t *__restrict__ first_sd,
+                                                         const int32_t *__restrict__ end_sd,
+                                                         int32_t *__restrict__ off_sd, int32_t *__restrict__ roots) {
+    __shared__ int32_t ws[kBThreads / 32];
+    __shared__ int32_t carry;
+    pdl_go();
+    pdl_after();
+    if (threadIdx.x == 0) carry = 0;
+    __syncthreads();
+    for (int32_t s0 = 0; s0 < M; s0 += kBThreads) {
+        const int32_t s = s0 + threadIdx.x;
+        int32_t n_s = 0;
+        if (s < M)
+            for (int32_t d = 0; d <= D; d++) n_s += group_size(first_sd, end_sd, s * (D + 1) + d);
+        int32_t tot;
+        const int32_t base = carry + block_excl_scan(n_s, ws, &tot);
+        if (s < M) {
+            roots[s] = base;
+            int32_t o = base;
+            for (int32_t d = 0; d <= D; d++) {
+                off_sd[s * (D + 1) + d] = o;
+                o += group_size(first_sd, end_sd, s * (D + 1) + d);
+            }
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) carry += tot;
+        __syncthreads();
+    }
+}
+
+// Renumbering, pass 3: final id of every level-order id.
+__global__ void k_b_map(const int32_t *__restrict__ ls, int32_t D, const int32_t *__restrict__ set_g,
+                        const int32_t *__restrict__ depth_g, const int32_t *__restrict__ first_sd,
+                        const int32_t *__restrict__ off_sd, int32_t *__restrict__ map) {
+    pdl_go();
+    pdl_after();
+    const int32_t n = ls[D + 1];
+    for (int32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
+        const int32_t k = set_g[g] * (D + 1) + depth_g[g];
+        map[g] = off_sd[k] + (g - first_sd[k]);
+    }
+}
+
+// Renumbering, pass 4: parent, label and terminal in the final layout.
+__global__ void k_b_permute(const int32_t *__restrict__ ls, int32_t D, const int32_t *__restrict__ map,
+                            const int32_t *__restrict__ parent_g, const uint8_t *__restrict__ label_g,
+                            const uint8_t *__restrict__ term_g, int32_t *__restrict__ parent,
+                            uint8_t *__restrict__ label, uint8_t *__restrict__ terminal) {
+    pdl_go();
+    pdl_after();
+    const int32_t n = ls[D + 1];
+    for (int32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
+        const int32_t f = map[g];
+        const int32_t p = parent_g[g];
+        parent[f] = p < 0 ? -1 : map[p];
+        label[f] = label_g[g];
+        terminal[f] = term_g[g];
+    }
+}
+
+}  // namespace
+
+// Scratch of one device build: the strings, level-order node arrays (at most
+// K_chars + M nodes), two child-label buffers of K rows, the level scans.
+struct DeviceBuild::Scratch {
+    void *base = nullptr;
+    uint8_t *bytes;
+    int64_t *off;
+    int32_t *set_off, *str_set, *cur, *parent_g, *set_g, *depth_g, *first, *tile_sum, *ls;
+    uint8_t *label_g, *term_g;
+    uint32_t *bits[2];
+    int32_t *end_sd, *first_sd, *off_sd, *roots, *map;
+    unsigned long long *n_chars;
+};
+
+DeviceBuild::~DeviceBuild() {
+    if (s_) {
+        if (s_->base) cudaFreeAsync(s_->base, stream_);
+        delete s_;
+    }
+}
+
+cudaError_t DeviceBuild::levels(const uint8_t *h_bytes, const int64_t *h_off, const int32_t *h_set_off, int32_t M,
+                                int32_t K, int64_t n_bytes, int32_t D, int num_sms, cudaMemPool_t pool,
+                                cudaStream_t st, int32_t *n_nodes,
+                                std::vector<int32_t> *roots, int64_t *n_chars) {
+    stream_ = st;
+    M_ = M;
+    D_ = D;
+    s_ = new Scratch();
+    const int64_t U = n_bytes + M;          // nodes at most
+    const int64_t W = std::max<int64_t>(K, M);  // parents of one level at most
+    const int64_t tiles = (W + kScanTile - 1) / kScanTile + 1;
+    const int64_t sd = int64_t(M) * (D + 1);
+    size_t total = 0;
+    auto add = [&](size_t b) {
+        const size_t o = total;
+        total += (b + 255) / 256 * 256;
+        return o;
+    };
+    const size_t o_bytes = add(size_t(n_bytes) + 16), o_off = add(8 * (size_t(K) + 1)),
+                 o_soff = add(4 * (size_t(M) + 1)), o_sset = add(4 * size_t(K)), o_cur = add(4 * size_t(K)),
+                 o_par = add(4 * size_t(U)), o_set = add(4 * size_t(U)), o_dep = add(4 * size_t(U)),
+                 o_first = add(4 * size_t(W)), o_ts = add(4 * size_t(tiles)), o_ls = add(4 * (size_t(D) + 2)),
+                 o_lab = add(size_t(U)), o_term = add(size_t(U)), o_b0 = add(32 * size_t(W) + 32),
+                 o_b1 = add(32 * size_t(W) + 32), o_end = add(4 * size_t(sd)), o_fsd = add(4 * size_t(sd)),
+                 o_osd = add(4 * size_t(sd)), o_roots = add(4 * size_t(M)), o_map = add(4 * size_t(U)),
+                 o_nch = add(8);
+    cudaError_t e = cudaMallocFromPoolAsync(&s_->base, total, pool, st);
+    if (e != cudaSuccess) return e;
+    char *b = static_cast<char *>(s_->base);
+    s_->bytes = reinterpret_cast<uint8_t *>(b + o_bytes);
+    s_->off = reinterpret_cast<int64_t *>(b + o_off);
+    s_->set_off = reinterpret_cast<int32_t *>(b + o_soff);
+    s_->str_set = reinterpret_cast<int32_t *>(b + o_sset);
+    s_->cur = reinterpret_cast<int32_t *>(b + o_cur);
+    s_->parent_g = reinterpret_cast<int32_t *>(b + o_par);
+    s_->set_g = reinterpret_cast<int32_t *>(b + o_set);
+    s_->depth_g = reinterpret_cast<int32_t *>(b + o_dep);
+    s_->first = reinterpret_cast<int32_t *>(b + o_first);
+    s_->tile_sum = reinterpret_cast<int32_t *>(b + o_ts);
+    s_->ls = reinterpret_cast<int32_t *>(b + o_ls);
+    s_->label_g = reinterpret_cast<uint8_t *>(b + o_lab);
+    s_->term_g = reinterpret_cast<uint8_t *>(b + o_term);
+    s_->bits[0] = reinterpret_cast<uint32_t *>(b + o_b0);
+    s_->bits[1] = reinterpret_cast<uint32_t *>(b + o_b1);
+    s_->end_sd = reinterpret_cast<int32_t *>(b + o_end);
+    s_->first_sd = reinterpret_cast<int32_t *>(b + o_fsd);
+    s_->off_sd = reinterpret_cast<int32_t *>(b + o_osd);
+    s_->roots = reinterpret_cast<int32_t *>(b + o_roots);
+    s_->map = reinterpret_cast<int32_t *>(b + o_map);
+    s_->n_chars = reinterpret_cast<unsigned long long *>(b + o_nch);
+    // inputs; zeroed flags, buffers and counters
+    if ((n_bytes > 0 &&
+         (e = cudaMemcpyAsync(s_->bytes, h_bytes, size_t(n_bytes), cudaMemcpyHostToDevice, st)) != cudaSuccess) ||
+        (e = cudaMemcpyAsync(s_->off, h_off, 8 * (size_t(K) + 1), cudaMemcpyHostToDevice, st)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(s_->set_off, h_set_off, 4 * (size_t(M) + 1), cudaMemcpyHostToDevice, st)) !=
+            cudaSuccess ||
+        (e = cudaMemsetAsync(s_->term_g, 0, size_t(U), st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s_->bits[0], 0, 32 * size_t(W) + 32, st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s_->bits[1], 0, 32 * size_t(W) + 32, st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s_->end_sd, 0, 4 * size_t(sd), st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s_->first_sd, 0x7F, 4 * size_t(sd), st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s_->n_chars, 0, 8, st)) != cudaSuccess)
+        return e;
+    const int64_t sgrid = (W + kBThreads - 1) / kBThreads;
+    if ((e = launch(k_b_init, sgrid, kBThreads, st, static_cast<const int64_t *>(s_->off),
+                    static_cast<const int32_t *>(s_->set_off), M, K, s_->str_set, s_->cur, s_->parent_g, s_->label_g,
+                    s_->term_g, s_->set_g, s_->depth_g, s_->ls)) != cudaSuccess)
+        return e;
+    const int64_t kgrid = (int64_t(K) + kBThreads - 1) / kBThreads;
+    const int32_t n_tiles = int32_t((W + kScanTile - 1) / kScanTile);
+    for (int32_t d = 0; d < D; d++) {
+        uint32_t *bits = s_->bits[d & 1];
+        if ((e = launch(k_b_bits, kgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
+                        static_cast<const int64_t *>(s_->off), K, d, static_cast<const int32_t *>(s_->cur),
+                        static_cast<const int32_t *>(s_->ls), bits)) != cudaSuccess ||
+            (e = launch(k_b_tile_sums, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
+                        static_cast<const uint32_t *>(bits), s_->tile_sum)) != cudaSuccess ||
+            (e = launch(k_b_tile_scan, 1, kBThreads, st, d, n_tiles, s_->ls, s_->tile_sum)) != cudaSuccess ||
+            (e = launch(k_b_first, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
+                        static_cast<const uint32_t *>(bits), static_cast<const int32_t *>(s_->tile_sum), s_->first,
+                        s_->bits[(d + 1) & 1])) != cudaSuccess ||
+            (e = launch(k_b_move, kgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
+                        static_cast<const int64_t *>(s_->off), K, d, static_cast<const int32_t *>(s_->ls),
+                        static_cast<const uint32_t *>(bits), static_cast<const int32_t *>(s_->first),
+                        static_cast<const int32_t *>(s_->str_set), s_->cur, s_->parent_g, s_->label_g, s_->term_g,
+                        s_->set_g, s_->depth_g)) != cudaSuccess)
+            return e;
+    }
+    const int64_t ngrid = std::min<int64_t>((U + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
+    if ((e = launch(k_b_count, ngrid, kBThreads, st, static_cast<const int32_t *>(s_->ls), D,
+                    static_cast<const int32_t *>(s_->set_g), static_cast<const int32_t *>(s_->depth_g),
+                    static_cast<const uint8_t *>(s_->term_g), s_->first_sd, s_->end_sd, s_->n_chars)) != cudaSuccess ||
+        (e = launch(k_b_offsets, 1, kBThreads, st, M, D, static_cast<const int32_t *>(s_->first_sd),
+                    static_cast<const int32_t *>(s_->end_sd), s_->off_sd, s_->roots)) != cudaSuccess ||
+        (e = launch(k_b_map, ngrid, kBThreads, st, static_cast<const int32_t *>(s_->ls), D,
+                    static_cast<const int32_t *>(s_->set_g), static_cast<const int32_t *>(s_->depth_g),
+                    static_cast<const int32_t *>(s_->first_sd), static_cast<const int32_t *>(s_->off_sd), s_->map)) !=
+            cudaSuccess)
+        return e;
+    // the node count, the roots and the characters (host-synchronous)
+    int32_t n = 0;
+    unsigned long long nc = 0;
+    roots->resize(size_t(M));
+    if ((e = cudaMemcpyAsync(&n, s_->ls + D + 1, 4, cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(roots->data(), s_->roots, 4 * size_t(M), cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(&nc, s_->n_chars, 8, cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaStreamSynchronize(st)) != cudaSuccess)
+        return e;
+    *n_nodes = n;
+    *n_chars = int64_t(nc);
+    n_ = n;
+    return cudaSuccess;
+}
+
+cudaError_t DeviceBuild::emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms) {
+    const int64_t ngrid = std::min<int64_t>((int64_t(n_) + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
+    return launch(k_b_permute, ngrid, kBThreads, stream_, static_cast<const int32_t *>(s_->ls), D_,
+                  static_cast<const int32_t *>(s_->map), static_cast<const int32_t *>(s_->parent_g),
+                  static_cast<const uint8_t *>(s_->label_g), static_cast<const uint8_t *>(s_->term_g), parent, label,
+                  terminal);
+}
+
+}  // namespace tmk

@@ -260,6 +260,40 @@ std::string build_forest(const uint8_t *bytes, const int64_t *offsets, const int
     return "";
 }
 
+// In breadth-first order with ascending sibling bytes, the children of a node
+// are consecutive ids after it, so a depth-first walk that visits them in id
+// order is the builder's pre-order (sorted strings); set i's walk fills
+// positions roots[i] .. roots[i + 1] - 1.
+void pre_order_from_parents(HostTrie *t) {
+    const int32_t n = t->n;
+    t->pre_node.resize(size_t(n));
+    t->pre_depth.resize(size_t(n));
+    t->pre_size.resize(size_t(n));
+    std::vector<int32_t> first(size_t(n), -1), cnt(size_t(n), 0), size(size_t(n), 1);
+    for (int32_t c = 0; c < n; c++) {
+        const int32_t p = t->parent[size_t(c)];
+        if (p < 0) continue;
+        if (first[size_t(p)] < 0) first[size_t(p)] = c;
+        cnt[size_t(p)]++;
+    }
+    for (int32_t c = n - 1; c > 0; c--)  // a child's id is above its parent's
+        if (t->parent[size_t(c)] >= 0) size[size_t(t->parent[size_t(c)])] += size[size_t(c)];
+    std::vector<std::pair<int32_t, int32_t>> stack;  // (node, depth)
+    int32_t pos = 0;
+    for (const int32_t r : t->roots) {
+        stack.emplace_back(r, 0);
+        while (!stack.empty()) {
+            const auto [x, d] = stack.back();
+            stack.pop_back();
+            t->pre_node[size_t(pos)] = x;
+            t->pre_depth[size_t(pos)] = d;
+            t->pre_size[size_t(pos)] = size[size_t(x)];
+            pos++;
+            for (int32_t k = cnt[size_t(x)] - 1; k >= 0; k--) stack.emplace_back(first[size_t(x)] + k, d + 1);
+        }
+    }
+}
+
 std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, HostVocab *out) {
     if (V < 2) return "V must be >= 2 (token V-1 is EOS)";
     if (offsets[0] < 0) return "vocab offsets must be non-negative";

@@ -113,11 +113,21 @@ extern "C" int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, 
     int rc = scratch_ptr(dev, &dscratch);
     if (rc != TRIE_OK) return rc;
 
-    // stage: trie arrays from the handle's host copy
+    // stage: trie arrays from the handle's host copy; a forest built on the
+    // device has none, and its device arrays are copied within the device
+    bool on_device;
+    {
+        std::lock_guard<std::mutex> hl(h->mu);
+        on_device = !h->host_arrays;
+    }
+    if (on_device && h->dev.device != dev)
+        return tmk::set_error(TRIE_EINVAL, "handle was built on another device");
     unsigned char *st = g_stage;
-    memcpy(st + o_par, t.parent.data(), 4 * n);
-    memcpy(st + o_lab, t.label.data(), n);
-    memcpy(st + o_term, t.terminal.data(), n);
+    if (!on_device) {
+        memcpy(st + o_par, t.parent.data(), 4 * n);
+        memcpy(st + o_lab, t.label.data(), n);
+        memcpy(st + o_term, t.terminal.data(), n);
+    }
     // stage: tokens 16-byte aligned, EOS and byte-less tokens with length 0
     uint32_t *toff = reinterpret_cast<uint32_t *>(st + o_toff);
     uint16_t *tlen = reinterpret_cast<uint16_t *>(st + o_tlen);
@@ -161,6 +171,13 @@ extern "C" int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, 
     }
 
     unsigned char *d = static_cast<unsigned char *>(dscratch);
+    if (on_device && n > 0 &&
+        ((e = cudaMemcpyAsync(d + o_par, h->dev.parent, 4 * n, cudaMemcpyDeviceToDevice, stream)) != cudaSuccess ||
+         (e = cudaMemcpyAsync(d + o_lab, h->dev.label, n, cudaMemcpyDeviceToDevice, stream)) != cudaSuccess ||
+         (e = cudaMemcpyAsync(d + o_term, h->dev.terminal, n, cudaMemcpyDeviceToDevice, stream)) != cudaSuccess)) {
+        cudaGetLastError();
+        return tmk::set_error(TRIE_ECUDA, "copy of the device-built trie into the no-alloc scratch failed");
+    }
     tmk::DevTrie dt;
     dt.device = dev;
     dt.parent = reinterpret_cast<const int32_t *>(d + o_par);

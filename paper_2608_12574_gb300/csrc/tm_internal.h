@@ -241,6 +241,36 @@ struct DevLazy {
     LazyNode *pre = nullptr;        // [n] by pre-order position
 };
 
+// A forest built on the device (device_build.cu): levels() runs the level
+// loop and the renumbering into its own scratch and returns the node count,
+// the roots and the characters (host-synchronous); emit() writes parent,
+// label and terminal of the final layout into the caller's device arrays
+// (asynchronous); the destructor frees the scratch after them.
+constexpr int32_t kDeviceBuildMaxDepth = 1024;        // longer strings: the host builder
+constexpr int64_t kDeviceBuildMaxGroups = int64_t(1) << 24;  // sets x (depths + 1) above: the host builder
+class DeviceBuild {
+public:
+    DeviceBuild() = default;
+    DeviceBuild(const DeviceBuild &) = delete;
+    DeviceBuild &operator=(const DeviceBuild &) = delete;
+    ~DeviceBuild();
+    cudaError_t levels(const uint8_t *h_bytes, const int64_t *h_off, const int32_t *h_set_off, int32_t M, int32_t K,
+                       int64_t n_bytes, int32_t D, int num_sms, cudaMemPool_t pool, cudaStream_t st,
+                       int32_t *n_nodes,
+                       std::vector<int32_t> *roots, int64_t *n_chars);
+    cudaError_t emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms);
+
+private:
+    struct Scratch;
+    Scratch *s_ = nullptr;
+    cudaStream_t stream_ = nullptr;
+    int32_t M_ = 0, D_ = 0, n_ = 0;
+};
+
+// The pre-order tables (pre_node / pre_depth / pre_size) of a trie or forest
+// from its breadth-first parent array (a depth-first walk per root).
+void pre_order_from_parents(HostTrie *t);
+
 // Character-position masks (App. K): formats of at most kFmtMaxLen positions
 // (their classes are staged in shared memory, 32 bytes per position).
 constexpr int32_t kFmtMaxLen = 1024;
@@ -263,6 +293,7 @@ struct fmt_s {
 struct trie_s {
     tmk::HostTrie host;
     std::mutex mu;                       // guards dev / vocab / mask fields
+    bool host_arrays = true;             // host parent / label / terminal / pre_* present (else on the device only)
     tmk::DevTrie dev;
     std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
@@ -277,6 +308,12 @@ namespace tmk {
 // Records msg as the calling thread's last error (trie_last_error) and
 // returns code.
 int set_error(int code, const char *msg);
+// Copies the host arrays of a device-built handle back from the device and
+// derives its pre-order tables (no-op for handles built on the host).
+int ensure_host_arrays(trie_s *h);
+// The library's device memory pool of device dev (created on first use;
+// nullptr if it cannot be created).
+cudaMemPool_t device_pool(int dev);
 
 // Kernel launchers (kernels.cu). Each returns the launch's cudaError_t.
 cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaStream_t st);

@@ -27,6 +27,7 @@ _P, _I32, _I64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
 SIGNATURES = {
     "trie_build": (ctypes.c_int, [_P, _P, _I32, _P]),
     "trie_build_many": (ctypes.c_int, [_P, _P, _P, _I32, _P]),
+    "trie_build_many_device": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_num_nodes": (_I32, [_P]),
     "trie_root": (_I32, [_P, _I32]),
     "trie_num_sets": (_I32, [_P]),
@@ -192,6 +193,19 @@ def trie_build_many(set_bytes, set_offsets, set_index) -> Trie:
     si = _host(set_index, np.int32)
     h = ctypes.c_void_p()
     _check(lib.trie_build_many(_hp(b), _hp(o), _hp(si), len(si) - 1, ctypes.byref(h)))
+    return Trie(h)
+
+
+def trie_build_many_device(set_bytes, set_offsets, set_index, stream=None) -> Trie:
+    """trie_build_many with the level loop on the current CUDA device (same node layout)."""
+    import torch
+    lib = load_library()
+    b = _host(set_bytes, np.uint8)
+    o = _host(set_offsets, np.int64)
+    si = _host(set_index, np.int32)
+    h = ctypes.c_void_p()
+    _check(lib.trie_build_many_device(_hp(b), _hp(o), _hp(si), len(si) - 1,
+                                      _stream(stream, torch.cuda.current_device()), ctypes.byref(h)))
     return Trie(h)
 
 

@@ -163,6 +163,27 @@ def test_build_many_argument_errors(lib):
                                ctypes.byref(h)) == T.TRIE_EINVAL
 
 
+def test_build_many_device_argument_errors(lib):
+    """Bad arguments are rejected before any device call (none is made here)."""
+    h = ctypes.c_void_p()
+    b = np.frombuffer(b"abcd", np.uint8).copy()
+    offs = np.array([0, 2, 4], np.int64)
+    bad_first = np.array([1, 2], np.int32)
+    bad_order = np.array([0, 2, 1], np.int32)
+    dec = np.array([0, 3, 2], np.int64)
+    ok = np.array([0, 2], np.int32)
+    f = lib.trie_build_many_device
+    assert f(b.ctypes.data, offs.ctypes.data, bad_first.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert f(b.ctypes.data, offs.ctypes.data, bad_order.ctypes.data, 2, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert f(b.ctypes.data, offs.ctypes.data, None, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert f(b.ctypes.data, offs.ctypes.data, ok.ctypes.data, 0, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert f(b.ctypes.data, offs.ctypes.data, ok.ctypes.data, 1, None, None) == T.TRIE_EINVAL
+    assert f(b.ctypes.data, dec.ctypes.data, ok.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert "non-decreasing" in T.trie_last_error()
+    assert f(None, offs.ctypes.data, ok.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    assert h.value is None
+
+
 def test_null_handle_queries(lib):
     assert lib.trie_num_nodes(None) == -1
     assert lib.trie_root(None, 0) == -1

@@ -1,0 +1,215 @@
+"""GPU: forests built on the device (trie_build_many_device) against the CPU
+oracle's tries and the host builder, through the C ABI.
+
+The node numbering is part of the ABI (breadth-first per set, siblings by
+ascending byte, sets concatenated in order), so a device-built forest must
+equal the host-built one array for array, and every set must equal the
+oracle's own trie of that set. The downstream calls (valid lists, lazy rows,
+the no-alloc compile, the fused decode step) must then give the same results
+on either handle.
+"""
+from __future__ import annotations
+
+import random
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_12574_gb300 import triemask as T
+from paper_2608_12574_gb300 import workloads as W
+from pins import random_case
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="session")
+def cuda():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_12574_gb300 import _build
+    _build.build()
+    T.load_library()
+    oracle.build()
+    return torch.device("cuda:0")
+
+
+def _np_u32(t):
+    import torch
+    return t.cpu().contiguous().view(torch.int32).numpy().view(np.uint32)
+
+
+def _forest(sets):
+    flat = [s for st in sets for s in st]
+    index = np.cumsum([0] + [len(s) for s in sets]).astype(np.int32)
+    sb, so = W.pack(flat)
+    return sb, so, index
+
+
+def _check_against_oracle(h, sets):
+    """Every set of h equals the oracle's trie of that set, at its root."""
+    c = h.csr()
+    assert h.num_sets == len(sets)
+    chars, depth = 0, 0
+    for i, st in enumerate(sets):
+        r = h.root(i)
+        ot = oracle.Trie(*W.pack(st))
+        n = ot.num_nodes
+        nxt = h.root(i + 1) if i + 1 < len(sets) else h.num_nodes
+        assert nxt - r == n, f"set {i}: {nxt - r} nodes, oracle {n}"
+        par = c["parent"][r:r + n].astype(np.int64)
+        par[par >= 0] -= r
+        assert np.array_equal(par, ot.parent), f"set {i}"
+        assert np.array_equal(c["label"][r:r + n], ot.label), f"set {i}"
+        assert np.array_equal(c["terminal"][r:r + n], ot.terminal), f"set {i}"
+        chars += ot.num_chars
+        depth = max(depth, int(ot.depth.max()))
+    assert h.num_chars == chars
+    assert h.max_depth == depth
+
+
+def _same_handles(a, b):
+    assert a.num_nodes == b.num_nodes and a.num_sets == b.num_sets
+    assert np.array_equal(a.roots(), b.roots())
+    assert a.num_chars == b.num_chars and a.max_depth == b.max_depth
+    ca, cb = a.csr(), b.csr()
+    for k in ca:
+        assert np.array_equal(ca[k], cb[k]), k
+
+
+def _random_sets(seed):
+    r = random.Random(seed)
+    sets = []
+    for j in range(r.randint(1, 12)):
+        if r.random() < 0.15:
+            sets.append([])  # a set with no strings: a lone, non-terminal root
+            continue
+        strings, _ = random_case(seed * 100 + j)
+        sets.append(strings)
+    return sets
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_device_forest_small_random(cuda, seed):
+    """Random forests (empty sets, empty strings, duplicates, prefixes of
+    other strings, bytes 0x00 / 0xFF): each set equals the oracle's trie, and
+    the whole forest equals the host builder's."""
+    sets = _random_sets(seed)
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _check_against_oracle(d, sets)
+    _same_handles(d, T.trie_build_many(sb, so, index))
+
+
+def test_device_forest_more_sets_than_strings(cuda):
+    """5,000 sets holding 3 strings in all: the root level is the widest."""
+    sets = [[] for _ in range(5000)]
+    sets[7] = [b"ab"]
+    sets[4000] = [b"", b"abc"]
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _same_handles(d, T.trie_build_many(sb, so, index))
+    c = d.csr()
+    assert d.num_nodes == 5000 + 2 + 3
+    assert d.root(7) == 7 and d.root(8) == 10 and c["terminal"][d.root(4000)] == 1
+
+
+def test_device_forest_single_set_mask_equals_oracle(cuda):
+    """A forest of one set (the K=100 tool names): the dense mask compiled on
+    the device-built handle equals the oracle's mask."""
+    import os
+    w = W.config(1)
+    d = T.trie_build_many_device(w.set_bytes, w.set_offsets, np.array([0, len(w.set_offsets) - 1], np.int32))
+    _same_handles(d, T.trie_build(w.set_bytes, w.set_offsets))
+    m = T.alloc_mask(d, w.V, cuda)
+    T.trie_compile_masks(d, w.vocab_bytes, w.vocab_offsets, w.V, m)
+    want = oracle.mask_all(oracle.Trie(w.set_bytes, w.set_offsets), oracle.Vocab(w.vocab_bytes, w.vocab_offsets),
+                           nthreads=os.cpu_count() or 1)
+    assert np.array_equal(_np_u32(m), want)
+
+
+def test_device_forest_long_strings_use_the_host_builder(cuda):
+    """Strings longer than the level loop's limit (1,024 bytes) go to the host
+    builder; the result is the same forest."""
+    rng = np.random.default_rng(11)
+    long = bytes(rng.integers(0, 3, 1500, dtype=np.uint8))
+    sets = [[long, long[:700], b"xy"], [long[:1100]]]
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _check_against_oracle(d, sets)
+    assert d.max_depth == 1500
+
+
+def test_device_forest_noalloc_compile(cuda):
+    """The no-alloc compile reads a device-built trie's arrays on the device;
+    its mask equals trie_compile_masks on the same handle."""
+    sets = _random_sets(3) + [[b"get", b"get_user", b"set"]]
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _, toks = random_case(77)
+    vb, vo = W.pack(toks)
+    V = len(toks)
+    m1 = T.alloc_mask(d, V, cuda)
+    m2 = T.alloc_mask(d, V, cuda)
+    m2.fill_(-1)
+    T.trie_compile_masks(d, vb, vo, V, m1)
+    T.trie_compile_masks_noalloc(d, vb, vo, V, m2)
+    assert np.array_equal(_np_u32(m1), _np_u32(m2))
+
+
+def test_device_forest_config5(cuda):
+    """The 256-request forest (4.8M nodes): equal to the host builder's; the
+    valid lists, lazy rows of sampled states and four fused list-driven
+    decode steps equal those of the host-built forest."""
+    import torch
+    w = W.config(5)
+    d = T.trie_build_many_device(w.set_bytes, w.set_offsets, w.set_index)
+    hst = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+    _same_handles(d, hst)
+    # sampled sets against the oracle
+    strings = W.unpack(w.set_bytes, w.set_offsets)
+    sel = [0, 1, 100, 255]
+    c = d.csr()
+    for i in sel:
+        ot = oracle.Trie(*W.pack(strings[w.set_index[i]:w.set_index[i + 1]]))
+        r, n = d.root(i), ot.num_nodes
+        assert np.array_equal(c["label"][r:r + n], ot.label)
+        assert np.array_equal(c["terminal"][r:r + n], ot.terminal)
+
+    T.trie_compile_lists(d, w.vocab_bytes, w.vocab_offsets, w.V)
+    T.trie_compile_lists(hst, w.vocab_bytes, w.vocab_offsets, w.V)
+    od, td = T.trie_copy_lists(d)
+    oh, th = T.trie_copy_lists(hst)
+    assert torch.equal(od, oh)
+    rows = np.repeat(np.arange(d.num_nodes, dtype=np.int64), np.diff(od.cpu().numpy()))
+    # the tokens of a row are in no particular order
+    assert np.array_equal(np.sort(rows * w.V + td.cpu().numpy()), np.sort(rows * w.V + th.cpu().numpy()))
+
+    B = 256
+    st = torch.as_tensor(d.roots()[:B].astype(np.int32), device=cuda)
+    sd, sh = st.clone(), st.clone()
+    tok = None
+    for step in range(5):
+        lg = W.logits(w, step, device="cuda", batch=B)
+        xd, xh = lg.clone(), lg.clone()
+        if tok is None:
+            T.trie_apply_lists(d, xd, sd)
+            T.trie_apply_lists(hst, xh, sh)
+        else:
+            nd, nh = torch.empty_like(sd), torch.empty_like(sh)
+            T.trie_advance_apply_lists(d, sd, tok, nd, xd)
+            T.trie_advance_apply_lists(hst, sh, tok, nh, xh)
+            assert torch.equal(nd, nh), f"step {step}"
+            sd, sh = nd, nh
+        assert torch.equal(xd.view(torch.int16), xh.view(torch.int16)), f"step {step}"
+        tok = torch.argmax(xd, dim=1).to(torch.int32)
+    assert int((sd >= 0).sum()) > 0  # the greedy walk stayed inside the tries
+
+    rng = np.random.default_rng(5)
+    states = rng.integers(0, d.num_nodes, 2048).astype(np.int32)
+    rows = []
+    for h in (d, hst):
+        T.trie_lazy_init(h, w.vocab_bytes, w.vocab_offsets, w.V, cache_rows=1024, max_batch=2048)
+        rows.append(_np_u32(T.trie_lazy_rows(h, torch.as_tensor(states, device=cuda), w.V)))
+    assert np.array_equal(rows[0], rows[1])
