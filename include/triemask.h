@@ -112,10 +112,16 @@ int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t 
  * of trie_build_many for the same arguments.
  *   Arguments as trie_build_many (all host, read during the call); stream is
  *   the stream the build kernels and the copies run on.
- * The strings are copied to the device and inserted level by level (depth
+ * The strings are staged on the device and inserted level by level (depth
  * d = 0, 1, ...) for all sets at once; the trie lives on the device only and
- * is bound to the current device. Host-synchronous: returns once the forest
- * is complete on `stream`. Calls that need the host arrays (trie_get_csr,
+ * is bound to the current device. Where the device reads pageable host
+ * memory coherently through the host's page tables (Grace CPUs over
+ * NVLink-C2C), a kernel reads the strings straight from the caller's arrays;
+ * elsewhere they are copied first (TRIEMASK_HOST_READ=copy in the
+ * environment forces the copies). The offsets are checked on the device.
+ * Host-synchronous: returns once the forest is complete on `stream`. Such a
+ * forest has no transition table: trie_advance and the fused calls walk the
+ * tokens' bytes. Calls that need the host arrays (trie_get_csr,
  * trie_lazy_init) copy them back once. Strings longer than 1024 bytes, more
  * than 2^24 (set, depth) pairs or more than 2^31-3 string bytes plus sets
  * are built by trie_build_many on the host instead. Device scratch (about

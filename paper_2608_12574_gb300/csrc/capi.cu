@@ -5,6 +5,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <memory>
 #include <mutex>
 #include <new>
@@ -177,7 +178,9 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
 // handle's own host arrays, which outlive them); the handle is bound to that
 // device.
 // Device arrays of a trie of n nodes (one allocation); nothing is uploaded.
-int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream) {
+// with_trans: also a transition table (8 or more slots per node) for the
+// compiles to record moves in.
+int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream, bool with_trans) {
     Layout L;
     const size_t o_par = L.add(sizeof(int32_t) * n);
     const size_t o_lab = L.add(n);
@@ -187,8 +190,8 @@ int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream) {
     const size_t o_win = L.add(sizeof(uint64_t) * 2 * n);
     const size_t o_d16 = L.add(n);
     const size_t o_anc = L.add(sizeof(int32_t) * 16 * n);
-    size_t trans_slots = 16;  // >= 8 per node, a power of two
-    while (trans_slots < 8 * n) trans_slots <<= 1;
+    size_t trans_slots = with_trans ? 16 : 0;  // >= 8 per node, a power of two
+    while (with_trans && trans_slots < 8 * n) trans_slots <<= 1;
     const size_t o_trans = L.add(sizeof(ulonglong2) * trans_slots);
     const size_t o_hits = L.add(sizeof(int2) * tmk::kHitSlots * n);  // compile scratch (probe -> scatter)
     const size_t o_hcnt = L.add(n);
@@ -206,8 +209,8 @@ int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream) {
     h->dev.window = reinterpret_cast<ulonglong2 *>(b + o_win);
     h->dev.depth16 = reinterpret_cast<uint8_t *>(b + o_d16);
     h->dev.anc = reinterpret_cast<int4 *>(b + o_anc);
-    h->dev.trans = reinterpret_cast<ulonglong2 *>(b + o_trans);
-    h->dev.trans_mask = uint32_t(trans_slots - 1);
+    h->dev.trans = with_trans ? reinterpret_cast<ulonglong2 *>(b + o_trans) : nullptr;
+    h->dev.trans_mask = with_trans ? uint32_t(trans_slots - 1) : 0u;
     h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
     h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
     return TRIE_OK;
@@ -240,7 +243,7 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     }
     const tmk::HostTrie &t = h->host;
     const size_t n = size_t(t.n);
-    int rc = alloc_device_trie(h, dev, n, stream);
+    int rc = alloc_device_trie(h, dev, n, stream, true);
     if (rc != TRIE_OK) return rc;
     struct Up { const void *dst; const void *src; size_t n; } ups[] = {
         {h->dev.parent, t.parent.data(), sizeof(int32_t) * n},
@@ -275,6 +278,30 @@ int prepare_trans(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, int sms, 
     if (e != cudaSuccess) return fail_cuda(e, "transition table clear");
     *fill = true;
     return TRIE_OK;
+}
+
+// Whether kernels on dev may read the caller's pageable host memory directly
+// (coherent access through the host's page tables, as on Grace systems over
+// NVLink-C2C). TRIEMASK_HOST_READ=copy in the environment forces the copy
+// path instead.
+bool host_memory_direct(int dev) {
+    static std::mutex mu;
+    static std::vector<int> cache;  // 0 unknown, 1 direct, 2 copy
+    std::lock_guard<std::mutex> lk(mu);
+    if (int(cache.size()) <= dev) cache.resize(size_t(dev) + 1, 0);
+    if (!cache[size_t(dev)]) {
+        int pageable = 0, host_tables = 0;
+        const char *env = getenv("TRIEMASK_HOST_READ");
+        const bool forced_copy = env && strcmp(env, "copy") == 0;
+        if (cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&host_tables, cudaDevAttrPageableMemoryAccessUsesHostPageTables, dev) !=
+                cudaSuccess) {
+            cudaGetLastError();
+            pageable = 0;
+        }
+        cache[size_t(dev)] = (!forced_copy && pageable == 1 && host_tables == 1) ? 1 : 2;
+    }
+    return cache[size_t(dev)] == 1;
 }
 
 int current_device(int *dev) {
@@ -459,41 +486,48 @@ int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const i
         if (set_offsets[i + 1] < set_offsets[i]) return fail(TRIE_EINVAL, "set_offsets must be non-decreasing");
     const int32_t K = set_offsets[M];
     if (K > 0 && !offsets) return fail(TRIE_EINVAL, "offsets is NULL");
-    if (K > 0 && offsets[K] > offsets[0] && !bytes) return fail(TRIE_EINVAL, "bytes is NULL");
-    int64_t max_len = 0;
-    for (int32_t i = 0; i < K; i++) {
-        if (offsets[i] < 0 || offsets[i + 1] < offsets[i])
-            return fail(TRIE_EINVAL, "offsets must be non-negative and non-decreasing");
-        max_len = std::max<int64_t>(max_len, offsets[i + 1] - offsets[i]);
-    }
-    const int64_t n_bytes = K > 0 ? offsets[K] - offsets[0] : 0;
-    // long strings (a long level loop), many sets with deep strings (the
-    // per-(set, depth) tables) or more bytes than node ids: the host builder
-    if (max_len > tmk::kDeviceBuildMaxDepth || int64_t(M) * (max_len + 1) > tmk::kDeviceBuildMaxGroups ||
-        n_bytes + M > int64_t(INT32_MAX) - 2)
+    static const int64_t zero = 0;
+    const int64_t *off = K > 0 ? offsets : &zero;
+    if (off[0] < 0 || off[K] < off[0]) return fail(TRIE_EINVAL, "offsets must be non-negative and non-decreasing");
+    const int64_t n_bytes = off[K] - off[0];
+    if (n_bytes > 0 && !bytes) return fail(TRIE_EINVAL, "bytes is NULL");
+    if (n_bytes + M > int64_t(INT32_MAX) - 2)  // more bytes than node ids: the host builder decides
         return trie_build_many(bytes, offsets, set_offsets, M, out);
     int dev, rc;
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    cudaMemPool_t pool = tmk::device_pool(dev);
+    if (!pool) return fail(TRIE_ECUDA, "creating the device memory pool for the forest build");
+    const int sms = num_sms(dev);
     trie_s *h = new (std::nothrow) trie_s;
     if (!h) return fail(TRIE_ENOMEM, "host allocation failed");
-    static const int64_t zero = 0;
-    const int64_t *off = K > 0 ? offsets : &zero;
-    const int sms = num_sms(dev);
-    int32_t n = 0;
+    int32_t n = 0, max_len = 0;
     int64_t n_chars = 0;
     cudaError_t e;
     {
         tmk::DeviceBuild db;
-        cudaMemPool_t pool = tmk::device_pool(dev);
-        e = pool ? db.levels(K > 0 ? bytes + off[0] : nullptr, off, set_offsets, M, K, n_bytes, int32_t(max_len),
-                             sms, pool, stream, &n, &h->host.roots, &n_chars)
-                 : cudaErrorMemoryAllocation;
+        bool ok = true;
+        e = db.stage(n_bytes > 0 ? bytes + off[0] : nullptr, off, set_offsets, M, K, n_bytes,
+                     host_memory_direct(dev), sms, pool, stream, &max_len, &ok);
+        if (e == cudaSuccess && !ok) {
+            delete h;
+            return fail(TRIE_EINVAL, "offsets must be non-negative and non-decreasing");
+        }
+        // long strings (a long level loop) or many sets with deep strings
+        // (the per-(set, depth) tables): the host builder
+        if (e == cudaSuccess &&
+            (max_len > tmk::kDeviceBuildMaxDepth || int64_t(M) * (max_len + 1) > tmk::kDeviceBuildMaxGroups)) {
+            delete h;
+            return trie_build_many(bytes, offsets, set_offsets, M, out);
+        }
+        if (e == cudaSuccess) e = db.levels(max_len, sms, &n, &h->host.roots, &n_chars);
         if (e == cudaSuccess) {
             h->host.n = n;
             h->host.n_chars = n_chars;
-            h->host.max_depth = int32_t(max_len);
+            h->host.max_depth = max_len;
             h->host_arrays = false;
-            if ((rc = alloc_device_trie(h, dev, size_t(n), stream)) != TRIE_OK) {
+            // per-batch sets are decoded for a few steps: no transition
+            // table to clear and fill (advance walks the tokens' bytes)
+            if ((rc = alloc_device_trie(h, dev, size_t(n), stream, false)) != TRIE_OK) {
                 delete h;
                 return rc;
             }
@@ -507,6 +541,7 @@ int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const i
     }
     if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
     if (e != cudaSuccess) {
+        cudaGetLastError();
         pool_free(h->dev.base);
         delete h;
         return fail_cuda(e, "building the forest on the device");

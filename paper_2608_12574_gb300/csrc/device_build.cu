@@ -44,13 +44,52 @@ cudaError_t launch(void (*kernel)(Params...), int64_t grid, int block, cudaStrea
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
 }
 
+// Staging: copies the strings' offsets, the set offsets and the bytes into
+// the scratch, checks the offsets (non-negative, non-decreasing) and finds
+// the longest string. The sources are either the caller's host memory, read
+// directly where the device accesses pageable memory coherently (Grace's
+// NVLink-C2C), or device copies of it (src_off == off: checked in place;
+// n_vec = 0: the bytes are in place). src_vec is the bytes' image in whole
+// 16-byte blocks (the first and last block may hold bytes outside the
+// strings; a 16-byte block never straddles a page).
+__global__ void k_b_stage(const int64_t *src_off, int32_t K, const int32_t *src_soff, int32_t M,
+                          const uint4 *src_vec, int64_t n_vec, int64_t *off, int32_t *soff, uint4 *vec,
+                          int32_t *__restrict__ flags) {
+    pdl_go();
+    pdl_after();
+    const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+    const int64_t i0 = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    int32_t longest = 0;
+    int32_t bad = 0;
+    for (int64_t i = i0; i <= K; i += stride) {
+        const int64_t o = src_off[i];
+        if (off != src_off) off[i] = o;
+        if (o < 0) bad = 1;
+        if (i < K) {
+            const int64_t o2 = src_off[i + 1];
+            if (o2 < o) bad = 1;
+            else longest = max(longest, int32_t(min(o2 - o, int64_t(INT32_MAX))));
+        }
+    }
+    if (soff != src_soff)
+        for (int64_t i = i0; i <= M; i += stride) soff[i] = src_soff[i];
+    for (int64_t k = i0; k < n_vec; k += stride) vec[k] = src_vec[k];
+    longest = __reduce_max_sync(0xffffffffu, longest);
+    bad = __any_sync(0xffffffffu, bad);
+    if ((threadIdx.x & 31) == 0) {
+        if (bad) atomicOr(flags, 1);
+        if (longest) atomicMax(flags + 1, longest);
+    }
+}
+
 // Strings: their set (from set_offsets), their node (the set's root), and the
-// roots of sets with an empty string are terminal. Level 0 = the M roots.
-__global__ void k_b_init(const int64_t *__restrict__ off, const int32_t *__restrict__ set_off, int32_t M,
-                         int32_t K, int32_t *__restrict__ str_set, int32_t *__restrict__ cur,
-                         int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
+// roots of sets with an empty string are terminal. Level 0 = the M roots;
+// every non-empty string sets its first byte in its root's child-label set.
+__global__ void k_b_init(const uint8_t *__restrict__ bytes, const int64_t *__restrict__ off,
+                         const int32_t *__restrict__ set_off, int32_t M, int32_t K, int32_t *__restrict__ str_set,
+                         int32_t *__restrict__ cur, int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
                          uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g,
-                         int32_t *__restrict__ ls) {
+                         int32_t *__restrict__ ls, uint32_t *__restrict__ bits0) {
     pdl_go();
     pdl_after();
     const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -73,22 +112,12 @@ __global__ void k_b_init(const int64_t *__restrict__ off, const int32_t *__restr
     }
     str_set[i] = lo;
     cur[i] = lo;
-    if (off[i + 1] == off[i]) term_g[lo] = 1;  // the empty string: the root is terminal
-}
-
-// Level d, pass 1: each string of length > d sets its byte d in its parent's
-// child-label set (bits of level d: row x - ls[d]).
-__global__ void k_b_bits(const uint8_t *__restrict__ bytes, const int64_t *__restrict__ off, int32_t K, int32_t d,
-                         const int32_t *__restrict__ cur, const int32_t *__restrict__ ls,
-                         uint32_t *__restrict__ bits) {
-    pdl_go();
-    pdl_after();
-    const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= K) return;
-    const int64_t a = off[i] - off[0];
-    if (off[i + 1] - off[i] <= d) return;
-    const uint32_t b = bytes[a + d];
-    atomicOr(bits + int64_t(cur[i] - ls[d]) * 8 + (b >> 5), 1u << (b & 31u));
+    if (off[i + 1] == off[i]) {
+        term_g[lo] = 1;  // the empty string: the root is terminal
+    } else {
+        const uint32_t b = bytes[off[i] - off[0]];
+        atomicOr(bits0 + int64_t(lo) * 8 + (b >> 5), 1u << (b & 31u));
+    }
 }
 
 __device__ __forceinline__ int32_t row_popc(const uint32_t *bits, int64_t row) {
@@ -124,7 +153,7 @@ __device__ __forceinline__ int32_t block_excl_scan(int32_t v, int32_t *warp_sums
     return before + x - v;
 }
 
-// Level d, pass 2: the children of every tile of kScanTile parents.
+// Level d, pass 1: the children of every tile of kScanTile parents.
 __global__ void __launch_bounds__(kBThreads) k_b_tile_sums(int32_t d, const int32_t *__restrict__ ls,
                                                            const uint32_t *__restrict__ bits,
                                                            int32_t *__restrict__ tile_sum) {
@@ -145,33 +174,14 @@ __global__ void __launch_bounds__(kBThreads) k_b_tile_sums(int32_t d, const int3
     if (threadIdx.x == 0) tile_sum[blockIdx.x] = tot;
 }
 
-// Level d, pass 3 (one CTA): exclusive scan of the tile sums; the end of level d + 1.
-__global__ void __launch_bounds__(kBThreads) k_b_tile_scan(int32_t d, int32_t n_tiles, int32_t *__restrict__ ls,
-                                                           int32_t *__restrict__ tile_sum) {
-    __shared__ int32_t ws[kBThreads / 32];
-    __shared__ int32_t carry;
-    pdl_go();
-    pdl_after();
-    if (threadIdx.x == 0) carry = 0;
-    __syncthreads();
-    for (int32_t t0 = 0; t0 < n_tiles; t0 += kBThreads) {
-        const int32_t t = t0 + threadIdx.x;
-        const int32_t v = t < n_tiles ? tile_sum[t] : 0;
-        int32_t tot;
-        const int32_t ex = block_excl_scan(v, ws, &tot);
-        if (t < n_tiles) tile_sum[t] = carry + ex;
-        __syncthreads();
-        if (threadIdx.x == 0) carry += tot;
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) ls[d + 2] = ls[d + 1] + carry;
-}
-
-// Level d, pass 4: first child of every parent of the level; also clears the
-// other bits buffer (level d - 1's rows) for level d + 1.
-__global__ void __launch_bounds__(kBThreads) k_b_first(int32_t d, const int32_t *__restrict__ ls,
+// Level d, pass 2: first child of every parent of the level (the level's
+// end + the children of the earlier tiles + an exclusive scan within the
+// tile); block 0 also writes the end of level d + 1. Clears the other bits
+// buffer (level d - 1's rows), into which the moves of level d set the
+// child-label sets of level d + 1.
+__global__ void __launch_bounds__(kBThreads) k_b_first(int32_t d, int32_t n_tiles, int32_t *__restrict__ ls,
                                                        const uint32_t *__restrict__ bits,
-                                                       const int32_t *__restrict__ tile_off,
+                                                       const int32_t *__restrict__ tile_sum,
                                                        int32_t *__restrict__ first, uint32_t *__restrict__ other) {
     __shared__ int32_t ws[kBThreads / 32];
     __shared__ int32_t carry;
@@ -186,9 +196,23 @@ __global__ void __launch_bounds__(kBThreads) k_b_first(int32_t d, const int32_t 
             r[0] = make_uint4(0u, 0u, 0u, 0u);
             r[1] = make_uint4(0u, 0u, 0u, 0u);
         }
-    if (t0 >= width) return;
-    if (threadIdx.x == 0) carry = ls[d + 1] + tile_off[blockIdx.x];
+    if (t0 >= width && blockIdx.x > 0) return;
+    // children of the tiles before this one (all tiles for block 0's total)
+    const int32_t upto = blockIdx.x > 0 ? int32_t(blockIdx.x) : n_tiles;
+    int32_t part = 0;
+    for (int32_t t = threadIdx.x; t < upto; t += kBThreads) part += tile_sum[t];
+    int32_t sum;
+    block_excl_scan(part, ws, &sum);
+    if (threadIdx.x == 0) {
+        if (blockIdx.x == 0) {
+            ls[d + 2] = ls[d + 1] + sum;
+            carry = ls[d + 1];
+        } else {
+            carry = ls[d + 1] + sum;
+        }
+    }
     __syncthreads();
+    if (t0 >= width) return;
     for (int32_t j0 = 0; j0 < kScanTile; j0 += kBThreads) {
         const int32_t x = t0 + j0 + threadIdx.x;
         const int32_t c = x < width ? row_popc(bits, x) : 0;
@@ -201,21 +225,24 @@ __global__ void __launch_bounds__(kBThreads) k_b_first(int32_t d, const int32_t 
     }
 }
 
-// Level d, pass 5: every string of length > d moves to its child at depth
+// Level d, pass 3: every string of length > d moves to its child at depth
 // d + 1, writing the child's parent, label, set, depth and terminal flag
-// (all strings through a child write the same values).
+// (all strings through a child write the same values), and sets its byte
+// d + 1, if any, in the child's child-label set (level d + 1's rows).
 __global__ void k_b_move(const uint8_t *__restrict__ bytes, const int64_t *__restrict__ off, int32_t K, int32_t d,
                          const int32_t *__restrict__ ls, const uint32_t *__restrict__ bits,
                          const int32_t *__restrict__ first, const int32_t *__restrict__ str_set,
                          int32_t *__restrict__ cur, int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
-                         uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g) {
+                         uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g,
+                         uint32_t *__restrict__ bits_next) {
     pdl_go();
     pdl_after();
     const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= K) return;
     const int64_t len = off[i + 1] - off[i];
     if (len <= d) return;
-    const uint32_t b = bytes[off[i] - off[0] + d];
+    const int64_t a = off[i] - off[0];
+    const uint32_t b = bytes[a + d];
     const int32_t x = cur[i];
     const int64_t row = x - ls[d];
     const uint32_t *r = bits + row * 8;
@@ -232,8 +259,13 @@ __global__ void k_b_move(const uint8_t *__restrict__ bytes, const int64_t *__res
     label_g[c] = uint8_t(b);
     set_g[c] = str_set[i];
     depth_g[c] = d + 1;
-    if (len == d + 1) term_g[c] = 1;
     cur[i] = c;
+    if (len == d + 1) {
+        term_g[c] = 1;
+    } else {
+        const uint32_t b1 = bytes[a + d + 1];
+        atomicOr(bits_next + int64_t(c - ls[d + 1]) * 8 + (b1 >> 5), 1u << (b1 & 31u));
+    }
 }
 
 // Renumbering, pass 1: the level-order range [first, end) of every (set,
@@ -327,13 +359,16 @@ __global__ void k_b_permute(const int32_t *__restrict__ ls, int32_t D, const int
 
 }  // namespace
 
-// Scratch of one device build: the strings, level-order node arrays (at most
-// K_chars + M nodes), two child-label buffers of K rows, the level scans.
+// Scratch of one device build. Staging part: the strings, level-order node
+// arrays (at most n_bytes + M nodes), two child-label buffers of
+// max(K, M) rows, the level scans, the flags. Level part (once the longest
+// string D is known): the level ends and the (set, depth) tables.
 struct DeviceBuild::Scratch {
-    void *base = nullptr;
+    void *base = nullptr, *base2 = nullptr;
     uint8_t *bytes;
+    uint4 *image;
     int64_t *off;
-    int32_t *set_off, *str_set, *cur, *parent_g, *set_g, *depth_g, *first, *tile_sum, *ls;
+    int32_t *set_off, *str_set, *cur, *parent_g, *set_g, *depth_g, *first, *tile_sum, *ls, *flags;
     uint8_t *label_g, *term_g;
     uint32_t *bits[2];
     int32_t *end_sd, *first_sd, *off_sd, *roots, *map;
@@ -343,40 +378,49 @@ struct DeviceBuild::Scratch {
 DeviceBuild::~DeviceBuild() {
     if (s_) {
         if (s_->base) cudaFreeAsync(s_->base, stream_);
+        if (s_->base2) cudaFreeAsync(s_->base2, stream_);
         delete s_;
     }
 }
 
-cudaError_t DeviceBuild::levels(const uint8_t *h_bytes, const int64_t *h_off, const int32_t *h_set_off, int32_t M,
-                                int32_t K, int64_t n_bytes, int32_t D, int num_sms, cudaMemPool_t pool,
-                                cudaStream_t st, int32_t *n_nodes,
-                                std::vector<int32_t> *roots, int64_t *n_chars) {
-    stream_ = st;
-    M_ = M;
-    D_ = D;
-    s_ = new Scratch();
-    const int64_t U = n_bytes + M;          // nodes at most
-    const int64_t W = std::max<int64_t>(K, M);  // parents of one level at most
-    const int64_t tiles = (W + kScanTile - 1) / kScanTile + 1;
-    const int64_t sd = int64_t(M) * (D + 1);
+namespace {
+
+struct Carver {
     size_t total = 0;
-    auto add = [&](size_t b) {
+    size_t add(size_t b) {
         const size_t o = total;
         total += (b + 255) / 256 * 256;
         return o;
-    };
-    const size_t o_bytes = add(size_t(n_bytes) + 16), o_off = add(8 * (size_t(K) + 1)),
-                 o_soff = add(4 * (size_t(M) + 1)), o_sset = add(4 * size_t(K)), o_cur = add(4 * size_t(K)),
-                 o_par = add(4 * size_t(U)), o_set = add(4 * size_t(U)), o_dep = add(4 * size_t(U)),
-                 o_first = add(4 * size_t(W)), o_ts = add(4 * size_t(tiles)), o_ls = add(4 * (size_t(D) + 2)),
-                 o_lab = add(size_t(U)), o_term = add(size_t(U)), o_b0 = add(32 * size_t(W) + 32),
-                 o_b1 = add(32 * size_t(W) + 32), o_end = add(4 * size_t(sd)), o_fsd = add(4 * size_t(sd)),
-                 o_osd = add(4 * size_t(sd)), o_roots = add(4 * size_t(M)), o_map = add(4 * size_t(U)),
-                 o_nch = add(8);
-    cudaError_t e = cudaMallocFromPoolAsync(&s_->base, total, pool, st);
+    }
+};
+
+}  // namespace
+
+cudaError_t DeviceBuild::stage(const uint8_t *h_bytes, const int64_t *h_off, const int32_t *h_set_off, int32_t M,
+                               int32_t K, int64_t n_bytes, bool direct, int num_sms, cudaMemPool_t pool,
+                               cudaStream_t st, int32_t *max_len, bool *offsets_ok) {
+    stream_ = st;
+    pool_ = pool;
+    M_ = M;
+    K_ = K;
+    n_bytes_ = n_bytes;
+    s_ = new Scratch();
+    const int64_t U = n_bytes + M;               // nodes at most
+    const int64_t W = std::max<int64_t>(K, M);   // parents of one level at most
+    const int64_t tiles = (W + kScanTile - 1) / kScanTile + 1;
+    Carver c;
+    const size_t o_img = c.add(size_t(n_bytes) + 32), o_off = c.add(8 * (size_t(K) + 1)),
+                 o_soff = c.add(4 * (size_t(M) + 1)), o_sset = c.add(4 * size_t(K)), o_cur = c.add(4 * size_t(K)),
+                 o_par = c.add(4 * size_t(U)), o_set = c.add(4 * size_t(U)), o_dep = c.add(4 * size_t(U)),
+                 o_first = c.add(4 * size_t(W)), o_ts = c.add(4 * size_t(tiles)), o_lab = c.add(size_t(U)),
+                 o_term = c.add(size_t(U)), o_b0 = c.add(32 * size_t(W) + 32), o_b1 = c.add(32 * size_t(W) + 32),
+                 o_roots = c.add(4 * size_t(M)), o_map = c.add(4 * size_t(U)), o_nch = c.add(8), o_flags = c.add(8);
+    cudaError_t e = cudaMallocFromPoolAsync(&s_->base, c.total, pool, st);
     if (e != cudaSuccess) return e;
     char *b = static_cast<char *>(s_->base);
-    s_->bytes = reinterpret_cast<uint8_t *>(b + o_bytes);
+    const size_t mis = reinterpret_cast<uintptr_t>(h_bytes) & 15u;  // the image keeps the source's alignment
+    s_->image = reinterpret_cast<uint4 *>(b + o_img);
+    s_->bytes = reinterpret_cast<uint8_t *>(b + o_img) + mis;
     s_->off = reinterpret_cast<int64_t *>(b + o_off);
     s_->set_off = reinterpret_cast<int32_t *>(b + o_soff);
     s_->str_set = reinterpret_cast<int32_t *>(b + o_sset);
@@ -386,53 +430,85 @@ cudaError_t DeviceBuild::levels(const uint8_t *h_bytes, const int64_t *h_off, co
     s_->depth_g = reinterpret_cast<int32_t *>(b + o_dep);
     s_->first = reinterpret_cast<int32_t *>(b + o_first);
     s_->tile_sum = reinterpret_cast<int32_t *>(b + o_ts);
-    s_->ls = reinterpret_cast<int32_t *>(b + o_ls);
     s_->label_g = reinterpret_cast<uint8_t *>(b + o_lab);
     s_->term_g = reinterpret_cast<uint8_t *>(b + o_term);
     s_->bits[0] = reinterpret_cast<uint32_t *>(b + o_b0);
     s_->bits[1] = reinterpret_cast<uint32_t *>(b + o_b1);
-    s_->end_sd = reinterpret_cast<int32_t *>(b + o_end);
-    s_->first_sd = reinterpret_cast<int32_t *>(b + o_fsd);
-    s_->off_sd = reinterpret_cast<int32_t *>(b + o_osd);
     s_->roots = reinterpret_cast<int32_t *>(b + o_roots);
     s_->map = reinterpret_cast<int32_t *>(b + o_map);
     s_->n_chars = reinterpret_cast<unsigned long long *>(b + o_nch);
-    // inputs; zeroed flags, buffers and counters
-    if ((n_bytes > 0 &&
-         (e = cudaMemcpyAsync(s_->bytes, h_bytes, size_t(n_bytes), cudaMemcpyHostToDevice, st)) != cudaSuccess) ||
-        (e = cudaMemcpyAsync(s_->off, h_off, 8 * (size_t(K) + 1), cudaMemcpyHostToDevice, st)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(s_->set_off, h_set_off, 4 * (size_t(M) + 1), cudaMemcpyHostToDevice, st)) !=
-            cudaSuccess ||
-        (e = cudaMemsetAsync(s_->term_g, 0, size_t(U), st)) != cudaSuccess ||
+    s_->flags = reinterpret_cast<int32_t *>(b + o_flags);
+    if ((e = cudaMemsetAsync(s_->term_g, 0, size_t(U), st)) != cudaSuccess ||
         (e = cudaMemsetAsync(s_->bits[0], 0, 32 * size_t(W) + 32, st)) != cudaSuccess ||
         (e = cudaMemsetAsync(s_->bits[1], 0, 32 * size_t(W) + 32, st)) != cudaSuccess ||
-        (e = cudaMemsetAsync(s_->end_sd, 0, 4 * size_t(sd), st)) != cudaSuccess ||
-        (e = cudaMemsetAsync(s_->first_sd, 0x7F, 4 * size_t(sd), st)) != cudaSuccess ||
-        (e = cudaMemsetAsync(s_->n_chars, 0, 8, st)) != cudaSuccess)
+        (e = cudaMemsetAsync(s_->n_chars, 0, 8, st)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s_->flags, 0, 8, st)) != cudaSuccess)
         return e;
+    const int64_t n_vec = n_bytes > 0 ? (int64_t(mis) + n_bytes + 15) / 16 : 0;
+    const int64_t items = std::max<int64_t>(std::max<int64_t>(K, M) + 1, n_vec);
+    const int64_t grid = std::min<int64_t>((items + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
+    if (direct) {
+        e = launch(k_b_stage, grid, kBThreads, st, h_off, K, h_set_off, M,
+                   reinterpret_cast<const uint4 *>(h_bytes - mis), n_vec, s_->off, s_->set_off, s_->image, s_->flags);
+    } else {
+        if ((n_bytes > 0 && (e = cudaMemcpyAsync(s_->bytes, h_bytes, size_t(n_bytes), cudaMemcpyHostToDevice, st)) !=
+                                cudaSuccess) ||
+            (e = cudaMemcpyAsync(s_->off, h_off, 8 * (size_t(K) + 1), cudaMemcpyHostToDevice, st)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(s_->set_off, h_set_off, 4 * (size_t(M) + 1), cudaMemcpyHostToDevice, st)) !=
+                cudaSuccess)
+            return e;
+        e = launch(k_b_stage, grid, kBThreads, st, static_cast<const int64_t *>(s_->off), K,
+                   static_cast<const int32_t *>(s_->set_off), M, static_cast<const uint4 *>(nullptr), int64_t(0),
+                   s_->off, s_->set_off, s_->image, s_->flags);
+    }
+    if (e != cudaSuccess) return e;
+    int32_t flags[2] = {0, 0};
+    if ((e = cudaMemcpyAsync(flags, s_->flags, sizeof(flags), cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaStreamSynchronize(st)) != cudaSuccess)
+        return e;
+    *offsets_ok = flags[0] == 0;
+    *max_len = flags[1];
+    return cudaSuccess;
+}
+
+cudaError_t DeviceBuild::levels(int32_t D, int num_sms, int32_t *n_nodes, std::vector<int32_t> *roots,
+                                int64_t *n_chars) {
+    const cudaStream_t st = stream_;
+    const int32_t M = M_, K = K_;
+    D_ = D;
+    const int64_t U = n_bytes_ + M;
+    const int64_t W = std::max<int64_t>(K, M);
+    const int64_t sd = int64_t(M) * (D + 1);
+    Carver c;
+    const size_t o_ls = c.add(4 * (size_t(D) + 2)), o_end = c.add(4 * size_t(sd)), o_fsd = c.add(4 * size_t(sd)),
+                 o_osd = c.add(4 * size_t(sd));
+    cudaError_t e = cudaMallocFromPoolAsync(&s_->base2, c.total, pool_, st);
+    if (e != cudaSuccess) return e;
+    char *b = static_cast<char *>(s_->base2);
+    s_->ls = reinterpret_cast<int32_t *>(b + o_ls);
+    s_->end_sd = reinterpret_cast<int32_t *>(b + o_end);
+    s_->first_sd = reinterpret_cast<int32_t *>(b + o_fsd);
+    s_->off_sd = reinterpret_cast<int32_t *>(b + o_osd);
+    if ((e = cudaMemsetAsync(s_->end_sd, 0, 4 * size_t(sd), st)) != cudaSuccess) return e;
     const int64_t sgrid = (W + kBThreads - 1) / kBThreads;
-    if ((e = launch(k_b_init, sgrid, kBThreads, st, static_cast<const int64_t *>(s_->off),
-                    static_cast<const int32_t *>(s_->set_off), M, K, s_->str_set, s_->cur, s_->parent_g, s_->label_g,
-                    s_->term_g, s_->set_g, s_->depth_g, s_->ls)) != cudaSuccess)
+    if ((e = launch(k_b_init, sgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
+                    static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M, K,
+                    s_->str_set, s_->cur, s_->parent_g, s_->label_g, s_->term_g, s_->set_g, s_->depth_g, s_->ls,
+                    s_->bits[0])) != cudaSuccess)
         return e;
     const int64_t kgrid = (int64_t(K) + kBThreads - 1) / kBThreads;
     const int32_t n_tiles = int32_t((W + kScanTile - 1) / kScanTile);
-    for (int32_t d = 0; d < D; d++) {
-        uint32_t *bits = s_->bits[d & 1];
-        if ((e = launch(k_b_bits, kgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
-                        static_cast<const int64_t *>(s_->off), K, d, static_cast<const int32_t *>(s_->cur),
-                        static_cast<const int32_t *>(s_->ls), bits)) != cudaSuccess ||
-            (e = launch(k_b_tile_sums, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
+    for (int32_t d = 0; d < D; d++) {  // level d: bits[d & 1] holds its child-label sets
+        uint32_t *bits = s_->bits[d & 1], *next = s_->bits[(d + 1) & 1];
+        if ((e = launch(k_b_tile_sums, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
                         static_cast<const uint32_t *>(bits), s_->tile_sum)) != cudaSuccess ||
-            (e = launch(k_b_tile_scan, 1, kBThreads, st, d, n_tiles, s_->ls, s_->tile_sum)) != cudaSuccess ||
-            (e = launch(k_b_first, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
-                        static_cast<const uint32_t *>(bits), static_cast<const int32_t *>(s_->tile_sum), s_->first,
-                        s_->bits[(d + 1) & 1])) != cudaSuccess ||
+            (e = launch(k_b_first, n_tiles, kBThreads, st, d, n_tiles, s_->ls, static_cast<const uint32_t *>(bits),
+                        static_cast<const int32_t *>(s_->tile_sum), s_->first, next)) != cudaSuccess ||
             (e = launch(k_b_move, kgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
                         static_cast<const int64_t *>(s_->off), K, d, static_cast<const int32_t *>(s_->ls),
                         static_cast<const uint32_t *>(bits), static_cast<const int32_t *>(s_->first),
                         static_cast<const int32_t *>(s_->str_set), s_->cur, s_->parent_g, s_->label_g, s_->term_g,
-                        s_->set_g, s_->depth_g)) != cudaSuccess)
+                        s_->set_g, s_->depth_g, next)) != cudaSuccess)
             return e;
     }
     const int64_t ngrid = std::min<int64_t>((U + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);

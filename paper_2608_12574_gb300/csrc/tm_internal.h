@@ -241,11 +241,14 @@ struct DevLazy {
     LazyNode *pre = nullptr;        // [n] by pre-order position
 };
 
-// A forest built on the device (device_build.cu): levels() runs the level
-// loop and the renumbering into its own scratch and returns the node count,
-// the roots and the characters (host-synchronous); emit() writes parent,
-// label and terminal of the final layout into the caller's device arrays
-// (asynchronous); the destructor frees the scratch after them.
+// A forest built on the device (device_build.cu): stage() copies the strings
+// into its own scratch (reading the caller's host memory directly when
+// `direct`), checks their offsets and returns the longest string's length
+// (host-synchronous); levels() runs the level loop and the renumbering and
+// returns the node count, the roots and the characters (host-synchronous);
+// emit() writes parent, label and terminal of the final layout into the
+// caller's device arrays (asynchronous); the destructor frees the scratch on
+// the stream after them.
 constexpr int32_t kDeviceBuildMaxDepth = 1024;        // longer strings: the host builder
 constexpr int64_t kDeviceBuildMaxGroups = int64_t(1) << 24;  // sets x (depths + 1) above: the host builder
 class DeviceBuild {
@@ -254,17 +257,19 @@ public:
     DeviceBuild(const DeviceBuild &) = delete;
     DeviceBuild &operator=(const DeviceBuild &) = delete;
     ~DeviceBuild();
-    cudaError_t levels(const uint8_t *h_bytes, const int64_t *h_off, const int32_t *h_set_off, int32_t M, int32_t K,
-                       int64_t n_bytes, int32_t D, int num_sms, cudaMemPool_t pool, cudaStream_t st,
-                       int32_t *n_nodes,
-                       std::vector<int32_t> *roots, int64_t *n_chars);
+    cudaError_t stage(const uint8_t *h_bytes, const int64_t *h_off, const int32_t *h_set_off, int32_t M, int32_t K,
+                      int64_t n_bytes, bool direct, int num_sms, cudaMemPool_t pool, cudaStream_t st,
+                      int32_t *max_len, bool *offsets_ok);
+    cudaError_t levels(int32_t D, int num_sms, int32_t *n_nodes, std::vector<int32_t> *roots, int64_t *n_chars);
     cudaError_t emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms);
 
 private:
     struct Scratch;
     Scratch *s_ = nullptr;
     cudaStream_t stream_ = nullptr;
-    int32_t M_ = 0, D_ = 0, n_ = 0;
+    cudaMemPool_t pool_ = nullptr;
+    int32_t M_ = 0, K_ = 0, D_ = 0, n_ = 0;
+    int64_t n_bytes_ = 0;
 };
 
 // The pre-order tables (pre_node / pre_depth / pre_size) of a trie or forest

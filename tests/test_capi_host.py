@@ -170,7 +170,6 @@ def test_build_many_device_argument_errors(lib):
     offs = np.array([0, 2, 4], np.int64)
     bad_first = np.array([1, 2], np.int32)
     bad_order = np.array([0, 2, 1], np.int32)
-    dec = np.array([0, 3, 2], np.int64)
     ok = np.array([0, 2], np.int32)
     f = lib.trie_build_many_device
     assert f(b.ctypes.data, offs.ctypes.data, bad_first.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
@@ -178,7 +177,11 @@ def test_build_many_device_argument_errors(lib):
     assert f(b.ctypes.data, offs.ctypes.data, None, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
     assert f(b.ctypes.data, offs.ctypes.data, ok.ctypes.data, 0, None, ctypes.byref(h)) == T.TRIE_EINVAL
     assert f(b.ctypes.data, offs.ctypes.data, ok.ctypes.data, 1, None, None) == T.TRIE_EINVAL
-    assert f(b.ctypes.data, dec.ctypes.data, ok.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    # offsets[0] < 0 or offsets[K] < offsets[0]: caught on the host (the rest on the device)
+    neg = np.array([-1, 2, 4], np.int64)
+    assert f(b.ctypes.data, neg.ctypes.data, ok.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
+    back = np.array([3, 4, 2], np.int64)
+    assert f(b.ctypes.data, back.ctypes.data, ok.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
     assert "non-decreasing" in T.trie_last_error()
     assert f(None, offs.ctypes.data, ok.ctypes.data, 1, None, ctypes.byref(h)) == T.TRIE_EINVAL
     assert h.value is None

@@ -115,6 +115,59 @@ def test_device_forest_more_sets_than_strings(cuda):
     assert d.root(7) == 7 and d.root(8) == 10 and c["terminal"][d.root(4000)] == 1
 
 
+def test_device_forest_offsets_checked_on_the_device(cuda):
+    """Offsets that decrease, or go negative, inside the list are found by the
+    staging kernel: TRIE_EINVAL, and no handle."""
+    import ctypes
+    lib = T.load_library()
+    b = np.frombuffer(b"abcdefgh", np.uint8).copy()
+    so = np.array([0, 3], np.int32)
+    h = ctypes.c_void_p()
+    for offs in ([0, 5, 2, 8], [0, 3, -1, 8], [0, 9, 4, 8]):
+        o = np.array(offs, np.int64)
+        rc = lib.trie_build_many_device(b.ctypes.data, o.ctypes.data, so.ctypes.data, 1, None, ctypes.byref(h))
+        assert rc == T.TRIE_EINVAL, offs
+        assert "non-decreasing" in T.trie_last_error()
+        assert h.value is None
+
+
+@pytest.mark.parametrize("shift", [0, 1, 5, 15])
+def test_device_forest_unaligned_bytes(cuda, shift):
+    """Byte arrays that start at any alignment, and offsets that do not start
+    at 0: the staged image keeps the source's alignment."""
+    sets = _random_sets(7) + [[b"get", b"get_user", b"", b"set"]]
+    sb, so, index = _forest(sets)
+    buf = np.zeros(len(sb) + 64, np.uint8)
+    view = buf[shift:shift + len(sb) + 3]
+    view[3:3 + len(sb)] = sb
+    d = T.trie_build_many_device(view, so + 3, index)
+    _check_against_oracle(d, sets)
+
+
+def test_device_forest_copy_path(cuda):
+    """The path for devices that cannot read pageable host memory (copies,
+    then the same checks on the device), forced in a fresh process."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    code = (
+        "import sys; sys.path[:0] = [%r, %r]\n"
+        "import numpy as np\n"
+        "from paper_2608_12574_gb300 import triemask as T\n"
+        "import test_gpu_device_build as t\n"
+        "for seed in range(12):\n"
+        "    sets = t._random_sets(seed)\n"
+        "    sb, so, index = t._forest(sets)\n"
+        "    d = T.trie_build_many_device(sb, so, index)\n"
+        "    t._check_against_oracle(d, sets)\n"
+        "    t._same_handles(d, T.trie_build_many(sb, so, index))\n"
+        "print('ok')\n" % (root, os.path.join(root, "tests")))
+    env = dict(os.environ, TRIEMASK_HOST_READ="copy")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
+
+
 def test_device_forest_single_set_mask_equals_oracle(cuda):
     """A forest of one set (the K=100 tool names): the dense mask compiled on
     the device-built handle equals the oracle's mask."""
