@@ -25,6 +25,7 @@ namespace tmk {
 namespace {
 
 constexpr int kBThreads = 256;
+constexpr int32_t kSetMaxStrings = 4096;  // forests whose sets all hold at most this many strings: one CTA per set
 constexpr int kScanTile = 1024;  // parents per tile of the level scan
 
 __device__ __forceinline__ void pdl_go() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
@@ -357,6 +358,198 @@ __global__ void k_b_permute(const int32_t *__restrict__ ls, int32_t D, const int
     }
 }
 
+// ---- Forests of small sets: one CTA per set (kSetThreads threads, each
+// owning up to kSetPer strings), the levels of that set in shared memory. The
+// set's nodes are created in the order of the level path restricted to the
+// set (breadth-first, sorted siblings) at local ids 0, 1, ..., written at
+// ub(s) = (bytes before set s) + s, room for the set's at most 1 + bytes
+// nodes; a scan of the node counts then gives every set its base.
+constexpr int kSetThreads = 512;
+constexpr int kSetPer = int(kSetMaxStrings / kSetThreads);
+
+__device__ __forceinline__ int32_t block_reduce_max(int32_t v, int32_t *ws) {
+    v = __reduce_max_sync(0xffffffffu, v);
+    if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = v;
+    __syncthreads();
+    int32_t m = 0;
+    for (int w = 0; w < int(blockDim.x >> 5); w++) m = max(m, ws[w]);
+    __syncthreads();
+    return m;
+}
+
+// Exclusive scan of one int per thread over a block of kSetThreads.
+__device__ __forceinline__ int32_t set_excl_scan(int32_t v, int32_t *ws, int32_t *total) {
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    int32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) ws[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+        int32_t w = lane < kSetThreads / 32 ? ws[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < kSetThreads / 32) ws[lane] = w;
+    }
+    __syncthreads();
+    const int32_t before = wid > 0 ? ws[wid - 1] : 0;
+    *total = ws[kSetThreads / 32 - 1];
+    __syncthreads();  // ws is reused by the next scan
+    return before + x - v;
+}
+
+// Dynamic shared memory: the child-label sets of the current level
+// (smax rows of 8 words) and the first child of each of its nodes.
+__global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restrict__ bytes,
+                                                        const int64_t *__restrict__ off,
+                                                        const int32_t *__restrict__ set_off, int32_t M, int32_t smax,
+                                                        int32_t *__restrict__ parent_ub, uint8_t *__restrict__ label_ub,
+                                                        uint8_t *__restrict__ term_ub, int32_t *__restrict__ count,
+                                                        unsigned long long *__restrict__ chars) {
+    extern __shared__ uint4 dyn[];
+    uint32_t *bits = reinterpret_cast<uint32_t *>(dyn);
+    int32_t *first = reinterpret_cast<int32_t *>(bits + int64_t(smax) * 8);
+    __shared__ int32_t ws[kSetThreads / 32];
+    __shared__ int32_t root_term;
+    pdl_go();
+    pdl_after();
+    const int tid = threadIdx.x;
+    for (int32_t r = tid; r < smax * 8; r += kSetThreads) bits[r] = 0u;
+    for (int32_t s = blockIdx.x; s < M; s += gridDim.x) {
+        const int32_t i0 = set_off[s], Ks = set_off[s + 1] - i0;
+        const int64_t ub = off[i0] - off[0] + s;
+        if (tid == 0) root_term = 0;
+        __syncthreads();
+        int32_t st[kSetPer], len[kSetPer], cur[kSetPer], nb[kSetPer];
+        int32_t longest = 0;
+#pragma unroll
+        for (int k = 0; k < kSetPer; k++) {
+            const int32_t j = tid + k * kSetThreads;
+            len[k] = -1;
+            cur[k] = 0;
+            nb[k] = 0;
+            st[k] = 0;
+            if (j < Ks) {
+                const int64_t a = off[i0 + j], e = off[i0 + j + 1];
+                st[k] = int32_t(a - off[0]);
+                len[k] = int32_t(e - a);
+                longest = max(longest, len[k]);
+                if (len[k] == 0) root_term = 1;
+                else nb[k] = bytes[st[k]];
+            }
+        }
+        const int32_t dmax = block_reduce_max(longest, ws);  // also orders root_term
+        if (tid == 0) {
+            parent_ub[ub] = -1;
+            label_ub[ub] = 0;
+            term_ub[ub] = uint8_t(root_term);
+        }
+        int32_t level_start = 0, level_end = 1;
+        unsigned long long my_chars = 0;
+        for (int32_t d = 0; d < dmax; d++) {
+            const int32_t width = level_end - level_start;
+#pragma unroll
+            for (int k = 0; k < kSetPer; k++)
+                if (len[k] > d)
+                    atomicOr(bits + (cur[k] - level_start) * 8 + (nb[k] >> 5), 1u << (nb[k] & 31));
+            __syncthreads();
+            // first child of every node of the level: a contiguous chunk of rows per thread
+            const int32_t per = (width + kSetThreads - 1) / kSetThreads;
+            const int32_t r0 = min(tid * per, width), r1 = min(r0 + per, width);
+            int32_t c = 0;
+            for (int32_t r = r0; r < r1; r++) c += row_popc(bits, r);
+            int32_t total;
+            int32_t at = level_end + set_excl_scan(c, ws, &total);
+            for (int32_t r = r0; r < r1; r++) {
+                first[r] = at;
+                at += row_popc(bits, r);
+            }
+            __syncthreads();
+#pragma unroll
+            for (int k = 0; k < kSetPer; k++) {
+                if (len[k] <= d) continue;
+                const uint32_t b = uint32_t(nb[k]);
+                const int32_t row = cur[k] - level_start;
+                const uint32_t *rw = bits + row * 8;
+                int32_t below = 0;
+#pragma unroll
+                for (int w = 0; w < 8; w++) {
+                    const int32_t lo = w * 32;
+                    if (int32_t(b) >= lo + 32) below += __popc(rw[w]);
+                    else if (int32_t(b) >= lo) below += __popc(rw[w] & ((1u << (b - lo)) - 1u));
+                }
+                const int32_t ch = first[row] + below;
+                const int64_t g = ub + ch;
+                parent_ub[g] = cur[k];
+                label_ub[g] = uint8_t(b);
+                if (len[k] == d + 1) term_ub[g] = 1;
+                else nb[k] = bytes[st[k] + d + 1];
+                cur[k] = ch;
+            }
+            __syncthreads();
+            for (int32_t r = tid; r < width * 8; r += kSetThreads) bits[r] = 0u;
+            for (int32_t x = level_end + tid; x < level_end + total; x += kSetThreads)
+                if (term_ub[ub + x]) my_chars += unsigned(d + 1);
+            level_start = level_end;
+            level_end += total;
+            __syncthreads();
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) my_chars += __shfl_down_sync(0xffffffffu, my_chars, o);
+        if ((tid & 31) == 0 && my_chars) atomicAdd(chars, my_chars);
+        if (tid == 0) count[s] = level_end;
+        __syncthreads();
+    }
+}
+
+// One CTA: every set's base (exclusive scan of the node counts) = its root,
+// and the total.
+__global__ void __launch_bounds__(kBThreads) k_b_set_scan(int32_t M, const int32_t *__restrict__ count,
+                                                          int32_t *__restrict__ roots, int32_t *__restrict__ total) {
+    __shared__ int32_t ws[kBThreads / 32];
+    __shared__ int32_t carry;
+    pdl_go();
+    pdl_after();
+    if (threadIdx.x == 0) carry = 0;
+    __syncthreads();
+    for (int32_t s0 = 0; s0 < M; s0 += kBThreads) {
+        const int32_t s = s0 + threadIdx.x;
+        int32_t tot;
+        const int32_t ex = block_excl_scan(s < M ? count[s] : 0, ws, &tot);
+        if (s < M) roots[s] = carry + ex;
+        __syncthreads();
+        if (threadIdx.x == 0) carry += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *total = carry;
+}
+
+// Every set's nodes from ub(s) + i to base(s) + i (CTA per set).
+__global__ void k_b_set_emit(const int64_t *__restrict__ off, const int32_t *__restrict__ set_off, int32_t M,
+                             const int32_t *__restrict__ count, const int32_t *__restrict__ roots,
+                             const int32_t *__restrict__ parent_ub, const uint8_t *__restrict__ label_ub,
+                             const uint8_t *__restrict__ term_ub, int32_t *__restrict__ parent,
+                             uint8_t *__restrict__ label, uint8_t *__restrict__ terminal) {
+    pdl_go();
+    pdl_after();
+    for (int32_t s = blockIdx.x; s < M; s += gridDim.x) {
+        const int64_t ub = off[set_off[s]] - off[0] + s;
+        const int32_t base = roots[s], n = count[s];
+        for (int32_t i = threadIdx.x; i < n; i += blockDim.x) {
+            const int32_t p = parent_ub[ub + i];
+            parent[base + i] = p < 0 ? -1 : base + p;
+            label[base + i] = label_ub[ub + i];
+            terminal[base + i] = term_ub[ub + i];
+        }
+    }
+}
+
 }  // namespace
 
 // Scratch of one device build. Staging part: the strings, level-order node
@@ -372,6 +565,7 @@ struct DeviceBuild::Scratch {
     uint8_t *label_g, *term_g;
     uint32_t *bits[2];
     int32_t *end_sd, *first_sd, *off_sd, *roots, *map;
+    int32_t *count, *total;  // small-set path: nodes per set, all nodes
     unsigned long long *n_chars;
 };
 
@@ -404,6 +598,9 @@ cudaError_t DeviceBuild::stage(const uint8_t *h_bytes, const int64_t *h_off, con
     M_ = M;
     K_ = K;
     n_bytes_ = n_bytes;
+    smax_ = 1;
+    for (int32_t i = 0; i < M; i++) smax_ = std::max(smax_, h_set_off[i + 1] - h_set_off[i]);
+    small_ = smax_ <= kSetMaxStrings;
     s_ = new Scratch();
     const int64_t U = n_bytes + M;               // nodes at most
     const int64_t W = std::max<int64_t>(K, M);   // parents of one level at most
@@ -476,6 +673,7 @@ cudaError_t DeviceBuild::levels(int32_t D, int num_sms, int32_t *n_nodes, std::v
     const cudaStream_t st = stream_;
     const int32_t M = M_, K = K_;
     D_ = D;
+    if (small_) return sets(num_sms, n_nodes, roots, n_chars);
     const int64_t U = n_bytes_ + M;
     const int64_t W = std::max<int64_t>(K, M);
     const int64_t sd = int64_t(M) * (D + 1);
@@ -537,7 +735,61 @@ cudaError_t DeviceBuild::levels(int32_t D, int num_sms, int32_t *n_nodes, std::v
     return cudaSuccess;
 }
 
+cudaError_t DeviceBuild::sets(int num_sms, int32_t *n_nodes, std::vector<int32_t> *roots, int64_t *n_chars) {
+    const cudaStream_t st = stream_;
+    const int32_t M = M_;
+    Carver c;
+    const size_t o_cnt = c.add(4 * size_t(M)), o_tot = c.add(4);
+    cudaError_t e = cudaMallocFromPoolAsync(&s_->base2, c.total, pool_, st);
+    if (e != cudaSuccess) return e;
+    char *b = static_cast<char *>(s_->base2);
+    s_->count = reinterpret_cast<int32_t *>(b + o_cnt);
+    s_->total = reinterpret_cast<int32_t *>(b + o_tot);
+    const size_t smem = size_t(smax_) * (8 * sizeof(uint32_t) + sizeof(int32_t));
+    int per_sm = 0;
+    if ((e = cudaFuncSetAttribute(k_b_sets, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem))) !=
+            cudaSuccess ||
+        (e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_b_sets, kSetThreads, smem)) != cudaSuccess)
+        return e;
+    const int64_t grid = std::min<int64_t>(M, int64_t(num_sms) * std::max(per_sm, 1));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(grid));
+    cfg.blockDim = dim3(unsigned(kSetThreads));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if ((e = cudaLaunchKernelEx(&cfg, k_b_sets, static_cast<const uint8_t *>(s_->bytes),
+                                static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M,
+                                smax_, s_->parent_g, s_->label_g, s_->term_g, s_->count, s_->n_chars)) !=
+            cudaSuccess ||
+        (e = launch(k_b_set_scan, 1, kBThreads, st, M, static_cast<const int32_t *>(s_->count), s_->roots,
+                    s_->total)) != cudaSuccess)
+        return e;
+    int32_t n = 0;
+    unsigned long long nc = 0;
+    roots->resize(size_t(M));
+    if ((e = cudaMemcpyAsync(&n, s_->total, 4, cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(roots->data(), s_->roots, 4 * size_t(M), cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(&nc, s_->n_chars, 8, cudaMemcpyDeviceToHost, st)) != cudaSuccess ||
+        (e = cudaStreamSynchronize(st)) != cudaSuccess)
+        return e;
+    *n_nodes = n;
+    *n_chars = int64_t(nc);
+    n_ = n;
+    return cudaSuccess;
+}
+
 cudaError_t DeviceBuild::emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms) {
+    if (small_)
+        return launch(k_b_set_emit, std::min<int64_t>(M_, int64_t(num_sms) * 8), kBThreads, stream_,
+                      static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M_,
+                      static_cast<const int32_t *>(s_->count), static_cast<const int32_t *>(s_->roots),
+                      static_cast<const int32_t *>(s_->parent_g), static_cast<const uint8_t *>(s_->label_g),
+                      static_cast<const uint8_t *>(s_->term_g), parent, label, terminal);
     const int64_t ngrid = std::min<int64_t>((int64_t(n_) + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
     return launch(k_b_permute, ngrid, kBThreads, stream_, static_cast<const int32_t *>(s_->ls), D_,
                   static_cast<const int32_t *>(s_->map), static_cast<const int32_t *>(s_->parent_g),

@@ -264,11 +264,15 @@ public:
     cudaError_t emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms);
 
 private:
+    // forests of small sets: one CTA per set (called by levels())
+    cudaError_t sets(int num_sms, int32_t *n_nodes, std::vector<int32_t> *roots, int64_t *n_chars);
     struct Scratch;
     Scratch *s_ = nullptr;
     cudaStream_t stream_ = nullptr;
     cudaMemPool_t pool_ = nullptr;
     int32_t M_ = 0, K_ = 0, D_ = 0, n_ = 0;
+    int32_t smax_ = 1;    // strings of the largest set
+    bool small_ = false;  // one CTA per set
     int64_t n_bytes_ = 0;
 };
 

@@ -102,6 +102,33 @@ def test_device_forest_small_random(cuda, seed):
     _same_handles(d, T.trie_build_many(sb, so, index))
 
 
+@pytest.mark.parametrize("big", [4096, 4097, 9000])
+def test_device_forest_set_size_paths(cuda, big):
+    """Sets of up to 4,096 strings are built one CTA per set (levels in shared
+    memory), larger ones by the level path over all sets: both sides of the
+    boundary, with small random sets beside the big one."""
+    r = random.Random(big)
+    alpha = [0x00, 0x41, 0x61, 0x5F, 0xFF]
+    big_set = [bytes(r.choice(alpha) for _ in range(r.randint(0, 9))) for _ in range(big)]
+    sets = _random_sets(big)[:3] + [big_set] + _random_sets(big + 1)[:3]
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _check_against_oracle(d, sets)
+    _same_handles(d, T.trie_build_many(sb, so, index))
+
+
+def test_device_forest_level_path_codes(cuda):
+    """The K = 10,000 ICD-style codes as one set (level path), between two
+    small sets."""
+    w = W.config(3)
+    codes = W.unpack(w.set_bytes, w.set_offsets)
+    sets = [[b"A01.1", b"A01"], codes, [b"", b"Z"]]
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _check_against_oracle(d, sets)
+    _same_handles(d, T.trie_build_many(sb, so, index))
+
+
 def test_device_forest_more_sets_than_strings(cuda):
     """5,000 sets holding 3 strings in all: the root level is the widest."""
     sets = [[] for _ in range(5000)]
