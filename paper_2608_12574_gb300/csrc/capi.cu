@@ -137,6 +137,9 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
     const size_t o_blob = L.add(hv.blob.size());
     const size_t o_key = L.add(sizeof(uint64_t) * hv.ht_key.size());
     const size_t o_val = L.add(sizeof(int32_t) * hv.ht_val.size());
+    // the probe's per-slot payload (blob offsets / 16 must fit in 27 bits)
+    const bool with_pay = !hv.dup_keys && hv.blob.size() < (size_t(1) << 31);
+    const size_t o_pay = with_pay ? L.add(sizeof(uint4) * hv.ht_key.size()) : 0;
     cudaError_t e = cudaMalloc(&dv->base, L.total);
     if (e != cudaSuccess) {
         dv->base = nullptr;
@@ -162,6 +165,13 @@ int get_vocab(const uint8_t *vb, const int64_t *vo, int32_t V, int dev,
     dv->dup_keys = hv.dup_keys;
     dv->ht_key = reinterpret_cast<const uint64_t *>(base + o_key);
     dv->ht_val = reinterpret_cast<const int32_t *>(base + o_val);
+    if (with_pay) {
+        uint4 *pay = reinterpret_cast<uint4 *>(base + o_pay);
+        if ((e = tmk::launch_vocab_pay(*dv, pay, num_sms(dev), 0)) != cudaSuccess ||
+            (e = cudaStreamSynchronize(0)) != cudaSuccess)
+            return fail_cuda(e, "building the token table's payload");
+        dv->ht_pay = pay;
+    }
     try {
         dv->src_offsets.assign(vo, vo + V + 1);
         dv->src_bytes.assign(vb ? vb + b0 : nullptr, vb ? vb + b1 : nullptr);
@@ -705,7 +715,8 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     tmk::DevLists &L = h->lists;
     if (!L.base) {  // per-row counters, cursors, offsets and scan scratch
         Layout lay;
-        const size_t o_cnt = lay.add(sizeof(int32_t) * 2 * size_t(n));
+        const size_t o_cnt = lay.add(sizeof(int32_t) * 3 * size_t(n));
+        const size_t o_rank = lay.add(sizeof(int32_t) * size_t(tmk::kHitSlots) * size_t(n));
         const size_t o_off = lay.add(sizeof(int64_t) * (size_t(n) + 1));
         const size_t o_tile = lay.add(sizeof(int64_t) * (size_t(n) / 4096 + 2));
         const size_t o_tot = lay.add(sizeof(int64_t));
@@ -715,6 +726,8 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         L.base = base;
         L.count = reinterpret_cast<int32_t *>(b + o_cnt);
         L.cursor = L.count + n;
+        L.over = L.count + 2 * int64_t(n);
+        L.rank = reinterpret_cast<int32_t *>(b + o_rank);
         L.off = reinterpret_cast<int64_t *>(b + o_off);
         L.tile_sum = reinterpret_cast<int64_t *>(b + o_tile);
         L.total = reinterpret_cast<int64_t *>(b + o_tot);

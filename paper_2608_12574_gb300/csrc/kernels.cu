@@ -135,6 +135,7 @@ struct PatchArgs {
     const uint32_t *tok_off;
     const uint16_t *tok_len;
     const uint8_t *blob;
+    const uint4 *ht_pay;  // per slot {token, min(len, 31) << 27 | blob offset / 16, bytes 0-3, 4-7}, or null
     int32_t lmax;
     uint32_t *mask;
     int64_t W;
@@ -148,6 +149,8 @@ struct PatchArgs {
     ulonglong2 *trans;         // transition table (row, token) -> end node, or null
     uint32_t trans_mask;       // slots - 1
     int32_t trans_fill;        // the probe inserts every transition it finds
+    int32_t *list_count;       // list compile: the probe counts the recorded hits per row, or null
+    int32_t *hit_rank;         // [n_nodes * kHitSlots]: each recorded hit's position in its row
 };
 
 // Transition table: open addressing over 16-byte slots {key, end node};
@@ -323,6 +326,24 @@ __device__ __forceinline__ void node_hits(const PatchArgs &a, int32_t m, Emit em
     }
 }
 
+// Payload of every slot of the token table (thread per slot): the token, its
+// length (saturated at 31) and blob offset / 16 in one word, and its first 8
+// bytes (the blob is zero-padded to 16 bytes per token). Empty slots: zero.
+__global__ void k_vocab_pay(const uint64_t *__restrict__ key, const int32_t *__restrict__ val,
+                            const uint16_t *__restrict__ tok_len, const uint32_t *__restrict__ tok_off,
+                            const uint8_t *__restrict__ blob, int64_t S, uint4 *__restrict__ pay) {
+    for (int64_t s = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; s < S; s += int64_t(gridDim.x) * blockDim.x) {
+        uint4 p = make_uint4(0u, 0u, 0u, 0u);
+        if (key[s]) {
+            const int32_t t = val[s];
+            const uint32_t len = tok_len[t], off = tok_off[t];
+            const uint2 b = *reinterpret_cast<const uint2 *>(blob + off);
+            p = make_uint4(uint32_t(t), (min(len, 31u) << 27) | (off >> 4), b.x, b.y);
+        }
+        pay[s] = p;
+    }
+}
+
 // Child links from parent and label (thread per node c): in breadth-first
 // order the children of a node are contiguous, so c is its parent's first
 // child iff c - 1 has another parent; every child sets its label's bit in its
@@ -477,21 +498,39 @@ __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, 
                 }
             }
             int32_t tid[8];
-#pragma unroll
-            for (int i = 0; i < 8; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
             int32_t tlen[8];
             uint32_t toff[8];
-#pragma unroll
-            for (int i = 0; i < 8; i++) {
-                tlen[i] = tid[i] >= 0 ? int32_t(__ldg(a.tok_len + tid[i])) : -1;
-                toff[i] = tid[i] >= 0 ? __ldg(a.tok_off + tid[i]) : 0u;
-            }
-            // token bytes: 16-byte aligned in the blob, which has 16 bytes of tail room
             uint4 tb[8];
+            if (a.ht_pay) {
+                // one load per match gives the token, its length, its offset
+                // and its first 8 bytes; suffixes of 9-16 bytes then read the
+                // rest from the blob
 #pragma unroll
-            for (int i = 0; i < 8; i++)
-                tb[i] = tlen[i] == k0 + i + 1 ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]))
-                                              : make_uint4(0u, 0u, 0u, 0u);
+                for (int i = 0; i < 8; i++) {
+                    const uint4 p = slot[i] >= 0 ? __ldg(a.ht_pay + slot[i]) : make_uint4(0u, 0u, 0u, 0u);
+                    tid[i] = slot[i] >= 0 ? int32_t(p.x) : -1;
+                    tlen[i] = slot[i] >= 0 ? int32_t(p.y >> 27) : -1;
+                    toff[i] = (p.y & 0x07FFFFFFu) << 4;
+                    tb[i] = make_uint4(p.z, p.w, 0u, 0u);
+                }
+#pragma unroll
+                for (int i = 0; i < 8; i++)
+                    if (k0 + i + 1 > 8 && tlen[i] == k0 + i + 1)
+                        tb[i] = __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]));
+            } else {
+#pragma unroll
+                for (int i = 0; i < 8; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
+#pragma unroll
+                for (int i = 0; i < 8; i++) {
+                    tlen[i] = tid[i] >= 0 ? int32_t(__ldg(a.tok_len + tid[i])) : -1;
+                    toff[i] = tid[i] >= 0 ? __ldg(a.tok_off + tid[i]) : 0u;
+                }
+                // token bytes: 16-byte aligned in the blob, which has 16 bytes of tail room
+#pragma unroll
+                for (int i = 0; i < 8; i++)
+                    tb[i] = tlen[i] == k0 + i + 1 ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]))
+                                                  : make_uint4(0u, 0u, 0u, 0u);
+            }
 #pragma unroll
             for (int i = 0; i < 8; i++) {
                 const int k = k0 + i + 1;  // suffix length
@@ -560,7 +599,10 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
         int32_t c = 0;
         int2 *slot = a.hits + int64_t(m) * kHitSlots;
         node_hits_window(a, m, [&](int32_t row, int32_t t) {
-            if (c < kHitSlots) slot[c] = make_int2(row, t);
+            if (c < kHitSlots) {
+                slot[c] = make_int2(row, t);
+                if (a.list_count) a.hit_rank[int64_t(m) * kHitSlots + c] = atomicAdd(a.list_count + row, 1);
+            }
             c++;
             if (a.trans_fill && t != a.eos) trans_insert(a.trans, a.trans_mask, row, t, m);
         });
@@ -818,18 +860,20 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
 // App. H.5): for every node, the ids of its allowed tokens (EOS included at
 // terminal nodes) in no particular order, as CSR offsets[N+1] + tokens.
 
-// Counts the allowed tokens of every row (the start node of each hit).
-__global__ void __launch_bounds__(kPatchThreads, 4) k_list_count(PatchArgs a, int32_t *__restrict__ row_count) {
+// The probe counted the hits it recorded (at most kHitSlots per node) and
+// gave each its position in its row; the hits beyond those, of nodes that
+// overflowed, are found again here (the search emits them in the same order)
+// and counted apart.
+__global__ void __launch_bounds__(kPatchThreads, 4) k_list_count_over(PatchArgs a, int32_t *__restrict__ over) {
     pdl_launch_dependents();
-    pdl_wait();  // hits from the probe, zeroed counters
+    pdl_wait();  // hits from the probe
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        const int32_t c = a.hit_count[m];
-        if (c == kHitOverflow) {
-            node_hits_window(a, m, [&](int32_t row, int32_t) { atomicAdd(row_count + row, 1); });
-            continue;
-        }
-        for (int32_t i = 0; i < c; i++) atomicAdd(row_count + a.hits[int64_t(m) * kHitSlots + i].x, 1);
+        if (a.hit_count[m] != kHitOverflow) continue;
+        int32_t i = 0;
+        node_hits_window(a, m, [&](int32_t row, int32_t) {
+            if (i++ >= kHitSlots) atomicAdd(over + row, 1);
+        });
     }
 }
 
@@ -866,7 +910,9 @@ __device__ __forceinline__ int64_t block_exclusive_scan(int64_t v, int64_t *smem
     return warp_base + x - v;
 }
 
-__global__ void __launch_bounds__(kScanThreads) k_scan_tiles(const int32_t *__restrict__ cnt, int32_t n,
+// The count of row i is cnt[i] (+ cnt2[i] when cnt2 is not null).
+__global__ void __launch_bounds__(kScanThreads) k_scan_tiles(const int32_t *__restrict__ cnt,
+                                                             const int32_t *__restrict__ cnt2, int32_t n,
                                                              int64_t *__restrict__ tile_sum) {
     pdl_launch_dependents();
     pdl_wait();
@@ -875,7 +921,7 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_tiles(const int32_t *__re
     int64_t v = 0;
 #pragma unroll
     for (int j = 0; j < kScanPer; j++)
-        if (base + j < n) v += cnt[base + j];
+        if (base + j < n) v += cnt[base + j] + (cnt2 ? cnt2[base + j] : 0);
     int64_t total;
     block_exclusive_scan(v, sw, &total);
     if (threadIdx.x == 0) tile_sum[blockIdx.x] = total;
@@ -898,7 +944,8 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_tile_sums(int64_t *__rest
     if (threadIdx.x == 0) *grand_total = carry;
 }
 
-__global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__restrict__ cnt, int32_t n,
+__global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__restrict__ cnt,
+                                                            const int32_t *__restrict__ cnt2, int32_t n,
                                                             const int64_t *__restrict__ tile_off,
                                                             const int64_t *__restrict__ grand_total,
                                                             int64_t *__restrict__ off) {
@@ -910,7 +957,7 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__res
     int64_t v = 0;
 #pragma unroll
     for (int j = 0; j < kScanPer; j++) {
-        c[j] = base + j < n ? cnt[base + j] : 0;
+        c[j] = base + j < n ? cnt[base + j] + (cnt2 ? cnt2[base + j] : 0) : 0;
         v += c[j];
     }
     int64_t total;
@@ -923,23 +970,28 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__res
     if (blockIdx.x == 0 && threadIdx.x == 0) off[n] = *grand_total;
 }
 
-// Writes every hit into its row (positions claimed with a per-row cursor).
+// Writes every hit into its row: a recorded hit at the position the probe
+// gave it; a hit beyond those of an overflowing node after the row's
+// recorded hits, at a position claimed with a per-row cursor.
 __global__ void __launch_bounds__(kPatchThreads, 4) k_list_scatter(PatchArgs a, const int64_t *__restrict__ off,
+                                                                const int32_t *__restrict__ count,
                                                                 int32_t *__restrict__ cursor,
                                                                 int32_t *__restrict__ toks) {
     pdl_launch_dependents();
     pdl_wait();
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        auto put = [&](int32_t row, int32_t t) { toks[off[row] + atomicAdd(cursor + row, 1)] = t; };
         const int32_t c = a.hit_count[m];
-        if (c == kHitOverflow) {
-            node_hits_window(a, m, put);
-            continue;
-        }
-        for (int32_t i = 0; i < c; i++) {
+        const int32_t rec = c == kHitOverflow ? kHitSlots : c;
+        for (int32_t i = 0; i < rec; i++) {
             const int2 hv = a.hits[int64_t(m) * kHitSlots + i];
-            put(hv.x, hv.y);
+            toks[off[hv.x] + a.hit_rank[int64_t(m) * kHitSlots + i]] = hv.y;
+        }
+        if (c == kHitOverflow) {
+            int32_t i = 0;
+            node_hits_window(a, m, [&](int32_t row, int32_t t) {
+                if (i++ >= kHitSlots) toks[off[row] + count[row] + atomicAdd(cursor + row, 1)] = t;
+            });
         }
     }
 }
@@ -1422,6 +1474,7 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.tok_off = v.tok_off;
     a.tok_len = v.tok_len;
     a.blob = v.blob;
+    a.ht_pay = v.ht_pay;
     a.lmax = lmax;
     a.mask = mask;
     a.W = W;
@@ -1435,6 +1488,8 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.trans = t.trans;
     a.trans_mask = t.trans_mask;
     a.trans_fill = 0;
+    a.list_count = nullptr;
+    a.hit_rank = nullptr;
     return a;
 }
 
@@ -1482,6 +1537,13 @@ cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st) {
     return launch_mask_fill(reinterpret_cast<uint32_t *>(t.trans), 4 * (int64_t(t.trans_mask) + 1), num_sms, st);
 }
 
+cudaError_t launch_vocab_pay(const DevVocab &v, uint4 *pay, int num_sms, cudaStream_t st) {
+    const int64_t S = int64_t(v.ht_mask) + 1;
+    const int grid = grid_for(S, 256, int64_t(num_sms) * 8);
+    k_vocab_pay<<<grid, 256, 0, st>>>(v.ht_key, v.ht_val, v.tok_len, v.tok_off, v.blob, S, pay);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
@@ -1498,9 +1560,13 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
     };
     const uint64_t S = uint64_t(v.ht_mask) + 1, nn = uint64_t(n_nodes), nv = uint64_t(v.V);
     add(v.ht_key, 8 * S);
-    add(v.ht_val, 4 * S);
-    add(v.tok_len, 2 * nv);
-    add(v.tok_off, 4 * nv);
+    if (v.ht_pay) {
+        add(v.ht_pay, 16 * S);
+    } else {
+        add(v.ht_val, 4 * S);
+        add(v.tok_len, 2 * nv);
+        add(v.tok_off, 4 * nv);
+    }
     add(v.blob, v.blob_bytes);
     add(t.window, 16 * nn);
     add(t.anc, 64 * nn);
@@ -1592,27 +1658,26 @@ cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab
                                const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
     a.trans_fill = fill_trans && t.trans;
+    a.list_count = L.count;
+    a.hit_rank = L.rank;
     Prefetch pf;
     pf.count = 0;
-    const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
-    cudaError_t e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf);
+    // count, cursor and over are adjacent: zero all three before the probe counts
+    cudaError_t e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), 3 * int64_t(n_nodes), num_sms, st);
     if (e != cudaSuccess) return e;
-    // count and cursor are adjacent: zero both
-    if ((e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), 2 * int64_t(n_nodes), num_sms, st)) !=
-        cudaSuccess)
-        return e;
-
+    const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
+    if ((e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf)) != cudaSuccess) return e;
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
-    if ((e = launch_pdl(k_list_count, grid, kPatchThreads, st, a, L.count)) != cudaSuccess) return e;
+    if ((e = launch_pdl(k_list_count_over, grid, kPatchThreads, st, a, L.over)) != cudaSuccess) return e;
     const int32_t n_tiles = int32_t((int64_t(n_nodes) + kScanTile - 1) / kScanTile);
-    if ((e = launch_pdl(k_scan_tiles, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count), n_nodes,
-                        L.tile_sum)) != cudaSuccess)
+    if ((e = launch_pdl(k_scan_tiles, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count),
+                        static_cast<const int32_t *>(L.over), n_nodes, L.tile_sum)) != cudaSuccess)
         return e;
     if ((e = launch_pdl(k_scan_tile_sums, 1, kScanThreads, st, L.tile_sum, n_tiles, L.total)) != cudaSuccess)
         return e;
-    if ((e = launch_pdl(k_scan_rows, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count), n_nodes,
-                        static_cast<const int64_t *>(L.tile_sum), static_cast<const int64_t *>(L.total),
-                        L.off)) != cudaSuccess)
+    if ((e = launch_pdl(k_scan_rows, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count),
+                        static_cast<const int32_t *>(L.over), n_nodes, static_cast<const int64_t *>(L.tile_sum),
+                        static_cast<const int64_t *>(L.total), L.off)) != cudaSuccess)
         return e;
     // the size decides the token buffer: read it back (the one host sync)
     if ((e = cudaMemcpyAsync(h_total, L.total, sizeof(int64_t), cudaMemcpyDeviceToHost, st)) != cudaSuccess)
@@ -1624,8 +1689,9 @@ cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVoc
                                  const DevLists &L, int num_sms, cudaStream_t st) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
-    return launch_pdl(k_list_scatter, grid, kPatchThreads, st, a, static_cast<const int64_t *>(L.off), L.cursor,
-                      L.toks);
+    a.hit_rank = L.rank;
+    return launch_pdl(k_list_scatter, grid, kPatchThreads, st, a, static_cast<const int64_t *>(L.off),
+                      static_cast<const int32_t *>(L.count), L.cursor, L.toks);
 }
 
 namespace {

@@ -138,6 +138,9 @@ struct DevVocab {
     int32_t dup_keys = 0;
     const uint64_t *ht_key = nullptr;
     const int32_t *ht_val = nullptr;
+    // per slot: token, min(len, 31) << 27 | blob offset / 16, first 8 bytes
+    // (null when the blob exceeds 2 GiB or two tokens share a key)
+    const uint4 *ht_pay = nullptr;
     // host copy of the caller's arrays, to recognise the same vocabulary later
     std::vector<uint8_t> src_bytes;
     std::vector<int64_t> src_offsets;
@@ -173,9 +176,11 @@ struct DevTrie {
 
 // Device storage of the sparse valid lists of a handle (library-owned).
 struct DevLists {
-    void *base = nullptr;           // count, cursor, off, tile_sum, total
-    int32_t *count = nullptr;       // [n] allowed tokens per row (cursor follows it)
-    int32_t *cursor = nullptr;      // [n]
+    void *base = nullptr;           // count, cursor, over, rank, off, tile_sum, total
+    int32_t *count = nullptr;       // [n] recorded hits per row (cursor and over follow it)
+    int32_t *cursor = nullptr;      // [n] positions claimed by overflow hits
+    int32_t *over = nullptr;        // [n] hits per row beyond the recorded ones
+    int32_t *rank = nullptr;        // [n * kHitSlots] position of each recorded hit in its row
     int64_t *off = nullptr;         // [n + 1]
     int64_t *tile_sum = nullptr;    // [tiles]
     int64_t *total = nullptr;       // [1]
@@ -339,6 +344,8 @@ cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cu
 cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
 // Zeroes the transition table (before it is filled for another vocabulary).
 cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st);
+// Fills the per-slot payload of the vocabulary's token table (S uint4).
+cudaError_t launch_vocab_pay(const DevVocab &v, uint4 *pay, int num_sms, cudaStream_t st);
 cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, const int32_t *states_in,
                            int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err, bool use_trans,
                            cudaStream_t st);
