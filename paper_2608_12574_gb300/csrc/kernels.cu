@@ -1559,10 +1559,8 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
         pf.count++;
     };
     const uint64_t S = uint64_t(v.ht_mask) + 1, nn = uint64_t(n_nodes), nv = uint64_t(v.V);
-    add(v.ht_key, 8 * S);
-    if (v.ht_pay) {
-        add(v.ht_pay, 16 * S);
-    } else {
+    add(v.ht_key, 8 * S);  // every suffix probe reads a slot pair
+    if (!v.ht_pay) {       // only matches read the payload: it is not prefetched
         add(v.ht_val, 4 * S);
         add(v.tok_len, 2 * nv);
         add(v.tok_off, 4 * nv);
