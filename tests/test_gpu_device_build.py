@@ -195,6 +195,36 @@ def test_device_forest_copy_path(cuda):
     assert r.returncode == 0 and r.stdout.strip().endswith("ok"), r.stdout + r.stderr
 
 
+def test_device_forest_repeated_builds_reuse_memory(cuda):
+    """Build, use and destroy forests of different sizes in turn, as a server
+    does per batch: every build is still equal to the host builder's (blocks
+    that the library's pool hands out again carry nothing over), and the
+    device memory in use stops growing once the pool holds its blocks."""
+    import torch
+    w = W.dynamic_requests(24)
+    small = [_forest(_random_sets(s)) for s in (41, 42)]
+    free = []
+    for it in range(6):
+        sb, so, index = (w.set_bytes, w.set_offsets, w.set_index) if it % 2 == 0 else small[it // 2 % 2]
+        d = T.trie_build_many_device(sb, so, index)
+        T.trie_compile_lists(d, w.vocab_bytes, w.vocab_offsets, w.V)
+        if it < 2 or it == 5:
+            h = T.trie_build_many(sb, so, index)
+            _same_handles(d, h)
+            T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, w.V)
+            od, td = T.trie_copy_lists(d)
+            oh, th = T.trie_copy_lists(h)
+            assert torch.equal(od, oh)
+            rows = np.repeat(np.arange(d.num_nodes, dtype=np.int64), np.diff(od.cpu().numpy()))
+            assert np.array_equal(np.sort(rows * w.V + td.cpu().numpy()), np.sort(rows * w.V + th.cpu().numpy()))
+            h.destroy()
+        d.destroy()
+        torch.cuda.synchronize()
+        free.append(torch.cuda.mem_get_info()[0])
+    # after the first large build the pool serves the later ones
+    assert free[-2] >= free[2] - (64 << 20), free
+
+
 def test_device_forest_single_set_mask_equals_oracle(cuda):
     """A forest of one set (the K=100 tool names): the dense mask compiled on
     the device-built handle equals the oracle's mask."""
