@@ -449,6 +449,100 @@ __device__ __forceinline__ int32_t anc_at(const int4 (&an)[4], int k) {
 // not in their first pair follow their chains together (find_slots). In a
 // vocabulary where some tokens share a key, a key whose first pair is full
 // takes the sequential probe, which finds every token under it.
+// One wavefront of node_hits_window: the suffixes of lengths k0 + 1 ..
+// k0 + 8 (those within depth) of node m. h and pw hold the hash of the
+// first k0 labels and B^k0 and are advanced over the batch; hit(i, row, t)
+// is called for every token t that is the suffix of length k0 + i + 1
+// (starting at row).
+template <typename Hit>
+__device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0, int32_t depth,
+                                           const uint32_t (&lab)[4], const int4 (&an)[4], uint64_t &h,
+                                           uint64_t &pw, Hit hit) {
+    const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
+    uint64_t key[8];
+    ulonglong2 first[8];
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+        key[i] = 0ull;
+        first[i] = make_ulonglong2(0ull, 0ull);
+        if (k0 + i < depth) {
+            h += (uint64_t(byte_at(lab, k0 + i)) + 1ull) * pw;
+            pw *= kHashBase;
+            key[i] = hash_finish(h, uint32_t(k0 + i + 1));
+            first[i] = __ldg(pairs + (uint32_t(key[i] >> 1) & a.pairs_mask));
+        }
+    }
+    int32_t slot[8];  // slot of the key, -1 none
+    uint32_t slow = 0;  // bit i: candidate i needs the sequential probe
+    if (!a.dup_keys) {
+        uint32_t pending = 0;
+#pragma unroll
+        for (int i = 0; i < 8; i++)
+            if (k0 + i < depth) pending |= 1u << i;
+        find_slots<8>(a, key, pending, first, slot);
+    } else {
+#pragma unroll
+        for (int i = 0; i < 8; i++) {
+            const bool m0 = first[i].x == key[i], m1 = first[i].y == key[i];
+            const uint32_t pr = uint32_t(key[i] >> 1) & a.pairs_mask;
+            slot[i] = (k0 + i < depth && (m0 || m1)) ? int32_t(2 * pr + (m0 ? 0 : 1)) : -1;
+            if (k0 + i < depth && first[i].y != 0ull) {
+                slow |= 1u << i;
+                slot[i] = -1;
+            }
+        }
+    }
+    int32_t tid[8];
+    int32_t tlen[8];
+    uint32_t toff[8];
+    uint4 tb[8];
+    if (a.ht_pay) {
+        // one load per match gives the token, its length, its offset
+        // and its first 8 bytes; suffixes of 9-16 bytes then read the
+        // rest from the blob
+#pragma unroll
+        for (int i = 0; i < 8; i++) {
+            const uint4 p = slot[i] >= 0 ? __ldg(a.ht_pay + slot[i]) : make_uint4(0u, 0u, 0u, 0u);
+            tid[i] = slot[i] >= 0 ? int32_t(p.x) : -1;
+            tlen[i] = slot[i] >= 0 ? int32_t(p.y >> 27) : -1;
+            toff[i] = (p.y & 0x07FFFFFFu) << 4;
+            tb[i] = make_uint4(p.z, p.w, 0u, 0u);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; i++)
+            if (k0 + i + 1 > 8 && tlen[i] == k0 + i + 1)
+                tb[i] = __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]));
+    } else {
+#pragma unroll
+        for (int i = 0; i < 8; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
+#pragma unroll
+        for (int i = 0; i < 8; i++) {
+            tlen[i] = tid[i] >= 0 ? int32_t(__ldg(a.tok_len + tid[i])) : -1;
+            toff[i] = tid[i] >= 0 ? __ldg(a.tok_off + tid[i]) : 0u;
+        }
+        // token bytes: 16-byte aligned in the blob, which has 16 bytes of tail room
+#pragma unroll
+        for (int i = 0; i < 8; i++)
+            tb[i] = tlen[i] == k0 + i + 1 ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]))
+                                          : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+        const int k = k0 + i + 1;  // suffix length
+        if (slow & (1u << i)) {
+            probe(a, key[i], k, &lab, m, [&](int32_t t) { hit(i, anc_at(an, k - 1), t); });
+        } else if (tlen[i] == k) {
+            // token byte j must equal the label k-1-j levels above m
+            const uint32_t tw[4] = {tb[i].x, tb[i].y, tb[i].z, tb[i].w};
+            bool eq = true;
+#pragma unroll
+            for (int j = 0; j < kMaxClimb; j++)
+                if (j < k) eq = eq && byte_at(tw, j) == byte_at(lab, k - 1 - j);
+            if (eq) hit(i, anc_at(an, k - 1), tid[i]);
+        }
+    }
+}
+
 template <typename Emit>
 __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, Emit emit) {
     const ulonglong2 win = __ldg(a.window + m);
@@ -459,94 +553,11 @@ __device__ __forceinline__ void node_hits_window(const PatchArgs &a, int32_t m, 
     const int32_t depth = a.lmax < d16 ? a.lmax : d16;
     const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y), uint32_t(win.y >> 32)};
     if (__ldg(a.terminal + m)) emit(m, a.eos);
-    const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
     uint64_t h = 0, pw = 1;
 #pragma unroll
     for (int k0 = 0; k0 < kMaxClimb; k0 += 8) {
-        if (k0 < depth) {
-            uint64_t key[8];
-            ulonglong2 first[8];
-#pragma unroll
-            for (int i = 0; i < 8; i++) {
-                key[i] = 0ull;
-                first[i] = make_ulonglong2(0ull, 0ull);
-                if (k0 + i < depth) {
-                    h += (uint64_t(byte_at(lab, k0 + i)) + 1ull) * pw;
-                    pw *= kHashBase;
-                    key[i] = hash_finish(h, uint32_t(k0 + i + 1));
-                    first[i] = __ldg(pairs + (uint32_t(key[i] >> 1) & a.pairs_mask));
-                }
-            }
-            int32_t slot[8];  // slot of the key, -1 none
-            uint32_t slow = 0;  // bit i: candidate i needs the sequential probe
-            if (!a.dup_keys) {
-                uint32_t pending = 0;
-#pragma unroll
-                for (int i = 0; i < 8; i++)
-                    if (k0 + i < depth) pending |= 1u << i;
-                find_slots<8>(a, key, pending, first, slot);
-            } else {
-#pragma unroll
-                for (int i = 0; i < 8; i++) {
-                    const bool m0 = first[i].x == key[i], m1 = first[i].y == key[i];
-                    const uint32_t pr = uint32_t(key[i] >> 1) & a.pairs_mask;
-                    slot[i] = (k0 + i < depth && (m0 || m1)) ? int32_t(2 * pr + (m0 ? 0 : 1)) : -1;
-                    if (k0 + i < depth && first[i].y != 0ull) {
-                        slow |= 1u << i;
-                        slot[i] = -1;
-                    }
-                }
-            }
-            int32_t tid[8];
-            int32_t tlen[8];
-            uint32_t toff[8];
-            uint4 tb[8];
-            if (a.ht_pay) {
-                // one load per match gives the token, its length, its offset
-                // and its first 8 bytes; suffixes of 9-16 bytes then read the
-                // rest from the blob
-#pragma unroll
-                for (int i = 0; i < 8; i++) {
-                    const uint4 p = slot[i] >= 0 ? __ldg(a.ht_pay + slot[i]) : make_uint4(0u, 0u, 0u, 0u);
-                    tid[i] = slot[i] >= 0 ? int32_t(p.x) : -1;
-                    tlen[i] = slot[i] >= 0 ? int32_t(p.y >> 27) : -1;
-                    toff[i] = (p.y & 0x07FFFFFFu) << 4;
-                    tb[i] = make_uint4(p.z, p.w, 0u, 0u);
-                }
-#pragma unroll
-                for (int i = 0; i < 8; i++)
-                    if (k0 + i + 1 > 8 && tlen[i] == k0 + i + 1)
-                        tb[i] = __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]));
-            } else {
-#pragma unroll
-                for (int i = 0; i < 8; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
-#pragma unroll
-                for (int i = 0; i < 8; i++) {
-                    tlen[i] = tid[i] >= 0 ? int32_t(__ldg(a.tok_len + tid[i])) : -1;
-                    toff[i] = tid[i] >= 0 ? __ldg(a.tok_off + tid[i]) : 0u;
-                }
-                // token bytes: 16-byte aligned in the blob, which has 16 bytes of tail room
-#pragma unroll
-                for (int i = 0; i < 8; i++)
-                    tb[i] = tlen[i] == k0 + i + 1 ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]))
-                                                  : make_uint4(0u, 0u, 0u, 0u);
-            }
-#pragma unroll
-            for (int i = 0; i < 8; i++) {
-                const int k = k0 + i + 1;  // suffix length
-                if (slow & (1u << i)) {
-                    probe(a, key[i], k, &lab, m, [&](int32_t t) { emit(anc_at(an, k - 1), t); });
-                } else if (tlen[i] == k) {
-                    // token byte j must equal the label k-1-j levels above m
-                    const uint32_t tw[4] = {tb[i].x, tb[i].y, tb[i].z, tb[i].w};
-                    bool eq = true;
-#pragma unroll
-                    for (int j = 0; j < kMaxClimb; j++)
-                        if (j < k) eq = eq && byte_at(tw, j) == byte_at(lab, k - 1 - j);
-                    if (eq) emit(anc_at(an, k - 1), tid[i]);
-                }
-            }
-        }
+        if (k0 < depth)
+            wavefront8(a, m, k0, depth, lab, an, h, pw, [&](int, int32_t row, int32_t t) { emit(row, t); });
     }
     // suffixes longer than the window (deep tries with long tokens)
     if (a.lmax > kMaxClimb && depth == kMaxClimb) {
@@ -607,6 +618,77 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
             if (a.trans_fill && t != a.eos) trans_insert(a.trans, a.trans_mask, row, t, m);
         });
         a.hit_count[m] = uint8_t(c > kHitSlots ? kHitOverflow : c);
+    }
+}
+
+// k_mask_probe with two threads per node, for tries so small that one
+// thread per node leaves most SMs idle and the probe's chain of dependent
+// loads sets the compile time: lanes 2j and 2j + 1 of a warp take node j of
+// the warp's 16, the even lane EOS and the suffixes of lengths 1-8, the odd
+// lane lengths 9-16, each as one wavefront (the same instructions on every
+// lane, k0 = 0 or 8). The pair then writes its hits in node_hits_window's
+// order (EOS, lengths 1..16) into the node's slots, so the hit buffer is
+// that of k_mask_probe. Only for vocabularies with the per-slot payload (at
+// most one token per suffix) and tokens of at most 16 bytes.
+__global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs a, Prefetch pf) {
+    pdl_wait();  // an earlier scatter may still read the hit buffer
+    if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
+    pdl_launch_dependents();
+    const int lane = threadIdx.x & 31;
+    const int half = lane & 1;
+    const int k0 = 8 * half;
+    const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+    const int64_t n2 = 2 * int64_t(a.n_nodes);
+    // every lane of a warp runs the same iterations (the shuffles below)
+    for (int64_t w0 = int64_t(blockIdx.x) * blockDim.x + (threadIdx.x & ~31); w0 < n2; w0 += stride) {
+        const int64_t t = w0 + lane;
+        const bool valid = t < n2;
+        const int32_t m = valid ? int32_t(t >> 1) : 0;
+        int32_t found[8];
+#pragma unroll
+        for (int i = 0; i < 8; i++) found[i] = -1;
+        int4 an[4] = {};
+        bool eos = false;
+        if (valid) {
+            const ulonglong2 win = __ldg(a.window + m);
+#pragma unroll
+            for (int q = 0; q < 4; q++) an[q] = __ldg(a.anc + int64_t(m) * 4 + q);
+            const int32_t d16 = __ldg(a.depth16 + m);
+            const int32_t depth = a.lmax < d16 ? a.lmax : d16;
+            const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y),
+                                     uint32_t(win.y >> 32)};
+            eos = half == 0 && __ldg(a.terminal + m);
+            uint64_t h = 0, pw = 1;
+#pragma unroll
+            for (int j = 0; j < 8; j++)  // the odd lane starts after the first 8 labels
+                if (half && j < depth) {
+                    h += (uint64_t(byte_at(lab, j)) + 1ull) * pw;
+                    pw *= kHashBase;
+                }
+            if (k0 < depth)
+                wavefront8(a, m, k0, depth, lab, an, h, pw, [&](int i, int32_t, int32_t tok) { found[i] = tok; });
+        }
+        int32_t c = eos ? 1 : 0;
+#pragma unroll
+        for (int i = 0; i < 8; i++) c += found[i] >= 0 ? 1 : 0;
+        const int32_t c0 = __shfl_sync(0xffffffffu, c, lane & ~1);
+        const int32_t c1 = __shfl_sync(0xffffffffu, c, lane | 1);
+        if (!valid) continue;
+        int2 *slot = a.hits + int64_t(m) * kHitSlots;
+        int32_t s = half ? c0 : 0;
+        auto rec = [&](int32_t row, int32_t tok) {
+            if (s < kHitSlots) {
+                slot[s] = make_int2(row, tok);
+                if (a.list_count) a.hit_rank[int64_t(m) * kHitSlots + s] = atomicAdd(a.list_count + row, 1);
+            }
+            s++;
+            if (a.trans_fill && tok != a.eos) trans_insert(a.trans, a.trans_mask, row, tok, m);
+        };
+        if (eos) rec(m, a.eos);
+#pragma unroll
+        for (int i = 0; i < 8; i++)
+            if (found[i] >= 0) rec(anc_at(an, k0 + i), found[i]);
+        if (half == 0) a.hit_count[m] = uint8_t(c0 + c1 > kHitSlots ? kHitOverflow : c0 + c1);
     }
 }
 
@@ -1500,6 +1582,20 @@ inline int grid_for(int64_t work, int64_t per_block, int64_t cap) {
     return int(g);
 }
 
+// The probe: two threads per node while even those fill at most half of the
+// resident slots (4 CTAs of kPatchThreads per SM) and the vocabulary allows
+// it (per-slot payload, tokens of at most 16 bytes), else one per node. Its
+// grid is resident at once (so that every CTA passes its entry wait and lets
+// the fill launch right away); nodes in a grid-stride loop.
+cudaError_t launch_probe(const PatchArgs &a, const Prefetch &pf, int num_sms, cudaStream_t st) {
+    const int64_t resident = int64_t(num_sms) * 4 * kPatchThreads;
+    if (a.ht_pay && a.lmax <= kMaxClimb && 2 * int64_t(a.n_nodes) * 2 <= resident)
+        return launch_pdl(k_mask_probe_pair, grid_for(2 * int64_t(a.n_nodes), kPatchThreads, int64_t(num_sms) * 4),
+                          kPatchThreads, st, a, pf);
+    return launch_pdl(k_mask_probe, grid_for(a.n_nodes, kPatchThreads, int64_t(num_sms) * 4), kPatchThreads, st, a,
+                      pf);
+}
+
 }  // namespace
 
 cudaError_t launch_mask_fill(uint32_t *mask, int64_t n_words, int num_sms, cudaStream_t st) {
@@ -1548,9 +1644,6 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
     a.trans_fill = fill_trans && t.trans;
-    // probe grid: every CTA resident at once (so that all of them pass their
-    // entry wait and let the fill launch right away), nodes in a grid-stride loop
-    const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
     Prefetch pf;
     pf.count = 0;
     auto add = [&](const void *p, uint64_t n) {
@@ -1570,7 +1663,7 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
     add(t.anc, 64 * nn);
     add(t.depth16, nn);
     add(t.terminal, nn);
-    cudaError_t e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf);
+    cudaError_t e = launch_probe(a, pf, num_sms, st);
     if (e != cudaSuccess) return e;
     const uintptr_t addr = reinterpret_cast<uintptr_t>(mask);
     const int64_t n_words = int64_t(n_nodes) * W;
@@ -1663,8 +1756,7 @@ cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab
     // count, cursor and over are adjacent: zero all three before the probe counts
     cudaError_t e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), 3 * int64_t(n_nodes), num_sms, st);
     if (e != cudaSuccess) return e;
-    const int probe_grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 4);
-    if ((e = launch_pdl(k_mask_probe, probe_grid, kPatchThreads, st, a, pf)) != cudaSuccess) return e;
+    if ((e = launch_probe(a, pf, num_sms, st)) != cudaSuccess) return e;
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
     if ((e = launch_pdl(k_list_count_over, grid, kPatchThreads, st, a, L.over)) != cudaSuccess) return e;
     const int32_t n_tiles = int32_t((int64_t(n_nodes) + kScanTile - 1) / kScanTile);
