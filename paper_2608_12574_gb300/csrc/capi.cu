@@ -554,6 +554,8 @@ int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const i
         cudaGetLastError();
         pool_free(h->dev.base);
         delete h;
+        if (e == cudaErrorMemoryAllocation)
+            return fail(TRIE_ENOMEM, "device allocation failed while building the forest");
         return fail_cuda(e, "building the forest on the device");
     }
     *out = h;

@@ -405,7 +405,8 @@ __device__ __forceinline__ int32_t set_excl_scan(int32_t v, int32_t *ws, int32_t
 }
 
 // Dynamic shared memory: the child-label sets of the current level
-// (smax rows of 8 words) and the first child of each of its nodes.
+// (smax rows of 8 words), the first child of each of its nodes, and a flag
+// per node of the next level that some string ends at.
 __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restrict__ bytes,
                                                         const int64_t *__restrict__ off,
                                                         const int32_t *__restrict__ set_off, int32_t M, int32_t smax,
@@ -415,12 +416,14 @@ __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restric
     extern __shared__ uint4 dyn[];
     uint32_t *bits = reinterpret_cast<uint32_t *>(dyn);
     int32_t *first = reinterpret_cast<int32_t *>(bits + int64_t(smax) * 8);
+    uint8_t *ends = reinterpret_cast<uint8_t *>(first + smax);
     __shared__ int32_t ws[kSetThreads / 32];
     __shared__ int32_t root_term;
     pdl_go();
     pdl_after();
     const int tid = threadIdx.x;
     for (int32_t r = tid; r < smax * 8; r += kSetThreads) bits[r] = 0u;
+    for (int32_t r = tid; r < smax; r += kSetThreads) ends[r] = 0;
     for (int32_t s = blockIdx.x; s < M; s += gridDim.x) {
         const int32_t i0 = set_off[s], Ks = set_off[s + 1] - i0;
         const int64_t ub = off[i0] - off[0] + s;
@@ -488,14 +491,21 @@ __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restric
                 const int64_t g = ub + ch;
                 parent_ub[g] = cur[k];
                 label_ub[g] = uint8_t(b);
-                if (len[k] == d + 1) term_ub[g] = 1;
-                else nb[k] = bytes[st[k] + d + 1];
+                if (len[k] == d + 1) {
+                    term_ub[g] = 1;
+                    ends[ch - level_end] = 1;
+                } else {
+                    nb[k] = bytes[st[k] + d + 1];
+                }
                 cur[k] = ch;
             }
             __syncthreads();
             for (int32_t r = tid; r < width * 8; r += kSetThreads) bits[r] = 0u;
-            for (int32_t x = level_end + tid; x < level_end + total; x += kSetThreads)
-                if (term_ub[ub + x]) my_chars += unsigned(d + 1);
+            for (int32_t x = tid; x < total; x += kSetThreads)
+                if (ends[x]) {
+                    my_chars += unsigned(d + 1);
+                    ends[x] = 0;
+                }
             level_start = level_end;
             level_end += total;
             __syncthreads();
@@ -745,7 +755,7 @@ cudaError_t DeviceBuild::sets(int num_sms, int32_t *n_nodes, std::vector<int32_t
     char *b = static_cast<char *>(s_->base2);
     s_->count = reinterpret_cast<int32_t *>(b + o_cnt);
     s_->total = reinterpret_cast<int32_t *>(b + o_tot);
-    const size_t smem = size_t(smax_) * (8 * sizeof(uint32_t) + sizeof(int32_t));
+    const size_t smem = size_t(smax_) * (8 * sizeof(uint32_t) + sizeof(int32_t) + 1);
     int per_sm = 0;
     if ((e = cudaFuncSetAttribute(k_b_sets, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem))) !=
             cudaSuccess ||

@@ -129,6 +129,16 @@ def test_device_forest_level_path_codes(cuda):
     _same_handles(d, T.trie_build_many(sb, so, index))
 
 
+@pytest.mark.parametrize("sets", [[[]], [[], [], []], [[b""]], [[], [b""], []]])
+def test_device_forest_without_bytes(cuda, sets):
+    """Forests without a single string byte: lone roots (terminal where the
+    set holds the empty string)."""
+    sb, so, index = _forest(sets)
+    d = T.trie_build_many_device(sb, so, index)
+    _check_against_oracle(d, sets)
+    _same_handles(d, T.trie_build_many(sb, so, index))
+
+
 def test_device_forest_more_sets_than_strings(cuda):
     """5,000 sets holding 3 strings in all: the root level is the widest."""
     sets = [[] for _ in range(5000)]
