@@ -1,0 +1,57 @@
+"""bench.py's reference arm (the CPU oracle) and its launch contract, on CPU.
+
+The reference arm needs no GPU: it times the oracle on this host's cores and
+prints one JSON line with the keys the driver reads. Under a multi-rank launch
+only rank 0 runs it; every other rank exits 0 without work or output.
+"""
+from __future__ import annotations
+
+import json
+import os
+import subprocess
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+ARGS = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "1",
+        "--steps", "1", "--warmup", "0"]
+
+
+def _run(extra_env: dict) -> subprocess.CompletedProcess:
+    env = dict(os.environ)
+    env.update(extra_env)
+    return subprocess.run(ARGS, cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+
+
+def test_reference_arm_prints_one_line():
+    r = _run({"RANK": "0", "WORLD_SIZE": "1"})
+    assert r.returncode == 0, r.stderr
+    lines = [ln for ln in r.stdout.splitlines() if ln.strip()]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference"
+    assert line["unit"] == "pairs/s" and line["higher_is_better"] is True
+    assert line["config"]["workload"] == "tools-K100-V32000-B1-f32"
+    assert line["config"]["N_nodes"] == 1384
+    assert line["value"] > 0 and line["steps"] == 1 and line["warmup"] == 0
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"]
+    assert cb["value"] == line["value"]
+    e2e = line["e2e"]
+    assert e2e == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}
+    # pairs/s of the sample: the sampled share of N x V pairs over one step's time
+    assert line["ms_per_step"] > 0
+    pairs = line["value"] * line["ms_per_step"] * 1e-3
+    assert abs(pairs - 1384 * 32000 * _share(cb)) <= 1e-3 * pairs   # the share is printed to 4 digits
+
+
+def _share(cb: dict) -> float:
+    # "... a 0.7756 slice of one ... step: 1074 of 1384 mask rows ..."
+    words = cb["sample"].split()
+    return float(words[words.index("slice") - 1]) if "slice" in words else float("nan")
+
+
+def test_reference_arm_other_ranks_exit_quietly():
+    r = _run({"RANK": "1", "WORLD_SIZE": "2"})
+    assert r.returncode == 0, r.stderr
+    assert r.stdout.strip() == ""
