@@ -125,9 +125,10 @@ int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t 
  * trie_lazy_init) copy them back once. Strings longer than 1024 bytes, more
  * than 2^24 (set, depth) pairs or more than 2^31-3 string bytes plus sets
  * are built by trie_build_many on the host instead. Device scratch (about
- * 20 bytes per string byte plus 90 per string) is taken with cudaMallocAsync
- * on `stream` and released there. Errors as trie_build_many; TRIE_ECUDA if
- * a CUDA call fails. */
+ * 20 bytes per string byte plus 90 per string) is taken from the library's
+ * device memory pool on `stream` and released there. Errors as
+ * trie_build_many; TRIE_ENOMEM if a device allocation fails, TRIE_ECUDA if
+ * another CUDA call fails. */
 int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
                            int32_t M, cudaStream_t stream, trie_t *out);
 
@@ -216,8 +217,8 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
 /* Sparse form of the masks: for every node the ids of its allowed tokens, as
  * the paper stores them (valid[n] as lists of 4-byte token ids, Sec. 4.2;
  * App. H.5), computed on the GPU without the dense bitmask. At K = 10,000 and
- * V = 152,064 the lists hold 46,899 ids (188 KB) where the bitmask takes
- * 439 MB.
+ * V = 152,064 the lists hold 56,899 ids (10,000 of them EOS; 228 KB) where the
+ * bitmask takes 439 MB.
  *   Arguments as trie_compile_masks; the lists are stored on the device by
  *   the library, with the handle (they replace those of an earlier call).
  *   Layout: offsets int64[num_nodes + 1] and tokens int32[offsets[N]]; the
