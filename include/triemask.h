@@ -13,7 +13,7 @@
  *   3. advances a batch of decode states by their sampled tokens,
  *      s' = delta*(s, bytes(token)) (Sec. 2, Eq. 1),
  *   4. writes -inf into the logits of every token not in valid[s]
- *      (Sec. 4.2 last paragraph; App. H.3 "bitmask application").
+ *      (Sec. 4.2 last paragraph; App. H.3, the cost of applying the bitmask).
  *
  * Conventions shared by every call
  * --------------------------------
