@@ -356,3 +356,20 @@ def test_mask_offset_pointer(cuda):
                            oracle.Vocab(w.vocab_bytes, w.vocab_offsets), nthreads=NCPU)
     assert np.array_equal(_np_u32(m), want)
     assert int(buf[0].item()) == 0 and int(buf[-3:].abs().sum().item()) == 0
+
+
+def test_compile_forest_full(cuda):
+    """256 per-request sets (4.8M nodes, 76 GB mask): every row of every set,
+    against the oracle's pairs (each set's Aho-Corasick pairs plus EOS at its
+    terminal nodes, offset by its root), compared on the device in chunks."""
+    import torch
+    from maskcheck import assert_mask_equals_pairs, forest_pairs
+    w = W.config(5)
+    h, m = _compile(cuda, w.set_bytes, w.set_offsets, w.vocab_bytes, w.vocab_offsets, w.set_index)
+    ac = oracle.AhoCorasick(oracle.Vocab(w.vocab_bytes, w.vocab_offsets))
+    rows, toks = forest_pairs(ac, W.unpack(w.set_bytes, w.set_offsets), w.set_index, h.roots(), w.V,
+                              nthreads=NCPU)
+    torch.cuda.synchronize()
+    assert_mask_equals_pairs(m, rows, toks)
+    del m
+    torch.cuda.empty_cache()
