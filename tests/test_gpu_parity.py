@@ -373,3 +373,62 @@ def test_compile_forest_full(cuda):
     assert_mask_equals_pairs(m, rows, toks)
     del m
     torch.cuda.empty_cache()
+
+
+def test_decode_loop_forest(cuda):
+    """The 256-request workload decoded as the bench decodes it: one forest of
+    the requests' sets, valid lists, the list-driven apply for step 0 and one
+    advance + apply launch per later step, greedy argmax in between. Every
+    request is then decoded by the oracle on its own set's trie (local node id
+    = forest id - the set's root) and compared at each of the 32 steps:
+    masked logits, token and state, and the error count."""
+    import torch
+    from concurrent.futures import ThreadPoolExecutor
+    w = W.config(5)
+    B, S = w.batch, w.steps
+    h = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
+    assert h.num_sets == B
+    T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, w.V)
+    roots = h.roots().astype(np.int64)
+    bufs = [torch.as_tensor(roots.astype(np.int32), device=cuda), torch.empty(B, dtype=torch.int32, device=cuda)]
+    err = torch.zeros(1, dtype=torch.int32, device=cuda)
+    raw, masked, toks, entering = [], [], [], []
+    tok = None
+    for t in range(S):
+        x = W.logits(w, t, device="cuda")
+        raw.append(_bits(x).copy())
+        if t == 0:
+            T.trie_apply_lists(h, x, bufs[0])
+        else:
+            T.trie_advance_apply_lists(h, bufs[(t - 1) % 2], tok, bufs[t % 2], x, err)
+        tok = torch.argmax(x, dim=1).to(torch.int32)
+        masked.append(_bits(x).copy())
+        toks.append(tok.cpu().numpy().copy())
+        entering.append(bufs[t % 2].cpu().numpy().copy())
+    T.trie_advance(h, bufs[(S - 1) % 2], tok, err)
+    entering.append(bufs[(S - 1) % 2].cpu().numpy().copy())     # the states after the last step
+    gpu_err = int(err.item())
+
+    ov = oracle.Vocab(w.vocab_bytes, w.vocab_offsets)
+    strings = W.unpack(w.set_bytes, w.set_offsets)
+
+    def check(b):
+        ot = oracle.Trie(*W.pack(strings[w.set_index[b]:w.set_index[b + 1]]))
+        om, otk, ost, oe = oracle.decode(ot, ov, [raw[t][b:b + 1] for t in range(S)], np.zeros(1, np.int32))
+        for t in range(S):
+            g = int(entering[t + 1][b])
+            g = g - int(roots[b]) if g >= 0 else g
+            if not np.array_equal(masked[t][b], om[t][0]):
+                return f"request {b}, step {t}: masked logits"
+            if int(toks[t][b]) != int(otk[t][0]):
+                return f"request {b}, step {t}: token"
+            if g != int(ost[t][0]):
+                return f"request {b}, step {t}: state {g} against {int(ost[t][0])}"
+        return oe
+
+    with ThreadPoolExecutor(max_workers=NCPU) as ex:
+        res = list(ex.map(check, range(B)))
+    bad = [r for r in res if isinstance(r, str)]
+    assert not bad, bad[:5]
+    assert gpu_err == sum(res) == 0
+    assert int(entering[0].astype(np.int64).sum()) == int(roots.sum())   # every request starts at its root
