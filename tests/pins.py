@@ -208,6 +208,22 @@ def check_golden(name: str) -> None:
                 assert got == want, (row["cite"], sorted(got))
             else:
                 assert want <= got, (row["cite"], sorted(got))
+    # token paths from the root: every step of a path that ends on a node or
+    # FINISHED is allowed by the row it leaves; the walk ends where stated
+    id_of = {name: i for i, name in name_of.items()}
+    ends = {"FINISHED": oracle.FINISHED, "DEAD": oracle.DEAD}
+    for path in ex.get("paths", []):
+        state = np.zeros(1, np.int32)
+        errors = 0
+        for name in path["tokens"]:
+            v = id_of[name]
+            if path["end"] != "DEAD" and state[0] >= 0:
+                assert v in row_ids(oracle.mask_rows(t, voc, [int(state[0])])[0], len(toks)), path["cite"]
+            state, e = oracle.advance(t, voc, state, np.array([v], np.int32))
+            errors += e
+        want = ends[path["end"]] if path["end"] in ends else ids[path["end"].encode()]
+        assert int(state[0]) == want, (path["cite"], int(state[0]))
+        assert errors == (1 if path["end"] == "DEAD" else 0), path["cite"]
 
 
 def check_chain(s: bytes) -> None:

@@ -54,6 +54,7 @@ MUTANTS = {
 def _all_pins():
     check_golden("appG1_worked_example.json")
     check_golden("fig2_alignment.json")
+    check_golden("appH9_noncanonical.json")
     check_argmax(7)
     check_chain(b"medical_billing")
     check_chain(bytes([0, 255, 0, 255, 7]))
