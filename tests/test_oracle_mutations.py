@@ -55,6 +55,7 @@ def _all_pins():
     check_golden("appG1_worked_example.json")
     check_golden("fig2_alignment.json")
     check_golden("appH9_noncanonical.json")
+    check_golden("sec42_prefix_values.json")
     check_argmax(7)
     check_chain(b"medical_billing")
     check_chain(bytes([0, 255, 0, 255, 7]))

@@ -10,7 +10,8 @@ from pins import (build, check_advance, check_apply, check_argmax, check_chain, 
                   check_masks, check_numbering, expected_row, prefix_ids, random_case, row_ids)
 
 
-@pytest.mark.parametrize("name", ["appG1_worked_example.json", "fig2_alignment.json", "appH9_noncanonical.json"])
+@pytest.mark.parametrize("name", ["appG1_worked_example.json", "fig2_alignment.json", "appH9_noncanonical.json",
+                                  "sec42_prefix_values.json"])
 def test_paper_worked_examples(oracle_lib, name):
     """App. G.1 Steps 1-4 (29 nodes, 44 chars, listed rows), Fig. 2's masks and
     App. H.9's canonical and non-canonical splits of one value."""
