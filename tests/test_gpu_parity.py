@@ -432,3 +432,30 @@ def test_decode_loop_forest(cuda):
     assert not bad, bad[:5]
     assert gpu_err == sum(res) == 0
     assert int(entering[0].astype(np.int64).sum()) == int(roots.sum())   # every request starts at its root
+
+
+@pytest.mark.parametrize("name", ["appG1_worked_example.json", "fig2_alignment.json",
+                                  "appH9_noncanonical.json", "sec42_prefix_values.json"])
+def test_golden_examples(cuda, name):
+    """The paper's worked examples (tests/golden): the GPU mask equals the
+    oracle's, and the GPU walks every listed token path to the oracle's state."""
+    import json
+    import torch
+    g = json.load(open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", name)))
+    toks = [b"" if s == "<EOS>" else s.encode() for s in g["vocab"]]
+    sb, so = W.pack([s.encode() for s in g["set"]])
+    vb, vo = W.pack(toks)
+    h, m = _compile(cuda, sb, so, vb, vo)
+    ot, ov = oracle.Trie(sb, so), oracle.Vocab(vb, vo)
+    assert np.array_equal(_np_u32(m), oracle.mask_all(ot, ov))
+    id_of = {s: i for i, s in enumerate(g["vocab"])}
+    for path in g["expect"].get("paths", []):
+        st = torch.zeros(1, dtype=torch.int32, device=cuda)
+        err = torch.zeros(1, dtype=torch.int32, device=cuda)
+        want = np.zeros(1, np.int32)
+        for s in path["tokens"]:
+            tok = np.array([id_of[s]], np.int32)
+            T.trie_advance(h, st, torch.as_tensor(tok, device=cuda), err)
+            want, _ = oracle.advance(ot, ov, want, tok)
+        assert int(st.item()) == int(want[0]), path["cite"]
+        assert int(err.item()) == (1 if path["end"] == "DEAD" else 0), path["cite"]
