@@ -55,3 +55,24 @@ def test_reference_arm_other_ranks_exit_quietly():
     r = _run({"RANK": "1", "WORLD_SIZE": "2"})
     assert r.returncode == 0, r.stderr
     assert r.stdout.strip() == ""
+
+
+def test_clock_summary_parses_nvidia_smi_samples():
+    """The clock record of the timed region: median SM clock, the maximum, and
+    every throttle reason seen Active in any sample (sw_power_cap included)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    c = bench.ClockSampler(None)
+    c.out = "\n".join([
+        "2070, 2070, 812.4, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+        "1980, 2070, 1391.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active",
+        "2055, 2070, 1102.7, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+        "[N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A], [N/A]",
+        "garbage",
+    ])
+    s = c.summary()
+    assert s == {"sm_mhz": 2055.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+    c.out = "1200, 2070, 900.0, 0x0000000000000008, Active, Not Active, Active, Not Active"
+    assert c.summary()["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
+    c.out = ""
+    assert c.summary()["reasons"] == ["no samples"]
