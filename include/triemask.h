@@ -260,8 +260,9 @@ int trie_apply_lists(trie_t h, void *d_logits, int dtype, const int32_t *d_state
  * uint32 words plus 16 bytes per trie node and 16 per batch row; replaces the
  * cache of an earlier trie_lazy_init on the handle (starting empty).
  *   vocab_bytes, vocab_offsets, V  as trie_compile_masks, 2 <= V <= 524,288
- *   cache_rows  rows kept between calls (rounded up to a multiple of 8; 0 =
- *               no cache, every row is recomputed). The cache is 8-way set
+ *   cache_rows  rows kept between calls, 0 <= cache_rows <= 2^30 (rounded up
+ *               to a multiple of 8; 0 = no cache, every row is recomputed;
+ *               TRIE_ENOMEM if the rows do not fit). The cache is 8-way set
  *               associative: a node may only use the 8 rows of its set, and
  *               a new row replaces the least recently used of them.
  *   max_batch   largest B of the calls below, 1 <= max_batch <= 4096

@@ -810,7 +810,8 @@ int trie_lazy_init(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_of
     if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
     if (V < 2 || (int64_t(V) + 31) / 32 > tmk::kLazyMaxWords)
         return fail(TRIE_EINVAL, "V must be in [2, " + std::to_string(tmk::kLazyMaxWords * 32) + "] for lazy rows");
-    if (cache_rows < 0) return fail(TRIE_EINVAL, "cache_rows must be >= 0");
+    if (cache_rows < 0 || cache_rows > tmk::kLazyMaxCacheRows)
+        return fail(TRIE_EINVAL, "cache_rows must be in [0, " + std::to_string(tmk::kLazyMaxCacheRows) + "]");
     if (max_batch < 1 || max_batch > tmk::kLazyMaxBatch)
         return fail(TRIE_EINVAL, "max_batch must be in [1, " + std::to_string(tmk::kLazyMaxBatch) + "]");
     int dev, rc;

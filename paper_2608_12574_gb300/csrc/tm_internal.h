@@ -195,6 +195,7 @@ struct DevLists {
 // replacement inside each set.
 constexpr int kLazyWays = 8;       // rows per cache set
 constexpr int kLazyMaxBatch = 4096;
+constexpr int32_t kLazyMaxCacheRows = int32_t(1) << 30;  // cache rows + call rows stay int32
 constexpr int64_t kLazyMaxWords = 16384;  // row built in shared memory (64 KB): V <= 524,288
 // A missing row whose subtree has more than kLazyPartNodes nodes is computed
 // in parts by several CTAs (at most kLazyMaxParts per row), for at most

@@ -227,6 +227,9 @@ def test_lazy_calls_checked_before_any_device_work(lib):
     assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 1, 8, 8) == T.TRIE_EINVAL       # V < 2
     assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 600000, 8, 8) == T.TRIE_EINVAL  # V too big
     assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, -1, 8) == T.TRIE_EINVAL      # cache_rows
+    for rows in ((1 << 30) + 1, 2**31 - 1):                  # rounding up must not overflow int32
+        assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, rows, 8) == T.TRIE_EINVAL
+        assert "cache_rows" in T.trie_last_error()
     assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, 8, 0) == T.TRIE_EINVAL       # max_batch
     assert L.trie_lazy_init(h.handle, vb.ctypes.data, vo.ctypes.data, 2, 8, 4097) == T.TRIE_EINVAL
     assert L.trie_lazy_init(h.handle, vb.ctypes.data, None, 2, 8, 8) == T.TRIE_EINVAL
