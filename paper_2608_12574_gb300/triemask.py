@@ -267,15 +267,11 @@ def trie_advance(h: Trie, d_states, d_tokens, d_err=None, stream=None) -> None:
 def trie_advance_apply(h: Trie, d_states_in, d_tokens, d_states_out, d_logits, d_err=None, stream=None) -> None:
     """states_out <- delta*(states_in, tokens); then mask d_logits ([B, V]) by states_out."""
     import torch
-    if d_logits.dim() != 2:
-        raise ValueError("d_logits must be [B, V]")
+    dtype = _logits_dtype(d_logits)
     B, V = d_logits.shape
     for t, name in ((d_states_in, "d_states_in"), (d_tokens, "d_tokens"), (d_states_out, "d_states_out")):
         if t.numel() != B:
             raise ValueError(f"{name} must have B entries")
-    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
-    if dtype is None:
-        raise TypeError("d_logits must be float32 or bfloat16")
     pe = _dev(d_err, (torch.int32,), "d_err") if d_err is not None else None
     _check(h._lib.trie_advance_apply(h.handle, _dev(d_states_in, (torch.int32,), "d_states_in"),
                                      _dev(d_tokens, (torch.int32,), "d_tokens"),
@@ -287,14 +283,10 @@ def trie_advance_apply(h: Trie, d_states_in, d_tokens, d_states_out, d_logits, d
 def trie_apply_mask(h: Trie, d_logits, d_states, stream=None) -> None:
     """-inf into disallowed entries of d_logits ([B, V] fp32 or bf16, CUDA), in place."""
     import torch
-    if d_logits.dim() != 2:
-        raise ValueError("d_logits must be [B, V]")
+    dtype = _logits_dtype(d_logits)
     B, V = d_logits.shape
     if d_states.numel() != B:
         raise ValueError("d_states must have B entries")
-    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
-    if dtype is None:
-        raise TypeError("d_logits must be float32 or bfloat16")
     pl = _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits")
     ps = _dev(d_states, (torch.int32,), "d_states")
     _check(h._lib.trie_apply_mask(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
@@ -333,14 +325,10 @@ def trie_copy_lists(h: Trie, device=None, stream=None):
 def trie_apply_lists(h: Trie, d_logits, d_states, stream=None) -> None:
     """trie_apply_mask driven by the handle's valid lists."""
     import torch
-    if d_logits.dim() != 2:
-        raise ValueError("d_logits must be [B, V]")
+    dtype = _logits_dtype(d_logits)
     B, V = d_logits.shape
     if d_states.numel() != B:
         raise ValueError("d_states must have B entries")
-    dtype = {torch.float32: TRIE_DTYPE_F32, torch.bfloat16: TRIE_DTYPE_BF16}.get(d_logits.dtype)
-    if dtype is None:
-        raise TypeError("d_logits must be float32 or bfloat16")
     pl = _dev(d_logits, (torch.float32, torch.bfloat16), "d_logits")
     ps = _dev(d_states, (torch.int32,), "d_states")
     _check(h._lib.trie_apply_lists(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
