@@ -140,6 +140,20 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def workload_config(w, n_nodes: int) -> dict:
+    """The `config` object of the JSON line, the same in both arms: the
+    workload and its sizes (N_chars = bytes of the distinct set strings, r =
+    N / N_chars as in App. H.7) and how L2 reuse is ruled out."""
+    from paper_2608_12574_gb300 import workloads as W
+    n_chars = sum(len(x) for x in set(W.unpack(w.set_bytes, w.set_offsets)))
+    elt = 2 if w.dtype == "bf16" else 4
+    mask_bytes = n_nodes * ((w.V + 31) // 32) * 4
+    return {"workload": w.name, "K": w.K, "V": w.V, "batch": w.batch, "decode_steps": w.steps,
+            "N_nodes": n_nodes, "N_chars": n_chars, "r": round(n_nodes / max(1, n_chars), 4),
+            "l2": f"inputs larger than L2: logits {w.steps * w.batch * w.V * elt / 1e9:.2f} GB, "
+                  f"mask {mask_bytes / 1e9:.2f} GB"}
+
+
 # --------------------------------------------------------------------------- oracle arm
 
 class OracleSample:
@@ -256,8 +270,7 @@ def run_reference(args, w):
             "warmup": warmup, "ms_per_step": cb["s_per_step"] * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "u32 mask / " + w.dtype, "data": "synthetic",
             "impl": "reference",
-            "config": {"workload": w.name, "K": w.K, "V": w.V, "batch": w.batch, "decode_steps": w.steps,
-                       "N_nodes": cb["N_nodes"]},
+            "config": workload_config(w, cb["N_nodes"]),
             "cpu_baseline": cb,
             "e2e": {"value": cb["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
@@ -409,21 +422,30 @@ def run_gpu(args, w, rank: int, world: int, dist):
 
         reps = max(20, min(200, args.steps // 4))
         compile_ms = timed(run_compile, reps)
+        # the same mask evaluated pair by pair (a lane per token, a warp
+        # ballot per word), the design the suffix search replaces
+        run_pairwise = capture(lambda: T.trie_compile_masks_pairwise(h, w.vocab_bytes, w.vocab_offsets, V, mask,
+                                                                     stream))
+        pairwise_ms = timed(run_pairwise, max(3, reps // 10))
+        run_compile()  # the mask of the suffix search again
         apply_avg = timed(run_apply, reps) / S
         advance_avg = timed(run_advance, reps) / S
         fused_avg = timed(run_fused, reps) / (S - 1)
-        # sparse valid lists: build (host-synchronous: it reads the size back)
-        # and the list-driven apply over the same 16 logits buffers
+        # sparse valid lists: the build (CUDA events around one call; no host
+        # sync inside it) and the list-driven apply over the same logits buffers
         with torch.cuda.stream(stream):
             n_valid = T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
         stream.synchronize()
         lt = []
         for _ in range(20):
-            t0 = time.perf_counter()
+            l0, l1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             with torch.cuda.stream(stream):
-                T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
-            lt.append(time.perf_counter() - t0)
-        lists_ms = sorted(lt)[len(lt) // 2] * 1e3
+                l0.record(stream)
+                T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
+                l1.record(stream)
+            stream.synchronize()
+            lt.append(l0.elapsed_time(l1))
+        lists_ms = sorted(lt)[len(lt) // 2]
 
         def apply_lists_only():
             for t in range(S):
@@ -433,6 +455,26 @@ def run_gpu(args, w, rank: int, world: int, dist):
         apply_lists_avg = timed(run_apply_lists, reps) / S
         lazy = run_lazy(w, logits, forced, dev, stream, capture, timed, reps)
         formats = run_formats(w, dev, stream, capture, timed, reps)
+    # a new schema with the vocabulary already cached (Sec. 4.2: the automaton
+    # over the vocabulary is made once per tokenizer, only the traversal runs
+    # per schema): a fresh host trie build, then its first compile, which
+    # uploads the trie (6 B per node), builds its per-node tables and fills
+    # its transition table. CUDA events around the compile call, median of 5.
+    ns_dev, ns_host = [], []
+    for _ in range(5):
+        t0 = time.perf_counter()
+        hn = T.trie_build(w.set_bytes, w.set_offsets)
+        ns_host.append((time.perf_counter() - t0) * 1e3)
+        n0, n1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            n0.record(stream)
+            T.trie_compile_masks(hn, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+            n1.record(stream)
+        stream.synchronize()
+        ns_dev.append(n0.elapsed_time(n1))
+        hn.destroy()
+    new_schema_ms = statistics.median(ns_dev)
+    new_schema_host_ms = statistics.median(ns_host)
     timing_src = (f"CUDA events around {reps} back-to-back replays of a graph of the {S - 1} fused "
                   f"advance+apply launches of a step (over {S - 1} logits buffers, "
                   f"{(S - 1) * B * V * elt / 1e9:.2f} GB > L2), launching stream, right after the timed region")
@@ -443,75 +485,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
     fused_gbs = fused_bytes / (fused_avg * 1e-3) / 1e9
     compile_gbs = compile_bytes / (compile_ms * 1e-3) / 1e9
 
-    # ---- e2e: host strings -> trie_build -> compile -> decode, with the logits
-    # and the step's tokens copied from pinned host memory and the states read
-    # back every decode step. The copies run on their own stream from the top
-    # of the step, so they overlap the host trie build, the compile and the
-    # earlier decode steps; decode step t waits only for its own logits.
-    host_logits = [lg.cpu().pin_memory() for lg in logits]
-    host_forced = forced.cpu().pin_memory()
-    host_states = torch.zeros((S, B), dtype=torch.int32).pin_memory()
-    copy_stream = torch.cuda.Stream(dev)
-    with torch.cuda.stream(stream):
-        dlogs = [torch.empty_like(lg) for lg in logits]
-        dtok = torch.empty((S, B), dtype=torch.int32, device=dev)
-        e2e_mask = torch.empty_like(mask)
-    arrived = [torch.cuda.Event() for _ in range(S + 1)]
-    consumed = torch.cuda.Event()
-    h2d = int(w.set_bytes.nbytes + w.set_offsets.nbytes + host_forced.numel() * 4
-              + sum(x.numel() * x.element_size() for x in host_logits))
-    d2h = S * B * 4
-
-    def e2e_step():
-        copy_stream.wait_event(consumed)  # the previous step is done with the buffers
-        with torch.cuda.stream(copy_stream):
-            dtok.copy_(host_forced, non_blocking=True)
-            arrived[S].record(copy_stream)
-            for t in range(S):
-                dlogs[t].copy_(host_logits[t], non_blocking=True)
-                arrived[t].record(copy_stream)
-        hh = T.trie_build(w.set_bytes, w.set_offsets)
-        T.trie_compile_masks(hh, w.vocab_bytes, w.vocab_offsets, V, e2e_mask, stream)
-        sbuf[0].zero_()
-        stream.wait_event(arrived[S])
-        cur = 0
-        for t in range(S):
-            stream.wait_event(arrived[t])
-            if t == 0:
-                T.trie_apply_mask(hh, dlogs[0], sbuf[0], stream)
-            else:
-                T.trie_advance_apply(hh, sbuf[cur], dtok[t - 1], sbuf[1 - cur], dlogs[t], err, stream)
-                cur = 1 - cur
-            host_states[t].copy_(sbuf[cur], non_blocking=True)
-        T.trie_advance(hh, sbuf[cur], dtok[S - 1], err, stream)
-        consumed.record(stream)
-        stream.synchronize()
-        hh.destroy()
-
-    with torch.cuda.stream(stream):
-        e2e_step()
-        if dist is not None:
-            dist.barrier()
-        t0 = time.perf_counter()
-        for _ in range(args.e2e_steps):
-            e2e_step()
-        e2e_s = (time.perf_counter() - t0) / args.e2e_steps
-    e2e_s = reduce_max(e2e_s, dist, dev)
-    # context: the step's host->device copies alone (the floor of the e2e
-    # step), the fastest of a few rounds timed with events on the copy stream
-    torch.cuda.synchronize()
-    rounds = []
-    for _ in range(5):
-        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        with torch.cuda.stream(copy_stream):
-            c0.record(copy_stream)
-            dtok.copy_(host_forced, non_blocking=True)
-            for t in range(S):
-                dlogs[t].copy_(host_logits[t], non_blocking=True)
-            c1.record(copy_stream)
-        copy_stream.synchronize()
-        rounds.append(c0.elapsed_time(c1) * 1e-3)
-    h2d_only_s = min(rounds)
+    e2e_s, h2d, d2h, h2d_only_s = run_e2e(w, N, logits, forced, dev, stream, args.e2e_steps, dist)
 
     if rank != 0:
         return
@@ -532,12 +506,9 @@ def run_gpu(args, w, rank: int, world: int, dist):
         "dtype": "u32 mask / " + w.dtype,
         "data": "synthetic",
         "impl": "gb300",
-        "config": {"workload": w.name, "K": w.K, "V": V, "batch": B, "decode_steps": S, "N_nodes": N,
-                   "N_chars": h.num_chars, "r": round(N / max(1, h.num_chars), 4),
-                   "parallelism": f"replicas x{world}",
-                   "l2": f"inputs larger than L2: logits {S * B * V * elt / 1e9:.2f} GB, "
-                         f"mask {compile_bytes / 1e9:.2f} GB",
-                   "graph": not args.no_graph},
+        "config": workload_config(w, N),
+        "parallelism": f"replicas x{world}",
+        "graph": not args.no_graph,
         "roofline": {"bound": "hbm", "achieved": fused_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": fused_gbs / hbm, "traffic": traffic, "kernel": "k_advance_apply_vec",
                      "bytes_per_launch": fused_bytes, "us_per_launch": fused_avg * 1e3,
@@ -554,18 +525,28 @@ def run_gpu(args, w, rank: int, world: int, dist):
                              "ms": compile_ms, "pairs_per_s": N * V / (compile_ms * 1e-3),
                              "peak_kind": peak_kind,
                              "timing": f"CUDA events around {reps} back-to-back replays of a graph of one compile"},
+        "compile_pairwise": {"ms": pairwise_ms, "pairs_per_s": N * V / (pairwise_ms * 1e-3),
+                             "frac_of_write_roofline": compile_bytes / (pairwise_ms * 1e-3) / 1e9 / hbm,
+                             "vs_suffix_search": pairwise_ms / compile_ms,
+                             "kernel": "k_mask_pairwise (a lane per token walks it from the node; "
+                                       "__ballot_sync per mask word)"},
         "sparse_lists": {"entries": n_valid, "bytes": n_valid * 4 + (N + 1) * 8,
-                         "compile_ms_host_sync": lists_ms,
+                         "compile_ms": lists_ms,
                          "apply_us_avg": apply_lists_avg * 1e3,
                          "apply_gbs": (B * V * elt + B * 4) / (apply_lists_avg * 1e-3) / 1e9,
-                         "note": "valid lists as the paper stores them (Sec. 4.2); compile includes its one "
-                                 "device-to-host read of the size"},
+                         "note": "valid lists as the paper stores them (Sec. 4.2); compile = median of 20 "
+                                 "calls, CUDA events"},
         "lazy_rows": lazy,
         "char_position_masks": formats,
         "breakdown": {"compile_ms": compile_ms, "apply_us_avg": apply_avg * 1e3,
                       "advance_us_avg": advance_avg * 1e3, "advance_apply_us_avg": fused_avg * 1e3,
                       "host_trie_build_ms": host_build_ms,
                       "cold_compile_ms": cold_compile_ms,
+                      "new_schema_compile_ms": new_schema_ms,
+                      "new_schema_host_build_ms": new_schema_host_ms,
+                      "new_schema_note": "fresh trie, vocabulary cached: upload, tables, transition table "
+                                         "clear and fill, compile (events around the call, median of 5); "
+                                         "compile_ms replays a compile whose transition table is complete",
                       "apply_gbs_conventional_rw": (2 * B * V * elt + B * Wd * 4) / (apply_avg * 1e-3) / 1e9},
         "e2e": {"value": job_throughput(N * V, world, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3,
@@ -574,13 +555,106 @@ def run_gpu(args, w, rank: int, world: int, dist):
         "clocks": clk.summary(),
     }
     if not args.no_dynamic:
-        del logits, mask, e2e_mask, dlogs
+        del logits, mask
         torch.cuda.empty_cache()
-        line["dynamic_sets"] = run_dynamic(dev, stream)
+        line["dynamic_sets"] = run_dynamic(dev, stream, rank=rank, world=world, dist=dist)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds / 5, 5, 1)
         line["cpu_paper_algorithm"] = cpu_paper_algorithm(w)
     print(json.dumps(line))
+
+
+def run_e2e(w, n_nodes: int, logits, forced, dev, stream, steps: int, dist=None):
+    """The e2e step through the C ABI from host buffers: per step the trie is
+    built from the host strings and compiled, the logits and tokens are
+    copied from pinned host memory and the states read back after every
+    decode step. Returns (seconds per step, H2D bytes, D2H bytes, seconds of
+    the step's H2D copies alone)."""
+    import torch
+    from paper_2608_12574_gb300 import triemask as T
+    V, B, S = w.V, w.batch, w.steps
+    sbuf = [torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(2)]
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    mask = torch.empty((n_nodes, T.mask_words(V)), dtype=torch.int32, device=dev)
+    # ---- e2e: host strings -> trie_build -> compile -> decode, with the logits
+    # and the step's tokens copied from pinned host memory and the states read
+    # back every decode step. Steps are pipelined as a server would run them:
+    # the copies run on their own stream into two alternating buffer sets, so
+    # step i + 1's copies follow step i's at once; decode step t waits only
+    # for its own logits; the next step's host trie build runs while the GPU
+    # works, and a step's handle is released in stream order (no device sync).
+    host_logits = [lg.cpu().pin_memory() for lg in logits]
+    host_forced = forced.cpu().pin_memory()
+    host_states = [torch.zeros((S, B), dtype=torch.int32).pin_memory() for _ in range(2)]
+    copy_stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        dlogs = [[torch.empty_like(lg) for lg in logits] for _ in range(2)]
+        dtok = [torch.empty((S, B), dtype=torch.int32, device=dev) for _ in range(2)]
+    arrived = [[torch.cuda.Event() for _ in range(S + 1)] for _ in range(2)]
+    consumed = [torch.cuda.Event() for _ in range(2)]
+    h2d = int(w.set_bytes.nbytes + w.set_offsets.nbytes + host_forced.numel() * 4
+              + sum(x.numel() * x.element_size() for x in host_logits))
+    d2h = S * B * 4
+
+    def e2e_step(i, hh):
+        """Queues step i on handle hh (built from the host strings); returns
+        the next step's handle, built while step i runs."""
+        k = i % 2
+        copy_stream.wait_event(consumed[k])  # step i - 2 is done with buffer set k
+        with torch.cuda.stream(copy_stream):
+            dtok[k].copy_(host_forced, non_blocking=True)
+            arrived[k][S].record(copy_stream)
+            for t in range(S):
+                dlogs[k][t].copy_(host_logits[t], non_blocking=True)
+                arrived[k][t].record(copy_stream)
+        T.trie_compile_masks(hh, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+        sbuf[0].zero_()
+        stream.wait_event(arrived[k][S])
+        cur = 0
+        for t in range(S):
+            stream.wait_event(arrived[k][t])
+            if t == 0:
+                T.trie_apply_mask(hh, dlogs[k][0], sbuf[0], stream)
+            else:
+                T.trie_advance_apply(hh, sbuf[cur], dtok[k][t - 1], sbuf[1 - cur], dlogs[k][t], err, stream)
+                cur = 1 - cur
+            host_states[k][t].copy_(sbuf[cur], non_blocking=True)
+        T.trie_advance(hh, sbuf[cur], dtok[k][S - 1], err, stream)
+        consumed[k].record(stream)
+        nxt = T.trie_build(w.set_bytes, w.set_offsets)  # host work beside the GPU's
+        hh.destroy_async(stream)
+        return nxt
+
+    with torch.cuda.stream(stream):
+        hh = T.trie_build(w.set_bytes, w.set_offsets)
+        for i in range(2):
+            hh = e2e_step(i, hh)
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for i in range(steps):
+            hh = e2e_step(i, hh)
+        torch.cuda.synchronize()
+        e2e_s = (time.perf_counter() - t0) / steps
+        hh.destroy()
+    e2e_s = reduce_max(e2e_s, dist, dev)
+    # context: the step's host->device copies alone (the floor of the e2e
+    # step), the fastest of a few rounds timed with events on the copy stream
+    torch.cuda.synchronize()
+    rounds = []
+    for _ in range(5):
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(copy_stream):
+            c0.record(copy_stream)
+            dtok[0].copy_(host_forced, non_blocking=True)
+            for t in range(S):
+                dlogs[0][t].copy_(host_logits[t], non_blocking=True)
+            c1.record(copy_stream)
+        copy_stream.synchronize()
+        rounds.append(c0.elapsed_time(c1) * 1e-3)
+    h2d_only_s = min(rounds)
+    return e2e_s, h2d, d2h, h2d_only_s
 
 
 def run_lazy(w, logits, forced, dev, stream, capture, timed, reps: int) -> dict:
@@ -651,7 +725,28 @@ def run_formats(w, dev, stream, capture, timed, reps: int) -> dict:
     return out
 
 
-def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
+def request_share(n_requests: int, rank: int, world: int) -> tuple[int, int]:
+    """Requests [lo, hi) of one rank: a contiguous block, sizes differing by at
+    most one, every request on exactly one rank."""
+    base, extra = divmod(n_requests, world)
+    lo = rank * base + min(rank, extra)
+    return lo, lo + base + (1 if rank < extra else 0)
+
+
+def share_of(w, lo: int, hi: int):
+    """The per-request forest workload restricted to requests [lo, hi): their
+    strings, and set_index rebased to start at 0 (vocabulary unchanged)."""
+    import dataclasses
+    import numpy as np
+    idx = w.set_index
+    s0, s1 = int(idx[lo]), int(idx[hi])
+    offs = w.set_offsets[s0:s1 + 1]
+    return dataclasses.replace(
+        w, set_bytes=w.set_bytes[int(offs[0]):int(offs[-1])], set_offsets=(offs - offs[0]).astype(np.int64),
+        set_index=(idx[lo:hi + 1] - idx[lo]).astype(np.int32), batch=hi - lo)
+
+
+def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, world: int = 1, dist=None) -> dict:
     """The dynamic per-query-set workload, end to end with logits resident:
     256 requests, each with its own set of K ~ U[300, 2000] names from a
     50,000-name pool; per batch the 256 tries are built as one forest (on the
@@ -661,9 +756,12 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
     import torch
     from paper_2608_12574_gb300 import triemask as T
     from paper_2608_12574_gb300 import workloads as W
-    w = W.config(5)
+    full = W.config(5)
+    lo, hi = request_share(full.batch, rank, world)
+    w = share_of(full, lo, hi) if world > 1 else full
     B, V = w.batch, w.V
-    out = {"workload": w.name, "requests": B, "V": V, "decode_steps": steps}
+    out = {"workload": full.name, "requests": full.batch, "V": V, "decode_steps": steps,
+           "ranks": world, "requests_per_rank": [request_share(full.batch, r, world) for r in range(world)]}
     t0 = time.perf_counter()
     h = T.trie_build_many(w.set_bytes, w.set_offsets, w.set_index)
     out["host_forest_build_ms"] = (time.perf_counter() - t0) * 1e3
@@ -707,15 +805,32 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
         e1.record(stream)
     stream.synchronize()
     out["decode_ms"] = e0.elapsed_time(e1) / reps
-    lt = []
+    lt, lw = [], []
     for _ in range(reps):
+        stream.synchronize()
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
-            n_valid = T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
-        lt.append(time.perf_counter() - t0)
-    out["lists_compile_ms"] = min(lt) * 1e3
+            e0.record(stream)
+            T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
+            e1.record(stream)
+        stream.synchronize()
+        lw.append(time.perf_counter() - t0)
+        lt.append(e0.elapsed_time(e1))
+    n_valid = T.trie_num_valid(h)
+    out["lists_compile_ms"] = min(lt)
+    out["lists_compile_wall_ms"] = min(lw) * 1e3
     out["list_entries"] = n_valid
     out["list_bytes"] = n_valid * 4 + (N + 1) * 8
+    # the list compile's algorithmic traffic: the entries and offsets written
+    # plus the per-node tables the walks read (window 16 B, anc 64 B, depth,
+    # terminal: 82 B per node, read by both walks)
+    peak, peak_kind = peaks()
+    list_bytes = out["list_bytes"] + 2 * 82 * N
+    out["roofline_lists"] = {"bound": "hbm", "achieved": list_bytes / (min(lt) * 1e-3) / 1e9, "peak": peak,
+                             "unit": "GB/s", "frac": list_bytes / (min(lt) * 1e-3) / 1e9 / peak,
+                             "bytes_per_launch": list_bytes, "peak_kind": peak_kind,
+                             "kernel": "k_list_walk (count) + scans + k_list_walk (write)",
+                             "timing": f"CUDA events around one trie_compile_lists, best of {reps}"}
     # end to end per batch of requests: forest build (on the device, or on the
     # host) + list compile + decode
     builders = {
@@ -735,7 +850,7 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
             t0 = time.perf_counter()
             hh = build()
             with torch.cuda.stream(stream):
-                T.trie_compile_lists(hh, w.vocab_bytes, w.vocab_offsets, V, stream)
+                T.trie_compile_lists(hh, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
                 st = [torch.as_tensor(hh.roots(), device=dev), torch.empty(B, dtype=torch.int32, device=dev)]
                 T.trie_apply_lists(hh, logits[0], st[0], stream)
                 for t in range(1, steps):
@@ -744,7 +859,12 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5) -> dict:
             stream.synchronize()
             et.append(time.perf_counter() - t0)
             hh.destroy()
-        out["end_to_end_ms" if kind == "device" else "end_to_end_host_build_ms"] = min(et) * 1e3
+        # with several ranks each holds a share of the requests: the batch is
+        # done when the slowest rank is (max over ranks; no data exchange)
+        key = "end_to_end_ms" if kind == "device" else "end_to_end_host_build_ms"
+        out[key] = reduce_max(min(et) * 1e3, dist, dev)
+    out["requests_per_s"] = full.batch / (out["end_to_end_ms"] * 1e-3)
+    out["scaling"] = "strong: the 256 requests are split across the ranks" if world > 1 else "single rank"
     # lazy rows (App. H.5) instead of the lists: no per-batch compile, each
     # step computes the rows its states reach (the requests are new every
     # batch, so no cache is kept)
@@ -826,11 +946,29 @@ def W_logits(w, s, dev):
     return W.logits(w, s, device=str(dev))
 
 
+def launch_ranks(n: int) -> int:
+    """Re-runs this command as n local ranks (one process per GPU), the way
+    the multi-GPU launch does: torch.distributed.run on 127.0.0.1."""
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr=127.0.0.1", f"--master-port={port}", os.path.abspath(__file__)] + sys.argv[1:]
+    return subprocess.call(cmd)
+
+
 def main():
     args = parse_args()
     from paper_2608_12574_gb300 import workloads as W
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
+    if args.gpus < 1:
+        sys.exit("--gpus must be >= 1")
+    if "WORLD_SIZE" not in os.environ and args.gpus > 1 and args.impl == "gb300":
+        sys.exit(launch_ranks(args.gpus))  # not under a launcher: start the ranks here
+    if "WORLD_SIZE" in os.environ and world != args.gpus:
+        sys.exit(f"--gpus {args.gpus} does not match WORLD_SIZE {world} of the launch")
     w = W.config(args.config)
     if args.impl == "reference":
         if rank == 0:

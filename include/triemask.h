@@ -214,6 +214,18 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
 int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_tokens, int32_t *d_states_out,
                        int32_t *d_err, void *d_logits, int dtype, int32_t B, int32_t V, cudaStream_t stream);
 
+/* The same mask as trie_compile_masks, computed pair by pair: for every node
+ * n and token v the GPU walks v's bytes down from n (the definition of
+ * Sec. 4.1: v is allowed iff prefix(n) . bytes(v) is a prefix of some set
+ * string, App. G.5), one token per lane, and a warp ballot assembles each
+ * 32-bit mask word. It costs N * V walks where trie_compile_masks does a few
+ * lookups per node; it is kept as the direct, measured alternative (the
+ * design that evaluates every pair) and as a second GPU derivation of the
+ * same mask. Arguments, layout, result and errors as trie_compile_masks; it
+ * does not record the mask, the vocabulary or transitions in the handle. */
+int trie_compile_masks_pairwise(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                                uint32_t *d_mask, cudaStream_t stream);
+
 /* Sparse form of the masks: for every node the ids of its allowed tokens, as
  * the paper stores them (valid[n] as lists of 4-byte token ids, Sec. 4.2;
  * App. H.5), computed on the GPU without the dense bitmask. At K = 10,000 and
@@ -224,15 +236,29 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
  *   Layout: offsets int64[num_nodes + 1] and tokens int32[offsets[N]]; the
  *   tokens of node n are tokens[offsets[n] .. offsets[n+1]), EOS (V-1)
  *   included where n is terminal, in no particular order.
- *   Host-synchronous: it reads the number of entries back to size the token
- *   buffer (one small device-to-host copy on `stream`). Records the
- *   vocabulary for trie_advance, like trie_compile_masks.
- *   Errors: TRIE_EINVAL, TRIE_ENOMEM, TRIE_ECUDA. */
+ *   Method: the tokens read backwards form a trie (built once per vocabulary
+ *   on the host, its edges inserted into a device table); from every node m
+ *   the GPU walks it with the labels above m, so that each token ending with
+ *   the last k edges into m is found and listed at the node k levels up
+ *   (the Aho-Corasick outputs of Sec. 4.2 step 2, found per node). One walk
+ *   counts every row's entries, a scan gives the offsets, a second walk
+ *   writes the tokens.
+ *   Asynchronous on `stream` while the bound on the entries (a node lists at
+ *   most one token string per length up to the longest token, each under
+ *   every id that spells it, plus EOS) is at most 2^28 entries or fits the
+ *   buffer of an earlier call: the token buffer is sized by it and nothing
+ *   is read back; trie_num_valid reads the size when asked. Beyond that the
+ *   exact count is read back between the walks (host-synchronous).
+ *   Records the vocabulary for trie_advance, like trie_compile_masks (it
+ *   neither reads nor fills the transition table).
+ *   Errors: TRIE_EINVAL (also for a vocabulary whose reversed-token trie
+ *   would exceed 2^24 - 2 nodes), TRIE_ENOMEM, TRIE_ECUDA. */
 int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
                        cudaStream_t stream);
 
 /* Number of (node, token) entries in the handle's lists; -1 before any
- * trie_compile_lists. */
+ * trie_compile_lists (or if reading the size back fails). The first call
+ * after a trie_compile_lists waits for that build to complete. */
 int64_t trie_num_valid(trie_t h);
 
 /* Copy the handle's lists into caller buffers (device; each may be NULL):
@@ -333,12 +359,18 @@ int trie_advance_apply_lists(trie_t h, const int32_t *d_states_in, const int32_t
  *   table of 12 bytes per slot, 4 slots per token with bytes) must fit in the
  *   scratch; otherwise TRIE_EINVAL with a message, and nothing is launched.
  *   The first call on a device looks up the device address of the scratch
- *   (cudaGetSymbolAddress) with that device current; make that first call
- *   before any stream capture.
+ *   (cudaGetSymbolAddress) and creates one event, with that device current;
+ *   make that first call before any stream capture. Both are kept until the
+ *   process exits: after cudaDeviceReset of a device, do not call this entry
+ *   point on that device again in the same process.
  *   All calls share the one scratch, which keeps the last call's contents
  *   (every byte a call uses is rewritten by it). Calls whose work overlaps on
  *   the GPU (other streams, other threads) race on it; order them, for
  *   example on one stream.
+ *   The host staging buffer is shared too: a call first waits on the host
+ *   until the previous call's copy out of it has completed on the GPU (which
+ *   includes the work queued before that copy on its stream), so calls queued
+ *   back to back on one stream without a synchronisation are safe.
  *   Unlike trie_compile_masks it does not record the mask or the vocabulary
  *   in the handle: trie_advance and trie_apply_mask keep using those of the
  *   last trie_compile_masks.
@@ -392,6 +424,18 @@ int fmt_destroy(fmt_t f);
 /* Release the handle, its host arrays and its device copy of the trie.
  * Synchronises the device first if device memory is held. NULL is a no-op. */
 int trie_destroy(trie_t h);
+
+/* Release the handle without synchronising: its device memory is freed in
+ * stream order on `stream` (it returns to the library's pool once the work
+ * queued on `stream` so far has completed), and its host arrays, which a
+ * queued upload may still be reading, by a host callback queued on `stream`
+ * after that work (a handle that never reached a device: at once). Every
+ * use of the handle on the device must be on `stream` or ordered before the
+ * work queued on it now (for example by an event); the handle must not be
+ * used by the host after the call. A server that builds a trie per request
+ * batch can then drop the batch's handle right after queueing its last
+ * kernel and go on building the next one. NULL is a no-op. */
+int trie_destroy_async(trie_t h, cudaStream_t stream);
 
 /* Message of the last error on the calling thread ("" if none). */
 const char *trie_last_error(void);

@@ -243,6 +243,8 @@ int finish_device_trie(trie_t h, int dev, cudaStream_t stream) {
     return TRIE_OK;
 }
 
+bool host_memory_direct(int dev);
+
 int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     std::lock_guard<std::mutex> lk(h->mu);
     if (h->dev.base) {
@@ -255,6 +257,20 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     const size_t n = size_t(t.n);
     int rc = alloc_device_trie(h, dev, n, stream, true);
     if (rc != TRIE_OK) return rc;
+    if (host_memory_direct(dev)) {
+        // the kernel reads the handle's host arrays itself: a pageable copy
+        // would wait on the host for the stream and for the copy engines
+        cudaError_t e = tmk::launch_copy3(const_cast<int32_t *>(h->dev.parent), t.parent.data(),
+                                          int64_t(sizeof(int32_t) * n), const_cast<uint8_t *>(h->dev.label),
+                                          t.label.data(), int64_t(n), const_cast<uint8_t *>(h->dev.terminal),
+                                          t.terminal.data(), int64_t(n), num_sms(dev), stream);
+        if (e != cudaSuccess) {
+            pool_free(h->dev.base);
+            h->dev = tmk::DevTrie();
+            return fail_cuda(e, "uploading the trie");
+        }
+        return finish_device_trie(h, dev, stream);
+    }
     struct Up { const void *dst; const void *src; size_t n; } ups[] = {
         {h->dev.parent, t.parent.data(), sizeof(int32_t) * n},
         {h->dev.label, t.label.data(), n},
@@ -431,9 +447,10 @@ int tmk::ensure_host_arrays(trie_s *h) {
 }
 
 tmk::DevVocab::~DevVocab() {
-    if (base) {
+    if (base || rt_base) {
         DeviceGuard g(device);
-        cudaFree(base);
+        if (base) cudaFree(base);
+        if (rt_base) cudaFree(rt_base);
     }
 }
 
@@ -703,6 +720,97 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
     return TRIE_OK;
 }
 
+// Token buffers of up to this many entries (1 GiB) are sized by the bound on
+// the number of list entries, with no read-back.
+constexpr int64_t kListBoundEntries = int64_t(1) << 28;
+
+// Whether the handle holds lists (their size may still be on the device).
+static bool lists_built(trie_t h) {
+    std::lock_guard<std::mutex> lk(h->mu);
+    return h->lists.n_valid_on_device || h->lists.n_valid >= 0;
+}
+
+// The vocabulary's reversed-token trie as a device edge table (the list
+// compile's walk), built on first use: on the host, then its edges inserted
+// on the device (host-synchronous, once per vocabulary and device).
+static int ensure_rev_trie(tmk::DevVocab *voc, const uint8_t *vb, const int64_t *vo, int32_t V) {
+    std::lock_guard<std::mutex> lk(voc->rt_mu);
+    if (voc->rt_state == 1) return TRIE_OK;
+    if (voc->rt_state < 0) return fail(TRIE_EINVAL, "the vocabulary is too large for the valid-list walk");
+    tmk::RevTokenTrie rt;
+    std::string err;
+    try {
+        err = tmk::build_reversed_token_trie(vb, vo, V, &rt);
+    } catch (const std::bad_alloc &) {
+        return fail(TRIE_ENOMEM, "host allocation failed while building the reversed-token trie");
+    }
+    if (!err.empty()) {
+        voc->rt_state = -1;
+        return fail(TRIE_EINVAL, err);
+    }
+    uint64_t S = 16;
+    while (S < 2 * uint64_t(rt.n)) S <<= 1;
+    Layout L;
+    const size_t o_edge = L.add(sizeof(uint4) * size_t(S));
+    const size_t o_next = rt.next.empty() ? 0 : L.add(sizeof(int32_t) * size_t(V));
+    Layout T;  // build-time arrays
+    const size_t t_par = T.add(sizeof(int32_t) * size_t(rt.n));
+    const size_t t_lab = T.add(size_t(rt.n));
+    const size_t t_tok = T.add(sizeof(int32_t) * size_t(rt.n));
+    DeviceGuard g(voc->device);
+    void *base = nullptr, *tmp = nullptr;
+    cudaError_t e = cudaMalloc(&base, L.total);
+    if (e == cudaSuccess) e = cudaMalloc(&tmp, T.total);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        if (base) cudaFree(base);
+        return fail(TRIE_ENOMEM, std::string("cudaMalloc for the reversed-token trie: ") + cudaGetErrorString(e));
+    }
+    char *b = static_cast<char *>(base), *t = static_cast<char *>(tmp);
+    if ((e = cudaMemcpy(t + t_par, rt.parent.data(), sizeof(int32_t) * size_t(rt.n), cudaMemcpyHostToDevice)) ==
+            cudaSuccess &&
+        (e = cudaMemcpy(t + t_lab, rt.label.data(), size_t(rt.n), cudaMemcpyHostToDevice)) == cudaSuccess &&
+        (e = cudaMemcpy(t + t_tok, rt.token.data(), sizeof(int32_t) * size_t(rt.n), cudaMemcpyHostToDevice)) ==
+            cudaSuccess &&
+        (rt.next.empty() || (e = cudaMemcpy(b + o_next, rt.next.data(), sizeof(int32_t) * size_t(V),
+                                            cudaMemcpyHostToDevice)) == cudaSuccess) &&
+        (e = tmk::launch_rt_build(reinterpret_cast<const int32_t *>(t + t_par),
+                                  reinterpret_cast<const uint8_t *>(t + t_lab),
+                                  reinterpret_cast<const int32_t *>(t + t_tok), rt.n,
+                                  reinterpret_cast<uint4 *>(b + o_edge), uint32_t(S - 1), num_sms(voc->device),
+                                  0)) == cudaSuccess)
+        e = cudaDeviceSynchronize();
+    cudaFree(tmp);
+    if (e != cudaSuccess) {
+        cudaFree(base);
+        return fail_cuda(e, "building the reversed-token trie");
+    }
+    voc->rt_base = base;
+    voc->rt_edge = reinterpret_cast<const uint4 *>(b + o_edge);
+    voc->rt_mask = uint32_t(S - 1);
+    voc->tok_next = rt.next.empty() ? nullptr : reinterpret_cast<const int32_t *>(b + o_next);
+    voc->rt_mult = rt.max_mult;
+    voc->rt_state = 1;
+    return TRIE_OK;
+}
+
+int trie_compile_masks_pairwise(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                                uint32_t *d_mask, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    if (!d_mask) return fail(TRIE_EINVAL, "d_mask is NULL");
+    if (reinterpret_cast<uintptr_t>(d_mask) & 3u) return fail(TRIE_EINVAL, "d_mask must be 4-byte aligned");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
+    cudaError_t e = tmk::launch_mask_pairwise(h->dev, h->host.n, *voc, d_mask, num_sms(dev), stream);
+    if (e != cudaSuccess) return fail_cuda(e, "pairwise mask compile launch");
+    return TRIE_OK;
+}
+
 int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
                        cudaStream_t stream) {
     if (!h) return fail(TRIE_EINVAL, "handle is NULL");
@@ -712,66 +820,102 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     std::shared_ptr<tmk::DevVocab> voc;
     if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    if ((rc = ensure_rev_trie(voc.get(), vocab_bytes, vocab_offsets, V)) != TRIE_OK) return rc;
     if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
     const int32_t n = h->host.n;
     tmk::DevLists &L = h->lists;
-    if (!L.base) {  // per-row counters, cursors, offsets and scan scratch
+    if (!L.base) {  // per-row counts, offsets and scan scratch
         Layout lay;
-        const size_t o_cnt = lay.add(sizeof(int32_t) * 3 * size_t(n));
-        const size_t o_rank = lay.add(sizeof(int32_t) * size_t(tmk::kHitSlots) * size_t(n));
+        const size_t o_cnt = lay.add(sizeof(int32_t) * size_t(n));
         const size_t o_off = lay.add(sizeof(int64_t) * (size_t(n) + 1));
         const size_t o_tile = lay.add(sizeof(int64_t) * (size_t(n) / 4096 + 2));
         const size_t o_tot = lay.add(sizeof(int64_t));
         void *base = nullptr;
         if ((rc = pool_alloc(dev, lay.total, stream, &base, "the valid lists")) != TRIE_OK) return rc;
+        cudaEvent_t done = nullptr;
+        cudaError_t e = cudaEventCreateWithFlags(&done, cudaEventDisableTiming);
+        if (e != cudaSuccess) {
+            pool_free(base);
+            return fail_cuda(e, "creating the valid lists' event");
+        }
         char *b = static_cast<char *>(base);
         L.base = base;
+        L.done = done;
         L.count = reinterpret_cast<int32_t *>(b + o_cnt);
-        L.cursor = L.count + n;
-        L.over = L.count + 2 * int64_t(n);
-        L.rank = reinterpret_cast<int32_t *>(b + o_rank);
         L.off = reinterpret_cast<int64_t *>(b + o_off);
         L.tile_sum = reinterpret_cast<int64_t *>(b + o_tile);
         L.total = reinterpret_cast<int64_t *>(b + o_tot);
     }
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
-    int64_t total = 0;
-    bool fill_trans;
-    if ((rc = prepare_trans(h, voc, sms, stream, &fill_trans)) != TRIE_OK) return rc;
-    cudaError_t e = tmk::launch_lists_count(h->dev, n, *voc, lmax, L, sms, fill_trans, stream, &total);
-    if (e != cudaSuccess) return fail_cuda(e, "valid-list count");
-    if (total > L.tok_cap) {  // grow the token buffer (by at least half)
-        const int64_t cap = std::max<int64_t>(total, L.tok_cap + L.tok_cap / 2);
+    // a node is the end of at most one path of each length up to lmax, each
+    // spelled by at most rt_mult ids, plus EOS. While that bound is modest the
+    // token buffer is sized by it and nothing is read back; otherwise the
+    // exact total is read back between the two walks (host-synchronous).
+    const int64_t bound = int64_t(n) * (int64_t(lmax) * voc->rt_mult + 1);
+    const bool by_bound = bound <= std::max<int64_t>(kListBoundEntries, L.tok_cap);
+    auto grow = [&](int64_t need) -> int {
+        if (need <= L.tok_cap) return TRIE_OK;
         pool_free(L.toks);  // earlier apply calls may still read it
         L.toks = nullptr;
         L.tok_cap = 0;
         void *toks = nullptr;
-        if ((rc = pool_alloc(dev, sizeof(int32_t) * size_t(std::max<int64_t>(cap, 1)), stream, &toks,
-                             "the valid-list tokens")) != TRIE_OK) {
-            L.n_valid = -1;
-            return rc;
-        }
+        int r = pool_alloc(dev, sizeof(int32_t) * size_t(std::max<int64_t>(need, 1)), stream, &toks,
+                           "the valid-list tokens");
+        if (r != TRIE_OK) return r;
         L.toks = static_cast<int32_t *>(toks);
-        L.tok_cap = cap;
+        L.tok_cap = need;
+        return TRIE_OK;
+    };
+    auto failed = [&](int r) {
+        L.n_valid = -1;
+        L.n_valid_on_device = false;
+        return r;
+    };
+    if (by_bound && (rc = grow(bound)) != TRIE_OK) return failed(rc);
+    cudaError_t e = tmk::launch_lists_count(h->dev, n, *voc, lmax, L, sms, stream);
+    if (e != cudaSuccess) return failed(fail_cuda(e, "valid-list count"));
+    if (!by_bound) {
+        int64_t total = 0;
+        if ((e = cudaMemcpyAsync(&total, L.total, sizeof(int64_t), cudaMemcpyDeviceToHost, stream)) != cudaSuccess ||
+            (e = cudaStreamSynchronize(stream)) != cudaSuccess)
+            return failed(fail_cuda(e, "reading the number of list entries back"));
+        if ((rc = grow(total + total / 2)) != TRIE_OK) return failed(rc);
     }
-    e = tmk::launch_lists_scatter(h->dev, n, *voc, lmax, L, sms, stream);
-    if (e != cudaSuccess) return fail_cuda(e, "valid-list scatter");
+    e = tmk::launch_lists_write(h->dev, n, *voc, lmax, L, sms, stream);
+    if (e == cudaSuccess) e = cudaEventRecord(L.done, stream);
+    if (e != cudaSuccess) return failed(fail_cuda(e, "valid-list write"));
     std::lock_guard<std::mutex> lk(h->mu);
-    L.n_valid = total;
+    L.n_valid_on_device = true;
     L.V = V;
-    h->trans_vocab = voc;
-    h->trans_complete = h->trans_complete || fill_trans;
     h->vocab = voc;
     return TRIE_OK;
 }
 
-int64_t trie_num_valid(trie_t h) { return h ? h->lists.n_valid : -1; }
+int64_t trie_num_valid(trie_t h) {
+    if (!h) return -1;
+    tmk::DevLists &L = h->lists;
+    std::lock_guard<std::mutex> lk(h->mu);
+    if (L.n_valid_on_device) {  // the total of the last build, once its kernels are done
+        int64_t total = -1;
+        DeviceGuard g(h->dev.device);
+        if (cudaEventSynchronize(L.done) != cudaSuccess ||
+            cudaMemcpy(&total, L.total, sizeof(int64_t), cudaMemcpyDeviceToHost) != cudaSuccess) {
+            cudaGetLastError();
+            fail(TRIE_ECUDA, "reading the number of list entries back failed");
+            return -1;
+        }
+        L.n_valid = total;
+        L.n_valid_on_device = false;
+    }
+    return L.n_valid;
+}
 
 int trie_copy_lists(trie_t h, int64_t *d_offsets, int32_t *d_tokens, cudaStream_t stream) {
     if (!h) return fail(TRIE_EINVAL, "handle is NULL");
     const tmk::DevLists &L = h->lists;
-    if (L.n_valid < 0) return fail(TRIE_ESTATE, "trie_copy_lists before trie_compile_lists on this handle");
+    if (!lists_built(h)) return fail(TRIE_ESTATE, "trie_copy_lists before trie_compile_lists on this handle");
+    if (trie_num_valid(h) < 0) return TRIE_ECUDA;
     if (d_offsets) {
         cudaError_t e = cudaMemcpyAsync(d_offsets, L.off, sizeof(int64_t) * (size_t(h->host.n) + 1),
                                         cudaMemcpyDeviceToDevice, stream);
@@ -791,7 +935,7 @@ int trie_apply_lists(trie_t h, void *d_logits, int dtype, const int32_t *d_state
     if (dtype != TRIE_DTYPE_F32 && dtype != TRIE_DTYPE_BF16) return fail(TRIE_EINVAL, "unknown dtype");
     if (B < 0) return fail(TRIE_EINVAL, "B must be >= 0");
     if (B > 0 && (!d_logits || !d_states)) return fail(TRIE_EINVAL, "d_logits / d_states is NULL");
-    if (h->lists.n_valid < 0) return fail(TRIE_ESTATE, "trie_apply_lists before trie_compile_lists on this handle");
+    if (!lists_built(h)) return fail(TRIE_ESTATE, "trie_apply_lists before trie_compile_lists on this handle");
     if (V != h->lists.V) return fail(TRIE_EINVAL, "V differs from the compiled lists' V");
     if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
         return fail(TRIE_EINVAL, "d_logits is not aligned to its element size");
@@ -936,7 +1080,7 @@ int trie_advance_apply_lists(trie_t h, const int32_t *d_states_in, const int32_t
         return fail(TRIE_EINVAL, "a device pointer is NULL");
     if (B > 0 && d_states_in == d_states_out)
         return fail(TRIE_EINVAL, "d_states_in and d_states_out must be different buffers");
-    if (h->lists.n_valid < 0)
+    if (!lists_built(h))
         return fail(TRIE_ESTATE, "trie_advance_apply_lists before trie_compile_lists on this handle");
     if (V != h->lists.V) return fail(TRIE_EINVAL, "V differs from the compiled lists' V");
     if (reinterpret_cast<uintptr_t>(d_logits) & uintptr_t(dtype == TRIE_DTYPE_F32 ? 3 : 1))
@@ -1091,9 +1235,56 @@ int trie_destroy(trie_t h) {
         pool_free(h->lists.toks);
         pool_free(h->lists.base);
         pool_free(h->dev.base);
+        if (h->lists.done) cudaEventDestroy(h->lists.done);
     }
     delete h;
     return TRIE_OK;
+}
+
+int trie_destroy_async(trie_t h, cudaStream_t stream) {
+    if (!h) return TRIE_OK;
+    int rc = TRIE_OK;
+    auto free_on = [&](void *p) {
+        if (!p) return;
+        cudaError_t e = cudaFreeAsync(p, stream);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            rc = fail_cuda(e, "stream-ordered free of the handle's device memory");
+        }
+    };
+    // the vocabularies are released here, on the calling thread (the last
+    // reference frees device memory, which a stream callback must not do)
+    std::shared_ptr<tmk::DevVocab> v1 = std::move(h->vocab), v2 = std::move(h->trans_vocab),
+                                   v3 = std::move(h->lazy.vocab);
+    int dev = h->dev.base || h->lists.base || h->lists.toks ? h->dev.device : h->lazy.device;
+    if (h->lazy.base) {
+        DeviceGuard g(h->lazy.device);
+        free_on(h->lazy.base);
+    }
+    if (h->dev.base || h->lists.base || h->lists.toks) {
+        DeviceGuard g(h->dev.device);
+        free_on(h->lists.toks);
+        free_on(h->lists.base);
+        free_on(h->dev.base);
+        // the event may still be pending: CUDA defers its destruction
+        if (h->lists.done) cudaEventDestroy(h->lists.done);
+    }
+    if (dev < 0) {
+        delete h;
+        return rc;
+    }
+    // the host arrays (which an upload kernel may still be reading) go once
+    // the work queued on the stream so far has run
+    DeviceGuard g(dev);
+    cudaError_t e = cudaLaunchHostFunc(stream, [](void *p) { delete static_cast<trie_t>(p); }, h);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        cudaStreamSynchronize(stream);
+        cudaGetLastError();
+        delete h;
+        if (rc == TRIE_OK) rc = fail_cuda(e, "queueing the release of the handle's host memory");
+    }
+    return rc;
 }
 
 }  // extern "C"

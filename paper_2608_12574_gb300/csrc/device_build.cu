@@ -28,23 +28,6 @@ constexpr int kBThreads = 256;
 constexpr int32_t kSetMaxStrings = 4096;  // forests whose sets all hold at most this many strings: one CTA per set
 constexpr int kScanTile = 1024;  // parents per tile of the level scan
 
-__device__ __forceinline__ void pdl_go() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void pdl_after() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
-template <typename... Params, typename... Args>
-cudaError_t launch(void (*kernel)(Params...), int64_t grid, int block, cudaStream_t st, Args... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(grid < 1 ? 1 : grid));
-    cfg.blockDim = dim3(unsigned(block));
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
-}
-
 // Staging: copies the strings' offsets, the set offsets and the bytes into
 // the scratch, checks the offsets (non-negative, non-decreasing) and finds
 // the longest string. The sources are either the caller's host memory, read
@@ -56,8 +39,8 @@ cudaError_t launch(void (*kernel)(Params...), int64_t grid, int block, cudaStrea
 __global__ void k_b_stage(const int64_t *src_off, int32_t K, const int32_t *src_soff, int32_t M,
                           const uint4 *src_vec, int64_t n_vec, int64_t *off, int32_t *soff, uint4 *vec,
                           int32_t *__restrict__ flags) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int64_t stride = int64_t(gridDim.x) * blockDim.x;
     const int64_t i0 = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
     int32_t longest = 0;
@@ -91,8 +74,8 @@ __global__ void k_b_init(const uint8_t *__restrict__ bytes, const int64_t *__res
                          int32_t *__restrict__ cur, int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
                          uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g,
                          int32_t *__restrict__ ls, uint32_t *__restrict__ bits0) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < M) {
         parent_g[i] = -1;
@@ -159,8 +142,8 @@ __global__ void __launch_bounds__(kBThreads) k_b_tile_sums(int32_t d, const int3
                                                            const uint32_t *__restrict__ bits,
                                                            int32_t *__restrict__ tile_sum) {
     __shared__ int32_t ws[kBThreads / 32];
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t width = ls[d + 1] - ls[d];
     const int32_t t0 = blockIdx.x * kScanTile;
     if (t0 >= width) {
@@ -186,8 +169,8 @@ __global__ void __launch_bounds__(kBThreads) k_b_first(int32_t d, int32_t n_tile
                                                        int32_t *__restrict__ first, uint32_t *__restrict__ other) {
     __shared__ int32_t ws[kBThreads / 32];
     __shared__ int32_t carry;
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t width = ls[d + 1] - ls[d];
     const int32_t prev = d > 0 ? ls[d] - ls[d - 1] : 0;
     const int32_t t0 = blockIdx.x * kScanTile;
@@ -236,8 +219,8 @@ __global__ void k_b_move(const uint8_t *__restrict__ bytes, const int64_t *__res
                          int32_t *__restrict__ cur, int32_t *__restrict__ parent_g, uint8_t *__restrict__ label_g,
                          uint8_t *__restrict__ term_g, int32_t *__restrict__ set_g, int32_t *__restrict__ depth_g,
                          uint32_t *__restrict__ bits_next) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= K) return;
     const int64_t len = off[i + 1] - off[i];
@@ -276,8 +259,8 @@ __global__ void k_b_count(const int32_t *__restrict__ ls, int32_t D, const int32
                           const int32_t *__restrict__ depth_g, const uint8_t *__restrict__ term_g,
                           int32_t *__restrict__ first_sd, int32_t *__restrict__ end_sd,
                           unsigned long long *__restrict__ n_chars) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t n = ls[D + 1];
     unsigned long long chars = 0;
     for (int32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
@@ -303,8 +286,8 @@ __global__ void __launch_bounds__(kBThreads) k_b_offsets(int32_t M, int32_t D, c
                                                          int32_t *__restrict__ off_sd, int32_t *__restrict__ roots) {
     __shared__ int32_t ws[kBThreads / 32];
     __shared__ int32_t carry;
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     if (threadIdx.x == 0) carry = 0;
     __syncthreads();
     for (int32_t s0 = 0; s0 < M; s0 += kBThreads) {
@@ -332,8 +315,8 @@ __global__ void __launch_bounds__(kBThreads) k_b_offsets(int32_t M, int32_t D, c
 __global__ void k_b_map(const int32_t *__restrict__ ls, int32_t D, const int32_t *__restrict__ set_g,
                         const int32_t *__restrict__ depth_g, const int32_t *__restrict__ first_sd,
                         const int32_t *__restrict__ off_sd, int32_t *__restrict__ map) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t n = ls[D + 1];
     for (int32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
         const int32_t k = set_g[g] * (D + 1) + depth_g[g];
@@ -346,8 +329,8 @@ __global__ void k_b_permute(const int32_t *__restrict__ ls, int32_t D, const int
                             const int32_t *__restrict__ parent_g, const uint8_t *__restrict__ label_g,
                             const uint8_t *__restrict__ term_g, int32_t *__restrict__ parent,
                             uint8_t *__restrict__ label, uint8_t *__restrict__ terminal) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int32_t n = ls[D + 1];
     for (int32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
         const int32_t f = map[g];
@@ -419,8 +402,8 @@ __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restric
     uint8_t *ends = reinterpret_cast<uint8_t *>(first + smax);
     __shared__ int32_t ws[kSetThreads / 32];
     __shared__ int32_t root_term;
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     const int tid = threadIdx.x;
     for (int32_t r = tid; r < smax * 8; r += kSetThreads) bits[r] = 0u;
     for (int32_t r = tid; r < smax; r += kSetThreads) ends[r] = 0;
@@ -524,8 +507,8 @@ __global__ void __launch_bounds__(kBThreads) k_b_set_scan(int32_t M, const int32
                                                           int32_t *__restrict__ roots, int32_t *__restrict__ total) {
     __shared__ int32_t ws[kBThreads / 32];
     __shared__ int32_t carry;
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     if (threadIdx.x == 0) carry = 0;
     __syncthreads();
     for (int32_t s0 = 0; s0 < M; s0 += kBThreads) {
@@ -546,8 +529,8 @@ __global__ void k_b_set_emit(const int64_t *__restrict__ off, const int32_t *__r
                              const int32_t *__restrict__ parent_ub, const uint8_t *__restrict__ label_ub,
                              const uint8_t *__restrict__ term_ub, int32_t *__restrict__ parent,
                              uint8_t *__restrict__ label, uint8_t *__restrict__ terminal) {
-    pdl_go();
-    pdl_after();
+    pdl_launch_dependents();
+    pdl_wait();
     for (int32_t s = blockIdx.x; s < M; s += gridDim.x) {
         const int64_t ub = off[set_off[s]] - off[0] + s;
         const int32_t base = roots[s], n = count[s];
@@ -655,7 +638,7 @@ cudaError_t DeviceBuild::stage(const uint8_t *h_bytes, const int64_t *h_off, con
     const int64_t items = std::max<int64_t>(std::max<int64_t>(K, M) + 1, n_vec);
     const int64_t grid = std::min<int64_t>((items + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
     if (direct) {
-        e = launch(k_b_stage, grid, kBThreads, st, h_off, K, h_set_off, M,
+        e = launch_pdl(k_b_stage, grid, kBThreads, st, h_off, K, h_set_off, M,
                    reinterpret_cast<const uint4 *>(h_bytes - mis), n_vec, s_->off, s_->set_off, s_->image, s_->flags);
     } else {
         if ((n_bytes > 0 && (e = cudaMemcpyAsync(s_->bytes, h_bytes, size_t(n_bytes), cudaMemcpyHostToDevice, st)) !=
@@ -664,7 +647,7 @@ cudaError_t DeviceBuild::stage(const uint8_t *h_bytes, const int64_t *h_off, con
             (e = cudaMemcpyAsync(s_->set_off, h_set_off, 4 * (size_t(M) + 1), cudaMemcpyHostToDevice, st)) !=
                 cudaSuccess)
             return e;
-        e = launch(k_b_stage, grid, kBThreads, st, static_cast<const int64_t *>(s_->off), K,
+        e = launch_pdl(k_b_stage, grid, kBThreads, st, static_cast<const int64_t *>(s_->off), K,
                    static_cast<const int32_t *>(s_->set_off), M, static_cast<const uint4 *>(nullptr), int64_t(0),
                    s_->off, s_->set_off, s_->image, s_->flags);
     }
@@ -699,7 +682,7 @@ cudaError_t DeviceBuild::levels(int32_t D, int num_sms, int32_t *n_nodes, std::v
     s_->off_sd = reinterpret_cast<int32_t *>(b + o_osd);
     if ((e = cudaMemsetAsync(s_->end_sd, 0, 4 * size_t(sd), st)) != cudaSuccess) return e;
     const int64_t sgrid = (W + kBThreads - 1) / kBThreads;
-    if ((e = launch(k_b_init, sgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
+    if ((e = launch_pdl(k_b_init, sgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
                     static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M, K,
                     s_->str_set, s_->cur, s_->parent_g, s_->label_g, s_->term_g, s_->set_g, s_->depth_g, s_->ls,
                     s_->bits[0])) != cudaSuccess)
@@ -708,11 +691,11 @@ cudaError_t DeviceBuild::levels(int32_t D, int num_sms, int32_t *n_nodes, std::v
     const int32_t n_tiles = int32_t((W + kScanTile - 1) / kScanTile);
     for (int32_t d = 0; d < D; d++) {  // level d: bits[d & 1] holds its child-label sets
         uint32_t *bits = s_->bits[d & 1], *next = s_->bits[(d + 1) & 1];
-        if ((e = launch(k_b_tile_sums, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
+        if ((e = launch_pdl(k_b_tile_sums, n_tiles, kBThreads, st, d, static_cast<const int32_t *>(s_->ls),
                         static_cast<const uint32_t *>(bits), s_->tile_sum)) != cudaSuccess ||
-            (e = launch(k_b_first, n_tiles, kBThreads, st, d, n_tiles, s_->ls, static_cast<const uint32_t *>(bits),
+            (e = launch_pdl(k_b_first, n_tiles, kBThreads, st, d, n_tiles, s_->ls, static_cast<const uint32_t *>(bits),
                         static_cast<const int32_t *>(s_->tile_sum), s_->first, next)) != cudaSuccess ||
-            (e = launch(k_b_move, kgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
+            (e = launch_pdl(k_b_move, kgrid, kBThreads, st, static_cast<const uint8_t *>(s_->bytes),
                         static_cast<const int64_t *>(s_->off), K, d, static_cast<const int32_t *>(s_->ls),
                         static_cast<const uint32_t *>(bits), static_cast<const int32_t *>(s_->first),
                         static_cast<const int32_t *>(s_->str_set), s_->cur, s_->parent_g, s_->label_g, s_->term_g,
@@ -720,12 +703,12 @@ cudaError_t DeviceBuild::levels(int32_t D, int num_sms, int32_t *n_nodes, std::v
             return e;
     }
     const int64_t ngrid = std::min<int64_t>((U + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
-    if ((e = launch(k_b_count, ngrid, kBThreads, st, static_cast<const int32_t *>(s_->ls), D,
+    if ((e = launch_pdl(k_b_count, ngrid, kBThreads, st, static_cast<const int32_t *>(s_->ls), D,
                     static_cast<const int32_t *>(s_->set_g), static_cast<const int32_t *>(s_->depth_g),
                     static_cast<const uint8_t *>(s_->term_g), s_->first_sd, s_->end_sd, s_->n_chars)) != cudaSuccess ||
-        (e = launch(k_b_offsets, 1, kBThreads, st, M, D, static_cast<const int32_t *>(s_->first_sd),
+        (e = launch_pdl(k_b_offsets, 1, kBThreads, st, M, D, static_cast<const int32_t *>(s_->first_sd),
                     static_cast<const int32_t *>(s_->end_sd), s_->off_sd, s_->roots)) != cudaSuccess ||
-        (e = launch(k_b_map, ngrid, kBThreads, st, static_cast<const int32_t *>(s_->ls), D,
+        (e = launch_pdl(k_b_map, ngrid, kBThreads, st, static_cast<const int32_t *>(s_->ls), D,
                     static_cast<const int32_t *>(s_->set_g), static_cast<const int32_t *>(s_->depth_g),
                     static_cast<const int32_t *>(s_->first_sd), static_cast<const int32_t *>(s_->off_sd), s_->map)) !=
             cudaSuccess)
@@ -776,7 +759,7 @@ cudaError_t DeviceBuild::sets(int num_sms, int32_t *n_nodes, std::vector<int32_t
                                 static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M,
                                 smax_, s_->parent_g, s_->label_g, s_->term_g, s_->count, s_->n_chars)) !=
             cudaSuccess ||
-        (e = launch(k_b_set_scan, 1, kBThreads, st, M, static_cast<const int32_t *>(s_->count), s_->roots,
+        (e = launch_pdl(k_b_set_scan, 1, kBThreads, st, M, static_cast<const int32_t *>(s_->count), s_->roots,
                     s_->total)) != cudaSuccess)
         return e;
     int32_t n = 0;
@@ -795,13 +778,13 @@ cudaError_t DeviceBuild::sets(int num_sms, int32_t *n_nodes, std::vector<int32_t
 
 cudaError_t DeviceBuild::emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms) {
     if (small_)
-        return launch(k_b_set_emit, std::min<int64_t>(M_, int64_t(num_sms) * 8), kBThreads, stream_,
+        return launch_pdl(k_b_set_emit, std::min<int64_t>(M_, int64_t(num_sms) * 8), kBThreads, stream_,
                       static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M_,
                       static_cast<const int32_t *>(s_->count), static_cast<const int32_t *>(s_->roots),
                       static_cast<const int32_t *>(s_->parent_g), static_cast<const uint8_t *>(s_->label_g),
                       static_cast<const uint8_t *>(s_->term_g), parent, label, terminal);
     const int64_t ngrid = std::min<int64_t>((int64_t(n_) + kBThreads - 1) / kBThreads, int64_t(num_sms) * 16);
-    return launch(k_b_permute, ngrid, kBThreads, stream_, static_cast<const int32_t *>(s_->ls), D_,
+    return launch_pdl(k_b_permute, ngrid, kBThreads, stream_, static_cast<const int32_t *>(s_->ls), D_,
                   static_cast<const int32_t *>(s_->map), static_cast<const int32_t *>(s_->parent_g),
                   static_cast<const uint8_t *>(s_->label_g), static_cast<const uint8_t *>(s_->term_g), parent, label,
                   terminal);

@@ -37,8 +37,6 @@ struct FmtArgs {
     int32_t V;
 };
 
-__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void pdl_wait_prior() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // Every byte of token v (len bytes at blob + off) lies in the class of its
 // position, starting at position p (the caller has checked p + len <= L).
@@ -99,8 +97,8 @@ __global__ void __launch_bounds__(kFmtThreads) k_fmt_compile(FmtArgs a, uint32_t
         }
     }
     __syncthreads();
-    pdl_trigger();
-    pdl_wait_prior();  // an earlier kernel may still read the mask
+    pdl_launch_dependents();
+    pdl_wait();  // an earlier kernel may still read the mask
     const int lane = threadIdx.x & 31;
     const int64_t warps = int64_t(gridDim.x) * (blockDim.x / 32);
     for (int64_t w = int64_t(blockIdx.x) * (blockDim.x / 32) + (threadIdx.x >> 5); w < W; w += warps) {
@@ -131,8 +129,8 @@ __global__ void __launch_bounds__(kFmtThreads) k_fmt_advance(FmtArgs a, const in
                                                              int32_t *states_out,
                                                              const int32_t *__restrict__ tokens, int32_t B,
                                                              int32_t *__restrict__ err) {
-    pdl_trigger();
-    pdl_wait_prior();  // states and tokens come from earlier kernels
+    pdl_launch_dependents();
+    pdl_wait();  // states and tokens come from earlier kernels
     const int32_t b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b >= B) return;
     const int32_t s = states_in[b], v = tokens[b];
@@ -145,20 +143,6 @@ __global__ void __launch_bounds__(kFmtThreads) k_fmt_advance(FmtArgs a, const in
     else nxt = fmt_allows(a, a.classes, s, v) ? s + int32_t(a.tok_len[v]) : kFmtDead;
     if (nxt == kFmtDead && s != kFmtDead && err) atomicAdd(err, 1);
     states_out[b] = nxt;
-}
-
-template <typename... Params, typename... Args>
-cudaError_t launch(void (*kernel)(Params...), int grid, int block, cudaStream_t st, Args... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(grid));
-    cfg.blockDim = dim3(unsigned(block));
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
 }
 
 FmtArgs fmt_args(const uint32_t *classes, int32_t L, const DevVocab &v) {
@@ -180,14 +164,14 @@ cudaError_t launch_fmt_compile(const uint32_t *classes, int32_t L, const DevVoca
     int64_t grid = (W + kFmtThreads / 32 - 1) / (kFmtThreads / 32);
     if (grid > int64_t(num_sms) * 8) grid = int64_t(num_sms) * 8;
     if (grid < 1) grid = 1;
-    return launch(k_fmt_compile, int(grid), kFmtThreads, st, fmt_args(classes, L, v), mask, W);
+    return launch_pdl(k_fmt_compile, int(grid), kFmtThreads, st, fmt_args(classes, L, v), mask, W);
 }
 
 cudaError_t launch_fmt_advance(const uint32_t *classes, int32_t L, const DevVocab &v, const int32_t *states_in,
                                int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err,
                                cudaStream_t st) {
     const int grid = (B + kFmtThreads - 1) / kFmtThreads;
-    return launch(k_fmt_advance, grid, kFmtThreads, st, fmt_args(classes, L, v), states_in, states_out, tokens, B,
+    return launch_pdl(k_fmt_advance, grid, kFmtThreads, st, fmt_args(classes, L, v), states_in, states_out, tokens, B,
                   err);
 }
 

@@ -294,12 +294,192 @@ void pre_order_from_parents(HostTrie *t) {
     }
 }
 
+void pack_token_bytes(const uint8_t *bytes, const int64_t *offsets, int32_t V, uint32_t *tok_off,
+                      uint16_t *tok_len, uint8_t *blob) {
+    uint32_t pos = 0;
+    for (int32_t v = 0; v < V; v++) {
+        const int64_t L = (v == V - 1) ? 0 : offsets[v + 1] - offsets[v];  // EOS bytes are ignored
+        tok_off[v] = pos;
+        tok_len[v] = uint16_t(L);
+        if (L > 0) memcpy(blob + pos, bytes + offsets[v], size_t(L));
+        pos += uint32_t((L + 15) / 16 * 16);
+    }
+}
+
+bool fill_token_table(const uint8_t *bytes, const int64_t *offsets, const uint16_t *tok_len, int32_t V,
+                      uint64_t S, uint64_t *key, int32_t *val) {
+    // load factor <= 1/4; slots are probed in aligned pairs (one 16-byte load
+    // holds two keys), pair after pair, the even slot of a pair filled first
+    std::fill(key, key + S, 0ull);
+    std::fill(val, val + S, -1);
+    const uint64_t pairs_mask = S / 2 - 1;
+    bool dup = false;
+    for (int32_t v = 0; v < V; v++) {
+        const uint32_t L = tok_len[v];
+        if (!L) continue;
+        const uint8_t *p = bytes + offsets[v];
+        uint64_t h = 0;
+        for (uint32_t j = 0; j < L; j++) h = h * kHashBase + uint64_t(p[j]) + 1;
+        const uint64_t k = hash_finish(h, L);
+        uint64_t pair = (k >> 1) & pairs_mask;
+        for (;;) {
+            const size_t s0 = size_t(2 * pair);
+            // an equal key: a repeated token string, or two strings whose hashes collide
+            if (key[s0] == k || key[s0 + 1] == k) dup = true;
+            if (!key[s0]) { key[s0] = k; val[s0] = v; break; }
+            if (!key[s0 + 1]) { key[s0 + 1] = k; val[s0 + 1] = v; break; }
+            pair = (pair + 1) & pairs_mask;
+        }
+    }
+    return dup;
+}
+
+uint64_t token_table_slots(int64_t n_tokens_with_bytes) {
+    uint64_t S = 16;
+    while (S < uint64_t(4 * n_tokens_with_bytes)) S <<= 1;
+    return S;
+}
+
+namespace {
+
+// One subtree of the reversed-token trie: the tokens whose last byte is b,
+// sorted by their reversed bytes, laid out in pre-order (local node 0 is the
+// root's child for b).
+struct RevPart {
+    hvec<int32_t> parent;  // local ids; -1 for local node 0
+    hvec<uint8_t> label;
+    hvec<int32_t> token;
+    std::vector<std::pair<int32_t, int32_t>> dup;  // (earlier id, later id) with equal bytes
+};
+
+void build_rev_part(const uint8_t *bytes, const int64_t *offsets, std::vector<int32_t> &ids, RevPart *out) {
+    // reversed byte i of token v
+    auto rb = [&](int32_t v, int64_t i) { return bytes[offsets[v + 1] - 1 - i]; };
+    auto len = [&](int32_t v) { return offsets[v + 1] - offsets[v]; };
+    std::vector<std::pair<uint64_t, int32_t>> keyed(ids.size());
+    for (size_t i = 0; i < ids.size(); i++) {
+        const int32_t v = ids[i];
+        uint64_t k = 0;
+        for (int j = 0; j < 8; j++) k = (k << 8) | (j < len(v) ? rb(v, j) : 0);
+        keyed[i] = {k, v};
+    }
+    auto less = [&](const std::pair<uint64_t, int32_t> &a, const std::pair<uint64_t, int32_t> &b) {
+        if (a.first != b.first) return a.first < b.first;
+        const int64_t la = len(a.second), lb = len(b.second), m = std::min(la, lb);
+        for (int64_t i = 8; i < m; i++) {
+            const uint8_t x = rb(a.second, i), y = rb(b.second, i);
+            if (x != y) return x < y;
+        }
+        if (la != lb) return la < lb;
+        return a.second < b.second;  // equal bytes: ascending id
+    };
+    std::sort(keyed.begin(), keyed.end(), less);
+    int64_t total = 0;
+    for (const auto &kv : keyed) total += len(kv.second);
+    out->parent.resize(size_t(total));
+    out->label.resize(size_t(total));
+    out->token.resize(size_t(total));
+    int32_t n = 0;
+    std::vector<int32_t> path;  // path[d] = local node at depth d + 1
+    int32_t prev = -1;
+    for (const auto &kv : keyed) {
+        const int32_t v = kv.second;
+        const int64_t L = len(v);
+        int64_t lcp = 0;
+        if (prev >= 0) {
+            const int64_t m = std::min(len(prev), L);
+            while (lcp < m && rb(prev, lcp) == rb(v, lcp)) lcp++;
+            if (lcp == L && len(prev) == L) {  // the same bytes as the previous token
+                out->dup.emplace_back(prev, v);
+                prev = v;
+                continue;
+            }
+        }
+        if (int64_t(path.size()) < L) path.resize(size_t(L));
+        for (int64_t d = lcp; d < L; d++) {
+            const int32_t id = n++;
+            out->parent[size_t(id)] = d == 0 ? -1 : path[size_t(d - 1)];
+            out->label[size_t(id)] = rb(v, d);
+            out->token[size_t(id)] = -1;
+            path[size_t(d)] = id;
+        }
+        out->token[size_t(path[size_t(L - 1)])] = v;
+        prev = v;
+    }
+    out->parent.resize(size_t(n));
+    out->label.resize(size_t(n));
+    out->token.resize(size_t(n));
+}
+
+}  // namespace
+
+std::string build_reversed_token_trie(const uint8_t *bytes, const int64_t *offsets, int32_t V,
+                                      RevTokenTrie *out) {
+    // tokens with bytes (EOS = V-1 excluded), bucketed by their last byte
+    std::vector<std::vector<int32_t>> bucket(256);
+    for (int32_t v = 0; v + 1 < V; v++)
+        if (offsets[v + 1] > offsets[v]) bucket[bytes[offsets[v + 1] - 1]].push_back(v);
+    std::vector<RevPart> part(256);
+    const unsigned hw = std::max(1u, std::thread::hardware_concurrency());
+    const unsigned nth = std::min<unsigned>(hw, 16u);
+    std::atomic<int> next(0);
+    auto loop = [&]() {
+        for (int b; (b = next.fetch_add(1)) < 256;)
+            if (!bucket[size_t(b)].empty()) build_rev_part(bytes, offsets, bucket[size_t(b)], &part[size_t(b)]);
+    };
+    std::vector<std::thread> th;
+    for (unsigned t = 1; t < nth; t++) th.emplace_back(loop);
+    loop();
+    for (auto &t : th) t.join();
+    int64_t n = 1;
+    std::vector<int64_t> base(256);
+    for (int b = 0; b < 256; b++) {
+        base[size_t(b)] = n;
+        n += int64_t(part[size_t(b)].parent.size());
+    }
+    if (n > kRevTrieMaxNodes) return "reversed-token trie would exceed 2^24 - 2 nodes";
+    out->n = int32_t(n);
+    out->parent.resize(size_t(n));
+    out->label.resize(size_t(n));
+    out->token.resize(size_t(n));
+    out->parent[0] = -1;
+    out->label[0] = 0;
+    out->token[0] = -1;
+    bool dups = false;
+    for (int b = 0; b < 256; b++) {
+        const RevPart &p = part[size_t(b)];
+        const int64_t g = base[size_t(b)];
+        for (size_t i = 0; i < p.parent.size(); i++) {
+            out->parent[size_t(g) + i] = p.parent[i] < 0 ? 0 : int32_t(g + p.parent[i]);
+            out->label[size_t(g) + i] = p.label[i];
+            out->token[size_t(g) + i] = p.token[i];
+        }
+        dups = dups || !p.dup.empty();
+    }
+    out->next.clear();
+    out->max_mult = 1;
+    if (dups) {
+        out->next.assign(size_t(V), -1);
+        std::vector<int32_t> is_later(size_t(V), 0);
+        for (const RevPart &p : part)
+            for (const auto &d : p.dup) {
+                out->next[size_t(d.first)] = d.second;
+                is_later[size_t(d.second)] = 1;
+            }
+        for (int32_t v = 0; v < V; v++) {  // chain heads: the longest chain
+            if (is_later[size_t(v)] || out->next[size_t(v)] < 0) continue;
+            int32_t len = 1;
+            for (int32_t u = out->next[size_t(v)]; u >= 0; u = out->next[size_t(u)]) len++;
+            out->max_mult = std::max(out->max_mult, len);
+        }
+    }
+    return "";
+}
+
 std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, HostVocab *out) {
     if (V < 2) return "V must be >= 2 (token V-1 is EOS)";
     if (offsets[0] < 0) return "vocab offsets must be non-negative";
     out->V = V;
-    out->tok_off.assign(size_t(V), 0);
-    out->tok_len.assign(size_t(V), 0);
     uint64_t pos = 0;
     int64_t n_ins = 0;
     int32_t max_len = 0;
@@ -308,8 +488,6 @@ std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, 
         if (e < a) return "vocab offsets must be non-decreasing";
         int64_t L = (v == V - 1) ? 0 : e - a;  // EOS bytes are ignored
         if (L > 65535) return "token " + std::to_string(v) + " is longer than 65535 bytes";
-        out->tok_off[size_t(v)] = uint32_t(pos);
-        out->tok_len[size_t(v)] = uint16_t(L);
         pos += uint64_t((L + 15) / 16 * 16);
         if (pos > 0xFFFFFFF0ull) return "packed vocabulary exceeds 4 GiB";
         if (L > 0) {
@@ -318,36 +496,17 @@ std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, 
         }
     }
     out->max_len = max_len;
+    out->tok_off.assign(size_t(V), 0);
+    out->tok_len.assign(size_t(V), 0);
     out->blob.assign(size_t(pos) + 16, 0);
-    for (int32_t v = 0; v < V; v++)
-        if (out->tok_len[size_t(v)])
-            memcpy(&out->blob[out->tok_off[size_t(v)]], bytes + offsets[v], out->tok_len[size_t(v)]);
-    // load factor <= 1/4; slots are probed in aligned pairs (one 16-byte load
-    // holds two keys), pair after pair, the even slot of a pair filled first
-    uint64_t S = 16;
-    while (S < uint64_t(4 * n_ins)) S <<= 1;
+    pack_token_bytes(bytes, offsets, V, out->tok_off.data(), out->tok_len.data(), out->blob.data());
+    const uint64_t S = token_table_slots(n_ins);
     if (S > (uint64_t(1) << 31)) return "vocabulary too large for the token hash table";
-    out->ht_key.assign(size_t(S), 0ull);
-    out->ht_val.assign(size_t(S), -1);
+    out->ht_key.resize(size_t(S));
+    out->ht_val.resize(size_t(S));
     out->ht_mask = uint32_t(S - 1);
-    const uint64_t pairs_mask = S / 2 - 1;
-    for (int32_t v = 0; v < V; v++) {
-        uint32_t L = out->tok_len[size_t(v)];
-        if (!L) continue;
-        const uint8_t *p = bytes + offsets[v];
-        uint64_t h = 0;
-        for (uint32_t j = 0; j < L; j++) h = h * kHashBase + uint64_t(p[j]) + 1;
-        const uint64_t key = hash_finish(h, L);
-        uint64_t pair = (key >> 1) & pairs_mask;
-        for (;;) {
-            size_t s0 = size_t(2 * pair);
-            // an equal key: a repeated token string, or two strings whose hashes collide
-            if (out->ht_key[s0] == key || out->ht_key[s0 + 1] == key) out->dup_keys = 1;
-            if (!out->ht_key[s0]) { out->ht_key[s0] = key; out->ht_val[s0] = v; break; }
-            if (!out->ht_key[s0 + 1]) { out->ht_key[s0 + 1] = key; out->ht_val[s0 + 1] = v; break; }
-            pair = (pair + 1) & pairs_mask;
-        }
-    }
+    out->dup_keys = fill_token_table(bytes, offsets, out->tok_len.data(), V, S, out->ht_key.data(),
+                                     out->ht_val.data()) ? 1 : 0;
     return "";
 }
 

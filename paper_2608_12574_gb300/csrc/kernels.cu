@@ -27,6 +27,8 @@
 // wait, so they overlap the fill.
 #include <stdint.h>
 
+#include <algorithm>
+
 #include <cuda_runtime.h>
 
 #include "tm_internal.h"
@@ -38,32 +40,6 @@ namespace {
 constexpr int32_t kDead = -1;
 constexpr int32_t kFinished = -2;
 constexpr int kMaxClimb = 16;  // suffix lengths kept in registers by the patch kernel
-
-__device__ __forceinline__ void pdl_launch_dependents() {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
-template <typename... Params, typename... Args>
-cudaError_t launch_pdl_smem(void (*kernel)(Params...), int grid, int block, size_t smem, cudaStream_t st,
-                            Args... args) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(grid));
-    cfg.blockDim = dim3(unsigned(block));
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
-}
-
-template <typename... Params, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(Params...), int grid, int block, cudaStream_t st, Args... args) {
-    return launch_pdl_smem(kernel, grid, block, 0, st, args...);
-}
 
 // ------------------------------------------------------------------ fill
 
@@ -149,8 +125,6 @@ struct PatchArgs {
     ulonglong2 *trans;         // transition table (row, token) -> end node, or null
     uint32_t trans_mask;       // slots - 1
     int32_t trans_fill;        // the probe inserts every transition it finds
-    int32_t *list_count;       // list compile: the probe counts the recorded hits per row, or null
-    int32_t *hit_rank;         // [n_nodes * kHitSlots]: each recorded hit's position in its row
 };
 
 // Transition table: open addressing over 16-byte slots {key, end node};
@@ -610,10 +584,7 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
         int32_t c = 0;
         int2 *slot = a.hits + int64_t(m) * kHitSlots;
         node_hits_window(a, m, [&](int32_t row, int32_t t) {
-            if (c < kHitSlots) {
-                slot[c] = make_int2(row, t);
-                if (a.list_count) a.hit_rank[int64_t(m) * kHitSlots + c] = atomicAdd(a.list_count + row, 1);
-            }
+            if (c < kHitSlots) slot[c] = make_int2(row, t);
             c++;
             if (a.trans_fill && t != a.eos) trans_insert(a.trans, a.trans_mask, row, t, m);
         });
@@ -677,10 +648,7 @@ __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs 
         int2 *slot = a.hits + int64_t(m) * kHitSlots;
         int32_t s = half ? c0 : 0;
         auto rec = [&](int32_t row, int32_t tok) {
-            if (s < kHitSlots) {
-                slot[s] = make_int2(row, tok);
-                if (a.list_count) a.hit_rank[int64_t(m) * kHitSlots + s] = atomicAdd(a.list_count + row, 1);
-            }
+            if (s < kHitSlots) slot[s] = make_int2(row, tok);
             s++;
             if (a.trans_fill && tok != a.eos) trans_insert(a.trans, a.trans_mask, row, tok, m);
         };
@@ -794,6 +762,60 @@ __global__ void __launch_bounds__(kAdvanceThreads) k_advance(AdvanceArgs a, cons
     states_out[b] = nxt;
 }
 
+// ------------------------------------------------------------ pairwise form
+// The compile as the pair-by-pair evaluation of the definition (Sec. 4.1,
+// App. G.5): bit[n][v] = 1 iff v is not EOS, has bytes, and every byte of v
+// finds a child walking down from n; bit[n][EOS] = terminal(n). One warp per
+// (node, 32 mask words): lane l tests token 32 i + l of word i by walking its
+// bytes (child-label set + first child, as the advance does), a warp ballot
+// assembles the word, and lane i keeps word i for one coalesced 128-byte
+// store. Kept as the measured alternative to the suffix search: its cost is
+// one walk per (node, token) pair, N * V walks, instead of a few probes per
+// node.
+constexpr int kPairwiseThreads = 256;
+
+__device__ __forceinline__ bool token_walks(const AdvanceArgs &a, int32_t n, int32_t t) {
+    const int32_t L = __ldg(a.tok_len + t);
+    if (L <= 0) return false;
+    const uint8_t *p = a.blob + __ldg(a.tok_off + t);
+    int32_t x = n;
+    for (int32_t j = 0; j < L; j++) {
+        const uint32_t c = __ldg(p + j);
+        const uint32_t wv = __ldg(a.child_bits + int64_t(x) * 8 + (c >> 5));
+        const uint32_t bit = c & 31u;
+        if (!((wv >> bit) & 1u)) return false;
+        uint32_t below = __popc(wv & ((1u << bit) - 1u));
+        for (uint32_t i = 0; i < (c >> 5); i++) below += __popc(__ldg(a.child_bits + int64_t(x) * 8 + i));
+        x = __ldg(a.first_child + x) + int32_t(below);
+    }
+    return true;
+}
+
+__global__ void __launch_bounds__(kPairwiseThreads) k_mask_pairwise(AdvanceArgs a, uint32_t *__restrict__ mask,
+                                                                    int64_t W, int64_t chunks) {
+    pdl_launch_dependents();
+    pdl_wait();  // an earlier kernel may still read the old mask
+    const int lane = threadIdx.x & 31;
+    const int64_t nwarps = (int64_t(gridDim.x) * blockDim.x) >> 5;
+    const int64_t tasks = int64_t(a.n_nodes) * chunks;
+    const int32_t eos = a.V - 1;
+    for (int64_t task = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; task < tasks; task += nwarps) {
+        const int32_t n = int32_t(task / chunks);
+        const int64_t w0 = (task - int64_t(n) * chunks) * 32;
+        const bool term = __ldg(a.terminal + n) != 0;
+        uint32_t out = 0u;
+        for (int i = 0; i < 32 && w0 + i < W; i++) {  // uniform across the warp
+            const int64_t t = (w0 + i) * 32 + lane;
+            bool ok = false;
+            if (t < eos) ok = token_walks(a, n, int32_t(t));
+            else if (t == eos) ok = term;
+            const uint32_t word = __ballot_sync(0xffffffffu, ok);
+            if (lane == i) out = word;
+        }
+        if (w0 + lane < W) mask[int64_t(n) * W + w0 + lane] = out;
+    }
+}
+
 // ------------------------------------------------------------------ apply
 
 constexpr int kApplyThreads = 256;
@@ -902,8 +924,10 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
 // Advance, then apply, in one launch (one decode step once the sampler has
 // picked tokens[b] for the previous logits): states_out[b] = delta*(states_in[b],
 // tokens[b]), and logits[b] (the next step's) are masked by the row of
-// states_out[b]. Lane 0 of every warp of row b computes the new state; the
-// warp of segment 0 stores it and counts a move into DEAD.
+// states_out[b]. CTA (row b, part p) covers segments 8p .. 8p + 7 of row b,
+// one warp each; its thread 0 computes the row's new state once for the CTA
+// (shared memory), and the CTA of part 0 stores it and counts a move into
+// DEAD.
 template <int kElt>
 __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs aa, uint4 *__restrict__ logits,
                                                                      const uint32_t *__restrict__ mask,
@@ -911,27 +935,30 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
                                                                      const int32_t *__restrict__ tokens,
                                                                      int32_t *__restrict__ states_out,
                                                                      int32_t *__restrict__ err, int32_t B,
-                                                                     int64_t W, int32_t segs) {
+                                                                     int64_t W, int32_t segs, int32_t parts) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     __shared__ __align__(128) uint4 tile[kSegChunks];
-    init_ninf_tile<kElt>(tile);
+    __shared__ int32_t next_state;
     pdl_launch_dependents();
-    pdl_wait();  // logits, states and tokens come from earlier kernels
+    const int32_t b = int32_t(blockIdx.x) / parts, part = int32_t(blockIdx.x) - b * parts;
+    for (int i = threadIdx.x; i < kSegChunks; i += blockDim.x) tile[i] = ninf16<kElt>();
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // tile visible to the bulk copies
+    if (threadIdx.x == 0) {
+        pdl_wait();  // states and tokens come from earlier kernels
+        const int32_t s = __ldg(states_in + b);
+        const int32_t nxt = advance_one(aa, s, __ldg(tokens + b));
+        next_state = nxt;
+        if (part == 0) {
+            states_out[b] = nxt;
+            if (nxt == kDead && s != kDead && err) atomicAdd(err, 1);
+        }
+    }
+    __syncthreads();
+    pdl_wait();  // logits come from earlier kernels
     const int lane = threadIdx.x & 31;
-    const int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
-    if (item >= B * segs) return;  // uniform per warp
-    const int32_t b = item / segs, seg = item - b * segs;
-    int32_t s = 0, nxt = 0;
-    if (lane == 0) {
-        s = __ldg(states_in + b);
-        nxt = advance_one(aa, s, __ldg(tokens + b));
-    }
-    nxt = __shfl_sync(0xffffffffu, nxt, 0);
-    if (seg == 0 && lane == 0) {
-        states_out[b] = nxt;
-        if (nxt == kDead && s != kDead && err) atomicAdd(err, 1);
-    }
-    const uint32_t word = row_word(mask, nxt, aa.n_nodes, W, int64_t(seg) * 32 + lane, aa.V - 1);
+    const int32_t seg = part * (kApplyThreads / 32) + int32_t(threadIdx.x >> 5);
+    if (seg >= segs) return;  // uniform per warp
+    const uint32_t word = row_word(mask, next_state, aa.n_nodes, W, int64_t(seg) * 32 + lane, aa.V - 1);
     const int64_t row_chunks = int64_t(aa.V) / (16 / kElt);
     write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
                         tile);
@@ -941,23 +968,6 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
 // Sparse form of the masks (the valid[n] lists the paper stores, Sec. 4.2 and
 // App. H.5): for every node, the ids of its allowed tokens (EOS included at
 // terminal nodes) in no particular order, as CSR offsets[N+1] + tokens.
-
-// The probe counted the hits it recorded (at most kHitSlots per node) and
-// gave each its position in its row; the hits beyond those, of nodes that
-// overflowed, are found again here (the search emits them in the same order)
-// and counted apart.
-__global__ void __launch_bounds__(kPatchThreads, 4) k_list_count_over(PatchArgs a, int32_t *__restrict__ over) {
-    pdl_launch_dependents();
-    pdl_wait();  // hits from the probe
-    const int32_t stride = gridDim.x * blockDim.x;
-    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        if (a.hit_count[m] != kHitOverflow) continue;
-        int32_t i = 0;
-        node_hits_window(a, m, [&](int32_t row, int32_t) {
-            if (i++ >= kHitSlots) atomicAdd(over + row, 1);
-        });
-    }
-}
 
 // Exclusive scan of the row counts into int64 offsets, in three passes over
 // tiles of kScanTile counts: tile sums, a scan of the tile sums by one CTA,
@@ -992,18 +1002,21 @@ __device__ __forceinline__ int64_t block_exclusive_scan(int64_t v, int64_t *smem
     return warp_base + x - v;
 }
 
-// The count of row i is cnt[i] (+ cnt2[i] when cnt2 is not null).
-__global__ void __launch_bounds__(kScanThreads) k_scan_tiles(const int32_t *__restrict__ cnt,
-                                                             const int32_t *__restrict__ cnt2, int32_t n,
+__global__ void __launch_bounds__(kScanThreads) k_scan_tiles(const int32_t *__restrict__ cnt, int32_t n,
                                                              int64_t *__restrict__ tile_sum) {
     pdl_launch_dependents();
     pdl_wait();
     __shared__ int64_t sw[32];
     const int64_t base = int64_t(blockIdx.x) * kScanTile + int64_t(threadIdx.x) * kScanPer;
     int64_t v = 0;
+    if (base + kScanPer <= n) {
+        const int4 q = *reinterpret_cast<const int4 *>(cnt + base);
+        v = int64_t(q.x) + q.y + q.z + q.w;
+    } else {
 #pragma unroll
-    for (int j = 0; j < kScanPer; j++)
-        if (base + j < n) v += cnt[base + j] + (cnt2 ? cnt2[base + j] : 0);
+        for (int j = 0; j < kScanPer; j++)
+            if (base + j < n) v += cnt[base + j];
+    }
     int64_t total;
     block_exclusive_scan(v, sw, &total);
     if (threadIdx.x == 0) tile_sum[blockIdx.x] = total;
@@ -1026,10 +1039,12 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_tile_sums(int64_t *__rest
     if (threadIdx.x == 0) *grand_total = carry;
 }
 
-__global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__restrict__ cnt,
-                                                            const int32_t *__restrict__ cnt2, int32_t n,
+// Exclusive sums of the row counts, written one place up: off[0] = 0 and
+// off[i + 1] = cnt[0] + .. + cnt[i - 1], the first position of row i. The
+// writing walk then claims row i's positions from off[i + 1], which ends at
+// cnt[0] + .. + cnt[i]: the offsets array is complete when the walk is.
+__global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__restrict__ cnt, int32_t n,
                                                             const int64_t *__restrict__ tile_off,
-                                                            const int64_t *__restrict__ grand_total,
                                                             int64_t *__restrict__ off) {
     pdl_launch_dependents();
     pdl_wait();
@@ -1037,47 +1052,169 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_rows(const int32_t *__res
     const int64_t base = int64_t(blockIdx.x) * kScanTile + int64_t(threadIdx.x) * kScanPer;
     int64_t c[kScanPer];
     int64_t v = 0;
+    if (base + kScanPer <= n) {
+        const int4 q = *reinterpret_cast<const int4 *>(cnt + base);
+        c[0] = q.x, c[1] = q.y, c[2] = q.z, c[3] = q.w;
+    } else {
 #pragma unroll
-    for (int j = 0; j < kScanPer; j++) {
-        c[j] = base + j < n ? cnt[base + j] + (cnt2 ? cnt2[base + j] : 0) : 0;
-        v += c[j];
+        for (int j = 0; j < kScanPer; j++) c[j] = base + j < n ? cnt[base + j] : 0;
     }
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++) v += c[j];
     int64_t total;
     int64_t run = tile_off[blockIdx.x] + block_exclusive_scan(v, sw, &total);
 #pragma unroll
     for (int j = 0; j < kScanPer; j++) {
-        if (base + j < n) off[base + j] = run;
+        if (base + j < n) off[base + j + 1] = run;
         run += c[j];
     }
-    if (blockIdx.x == 0 && threadIdx.x == 0) off[n] = *grand_total;
+    if (blockIdx.x == 0 && threadIdx.x == 0) off[0] = 0;
 }
 
-// Writes every hit into its row: a recorded hit at the position the probe
-// gave it; a hit beyond those of an overflowing node after the row's
-// recorded hits, at a position claimed with a per-row cursor.
-__global__ void __launch_bounds__(kPatchThreads, 4) k_list_scatter(PatchArgs a, const int64_t *__restrict__ off,
-                                                                const int32_t *__restrict__ count,
-                                                                int32_t *__restrict__ cursor,
-                                                                int32_t *__restrict__ toks) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int32_t stride = gridDim.x * blockDim.x;
-    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        const int32_t c = a.hit_count[m];
-        const int32_t rec = c == kHitOverflow ? kHitSlots : c;
-        for (int32_t i = 0; i < rec; i++) {
-            const int2 hv = a.hits[int64_t(m) * kHitSlots + i];
-            toks[off[hv.x] + a.hit_rank[int64_t(m) * kHitSlots + i]] = hv.y;
+// ------------------------------------------------------------ list walk
+// The valid lists from the reversed-token trie (the vocabulary's tokens read
+// backwards, as an edge table): from every node m the walk follows the labels
+// above m, the label into m first. After j + 1 steps it stands on the
+// reversed prefix of every token that ends with the last j + 1 edges into m;
+// a token ending there is allowed at the node j + 1 levels above m (Sec. 4.2
+// step 2: an output found at the current node belongs to the node |token|
+// characters up). The walk stops at the first label no token continues with,
+// so it costs one exact edge lookup per step and no hashing of whole
+// suffixes. Two walks: the first counts the entries of every row, the second
+// writes them at positions claimed from the rows' offsets (order within a row
+// unspecified).
+
+struct WalkArgs {
+    const uint8_t *terminal;
+    const ulonglong2 *window;  // last 16 labels into each node (byte i = i levels up)
+    const uint8_t *depth16;    // min(depth, 16)
+    const int32_t *anc;        // [n * 16]: ancestors 1..16 levels up
+    const int32_t *parent;
+    const uint8_t *label;
+    int32_t n_nodes;
+    int32_t lmax;              // min(longest token, trie depth)
+    int32_t eos;
+    const uint4 *edge;         // {(parent << 8 | byte) + 1, child, token or -1, 0}; key 0 = empty
+    uint32_t edge_mask;        // slots - 1
+    uint32_t edge_shift;       // 32 - log2(slots)
+    const int32_t *tok_next;   // tokens with the same bytes, or null
+    int32_t *count;            // [n] entries per row (counting walk)
+    unsigned long long *off;   // [n + 1]: off[i + 1] = next position of row i (writing walk)
+    int32_t *toks;
+    unsigned long long tok_cap;  // entries toks holds (a write past it is dropped)
+};
+
+constexpr int kWalkThreads = 256;  // also the 256 root edges each CTA stages
+
+__device__ __forceinline__ uint32_t edge_slot(uint32_t key, uint32_t shift) { return (key * 0x9E3779B1u) >> shift; }
+
+// The edge of reversed-trie node x for byte c (e.y = child, e.z = token
+// ending at the child or -1); false if there is none. The table is at most
+// half full, so an empty slot ends every probe sequence.
+__device__ __forceinline__ bool rt_step(const uint4 *__restrict__ edge, uint32_t mask, uint32_t shift, int32_t x,
+                                        uint32_t c, uint4 *out) {
+    const uint32_t key = ((uint32_t(x) << 8) | c) + 1u;
+    uint32_t s = edge_slot(key, shift);
+    for (uint32_t i = 0; i <= mask; i++) {
+        const uint4 e = __ldg(edge + s);
+        if (e.x == key) {
+            *out = e;
+            return true;
         }
-        if (c == kHitOverflow) {
-            int32_t i = 0;
-            node_hits_window(a, m, [&](int32_t row, int32_t t) {
-                if (i++ >= kHitSlots) toks[off[row] + count[row] + atomicAdd(cursor + row, 1)] = t;
-            });
+        if (e.x == 0u) return false;
+        s = (s + 1u) & mask;
+    }
+    return false;
+}
+
+// Inserts the edge into every node c > 0 of a reversed-token trie.
+__global__ void k_rt_insert(const int32_t *__restrict__ parent, const uint8_t *__restrict__ label,
+                            const int32_t *__restrict__ token, int32_t n, uint4 *__restrict__ edge, uint32_t mask,
+                            uint32_t shift) {
+    for (int32_t c = 1 + blockIdx.x * blockDim.x + threadIdx.x; c < n; c += gridDim.x * blockDim.x) {
+        const uint32_t key = ((uint32_t(parent[c]) << 8) | label[c]) + 1u;
+        uint32_t s = edge_slot(key, shift);
+        for (uint32_t i = 0; i <= mask; i++) {  // keys are distinct: the first empty slot takes it
+            if (atomicCAS(&edge[s].x, 0u, key) == 0u) {
+                edge[s].y = uint32_t(c);
+                edge[s].z = uint32_t(token[c]);
+                break;
+            }
+            s = (s + 1u) & mask;
         }
     }
 }
 
+// Every (row, token) entry whose path ends at node m: EOS at m if m is
+// terminal (App. G.5), then the tokens met by the walk (row = the node as
+// many levels above m as the token has bytes). root[c] = {child, token} of
+// the reversed trie's root for byte c.
+template <typename Tok>
+__device__ __forceinline__ void walk_node(const WalkArgs &a, const int2 *root, int32_t m, Tok tok) {
+    if (__ldg(a.terminal + m)) tok(m, a.eos);
+    const int32_t d16 = __ldg(a.depth16 + m);
+    const int32_t lim = a.lmax < d16 ? a.lmax : d16;
+    if (lim <= 0) return;
+    const ulonglong2 win = __ldg(a.window + m);
+    const int32_t *up = a.anc + int64_t(m) * 16;
+    const int2 r0 = root[uint32_t(win.x) & 0xFFu];
+    int32_t x = r0.x;
+    if (x < 0) return;
+    if (r0.y >= 0) tok(__ldg(up), r0.y);
+    for (int32_t j = 1; j < lim; j++) {
+        const uint32_t c = uint32_t((j < 8 ? win.x >> (8 * j) : win.y >> (8 * (j - 8))) & 0xFFu);
+        uint4 e;
+        if (!rt_step(a.edge, a.edge_mask, a.edge_shift, x, c, &e)) return;
+        x = int32_t(e.y);
+        if (int32_t(e.z) >= 0) tok(__ldg(up + j), int32_t(e.z));
+    }
+    // tokens longer than the 16-label window, in a trie deeper than 16
+    if (lim == 16 && a.lmax > 16) {
+        int32_t y = __ldg(up + 15);  // 16 levels above m: its label is the 17th
+        for (int32_t j = 16; j < a.lmax; j++) {
+            const int32_t p = __ldg(a.parent + y);
+            if (p < 0) return;
+            uint4 e;
+            if (!rt_step(a.edge, a.edge_mask, a.edge_shift, x, __ldg(a.label + y), &e)) return;
+            x = int32_t(e.y);
+            if (int32_t(e.z) >= 0) tok(p, int32_t(e.z));
+            y = p;
+        }
+    }
+}
+
+// kWrite = false: count[row] += 1 for every entry; true: the entry's token
+// at the position claimed from off[row + 1]. Persistent grid (each CTA first
+// stages the reversed trie's 256 root edges in shared memory), a node per
+// thread in a grid-stride loop.
+template <bool kWrite>
+__global__ void __launch_bounds__(kWalkThreads) k_list_walk(WalkArgs a) {
+    __shared__ int2 root[256];
+    {
+        uint4 e;
+        root[threadIdx.x] = rt_step(a.edge, a.edge_mask, a.edge_shift, 0, threadIdx.x, &e)
+                                ? make_int2(int32_t(e.y), int32_t(e.z))
+                                : make_int2(-1, -1);
+    }
+    __syncthreads();
+    pdl_launch_dependents();
+    pdl_wait();  // counts zeroed, or offsets scanned, by the previous kernels
+    auto emit = [&](int32_t row, int32_t t) {
+        if (kWrite) {
+            const unsigned long long p = atomicAdd(a.off + row + 1, 1ull);
+            if (p < a.tok_cap) a.toks[p] = t;
+        } else {
+            atomicAdd(a.count + row, 1);
+        }
+    };
+    auto tok = [&](int32_t row, int32_t t) {
+        emit(row, t);
+        if (a.tok_next)
+            for (int32_t u = __ldg(a.tok_next + t); u >= 0; u = __ldg(a.tok_next + u)) emit(row, u);
+    };
+    const int32_t stride = gridDim.x * blockDim.x;
+    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) walk_node(a, root, m, tok);
+}
 // Apply from the lists: CTA (row b, part p) covers 8 segments (8,192 tokens).
 // It rebuilds their 256 mask words in shared memory from the row's list and
 // writes them like k_apply_vec (kVec) or one logit per thread (any V and
@@ -1570,8 +1707,6 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.trans = t.trans;
     a.trans_mask = t.trans_mask;
     a.trans_fill = 0;
-    a.list_count = nullptr;
-    a.hit_rank = nullptr;
     return a;
 }
 
@@ -1691,6 +1826,14 @@ AdvanceArgs advance_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, b
     return a;
 }
 
+cudaError_t launch_mask_pairwise(const DevTrie &t, int32_t n_nodes, const DevVocab &v, uint32_t *mask, int num_sms,
+                                 cudaStream_t st) {
+    const AdvanceArgs a = advance_args(t, n_nodes, v, false);
+    const int64_t W = (int64_t(v.V) + 31) / 32, chunks = (W + 31) / 32;
+    const int grid = grid_for(int64_t(n_nodes) * chunks, kPairwiseThreads / 32, int64_t(num_sms) * 8);
+    return launch_pdl(k_mask_pairwise, grid, kPairwiseThreads, st, a, mask, W, chunks);
+}
+
 cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v, const int32_t *states_in,
                            int32_t *states_out, const int32_t *tokens, int32_t B, int32_t *err, bool use_trans,
                            cudaStream_t st) {
@@ -1715,12 +1858,14 @@ cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVoc
         return launch_apply(logits, dtype, mask, states_out, B, V, n_nodes, num_sms, st);
     }
     const AdvanceArgs aa = advance_args(t, n_nodes, v, use_trans);
-    const int grid = grid_for(int64_t(B) * segs, kApplyThreads / 32, INT32_MAX);
+    const int32_t parts = (segs + kApplyThreads / 32 - 1) / (kApplyThreads / 32);
+    const int64_t grid = int64_t(B) * parts;
+    if (grid > INT32_MAX) return cudaErrorInvalidValue;
     if (elt == 2)
         return launch_pdl(k_advance_apply_vec<2>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
-                          states_in, tokens, states_out, err, B, W, segs);
+                          states_in, tokens, states_out, err, B, W, segs, parts);
     return launch_pdl(k_advance_apply_vec<4>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
-                      states_in, tokens, states_out, err, B, W, segs);
+                      states_in, tokens, states_out, err, B, W, segs, parts);
 }
 
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
@@ -1745,43 +1890,110 @@ cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const in
     return launch_pdl(k_apply_scalar<4>, grid, kApplyThreads, st, logits, mask, states, B, V, W, n_nodes);
 }
 
+namespace {
+
+// Up to three copies in one launch, reading the sources directly (host memory
+// that the device reads coherently, or device memory): 16-byte blocks where
+// both ends are 16-byte aligned, else bytes.
+struct CopySeg {
+    uint8_t *dst;
+    const uint8_t *src;
+    int64_t bytes;
+};
+
+__global__ void k_copy_segments(CopySeg s0, CopySeg s1, CopySeg s2) {
+    pdl_launch_dependents();
+    pdl_wait();  // the destination may still be read by an earlier kernel
+    const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+    const int64_t i0 = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+    const CopySeg seg[3] = {s0, s1, s2};
+#pragma unroll
+    for (int k = 0; k < 3; k++) {
+        const CopySeg c = seg[k];
+        int64_t done = 0;
+        if (((reinterpret_cast<uintptr_t>(c.dst) | reinterpret_cast<uintptr_t>(c.src)) & 15u) == 0) {
+            const int64_t nv = c.bytes >> 4;
+            for (int64_t i = i0; i < nv; i += stride)
+                reinterpret_cast<uint4 *>(c.dst)[i] = reinterpret_cast<const uint4 *>(c.src)[i];
+            done = nv << 4;
+        }
+        for (int64_t i = done + i0; i < c.bytes; i += stride) c.dst[i] = c.src[i];
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_copy3(void *d0, const void *s0, int64_t b0, void *d1, const void *s1, int64_t b1, void *d2,
+                         const void *s2, int64_t b2, int num_sms, cudaStream_t st) {
+    const int64_t most = std::max(b0, std::max(b1, b2));
+    if (most <= 0) return cudaSuccess;
+    const int grid = grid_for((most + 15) / 16, 256, int64_t(num_sms) * 4);
+    return launch_pdl(k_copy_segments, grid, 256, st,
+                      CopySeg{static_cast<uint8_t *>(d0), static_cast<const uint8_t *>(s0), b0},
+                      CopySeg{static_cast<uint8_t *>(d1), static_cast<const uint8_t *>(s1), b1},
+                      CopySeg{static_cast<uint8_t *>(d2), static_cast<const uint8_t *>(s2), b2});
+}
+
+cudaError_t launch_rt_build(const int32_t *parent, const uint8_t *label, const int32_t *token, int32_t n,
+                            uint4 *edge, uint32_t mask, int num_sms, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(edge, 0, sizeof(uint4) * (size_t(mask) + 1), st);
+    if (e != cudaSuccess || n <= 1) return e;
+    const uint32_t shift = 32u - uint32_t(__builtin_popcount(mask));
+    const int grid = grid_for(n, 256, int64_t(num_sms) * 8);
+    k_rt_insert<<<grid, 256, 0, st>>>(parent, label, token, n, edge, mask, shift);
+    return cudaGetLastError();
+}
+
+namespace {
+
+WalkArgs walk_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax, const DevLists &L) {
+    WalkArgs a;
+    a.terminal = t.terminal;
+    a.window = t.window;
+    a.depth16 = t.depth16;
+    a.anc = reinterpret_cast<const int32_t *>(t.anc);
+    a.parent = t.parent;
+    a.label = t.label;
+    a.n_nodes = n_nodes;
+    a.lmax = lmax;
+    a.eos = v.V - 1;
+    a.edge = v.rt_edge;
+    a.edge_mask = v.rt_mask;
+    a.edge_shift = 32u - uint32_t(__builtin_popcount(v.rt_mask));
+    a.tok_next = v.tok_next;
+    a.count = L.count;
+    a.off = reinterpret_cast<unsigned long long *>(L.off);
+    a.toks = L.toks;
+    a.tok_cap = static_cast<unsigned long long>(L.tok_cap);
+    return a;
+}
+
+}  // namespace
+
 cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                               const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total) {
-    PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
-    a.trans_fill = fill_trans && t.trans;
-    a.list_count = L.count;
-    a.hit_rank = L.rank;
-    Prefetch pf;
-    pf.count = 0;
-    // count, cursor and over are adjacent: zero all three before the probe counts
-    cudaError_t e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), 3 * int64_t(n_nodes), num_sms, st);
+                               const DevLists &L, int num_sms, cudaStream_t st) {
+    const WalkArgs a = walk_args(t, n_nodes, v, lmax, L);
+    cudaError_t e = launch_mask_fill(reinterpret_cast<uint32_t *>(L.count), int64_t(n_nodes), num_sms, st);
     if (e != cudaSuccess) return e;
-    if ((e = launch_probe(a, pf, num_sms, st)) != cudaSuccess) return e;
-    const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
-    if ((e = launch_pdl(k_list_count_over, grid, kPatchThreads, st, a, L.over)) != cudaSuccess) return e;
+    const int grid = grid_for(n_nodes, kWalkThreads, int64_t(num_sms) * 8);
+    if ((e = launch_pdl(k_list_walk<false>, grid, kWalkThreads, st, a)) != cudaSuccess) return e;
     const int32_t n_tiles = int32_t((int64_t(n_nodes) + kScanTile - 1) / kScanTile);
-    if ((e = launch_pdl(k_scan_tiles, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count),
-                        static_cast<const int32_t *>(L.over), n_nodes, L.tile_sum)) != cudaSuccess)
+    if ((e = launch_pdl(k_scan_tiles, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count), n_nodes,
+                        L.tile_sum)) != cudaSuccess)
         return e;
     if ((e = launch_pdl(k_scan_tile_sums, 1, kScanThreads, st, L.tile_sum, n_tiles, L.total)) != cudaSuccess)
         return e;
-    if ((e = launch_pdl(k_scan_rows, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count),
-                        static_cast<const int32_t *>(L.over), n_nodes, static_cast<const int64_t *>(L.tile_sum),
-                        static_cast<const int64_t *>(L.total), L.off)) != cudaSuccess)
+    if ((e = launch_pdl(k_scan_rows, n_tiles, kScanThreads, st, static_cast<const int32_t *>(L.count), n_nodes,
+                        static_cast<const int64_t *>(L.tile_sum), L.off)) != cudaSuccess)
         return e;
-    // the size decides the token buffer: read it back (the one host sync)
-    if ((e = cudaMemcpyAsync(h_total, L.total, sizeof(int64_t), cudaMemcpyDeviceToHost, st)) != cudaSuccess)
-        return e;
-    return cudaStreamSynchronize(st);
+    return cudaSuccess;
 }
 
-cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                                 const DevLists &L, int num_sms, cudaStream_t st) {
-    PatchArgs a = patch_args(t, n_nodes, v, lmax, nullptr, 0);
-    const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 16);
-    a.hit_rank = L.rank;
-    return launch_pdl(k_list_scatter, grid, kPatchThreads, st, a, static_cast<const int64_t *>(L.off),
-                      static_cast<const int32_t *>(L.count), L.cursor, L.toks);
+cudaError_t launch_lists_write(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                               const DevLists &L, int num_sms, cudaStream_t st) {
+    const WalkArgs a = walk_args(t, n_nodes, v, lmax, L);
+    const int grid = grid_for(n_nodes, kWalkThreads, int64_t(num_sms) * 8);
+    return launch_pdl(k_list_walk<true>, grid, kWalkThreads, st, a);
 }
 
 namespace {

@@ -9,8 +9,10 @@
 // serves them: the trie and vocabulary go into one fixed-size array declared
 // in this file (g_scratch, TRIE_NOALLOC_SCRATCH_BYTES), reserved when the
 // library's module is loaded on a device and held until the process exits.
-// The host packing likewise goes through a static staging buffer. Only the
-// caller's inputs and output are touched besides.
+// The host packing likewise goes through a static staging buffer, which a call
+// rewrites only after the previous call's copy out of it has completed (an
+// event recorded after that copy). Only the caller's inputs and output are
+// touched besides.
 #include <stdint.h>
 #include <string.h>
 
@@ -31,26 +33,41 @@ __device__ __align__(256) unsigned char g_scratch[TRIE_NOALLOC_SCRATCH_BYTES];
 alignas(256) unsigned char g_stage[TRIE_NOALLOC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-std::mutex g_mu;                          // serialises use of g_stage and g_dev_ptr
-void *g_dev_ptr[kMaxDevices] = {nullptr};  // device address of g_scratch per device
+std::mutex g_mu;  // serialises use of g_stage and of the per-device state
+
+// Per device, set up by its first call with the device current: the device
+// address of g_scratch and an event recorded after each copy out of g_stage.
+struct DevState {
+    void *scratch = nullptr;
+    cudaEvent_t staged = nullptr;
+};
+DevState g_dev[kMaxDevices];
+cudaEvent_t g_pending = nullptr;  // event of the last copy out of g_stage (any device)
 
 size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
-// Device address of g_scratch on `dev` (the current device). The host-side
-// name g_scratch is only a stand-in for the symbol, so the address is looked
-// up once per device with that device current.
-int scratch_ptr(int dev, void **out) {
+// The host-side name g_scratch is only a stand-in for the symbol, so its
+// device address is looked up once per device; the address and the event are
+// kept for the life of the process (they do not survive cudaDeviceReset).
+int device_state(int dev, DevState **out) {
     if (dev < 0 || dev >= kMaxDevices) return tmk::set_error(TRIE_EINVAL, "device ordinal out of range");
-    if (!g_dev_ptr[dev]) {
+    DevState &d = g_dev[dev];
+    if (!d.scratch) {
         void *p = nullptr;
         cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
         if (e != cudaSuccess || !p) {
             cudaGetLastError();
             return tmk::set_error(TRIE_ECUDA, "cudaGetSymbolAddress of the no-alloc scratch failed");
         }
-        g_dev_ptr[dev] = p;
+        cudaEvent_t ev = nullptr;
+        if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming)) != cudaSuccess) {
+            cudaGetLastError();
+            return tmk::set_error(TRIE_ECUDA, "creating the no-alloc staging event failed");
+        }
+        d.scratch = p;
+        d.staged = ev;
     }
-    *out = g_dev_ptr[dev];
+    *out = &d;
     return TRIE_OK;
 }
 
@@ -81,8 +98,7 @@ extern "C" int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, 
             if (L > max_len) max_len = int32_t(L);
         }
     }
-    uint64_t S = 16;
-    while (S < uint64_t(4 * n_ins)) S <<= 1;
+    const uint64_t S = tmk::token_table_slots(n_ins);
     const tmk::HostTrie &t = h->host;
     const size_t n = size_t(t.n);
     size_t off = 0;
@@ -109,12 +125,11 @@ extern "C" int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, 
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 1;
 
     std::lock_guard<std::mutex> lk(g_mu);
-    void *dscratch = nullptr;
-    int rc = scratch_ptr(dev, &dscratch);
+    DevState *ds = nullptr;
+    int rc = device_state(dev, &ds);
     if (rc != TRIE_OK) return rc;
+    void *dscratch = ds->scratch;
 
-    // stage: trie arrays from the handle's host copy; a forest built on the
-    // device has none, and its device arrays are copied within the device
     bool on_device;
     {
         std::lock_guard<std::mutex> hl(h->mu);
@@ -122,53 +137,47 @@ extern "C" int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, 
     }
     if (on_device && h->dev.device != dev)
         return tmk::set_error(TRIE_EINVAL, "handle was built on another device");
+    // the previous call's copy may still be reading g_stage (an asynchronous
+    // copy from pageable memory need not have staged it before returning)
+    if (g_pending) {
+        e = cudaEventSynchronize(g_pending);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return tmk::set_error(TRIE_ECUDA, "waiting for the previous no-alloc copy failed");
+        }
+        g_pending = nullptr;
+    }
+    // stage: trie arrays from the handle's host copy; a forest built on the
+    // device has none, and its device arrays are copied within the device
     unsigned char *st = g_stage;
     if (!on_device) {
         memcpy(st + o_par, t.parent.data(), 4 * n);
         memcpy(st + o_lab, t.label.data(), n);
         memcpy(st + o_term, t.terminal.data(), n);
     }
-    // stage: tokens 16-byte aligned, EOS and byte-less tokens with length 0
+    // stage: tokens 16-byte aligned (EOS and byte-less tokens with length 0)
+    // and the (length, bytes) -> id table, as trie_compile_masks packs them
     uint32_t *toff = reinterpret_cast<uint32_t *>(st + o_toff);
     uint16_t *tlen = reinterpret_cast<uint16_t *>(st + o_tlen);
-    unsigned char *bl = st + o_blob;
-    memset(bl, 0, size_t(blob) + 16);
-    uint32_t pos = 0;
-    for (int32_t v = 0; v < V; v++) {
-        const int64_t L = (v == V - 1) ? 0 : vocab_offsets[v + 1] - vocab_offsets[v];
-        toff[v] = pos;
-        tlen[v] = uint16_t(L);
-        if (L > 0) memcpy(bl + pos, vocab_bytes + vocab_offsets[v], size_t(L));
-        pos += uint32_t((L + 15) / 16 * 16);
-    }
-    // stage: (length, bytes) -> id table in aligned slot pairs, load <= 1/4,
-    // the same hash and probe order as the kernel's lookups
-    uint64_t *key = reinterpret_cast<uint64_t *>(st + o_key);
-    int32_t *val = reinterpret_cast<int32_t *>(st + o_val);
-    memset(key, 0, 8 * size_t(S));
-    memset(val, 0xff, 4 * size_t(S));
-    const uint64_t pairs_mask = S / 2 - 1;
-    for (int32_t v = 0; v + 1 < V; v++) {
-        const uint32_t L = tlen[v];
-        if (!L) continue;
-        const uint8_t *p = vocab_bytes + vocab_offsets[v];
-        uint64_t hsh = 0;
-        for (uint32_t j = 0; j < L; j++) hsh = hsh * tmk::kHashBase + uint64_t(p[j]) + 1;
-        const uint64_t k = tmk::hash_finish(hsh, L);
-        uint64_t pair = (k >> 1) & pairs_mask;
-        for (;;) {
-            if (!key[2 * pair]) { key[2 * pair] = k; val[2 * pair] = v; break; }
-            if (!key[2 * pair + 1]) { key[2 * pair + 1] = k; val[2 * pair + 1] = v; break; }
-            pair = (pair + 1) & pairs_mask;
-        }
-    }
-    // one copy into the device scratch, ordered on the caller's stream; from
-    // pageable memory it returns once the staging buffer has been read
+    memset(st + o_blob, 0, size_t(blob) + 16);
+    tmk::pack_token_bytes(vocab_bytes, vocab_offsets, V, toff, tlen, st + o_blob);
+    const bool dup_keys = tmk::fill_token_table(vocab_bytes, vocab_offsets, tlen, V, S,
+                                                reinterpret_cast<uint64_t *>(st + o_key),
+                                                reinterpret_cast<int32_t *>(st + o_val));
+    // one copy into the device scratch, ordered on the caller's stream; the
+    // next call waits for its event before it rewrites g_stage
     e = cudaMemcpyAsync(dscratch, g_stage, total, cudaMemcpyHostToDevice, stream);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return tmk::set_error(TRIE_ECUDA, "copy into the no-alloc scratch failed");
     }
+    if ((e = cudaEventRecord(ds->staged, stream)) != cudaSuccess) {
+        cudaGetLastError();
+        cudaStreamSynchronize(stream);  // no event to wait for: g_stage must be free on return
+        cudaGetLastError();
+        return tmk::set_error(TRIE_ECUDA, "recording the no-alloc staging event failed");
+    }
+    g_pending = ds->staged;
 
     unsigned char *d = static_cast<unsigned char *>(dscratch);
     if (on_device && n > 0 &&
@@ -193,6 +202,7 @@ extern "C" int trie_compile_masks_noalloc(trie_t h, const uint8_t *vocab_bytes, 
     dv.blob = d + o_blob;
     dv.ht_key = reinterpret_cast<const uint64_t *>(d + o_key);
     dv.ht_val = reinterpret_cast<const int32_t *>(d + o_val);
+    dv.dup_keys = dup_keys ? 1 : 0;
     const int64_t W = (int64_t(V) + 31) / 32;
     const int32_t lmax = max_len < t.max_depth ? max_len : t.max_depth;
     e = tmk::launch_mask_fill(d_mask, int64_t(t.n) * W, sms, stream);

@@ -16,6 +16,40 @@
 
 namespace tmk {
 
+#if defined(__CUDACC__)
+// Programmatic dependent launch (PDL). Every kernel of the library is launched
+// with programmatic stream serialization: it may let the next kernel of its
+// stream launch early (pdl_launch_dependents) and waits for the previous one
+// (pdl_wait, the hardware grid dependency: the previous grid never waits on
+// this one, so the wait always resolves) before it touches memory that kernel
+// may write or read.
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl_smem(void (*kernel)(Params...), int64_t grid, int block, size_t smem, cudaStream_t st,
+                            Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(grid < 1 ? 1 : grid));
+    cfg.blockDim = dim3(unsigned(block));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Params>(args)...);
+}
+
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), int64_t grid, int block, cudaStream_t st, Args... args) {
+    return launch_pdl_smem(kernel, grid, block, 0, st, args...);
+}
+#endif
+
 // Blocks of at least 2 MB for the builder's arrays come from a process-wide
 // cache of freed blocks (whole 2 MB classes, at most 1 GB held): a server that
 // builds a new forest for every batch then reuses pages it has already
@@ -109,6 +143,38 @@ struct HostVocab {
 
 std::string pack_vocab(const uint8_t *bytes, const int64_t *offsets, int32_t V, HostVocab *out);
 
+// The tokens read backwards, as a trie (root 0): the path from the root
+// spelling b_{L-1} .. b_0 ends at the node of token b_0 .. b_{L-1}. Walking it
+// with the labels above a node m of a set trie (the label into m first) meets,
+// after k steps, exactly the tokens that spell the last k edges into m: the
+// Aho-Corasick outputs at m of Sec. 4.2 step 2, without failure links. Node
+// ids in pre-order; token[x] = the smallest id whose bytes end at x, or -1;
+// next[v] = the next larger id with the same bytes as v, or -1 (empty when
+// all token strings differ). Built once per vocabulary, on the host.
+constexpr int64_t kRevTrieMaxNodes = (int64_t(1) << 24) - 2;  // edge keys (parent << 8 | byte) + 1 fit 32 bits
+struct RevTokenTrie {
+    int32_t n = 0;
+    hvec<int32_t> parent;
+    hvec<uint8_t> label;
+    hvec<int32_t> token;
+    std::vector<int32_t> next;
+    int32_t max_mult = 1;  // most ids sharing one byte string
+};
+std::string build_reversed_token_trie(const uint8_t *bytes, const int64_t *offsets, int32_t V,
+                                      RevTokenTrie *out);
+
+// The two halves of pack_vocab, writing into caller-supplied arrays (the
+// no-alloc compile stages into a static buffer). pack_token_bytes: token v's
+// bytes at tok_off[v] (16-byte aligned, blob zeroed by the caller), its length
+// in tok_len[v]; EOS (V-1) gets length 0. fill_token_table: the (length,
+// bytes) -> id table of S slots (token_table_slots), returns whether two
+// tokens share a key. Offsets must already be validated.
+void pack_token_bytes(const uint8_t *bytes, const int64_t *offsets, int32_t V, uint32_t *tok_off,
+                      uint16_t *tok_len, uint8_t *blob);
+bool fill_token_table(const uint8_t *bytes, const int64_t *offsets, const uint16_t *tok_len, int32_t V,
+                      uint64_t S, uint64_t *key, int32_t *val);
+uint64_t token_table_slots(int64_t n_tokens_with_bytes);
+
 // Polynomial string hash used by the table: Horner over (byte + 1) with base
 // kHashBase, modulo 2^64, then mixed with the length. The kernel extends it
 // one byte to the left per trie edge it climbs.
@@ -141,6 +207,16 @@ struct DevVocab {
     // per slot: token, min(len, 31) << 27 | blob offset / 16, first 8 bytes
     // (null when the blob exceeds 2 GiB or two tokens share a key)
     const uint4 *ht_pay = nullptr;
+    // The reversed-token trie (RevTokenTrie) as an open-addressing edge table
+    // for the list compile's walk, built on first use: slot {(parent << 8 |
+    // byte) + 1, child, token ending at child or -1, 0}, key 0 = empty.
+    std::mutex rt_mu;
+    int32_t rt_state = 0;                // 0 not built, 1 built, -1 too large (walk unavailable)
+    void *rt_base = nullptr;
+    const uint4 *rt_edge = nullptr;
+    uint32_t rt_mask = 0;                // slots - 1
+    const int32_t *tok_next = nullptr;   // [V] next id with the same bytes, or null (all strings differ)
+    int32_t rt_mult = 1;                 // most ids sharing one byte string
     // host copy of the caller's arrays, to recognise the same vocabulary later
     std::vector<uint8_t> src_bytes;
     std::vector<int64_t> src_offsets;
@@ -176,17 +252,16 @@ struct DevTrie {
 
 // Device storage of the sparse valid lists of a handle (library-owned).
 struct DevLists {
-    void *base = nullptr;           // count, cursor, over, rank, off, tile_sum, total
-    int32_t *count = nullptr;       // [n] recorded hits per row (cursor and over follow it)
-    int32_t *cursor = nullptr;      // [n] positions claimed by overflow hits
-    int32_t *over = nullptr;        // [n] hits per row beyond the recorded ones
-    int32_t *rank = nullptr;        // [n * kHitSlots] position of each recorded hit in its row
+    void *base = nullptr;           // count, off, tile_sum, total
+    int32_t *count = nullptr;       // [n] entries per row (the counting walk)
     int64_t *off = nullptr;         // [n + 1]
     int64_t *tile_sum = nullptr;    // [tiles]
     int64_t *total = nullptr;       // [1]
     int32_t *toks = nullptr;        // [tok_cap], separate allocation
     int64_t tok_cap = 0;
-    int64_t n_valid = -1;           // entries of the last build, -1 before any
+    int64_t n_valid = -1;           // entries of the last build, -1 before any (read back on demand)
+    bool n_valid_on_device = false; // n_valid is still only in *total
+    cudaEvent_t done = nullptr;     // recorded after the last build's kernels
     int32_t V = 0;
 };
 
@@ -357,12 +432,29 @@ cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVoc
                                  int num_sms, cudaStream_t st);
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
                          int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st);
-// Valid lists: probe, per-row counts and their scan; ends by reading the
-// total into *h_total (host-synchronous). Then the scatter into L.toks.
+// Copies (d_k, s_k, b_k bytes), k = 0..2, in one launch; the sources are read
+// by the kernel itself (device memory, or host memory the device reads
+// coherently), so no copy engine and no host synchronisation is involved.
+cudaError_t launch_copy3(void *d0, const void *s0, int64_t b0, void *d1, const void *s1, int64_t b1, void *d2,
+                         const void *s2, int64_t b2, int num_sms, cudaStream_t st);
+// The pairwise form of the dense compile (one walk per (node, token) pair,
+// a warp ballot per mask word), kept for comparison with the suffix search.
+cudaError_t launch_mask_pairwise(const DevTrie &t, int32_t n_nodes, const DevVocab &v, uint32_t *mask, int num_sms,
+                                 cudaStream_t st);
+// Edge table of a reversed-token trie (parent, label, token arrays of n
+// nodes on the device): zeroes the S = mask + 1 slots and inserts every edge.
+cudaError_t launch_rt_build(const int32_t *parent, const uint8_t *label, const int32_t *token, int32_t n,
+                            uint4 *edge, uint32_t mask, int num_sms, cudaStream_t st);
+// Valid lists by walking the reversed-token trie from every node. Count:
+// zero the per-row counts, count every (row, token) entry, scan the counts
+// into L.off (shifted one place up: off[i + 1] = the first position of row
+// i) and *L.total. Write: walk again, writing every entry at the position
+// claimed from off[row + 1] into L.toks (entries past L.tok_cap are
+// dropped); afterwards L.off holds the rows' offsets.
 cudaError_t launch_lists_count(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                               const DevLists &L, int num_sms, bool fill_trans, cudaStream_t st, int64_t *h_total);
-cudaError_t launch_lists_scatter(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                                 const DevLists &L, int num_sms, cudaStream_t st);
+                               const DevLists &L, int num_sms, cudaStream_t st);
+cudaError_t launch_lists_write(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
+                               const DevLists &L, int num_sms, cudaStream_t st);
 // Lazy rows: pos_of from the pre-order tables and the path hashes (once, at set-up).
 cudaError_t launch_lazy_tables(const DevTrie &t, const DevLazy &L, int32_t n_nodes, cudaStream_t st);
 // One lazy call: map the batch's states (after the advance when tokens is not

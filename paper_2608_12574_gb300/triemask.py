@@ -35,6 +35,7 @@ SIGNATURES = {
     "trie_max_depth": (_I32, [_P]),
     "trie_get_csr": (ctypes.c_int, [_P, _P, _P, _P, _P]),
     "trie_compile_masks": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
+    "trie_compile_masks_pairwise": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_compile_masks_noalloc": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_compile_lists": (ctypes.c_int, [_P, _P, _P, _I32, _P]),
     "trie_num_valid": (_I64, [_P]),
@@ -56,6 +57,7 @@ SIGNATURES = {
     "fmt_apply_mask": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
     "fmt_destroy": (ctypes.c_int, [_P]),
     "trie_destroy": (ctypes.c_int, [_P]),
+    "trie_destroy_async": (ctypes.c_int, [_P, _P]),
     "trie_last_error": (ctypes.c_char_p, []),
 }
 
@@ -164,6 +166,13 @@ class Trie:
             self._lib.trie_destroy(self.handle)
             self.handle = None
 
+    def destroy_async(self, stream=None) -> None:
+        """Release the handle; its device memory is freed in stream order."""
+        import torch
+        if self.handle:
+            h, self.handle = self.handle, None
+            _check(self._lib.trie_destroy_async(h, _stream(stream, torch.cuda.current_device())))
+
     def __del__(self):
         try:
             self.destroy()
@@ -238,6 +247,20 @@ def trie_compile_masks(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stre
                                      _stream(stream, d_mask.device)))
 
 
+def trie_compile_masks_pairwise(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stream=None) -> None:
+    """The dense mask evaluated pair by pair (one token per lane, a warp ballot per word)."""
+    import torch
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    p = _dev(d_mask, (torch.int32,), "d_mask")
+    if d_mask.numel() < h.num_nodes * mask_words(V):
+        raise ValueError("d_mask is smaller than num_nodes * ceil(V/32) words")
+    _check(h._lib.trie_compile_masks_pairwise(h.handle, _hp(vb), _hp(vo), V, p,
+                                              _stream(stream, d_mask.device)))
+
+
 def trie_compile_masks_noalloc(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stream=None) -> None:
     """trie_compile_masks without device allocation (fixed 32 MiB library scratch)."""
     import torch
@@ -292,8 +315,11 @@ def trie_apply_mask(h: Trie, d_logits, d_states, stream=None) -> None:
     _check(h._lib.trie_apply_mask(h.handle, pl, dtype, ps, B, V, _stream(stream, d_logits.device)))
 
 
-def trie_compile_lists(h: Trie, vocab_bytes, vocab_offsets, V: int, stream=None, device=None) -> int:
-    """Build the handle's sparse valid lists on the GPU; returns the number of entries."""
+def trie_compile_lists(h: Trie, vocab_bytes, vocab_offsets, V: int, stream=None, device=None,
+                       count: bool = True) -> int | None:
+    """Build the handle's sparse valid lists on the GPU (asynchronous on the
+    stream). Returns the number of entries, which waits for the build; with
+    count=False it returns None and does not wait."""
     import torch
     vb = _host(vocab_bytes, np.uint8)
     vo = _host(vocab_offsets, np.int64)
@@ -301,7 +327,7 @@ def trie_compile_lists(h: Trie, vocab_bytes, vocab_offsets, V: int, stream=None,
         raise ValueError("vocab_offsets must have V+1 entries")
     _check(h._lib.trie_compile_lists(h.handle, _hp(vb), _hp(vo), V,
                                      _stream(stream, device if device is not None else torch.cuda.current_device())))
-    return h._lib.trie_num_valid(h.handle)
+    return h._lib.trie_num_valid(h.handle) if count else None
 
 
 def trie_num_valid(h: Trie) -> int:
@@ -421,6 +447,10 @@ def trie_advance_apply_lists(h: Trie, d_states_in, d_tokens, d_states_out, d_log
 
 def trie_destroy(h: Trie) -> None:
     h.destroy()
+
+
+def trie_destroy_async(h: Trie, stream=None) -> None:
+    h.destroy_async(stream)
 
 
 # ------------------------------------------------------------ fixed formats

@@ -16,10 +16,10 @@ ARGS = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "
         "--steps", "1", "--warmup", "0"]
 
 
-def _run(extra_env: dict) -> subprocess.CompletedProcess:
+def _run(extra_env: dict, extra_args: tuple = ()) -> subprocess.CompletedProcess:
     env = dict(os.environ)
     env.update(extra_env)
-    return subprocess.run(ARGS, cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    return subprocess.run(ARGS + list(extra_args), cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
 
 
 def test_reference_arm_prints_one_line():
@@ -32,6 +32,13 @@ def test_reference_arm_prints_one_line():
     assert line["unit"] == "pairs/s" and line["higher_is_better"] is True
     assert line["config"]["workload"] == "tools-K100-V32000-B1-f32"
     assert line["config"]["N_nodes"] == 1384
+    # the GPU arm prints the same config object (bench.workload_config), so the
+    # two arms' lines describe one workload key for key
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_12574_gb300 import workloads as W
+    assert line["config"] == bench.workload_config(W.config(1), 1384)
+    assert set(line["config"]) == {"workload", "K", "V", "batch", "decode_steps", "N_nodes", "N_chars", "r", "l2"}
     assert line["value"] > 0 and line["steps"] == 1 and line["warmup"] == 0
     cb = line["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"]
@@ -52,9 +59,17 @@ def _share(cb: dict) -> float:
 
 
 def test_reference_arm_other_ranks_exit_quietly():
-    r = _run({"RANK": "1", "WORLD_SIZE": "2"})
+    r = _run({"RANK": "1", "WORLD_SIZE": "2"}, ("--gpus", "2"))
     assert r.returncode == 0, r.stderr
     assert r.stdout.strip() == ""
+
+
+def test_gpus_must_match_the_launch():
+    """A launch of WORLD_SIZE ranks whose --gpus says otherwise fails loudly
+    instead of reporting a different number of GPUs."""
+    r = _run({"RANK": "0", "WORLD_SIZE": "2"}, ("--gpus", "4"))
+    assert r.returncode != 0
+    assert "does not match WORLD_SIZE" in r.stderr
 
 
 def test_clock_summary_parses_nvidia_smi_samples():

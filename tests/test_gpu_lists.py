@@ -93,6 +93,48 @@ def test_lists_configs(cuda, cfg):
     assert np.array_equal(_key(*got, w.V), _key(want_r, want_t, w.V))
 
 
+@pytest.mark.parametrize("seed", range(3))
+def test_lists_long_tokens_deep_trie(cuda, seed):
+    """Tokens longer than 16 bytes in a trie deeper than 16: the walk leaves
+    the 16-label window and climbs parent links; repeated token strings are
+    listed under every id."""
+    r = np.random.default_rng(77 + seed)
+    alpha = np.frombuffer(b"ab", np.uint8)
+    strings = [bytes(r.choice(alpha, r.integers(1, 48))) for _ in range(40)]
+    toks = [bytes([c]) for c in range(256)]
+    toks += [bytes(r.choice(alpha, r.integers(2, 31))) for _ in range(400)]
+    toks += [s_[i:i + L] for s_ in strings[:10] for i in range(0, 5) for L in (17, 23, 30) if len(s_) >= i + L]
+    toks += toks[300:320]  # repeated strings
+    toks.append(b"")
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    V = len(toks)
+    h = T.trie_build(sb, so)
+    n = T.trie_compile_lists(h, vb, vo, V)
+    want = _oracle_pairs_from_mask(oracle.mask_all(oracle.Trie(sb, so), oracle.Vocab(vb, vo)), V)
+    assert n == len(want[0])
+    assert np.array_equal(_key(*_gpu_pairs(h), V), _key(*want, V))
+
+
+def test_lists_many_repeated_tokens(cuda):
+    """One token string under 20,000 ids: the bound on the entries (one per
+    id and length) is too large to allocate, so the list compile reads the
+    exact count back between its two walks."""
+    r = np.random.default_rng(5)
+    alpha = np.frombuffer(b"ab", np.uint8)
+    strings = [bytes(r.choice(alpha, r.integers(10, 30))) for _ in range(100)]
+    toks = [bytes([c]) for c in range(256)] + [b"ab"] * 20000 + [b"ba", b"aab", b""]
+    sb, so = W.pack(strings)
+    vb, vo = W.pack(toks)
+    V = len(toks)
+    h = T.trie_build(sb, so)
+    assert h.num_nodes * (16 * 20000 + 1) > (1 << 28)
+    n = T.trie_compile_lists(h, vb, vo, V)
+    want = _oracle_pairs_from_mask(oracle.mask_all(oracle.Trie(sb, so), oracle.Vocab(vb, vo)), V)
+    assert n == len(want[0])
+    assert np.array_equal(_key(*_gpu_pairs(h), V), _key(*want, V))
+
+
 def test_lists_forest(cuda):
     """The 256-request forest: every set's entries, offset by its root."""
     w = W.config(5)

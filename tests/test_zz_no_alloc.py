@@ -61,6 +61,61 @@ def test_noalloc_equals_compile_on_consecutive_calls(cuda):
         assert torch.equal(out, ref), f"workload {w.name}: no-alloc mask differs"
 
 
+def test_noalloc_back_to_back_without_sync(cuda):
+    """Calls queued on one stream with no synchronisation between them: each
+    call rewrites the shared host staging buffer only after the previous
+    call's copy out of it has completed, so both masks must be right."""
+    import torch
+    lib = T.load_library()
+    stream = torch.cuda.Stream(cuda)
+    ws = [W.config(c) for c in (3, 1, 2)]
+    hs = [T.trie_build(w.set_bytes, w.set_offsets) for w in ws]
+    refs = []
+    for w, h in zip(ws, hs):
+        ref = T.alloc_mask(h, w.V, cuda)
+        T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, w.V, ref)
+        refs.append(ref)
+    torch.cuda.synchronize()
+    outs = [torch.full_like(r, -1) for r in refs]
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        # a long kernel ahead of the first copy keeps the stream busy
+        big = torch.empty(1 << 28, dtype=torch.int32, device=cuda)
+        big.fill_(7)
+        for w, h, out in zip(ws, hs, outs):
+            rc = _noalloc(lib, h, w.vocab_bytes, w.vocab_offsets, w.V, out, stream)
+            assert rc == T.TRIE_OK, T.trie_last_error()
+    stream.synchronize()
+    for w, out, ref in zip(ws, outs, refs):
+        assert torch.equal(out, ref), f"workload {w.name}: queued no-alloc mask differs"
+
+
+def test_noalloc_device_built_forest(cuda):
+    """A forest built on the device keeps its trie only in device memory; the
+    no-alloc compile copies those arrays within the device."""
+    import torch
+    lib = T.load_library()
+    stream = torch.cuda.current_stream(cuda)
+    w = W.config(1)
+    names = W.unpack(w.set_bytes, w.set_offsets)
+    sets = [names[:30], names[30:31] + [b""], names[31:], names[5:60]]
+    fb, fo = W.pack([x for s in sets for x in s])
+    fi = np.cumsum([0] + [len(s) for s in sets]).astype(np.int32)
+    for _ in range(2):  # two calls in a row
+        hd = T.trie_build_many_device(fb, fo, fi)
+        hh = T.trie_build_many(fb, fo, fi)
+        ref = T.alloc_mask(hh, w.V, cuda)
+        T.trie_compile_masks(hh, w.vocab_bytes, w.vocab_offsets, w.V, ref)
+        out = torch.full_like(ref, -1)
+        rc = _noalloc(lib, hd, w.vocab_bytes, w.vocab_offsets, w.V, out, stream)
+        assert rc == T.TRIE_OK, T.trie_last_error()
+        torch.cuda.synchronize()
+        assert hd.num_nodes == hh.num_nodes
+        assert torch.equal(out, ref), "no-alloc mask of the device-built forest differs"
+        hd.destroy()
+        hh.destroy()
+
+
 def test_noalloc_rejects_oversized_input(cuda):
     import torch
     lib = T.load_library()
