@@ -56,6 +56,13 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-dynamic", action="store_true", help="skip the dynamic per-query-set measurement")
     p.add_argument("--no-graph", action="store_true", help="run the steps eagerly instead of as CUDA graphs")
+    p.add_argument("--profile", choices=["compile", "pairwise", "lists", "lazy", "step"],
+                   help="run one part of the path alone (for profilers) and print its CUDA-event time "
+                        "instead of the JSON line")
+    p.add_argument("--requests", type=int, default=256, help="--profile lists: requests of the forest")
+    p.add_argument("--device-build", action="store_true", help="--profile lists: build the forest on the GPU")
+    p.add_argument("--cache-rows", type=int, default=0, help="--profile lazy: row cache size")
+    p.add_argument("--reps", type=int, default=5, help="--profile: repetitions")
     return p.parse_args()
 
 
@@ -330,22 +337,25 @@ def run_gpu(args, w, rank: int, world: int, dist):
 
     sbuf = [states, torch.zeros_like(states)]
 
-    def decode(logits_t, state0):
+    def decode(logits_t):
         """The decode loop: mask step 0, then per step advance by the previous
         step's token and mask this step's logits in one launch, then the last
-        advance. Returns the buffer holding the final states."""
-        state0.copy_(states0)
-        T.trie_apply_mask(h, logits_t[0], state0, stream)
-        cur = 0
+        advance. The initial states (states0) are only read; returns the
+        buffer holding the final states."""
+        T.trie_apply_mask(h, logits_t[0], states0, stream)
+        prev = states0
         for t in range(1, S):
-            T.trie_advance_apply(h, sbuf[cur], forced[t - 1], sbuf[1 - cur], logits_t[t], err, stream)
-            cur = 1 - cur
-        T.trie_advance(h, sbuf[cur], forced[S - 1], err, stream)
-        return sbuf[cur]
+            T.trie_advance_apply(h, prev, forced[t - 1], sbuf[t % 2], logits_t[t], err, stream)
+            prev = sbuf[t % 2]
+        if prev is states0:  # a one-step loop: advance a copy
+            sbuf[1].copy_(states0)
+            prev = sbuf[1]
+        T.trie_advance(h, prev, forced[S - 1], err, stream)
+        return prev
 
     def step():
         T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
-        decode(logits, sbuf[0])
+        decode(logits)
 
     # kernel-level graphs: the compile alone; the 16 applies of a step, back to
     # back over the 16 logits buffers with the states each decode step sees
@@ -478,7 +488,21 @@ def run_gpu(args, w, rank: int, world: int, dist):
     timing_src = (f"CUDA events around {reps} back-to-back replays of a graph of the {S - 1} fused "
                   f"advance+apply launches of a step (over {S - 1} logits buffers, "
                   f"{(S - 1) * B * V * elt / 1e9:.2f} GB > L2), launching stream, right after the timed region")
-    apply_bytes = B * V * elt + B * Wd * 4 + B * 4
+    # bytes an apply must move: the B x V logits written, the states, and of
+    # each state's mask row the segment summary plus the 1,024-token segments
+    # that hold an allowed token (the compile's summary lets the apply skip
+    # reading the others), averaged over the decode steps' states
+    segs = (Wd + 31) // 32
+    seg_words = (segs + 31) // 32
+    occupied = 0
+    for t in range(S):
+        sv = hist[t].long()
+        node = (sv >= 0) & (sv < N)
+        rows = mask[sv.clamp(0, N - 1)]
+        rows = torch.nn.functional.pad(rows, (0, segs * 32 - Wd)).view(B, segs, 32)
+        occ = (rows != 0).any(dim=2) & node[:, None]
+        occupied += int(occ.sum().item())  # FINISHED / DEAD rows ({EOS}) read no mask word
+    apply_bytes = B * V * elt + B * 4 + B * seg_words * 4 + (occupied / S) * 128
     fused_bytes = apply_bytes + 2 * B * 4  # + tokens read, new states written
     compile_bytes = N * Wd * 4
     apply_gbs = apply_bytes / (apply_avg * 1e-3) / 1e9
@@ -805,6 +829,19 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
         e1.record(stream)
     stream.synchronize()
     out["decode_ms"] = e0.elapsed_time(e1) / reps
+    # one list-driven apply (the fused advance + apply of a step): the B x V
+    # logits written and the states read (the rows' list entries, a few KB
+    # read from L2, are left out)
+    peak, peak_kind = peaks()
+    elt = 2 if w.dtype == "bf16" else 4
+    per_launch_us = out["decode_ms"] * 1e3 / steps
+    ab = B * V * elt + 3 * B * 4
+    out["roofline_apply_lists"] = {"bound": "hbm", "achieved": ab / (per_launch_us * 1e-6) / 1e9, "peak": peak,
+                                   "unit": "GB/s", "frac": ab / (per_launch_us * 1e-6) / 1e9 / peak,
+                                   "bytes_per_launch": ab, "us_per_launch": per_launch_us,
+                                   "peak_kind": peak_kind, "kernel": "k_apply_lists",
+                                   "timing": f"the {steps}-step decode graph (1 + {steps - 1} launches) over "
+                                             f"its launches, CUDA events around {reps} replays"}
     lt, lw = [], []
     for _ in range(reps):
         stream.synchronize()
@@ -841,17 +878,23 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
     for _ in range(reps):
         t0 = time.perf_counter()
         hh = builders["device"]()
+        stream.synchronize()  # the build returns before its last kernels have run
         bt.append(time.perf_counter() - t0)
         hh.destroy()
     out["device_forest_build_ms"] = min(bt) * 1e3
+    # the batch's initial states (the roots) go up through a pinned buffer,
+    # queued before the compile: a pageable copy would wait for the stream
+    roots_host = torch.empty(B, dtype=torch.int32).pin_memory()
+    st = [torch.empty(B, dtype=torch.int32, device=dev) for _ in range(2)]
     for kind, build in builders.items():
         et = []
         for _ in range(reps):
             t0 = time.perf_counter()
             hh = build()
             with torch.cuda.stream(stream):
+                roots_host.numpy()[:] = hh.roots()
+                st[0].copy_(roots_host, non_blocking=True)
                 T.trie_compile_lists(hh, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
-                st = [torch.as_tensor(hh.roots(), device=dev), torch.empty(B, dtype=torch.int32, device=dev)]
                 T.trie_apply_lists(hh, logits[0], st[0], stream)
                 for t in range(1, steps):
                     T.trie_advance_apply_lists(hh, st[(t - 1) % 2], forced[t - 1], st[t % 2], logits[t], err,
@@ -946,6 +989,85 @@ def W_logits(w, s, dev):
     return W.logits(w, s, device=str(dev))
 
 
+def run_profile(args, w) -> None:
+    """One part of the path alone, --reps times after one untimed call, with
+    CUDA events around the repetitions on the launching stream (eager
+    launches, no graph): the commands the ncu summaries were made with."""
+    import torch
+    from paper_2608_12574_gb300 import _build
+    from paper_2608_12574_gb300 import triemask as T
+    from paper_2608_12574_gb300 import workloads as W
+    _build.build()
+    dev = torch.device("cuda:0")
+    stream = torch.cuda.Stream(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn, what):
+        with torch.cuda.stream(stream):
+            fn()
+            e0.record(stream)
+            for _ in range(args.reps):
+                fn()
+            e1.record(stream)
+        stream.synchronize()
+        print(f"{what}: {e0.elapsed_time(e1) * 1e3 / max(1, args.reps):.2f} us per call", flush=True)
+
+    if args.profile in ("compile", "pairwise", "lazy", "step"):
+        h = T.trie_build(w.set_bytes, w.set_offsets)
+        mask = T.alloc_mask(h, w.V, dev)
+        T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, w.V, mask)
+        if args.profile == "compile":
+            timed(lambda: T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, w.V, mask, stream),
+                  f"{w.name} trie_compile_masks, {h.num_nodes} nodes")
+        elif args.profile == "pairwise":
+            timed(lambda: T.trie_compile_masks_pairwise(h, w.vocab_bytes, w.vocab_offsets, w.V, mask, stream),
+                  f"{w.name} trie_compile_masks_pairwise, {h.num_nodes} nodes")
+        else:
+            V, B, S = w.V, w.batch, w.steps
+            logits = [W.logits(w, s, device=str(dev)) for s in range(S)]
+            states = torch.zeros(B, dtype=torch.int32, device=dev)
+            err = torch.zeros(1, dtype=torch.int32, device=dev)
+            forced = torch.zeros((S, B), dtype=torch.int32, device=dev)
+            for t in range(S):  # greedy tokens, replayed below
+                x = logits[t].clone()
+                T.trie_apply_mask(h, x, states)
+                forced[t].copy_(torch.argmax(x, dim=1))
+                T.trie_advance(h, states, forced[t], err)
+            s0 = torch.zeros(B, dtype=torch.int32, device=dev)
+            sb = [torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(2)]
+            if args.profile == "lazy":
+                T.trie_lazy_init(h, w.vocab_bytes, w.vocab_offsets, V, args.cache_rows, B)
+
+                def loop():
+                    T.trie_lazy_apply(h, logits[0], s0, stream)
+                    prev = s0
+                    for t in range(1, S):
+                        T.trie_lazy_advance_apply(h, prev, forced[t - 1], sb[t % 2], logits[t], err, stream)
+                        prev = sb[t % 2]
+
+                timed(loop, f"{w.name} lazy decode loop ({S} steps, cache {args.cache_rows} rows)")
+            else:
+                def loop():
+                    T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+                    T.trie_apply_mask(h, logits[0], s0, stream)
+                    prev = s0
+                    for t in range(1, S):
+                        T.trie_advance_apply(h, prev, forced[t - 1], sb[t % 2], logits[t], err, stream)
+                        prev = sb[t % 2]
+                    T.trie_advance(h, prev, forced[S - 1], err, stream)
+
+                timed(loop, f"{w.name} step (compile + {S} decode steps, eager)")
+        return
+    full = W.dynamic_requests(args.requests)
+    if args.device_build:
+        h = T.trie_build_many_device(full.set_bytes, full.set_offsets, full.set_index, stream)
+    else:
+        h = T.trie_build_many(full.set_bytes, full.set_offsets, full.set_index)
+    timed(lambda: T.trie_compile_lists(h, full.vocab_bytes, full.vocab_offsets, full.V, stream, count=False),
+          f"{args.requests}-request forest trie_compile_lists, {h.num_nodes} nodes")
+    print(f"{T.trie_num_valid(h)} entries")
+
+
 def launch_ranks(n: int) -> int:
     """Re-runs this command as n local ranks (one process per GPU), the way
     the multi-GPU launch does: torch.distributed.run on 127.0.0.1."""
@@ -970,6 +1092,9 @@ def main():
     if "WORLD_SIZE" in os.environ and world != args.gpus:
         sys.exit(f"--gpus {args.gpus} does not match WORLD_SIZE {world} of the launch")
     w = W.config(args.config)
+    if args.profile:
+        run_profile(args, w)
+        return
     if args.impl == "reference":
         if rank == 0:
             run_reference(args, w)

@@ -48,7 +48,10 @@
  * passes (mask, states, tokens, logits, error counter). The mask passed to
  * trie_compile_masks must stay allocated and unchanged while the handle is
  * used by trie_apply_mask (the handle keeps a non-owning pointer to it).
- * A handle's device memory (trie arrays, valid lists, lazy rows) and the
+ * A handle's device memory (trie arrays and per-node tables, 123 B per
+ * node, plus a transition table of at least 128 B per node for a single trie;
+ * the dense compile's hit buffer, 129 B per node, allocated by the
+ * handle's first trie_compile_masks; valid lists; lazy rows) and the
  * scratch of trie_build_many_device come from a memory pool per device that
  * the library creates on first use; up to 8 GiB of memory freed by
  * trie_destroy stays reserved in it for later handles until the process
@@ -119,7 +122,12 @@ int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t 
  * NVLink-C2C), a kernel reads the strings straight from the caller's arrays;
  * elsewhere they are copied first (TRIEMASK_HOST_READ=copy in the
  * environment forces the copies). The offsets are checked on the device.
- * Host-synchronous: returns once the forest is complete on `stream`. Such a
+ * Returns once the node count and the roots are known on the host (read back
+ * after the level insertion; the caller's arrays have been read by then):
+ * the last kernels (the breadth-first layout, child links and per-node
+ * tables) are still queued on `stream`, so use the handle on `stream` or
+ * after synchronising it (calls that copy arrays back synchronise the device
+ * first); an error in those kernels surfaces on a later call. Such a
  * forest has no transition table: trie_advance and the fused calls walk the
  * tokens' bytes. Calls that need the host arrays (trie_get_csr,
  * trie_lazy_init) copy them back once. Strings longer than 1024 bytes, more
@@ -137,6 +145,9 @@ int32_t trie_num_nodes(trie_t h);
 
 /* Root node id of set i (0 for a single trie); -1 if i is out of range. */
 int32_t trie_root(trie_t h, int32_t i);
+/* All roots at once: roots (host int32[trie_num_sets(h)]) receives the root
+ * node id of every set, in set order (a forest of many sets, in one call). */
+int trie_copy_roots(trie_t h, int32_t *roots);
 
 /* Number of sets in the handle (1 for trie_build). */
 int32_t trie_num_sets(trie_t h);
@@ -427,9 +438,10 @@ int trie_destroy(trie_t h);
 
 /* Release the handle without synchronising: its device memory is freed in
  * stream order on `stream` (it returns to the library's pool once the work
- * queued on `stream` so far has completed), and its host arrays, which a
- * queued upload may still be reading, by a host callback queued on `stream`
- * after that work (a handle that never reached a device: at once). Every
+ * queued on `stream` so far has completed); its host arrays, which a queued
+ * upload may still be reading, once an event recorded on `stream` now has
+ * completed: a later trie_destroy_async or trie_build* call frees them (a
+ * handle that never reached a device: at once). Every
  * use of the handle on the device must be on `stream` or ordered before the
  * work queued on it now (for example by an event); the handle must not be
  * used by the host after the call. A server that builds a trie per request

@@ -203,8 +203,6 @@ int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream, bool wit
     size_t trans_slots = with_trans ? 16 : 0;  // >= 8 per node, a power of two
     while (with_trans && trans_slots < 8 * n) trans_slots <<= 1;
     const size_t o_trans = L.add(sizeof(ulonglong2) * trans_slots);
-    const size_t o_hits = L.add(sizeof(int2) * tmk::kHitSlots * n);  // compile scratch (probe -> scatter)
-    const size_t o_hcnt = L.add(n);
     void *base = nullptr;
     const int rc = pool_alloc(dev, L.total, stream, &base, "the trie");
     if (rc != TRIE_OK) return rc;
@@ -221,8 +219,6 @@ int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream, bool wit
     h->dev.anc = reinterpret_cast<int4 *>(b + o_anc);
     h->dev.trans = with_trans ? reinterpret_cast<ulonglong2 *>(b + o_trans) : nullptr;
     h->dev.trans_mask = with_trans ? uint32_t(trans_slots - 1) : 0u;
-    h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
-    h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
     return TRIE_OK;
 }
 
@@ -255,7 +251,9 @@ int ensure_device_trie(trie_t h, int dev, cudaStream_t stream) {
     }
     const tmk::HostTrie &t = h->host;
     const size_t n = size_t(t.n);
-    int rc = alloc_device_trie(h, dev, n, stream, true);
+    // a transition table for a single trie; a forest's per-request sets are
+    // decoded for a few steps, where byte walks cost less than the table
+    int rc = alloc_device_trie(h, dev, n, stream, t.roots.size() <= 1);
     if (rc != TRIE_OK) return rc;
     if (host_memory_direct(dev)) {
         // the kernel reads the handle's host arrays itself: a pageable copy
@@ -420,6 +418,11 @@ cudaMemPool_t tmk::device_pool(int dev) {
 int tmk::ensure_host_arrays(trie_s *h) {
     std::lock_guard<std::mutex> lk(h->mu);
     if (h->host_arrays) return TRIE_OK;
+    {  // the build's last kernels may still be queued (on the caller's stream)
+        DeviceGuard g(h->dev.device);
+        const cudaError_t e = cudaDeviceSynchronize();
+        if (e != cudaSuccess) return fail_cuda(e, "waiting for the forest build");
+    }
     tmk::HostTrie &t = h->host;
     const size_t n = size_t(t.n);
     try {
@@ -458,7 +461,10 @@ extern "C" {
 
 const char *trie_last_error(void) { return g_last_error.c_str(); }
 
+static void sweep_retired();
+
 int trie_build(const uint8_t *bytes, const int64_t *offsets, int32_t K, trie_t *out) {
+    sweep_retired();
     if (!out) return fail(TRIE_EINVAL, "out is NULL");
     *out = nullptr;
     if (K < 0) return fail(TRIE_EINVAL, "K must be >= 0");
@@ -479,6 +485,7 @@ int trie_build(const uint8_t *bytes, const int64_t *offsets, int32_t K, trie_t *
 
 int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets,
                     int32_t M, trie_t *out) {
+    sweep_retired();
     if (!out) return fail(TRIE_EINVAL, "out is NULL");
     *out = nullptr;
     if (M < 1) return fail(TRIE_EINVAL, "M must be >= 1");
@@ -504,6 +511,7 @@ int trie_build_many(const uint8_t *bytes, const int64_t *offsets, const int32_t 
 
 int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const int32_t *set_offsets, int32_t M,
                            cudaStream_t stream, trie_t *out) {
+    sweep_retired();
     if (!out) return fail(TRIE_EINVAL, "out is NULL");
     *out = nullptr;
     if (M < 1) return fail(TRIE_EINVAL, "M must be >= 1");
@@ -566,7 +574,10 @@ int trie_build_many_device(const uint8_t *bytes, const int64_t *offsets, const i
         delete h;
         return rc;
     }
-    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    // no synchronisation here: the node count and roots are on the host, the
+    // caller's arrays have been read, and the last kernels (breadth-first
+    // layout, child links, per-node tables) finish on `stream` while the host
+    // goes on (a later call on `stream` is ordered after them)
     if (e != cudaSuccess) {
         cudaGetLastError();
         pool_free(h->dev.base);
@@ -586,6 +597,13 @@ int32_t trie_num_sets(trie_t h) { return h ? int32_t(h->host.roots.size()) : -1;
 int32_t trie_root(trie_t h, int32_t i) {
     if (!h || i < 0 || i >= int32_t(h->host.roots.size())) return -1;
     return h->host.roots[size_t(i)];
+}
+
+int trie_copy_roots(trie_t h, int32_t *roots) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!roots && !h->host.roots.empty()) return fail(TRIE_EINVAL, "roots is NULL");
+    std::copy(h->host.roots.begin(), h->host.roots.end(), roots);
+    return TRIE_OK;
 }
 
 int64_t trie_num_chars(trie_t h) { return h ? h->host.n_chars : -1; }
@@ -608,6 +626,48 @@ int trie_get_csr(trie_t h, int32_t *parent, uint8_t *label, uint8_t *terminal, i
     return TRIE_OK;
 }
 
+// The dense compile's hit buffer (the probe's records for the scatter), on
+// the first dense compile of the handle: the valid lists and the lazy rows
+// never need it, so a forest compiled to lists does not hold 129 B per node.
+static int ensure_hits(trie_t h, int dev, cudaStream_t stream) {
+    std::lock_guard<std::mutex> lk(h->mu);
+    if (h->dev.hits_base) return TRIE_OK;
+    const size_t n = size_t(h->host.n);
+    Layout L;
+    const size_t o_hits = L.add(sizeof(int2) * tmk::kHitSlots * n);
+    const size_t o_hcnt = L.add(n);
+    void *base = nullptr;
+    const int rc = pool_alloc(dev, L.total, stream, &base, "the compile's hit buffer");
+    if (rc != TRIE_OK) return rc;
+    char *b = static_cast<char *>(base);
+    h->dev.hits_base = base;
+    h->dev.hits = reinterpret_cast<int2 *>(b + o_hits);
+    h->dev.hit_count = reinterpret_cast<uint8_t *>(b + o_hcnt);
+    return TRIE_OK;
+}
+
+// The segment summary of the dense mask (bit g of row r set iff the row allows
+// a token of the 1,024-token segment g), which lets the apply skip reading
+// the mask words of empty segments; none when it would exceed 256 MB.
+static uint32_t *ensure_seg(trie_t h, int dev, cudaStream_t stream, int32_t words) {
+    const int64_t need = int64_t(h->host.n) * words;
+    if (need * 4 > (int64_t(256) << 20)) return nullptr;
+    std::lock_guard<std::mutex> lk(h->mu);
+    if (h->dev.seg_cap < need) {
+        pool_free(h->dev.seg_any);  // an earlier apply may still read it
+        h->dev.seg_any = nullptr;
+        h->dev.seg_cap = 0;
+        void *p = nullptr;
+        if (pool_alloc(dev, size_t(need) * 4, stream, &p, "the mask's segment summary") != TRIE_OK) {
+            cudaGetLastError();
+            return nullptr;  // the compile and the apply work without it
+        }
+        h->dev.seg_any = static_cast<uint32_t *>(p);
+        h->dev.seg_cap = need;
+    }
+    return h->dev.seg_any;
+}
+
 int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
                        uint32_t *d_mask, cudaStream_t stream) {
     if (!h) return fail(TRIE_EINVAL, "handle is NULL");
@@ -620,13 +680,18 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     std::shared_ptr<tmk::DevVocab> voc;
     if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
     if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
+    if ((rc = ensure_hits(h, dev, stream)) != TRIE_OK) return rc;
     const int64_t W = (int64_t(V) + 31) / 32;
     const int32_t n = h->host.n;
     const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
     bool fill_trans;
     if ((rc = prepare_trans(h, voc, sms, stream, &fill_trans)) != TRIE_OK) return rc;
-    cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, fill_trans, stream);
+    const int32_t seg_words = int32_t(((W + 31) / 32 + 31) / 32);
+    uint32_t *seg = ensure_seg(h, dev, stream, seg_words);
+    bool seg_written = false;
+    cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, fill_trans, stream, seg,
+                                              seg_words, &seg_written);
     if (e != cudaSuccess) return fail_cuda(e, "mask compile launch");
     std::lock_guard<std::mutex> lk(h->mu);
     h->trans_vocab = voc;
@@ -634,6 +699,8 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     h->vocab = voc;
     h->mask = d_mask;
     h->mask_V = V;
+    h->mask_seg = seg_written ? seg : nullptr;
+    h->mask_seg_words = seg_words;
     return TRIE_OK;
 }
 
@@ -673,12 +740,16 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
     uint32_t *mask;
     int32_t mV;
     bool use_trans;
+    const uint32_t *seg;
+    int32_t seg_words;
     {
         std::lock_guard<std::mutex> lk(h->mu);
         voc = h->vocab;
         mask = h->mask;
         mV = h->mask_V;
         use_trans = h->trans_vocab == voc;
+        seg = h->mask_seg;
+        seg_words = h->mask_seg_words;
     }
     if (!mask || !voc) return fail(TRIE_ESTATE, "trie_advance_apply before trie_compile_masks on this handle");
     if (V != mV || V != voc->V) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
@@ -689,7 +760,8 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
     cudaError_t e = tmk::launch_advance_apply(h->dev, h->host.n, *voc, use_trans, d_states_in, d_tokens,
-                                              d_states_out, d_err, d_logits, dtype, mask, B, num_sms(dev), stream);
+                                              d_states_out, d_err, d_logits, dtype, mask, B, num_sms(dev), stream,
+                                              seg, seg_words);
     if (e != cudaSuccess) return fail_cuda(e, "advance-apply launch");
     return TRIE_OK;
 }
@@ -702,10 +774,14 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
     if (B > 0 && (!d_logits || !d_states)) return fail(TRIE_EINVAL, "d_logits / d_states is NULL");
     uint32_t *mask;
     int32_t mV;
+    const uint32_t *seg;
+    int32_t seg_words;
     {
         std::lock_guard<std::mutex> lk(h->mu);
         mask = h->mask;
         mV = h->mask_V;
+        seg = h->mask_seg;
+        seg_words = h->mask_seg_words;
     }
     if (!mask) return fail(TRIE_ESTATE, "trie_apply_mask before trie_compile_masks on this handle");
     if (V != mV) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
@@ -715,9 +791,61 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
     int dev, rc;
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
-    cudaError_t e = tmk::launch_apply(d_logits, dtype, mask, d_states, B, V, h->host.n, num_sms(dev), stream);
+    cudaError_t e = tmk::launch_apply(d_logits, dtype, mask, d_states, B, V, h->host.n, num_sms(dev), stream, seg,
+                                      seg_words);
     if (e != cudaSuccess) return fail_cuda(e, "apply launch");
     return TRIE_OK;
+}
+
+// Blocks of released valid lists kept for the next handles' lists: a fresh
+// block from the pool cost 0.3-0.4 ms of host time for the 4.8 M-node forest
+// (381 MB), more than the list compile's kernels. A block is reused once the
+// event recorded at its release (if any) has completed; at most
+// kSpareListBlocks are kept per device, the rest go back to the pool.
+constexpr size_t kSpareListBlocks = 2;
+struct SpareBlock {
+    int dev;
+    void *p;
+    size_t bytes;
+    cudaEvent_t ready;  // null: free for use at once
+};
+static std::mutex g_spare_mu;
+static std::vector<SpareBlock> &g_spare = *new std::vector<SpareBlock>();
+
+static void *take_spare_block(int dev, size_t bytes) {
+    std::lock_guard<std::mutex> lk(g_spare_mu);
+    for (size_t i = 0; i < g_spare.size(); i++) {
+        SpareBlock &b = g_spare[i];
+        if (b.dev != dev || b.bytes < bytes || b.bytes > 2 * bytes) continue;
+        if (b.ready) {
+            const cudaError_t q = cudaEventQuery(b.ready);
+            if (q == cudaErrorNotReady) continue;
+            cudaGetLastError();
+            cudaEventDestroy(b.ready);
+        }
+        void *p = b.p;
+        g_spare.erase(g_spare.begin() + long(i));
+        return p;
+    }
+    return nullptr;
+}
+
+// Takes a block of `bytes` on device dev (current) whose last use is queued
+// before `ready` (null: none pending); frees it in stream order on `stream`
+// when the cache is full.
+static void give_spare_block(int dev, void *p, size_t bytes, cudaEvent_t ready, cudaStream_t stream) {
+    {
+        std::lock_guard<std::mutex> lk(g_spare_mu);
+        size_t held = 0;
+        for (const SpareBlock &b : g_spare) held += b.dev == dev;
+        if (held < kSpareListBlocks) {
+            g_spare.push_back(SpareBlock{dev, p, bytes, ready});
+            return;
+        }
+    }
+    if (ready) cudaEventDestroy(ready);
+    cudaFreeAsync(p, stream);
+    cudaGetLastError();
 }
 
 // Token buffers of up to this many entries (1 GiB) are sized by the bound on
@@ -824,14 +952,22 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
     const int32_t n = h->host.n;
     tmk::DevLists &L = h->lists;
-    if (!L.base) {  // per-row counts, offsets and scan scratch
+    const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
+    // a node is the end of at most one path of each length up to lmax, each
+    // spelled by at most rt_mult ids, plus EOS. While that bound is modest the
+    // token buffer is sized by it and nothing is read back; otherwise the
+    // exact total is read back between the two walks (host-synchronous).
+    const int64_t bound = int64_t(n) * (int64_t(lmax) * voc->rt_mult + 1);
+    const bool by_bound = bound <= std::max<int64_t>(kListBoundEntries, L.tok_cap);
+    if (!L.base) {  // per-row counts, offsets, scan scratch (and a first token buffer, in one block)
         Layout lay;
         const size_t o_cnt = lay.add(sizeof(int32_t) * size_t(n));
         const size_t o_off = lay.add(sizeof(int64_t) * (size_t(n) + 1));
         const size_t o_tile = lay.add(sizeof(int64_t) * (size_t(n) / 4096 + 2));
         const size_t o_tot = lay.add(sizeof(int64_t));
-        void *base = nullptr;
-        if ((rc = pool_alloc(dev, lay.total, stream, &base, "the valid lists")) != TRIE_OK) return rc;
+        const size_t o_tok = by_bound ? lay.add(sizeof(int32_t) * size_t(std::max<int64_t>(bound, 1))) : 0;
+        void *base = take_spare_block(dev, lay.total);
+        if (!base && (rc = pool_alloc(dev, lay.total, stream, &base, "the valid lists")) != TRIE_OK) return rc;
         cudaEvent_t done = nullptr;
         cudaError_t e = cudaEventCreateWithFlags(&done, cudaEventDisableTiming);
         if (e != cudaSuccess) {
@@ -840,24 +976,23 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         }
         char *b = static_cast<char *>(base);
         L.base = base;
+        L.base_bytes = lay.total;
         L.done = done;
         L.count = reinterpret_cast<int32_t *>(b + o_cnt);
         L.off = reinterpret_cast<int64_t *>(b + o_off);
         L.tile_sum = reinterpret_cast<int64_t *>(b + o_tile);
         L.total = reinterpret_cast<int64_t *>(b + o_tot);
+        if (by_bound) {
+            L.toks = reinterpret_cast<int32_t *>(b + o_tok);
+            L.tok_cap = std::max<int64_t>(bound, 1);
+            L.toks_separate = false;
+        }
     }
-    const int32_t lmax = std::min(voc->max_len, h->host.max_depth);
     const int sms = num_sms(dev);
-    // a node is the end of at most one path of each length up to lmax, each
-    // spelled by at most rt_mult ids, plus EOS. While that bound is modest the
-    // token buffer is sized by it and nothing is read back; otherwise the
-    // exact total is read back between the two walks (host-synchronous).
-    const int64_t bound = int64_t(n) * (int64_t(lmax) * voc->rt_mult + 1);
-    const bool by_bound = bound <= std::max<int64_t>(kListBoundEntries, L.tok_cap);
     auto grow = [&](int64_t need) -> int {
         if (need <= L.tok_cap) return TRIE_OK;
-        pool_free(L.toks);  // earlier apply calls may still read it
-        L.toks = nullptr;
+        if (L.toks_separate) pool_free(L.toks);  // earlier apply calls may still read it
+        L.toks = nullptr;                         // (a buffer inside the block at base stays there)
         L.tok_cap = 0;
         void *toks = nullptr;
         int r = pool_alloc(dev, sizeof(int32_t) * size_t(std::max<int64_t>(need, 1)), stream, &toks,
@@ -865,6 +1000,7 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         if (r != TRIE_OK) return r;
         L.toks = static_cast<int32_t *>(toks);
         L.tok_cap = need;
+        L.toks_separate = true;
         return TRIE_OK;
     };
     auto failed = [&](int r) {
@@ -1229,16 +1365,56 @@ int trie_destroy(trie_t h) {
         DeviceGuard g(h->lazy.device);
         pool_free(h->lazy.base);
     }
-    if (h->dev.base || h->lists.base || h->lists.toks) {
+    if (h->dev.base || h->lists.base) {
         DeviceGuard g(h->dev.device);
         // after the work on the device that may still read these
-        pool_free(h->lists.toks);
-        pool_free(h->lists.base);
+        if (h->lists.toks_separate) pool_free(h->lists.toks);
+        if (h->lists.base) {
+            cudaDeviceSynchronize();  // no queued work still uses the block
+            give_spare_block(h->dev.device, h->lists.base, h->lists.base_bytes, nullptr, 0);
+        }
+        pool_free(h->dev.hits_base);
+        pool_free(h->dev.seg_any);
         pool_free(h->dev.base);
         if (h->lists.done) cudaEventDestroy(h->lists.done);
     }
     delete h;
     return TRIE_OK;
+}
+
+// Handles released by trie_destroy_async whose host arrays may still be read
+// by queued work: each waits for its event, and every release (and every
+// build) frees those whose event has completed.
+static std::mutex g_retired_mu;
+static std::vector<std::pair<cudaEvent_t, trie_t>> &g_retired =
+    *new std::vector<std::pair<cudaEvent_t, trie_t>>();
+
+static void sweep_retired() {
+    std::vector<trie_t> done;
+    {
+        std::lock_guard<std::mutex> lk(g_retired_mu);
+        size_t keep = 0;
+        for (size_t i = 0; i < g_retired.size(); i++) {
+            const cudaError_t q = cudaEventQuery(g_retired[i].first);
+            if (q == cudaErrorNotReady) {
+                g_retired[keep++] = g_retired[i];
+                continue;
+            }
+            cudaGetLastError();
+            cudaEventDestroy(g_retired[i].first);
+            done.push_back(g_retired[i].second);
+        }
+        g_retired.resize(keep);
+    }
+    for (trie_t h : done) delete h;
+}
+
+static void retire_handle(trie_t h, cudaEvent_t ev) {
+    {
+        std::lock_guard<std::mutex> lk(g_retired_mu);
+        g_retired.emplace_back(ev, h);
+    }
+    sweep_retired();
 }
 
 int trie_destroy_async(trie_t h, cudaStream_t stream) {
@@ -1263,8 +1439,20 @@ int trie_destroy_async(trie_t h, cudaStream_t stream) {
     }
     if (h->dev.base || h->lists.base || h->lists.toks) {
         DeviceGuard g(h->dev.device);
-        free_on(h->lists.toks);
-        free_on(h->lists.base);
+        if (h->lists.toks_separate) free_on(h->lists.toks);
+        if (h->lists.base) {  // kept for a later handle once the queued work is done
+            cudaEvent_t ev = nullptr;
+            if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess &&
+                cudaEventRecord(ev, stream) == cudaSuccess) {
+                give_spare_block(h->dev.device, h->lists.base, h->lists.base_bytes, ev, stream);
+            } else {
+                cudaGetLastError();
+                if (ev) cudaEventDestroy(ev);
+                free_on(h->lists.base);
+            }
+        }
+        free_on(h->dev.hits_base);
+        free_on(h->dev.seg_any);
         free_on(h->dev.base);
         // the event may still be pending: CUDA defers its destruction
         if (h->lists.done) cudaEventDestroy(h->lists.done);
@@ -1274,16 +1462,23 @@ int trie_destroy_async(trie_t h, cudaStream_t stream) {
         return rc;
     }
     // the host arrays (which an upload kernel may still be reading) go once
-    // the work queued on the stream so far has run
+    // the work queued on the stream so far has run: an event marks that
+    // point and a later call frees the handle once the event has completed
+    // (no stream callback, which would hold up the stream's later work)
     DeviceGuard g(dev);
-    cudaError_t e = cudaLaunchHostFunc(stream, [](void *p) { delete static_cast<trie_t>(p); }, h);
+    cudaEvent_t ev = nullptr;
+    cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventRecord(ev, stream);
     if (e != cudaSuccess) {
         cudaGetLastError();
+        if (ev) cudaEventDestroy(ev);
         cudaStreamSynchronize(stream);
         cudaGetLastError();
         delete h;
         if (rc == TRIE_OK) rc = fail_cuda(e, "queueing the release of the handle's host memory");
+        return rc;
     }
+    retire_handle(h, ev);
     return rc;
 }
 

@@ -125,6 +125,8 @@ struct PatchArgs {
     ulonglong2 *trans;         // transition table (row, token) -> end node, or null
     uint32_t trans_mask;       // slots - 1
     int32_t trans_fill;        // the probe inserts every transition it finds
+    uint32_t *seg_any;         // [n_nodes * seg_words]: bit g of row r = some token of segment g allowed, or null
+    int32_t seg_words;         // words per row of seg_any (segments of 1,024 tokens)
 };
 
 // Transition table: open addressing over 16-byte slots {key, end node};
@@ -159,6 +161,14 @@ __device__ __forceinline__ void trans_insert(ulonglong2 *tab, uint32_t mask, int
 }
 
 constexpr int kHitOverflow = 255;
+
+// Masks up to this size are compiled in two kernels (fill, then a search that
+// ORs its hits itself): at K = 100 (5.5 MB) 10.4 us against 16.4 us for three
+// kernels. Larger ones by the search beside the fill and a scatter of the
+// recorded hits: there the search starts only once the fill's last wave is
+// running and no longer hides under it (K = 1,000, 184 MB: 37.2 us against
+// 33.4 us).
+constexpr int64_t kSmallMaskBytes = int64_t(32) << 20;
 
 // Read-only arrays the probe reads, for a bulk L2 prefetch.
 struct Prefetch {
@@ -333,10 +343,17 @@ __global__ void k_trie_links(const int32_t *__restrict__ parent, const uint8_t *
     }
 }
 
-// Per-node tables of the probe (one thread per node, climbing at most 16
-// parents): the last 16 edge labels into m, min(depth, 16), and the 16
-// nearest ancestors. Siblings and cousins are neighbours in breadth-first
-// order, so a warp's climbs read neighbouring entries.
+// Per-node tables of the probe and of the list walk (one thread per node,
+// climbing at most 16 parents): the last 16 edge labels into m (byte i = the
+// label i levels up, 0 past the root), min(depth, 16), and the 16 nearest
+// ancestors (-1 past the root), stored as four 16-byte rows. Siblings and
+// cousins are neighbours in breadth-first order, so a warp's climbs read
+// neighbouring entries of the parent and label arrays, which stay in L2.
+// (Two alternatives measured slower on the 4.77 M-node forest: rows built by
+// doubling from the rows of the ancestors 4, 8 and 12 levels up, 230 us, whose
+// reads of the 64-byte ancestor rows come from DRAM; and two climbs per thread
+// storing each ancestor as found, 404 us, whose 4-byte stores multiply the L2
+// write traffic. This form: 114 us.)
 constexpr int kTableThreads = 256;
 __global__ void __launch_bounds__(kTableThreads) k_trie_tables(const int32_t *__restrict__ parent,
                                                                const uint8_t *__restrict__ label, int32_t n,
@@ -552,6 +569,27 @@ __device__ __forceinline__ void set_mask_bit(const PatchArgs &a, int32_t row, in
     atomicOr(a.mask + int64_t(row) * a.W + (t >> 5), 1u << (t & 31));
 }
 
+// The bit, and the row's segment bit in the summary the apply reads first
+// (a 1,024-token segment whose bit is clear holds no allowed token).
+__device__ __forceinline__ void set_mask_bit_seg(const PatchArgs &a, int32_t row, int32_t t) {
+    set_mask_bit(a, row, t);
+    if (a.seg_any) {  // most hits of a row share a few segments: set a bit only once
+        const int32_t g = t >> 10;
+        uint32_t *w = a.seg_any + int64_t(row) * a.seg_words + (g >> 5);
+        const uint32_t bit = 1u << (g & 31);
+        if (!(*reinterpret_cast<volatile uint32_t *>(w) & bit)) atomicOr(w, bit);
+    }
+}
+
+// Zeroes the segment summary (grid-stride; called by the probe, which runs
+// before the scatter that sets it).
+__device__ __forceinline__ void clear_seg_any(const PatchArgs &a) {
+    if (!a.seg_any) return;
+    const int64_t n = int64_t(a.n_nodes) * a.seg_words;
+    for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += int64_t(gridDim.x) * blockDim.x)
+        a.seg_any[i] = 0u;
+}
+
 // Fill-then-patch form (two kernels): climbs and probes overlap the fill,
 // the bits are set once the fill has completed.
 __global__ void __launch_bounds__(kPatchThreads) k_mask_patch(PatchArgs a) {
@@ -576,9 +614,10 @@ __global__ void __launch_bounds__(kPatchThreads) k_mask_patch(PatchArgs a) {
 // its tables into L2 (its dependent loads then hit L2 while the fill
 // saturates HBM) and only then lets the fill launch, which runs beside it.
 __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Prefetch pf) {
-    pdl_wait();  // an earlier scatter may still read the hit buffer
+    pdl_wait();  // an earlier scatter may still read the hit buffer (an apply, the summary)
     if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
     pdl_launch_dependents();
+    clear_seg_any(a);
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
         int32_t c = 0;
@@ -601,9 +640,17 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
 // order (EOS, lengths 1..16) into the node's slots, so the hit buffer is
 // that of k_mask_probe. Only for vocabularies with the per-slot payload (at
 // most one token per suffix) and tokens of at most 16 bytes.
+//
+// kOr: the two-kernel form for small masks. The zero fill runs first; this
+// kernel searches (read-only tables) while the fill runs, waits for it, and
+// ORs its hits into the mask itself: no hit buffer, no scatter launch.
+template <bool kOr>
 __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs a, Prefetch pf) {
-    pdl_wait();  // an earlier scatter may still read the hit buffer
-    if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
+    if (!kOr) {
+        pdl_wait();  // an earlier scatter may still read the hit buffer (an apply, the summary)
+        if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
+        clear_seg_any(a);
+    }
     pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int half = lane & 1;
@@ -645,18 +692,23 @@ __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs 
         const int32_t c0 = __shfl_sync(0xffffffffu, c, lane & ~1);
         const int32_t c1 = __shfl_sync(0xffffffffu, c, lane | 1);
         if (!valid) continue;
+        if (kOr) pdl_wait();  // the fill of this mask (and of the transition table) is complete
         int2 *slot = a.hits + int64_t(m) * kHitSlots;
         int32_t s = half ? c0 : 0;
         auto rec = [&](int32_t row, int32_t tok) {
-            if (s < kHitSlots) slot[s] = make_int2(row, tok);
-            s++;
+            if (kOr) {
+                set_mask_bit(a, row, tok);
+            } else {
+                if (s < kHitSlots) slot[s] = make_int2(row, tok);
+                s++;
+            }
             if (a.trans_fill && tok != a.eos) trans_insert(a.trans, a.trans_mask, row, tok, m);
         };
         if (eos) rec(m, a.eos);
 #pragma unroll
         for (int i = 0; i < 8; i++)
             if (found[i] >= 0) rec(anc_at(an, k0 + i), found[i]);
-        if (half == 0) a.hit_count[m] = uint8_t(c0 + c1 > kHitSlots ? kHitOverflow : c0 + c1);
+        if (!kOr && half == 0) a.hit_count[m] = uint8_t(c0 + c1 > kHitSlots ? kHitOverflow : c0 + c1);
     }
 }
 
@@ -666,7 +718,7 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_scatter(PatchArgs a) 
     pdl_wait();  // fill complete, and through it the probe
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        auto emit = [&](int32_t row, int32_t t) { set_mask_bit(a, row, t); };
+        auto emit = [&](int32_t row, int32_t t) { set_mask_bit_seg(a, row, t); };
         const int32_t c = a.hit_count[m];
         if (c == kHitOverflow) {
             node_hits_window(a, m, emit);
@@ -829,6 +881,18 @@ __device__ __forceinline__ uint32_t row_word(const uint32_t *__restrict__ mask, 
     return (w == (eos >> 5)) ? (1u << (eos & 31)) : 0u;
 }
 
+// Mask word w of state s's row, reading the row only when the segment
+// summary (if any) says segment seg holds an allowed token.
+__device__ __forceinline__ uint32_t seg_row_word(const uint32_t *__restrict__ mask,
+                                                 const uint32_t *__restrict__ seg_any, int32_t seg_words,
+                                                 int32_t s, int32_t n_nodes, int64_t W, int32_t seg, int64_t w,
+                                                 int32_t eos) {
+    if (seg_any && s >= 0 && s < n_nodes &&
+        !((__ldg(seg_any + int64_t(s) * seg_words + (seg >> 5)) >> (seg & 31)) & 1u))
+        return 0u;
+    return row_word(mask, s, n_nodes, W, w, eos);
+}
+
 // -inf pattern of 16 bytes of logits.
 template <int kElt>
 __device__ __forceinline__ uint4 ninf16() {
@@ -905,7 +969,8 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
                                                              const uint32_t *__restrict__ mask,
                                                              const int32_t *__restrict__ states, int32_t B,
                                                              int32_t V, int64_t W, int32_t n_nodes,
-                                                             int32_t segs) {
+                                                             int32_t segs, const uint32_t *__restrict__ seg_any,
+                                                             int32_t seg_words) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     __shared__ __align__(128) uint4 tile[kSegChunks];
     init_ninf_tile<kElt>(tile);
@@ -915,7 +980,8 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
     const int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
     if (item >= B * segs) return;  // uniform per warp
     const int32_t b = item / segs, seg = item - b * segs;
-    const uint32_t word = row_word(mask, __ldg(states + b), n_nodes, W, int64_t(seg) * 32 + lane, V - 1);
+    const uint32_t word = seg_row_word(mask, seg_any, seg_words, __ldg(states + b), n_nodes, W, seg,
+                                       int64_t(seg) * 32 + lane, V - 1);
     const int64_t row_chunks = int64_t(V) / (16 / kElt);
     write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
                         tile);
@@ -935,7 +1001,9 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
                                                                      const int32_t *__restrict__ tokens,
                                                                      int32_t *__restrict__ states_out,
                                                                      int32_t *__restrict__ err, int32_t B,
-                                                                     int64_t W, int32_t segs, int32_t parts) {
+                                                                     int64_t W, int32_t segs, int32_t parts,
+                                                                     const uint32_t *__restrict__ seg_any,
+                                                                     int32_t seg_words) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     __shared__ __align__(128) uint4 tile[kSegChunks];
     __shared__ int32_t next_state;
@@ -958,7 +1026,8 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
     const int lane = threadIdx.x & 31;
     const int32_t seg = part * (kApplyThreads / 32) + int32_t(threadIdx.x >> 5);
     if (seg >= segs) return;  // uniform per warp
-    const uint32_t word = row_word(mask, next_state, aa.n_nodes, W, int64_t(seg) * 32 + lane, aa.V - 1);
+    const uint32_t word = seg_row_word(mask, seg_any, seg_words, next_state, aa.n_nodes, W, seg,
+                                       int64_t(seg) * 32 + lane, aa.V - 1);
     const int64_t row_chunks = int64_t(aa.V) / (16 / kElt);
     write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
                         tile);
@@ -1707,6 +1776,8 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.trans = t.trans;
     a.trans_mask = t.trans_mask;
     a.trans_fill = 0;
+    a.seg_any = nullptr;
+    a.seg_words = 0;
     return a;
 }
 
@@ -1722,11 +1793,16 @@ inline int grid_for(int64_t work, int64_t per_block, int64_t cap) {
 // it (per-slot payload, tokens of at most 16 bytes), else one per node. Its
 // grid is resident at once (so that every CTA passes its entry wait and lets
 // the fill launch right away); nodes in a grid-stride loop.
-cudaError_t launch_probe(const PatchArgs &a, const Prefetch &pf, int num_sms, cudaStream_t st) {
+bool pair_probe(const PatchArgs &a, int num_sms) {
     const int64_t resident = int64_t(num_sms) * 4 * kPatchThreads;
-    if (a.ht_pay && a.lmax <= kMaxClimb && 2 * int64_t(a.n_nodes) * 2 <= resident)
-        return launch_pdl(k_mask_probe_pair, grid_for(2 * int64_t(a.n_nodes), kPatchThreads, int64_t(num_sms) * 4),
-                          kPatchThreads, st, a, pf);
+    return a.ht_pay && a.lmax <= kMaxClimb && 2 * int64_t(a.n_nodes) * 2 <= resident;
+}
+
+cudaError_t launch_probe(const PatchArgs &a, const Prefetch &pf, int num_sms, cudaStream_t st) {
+    if (pair_probe(a, num_sms))
+        return launch_pdl(k_mask_probe_pair<false>,
+                          grid_for(2 * int64_t(a.n_nodes), kPatchThreads, int64_t(num_sms) * 4), kPatchThreads, st,
+                          a, pf);
     return launch_pdl(k_mask_probe, grid_for(a.n_nodes, kPatchThreads, int64_t(num_sms) * 4), kPatchThreads, st, a,
                       pf);
 }
@@ -1776,9 +1852,11 @@ cudaError_t launch_vocab_pay(const DevVocab &v, uint4 *pay, int num_sms, cudaStr
 }
 
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                                 uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st) {
+                                 uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st,
+                                 uint32_t *seg_any, int32_t seg_words, bool *seg_written) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
     a.trans_fill = fill_trans && t.trans;
+    *seg_written = false;
     Prefetch pf;
     pf.count = 0;
     auto add = [&](const void *p, uint64_t n) {
@@ -1786,6 +1864,17 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
         pf.bytes[pf.count] = n;
         pf.count++;
     };
+    const int64_t n_words = int64_t(n_nodes) * W;
+    if (pair_probe(a, num_sms) && n_words * 4 <= kSmallMaskBytes) {
+        // small masks: the zero fill, then the search ORing its hits itself
+        cudaError_t e = launch_mask_fill(mask, n_words, num_sms, st);
+        if (e != cudaSuccess) return e;
+        return launch_pdl(k_mask_probe_pair<true>, grid_for(2 * int64_t(n_nodes), kPatchThreads, int64_t(num_sms) * 4),
+                          kPatchThreads, st, a, pf);
+    }
+    a.seg_any = seg_any;  // the probe clears it, the scatter sets it
+    a.seg_words = seg_words;
+    *seg_written = seg_any != nullptr;
     const uint64_t S = uint64_t(v.ht_mask) + 1, nn = uint64_t(n_nodes), nv = uint64_t(v.V);
     add(v.ht_key, 8 * S);  // every suffix probe reads a slot pair
     if (!v.ht_pay) {       // only matches read the payload: it is not prefetched
@@ -1801,7 +1890,6 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
     cudaError_t e = launch_probe(a, pf, num_sms, st);
     if (e != cudaSuccess) return e;
     const uintptr_t addr = reinterpret_cast<uintptr_t>(mask);
-    const int64_t n_words = int64_t(n_nodes) * W;
     int64_t head = int64_t(((16u - (addr & 15u)) & 15u) >> 2);
     if (head > n_words) head = n_words;
     const int fill_grid = grid_for((n_words - head) >> 2, kFillThreads * kFillVecs, INT32_MAX);
@@ -1845,7 +1933,7 @@ cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v,
 cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
                                  const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                                  int32_t *err, void *logits, int dtype, const uint32_t *mask, int32_t B,
-                                 int num_sms, cudaStream_t st) {
+                                 int num_sms, cudaStream_t st, const uint32_t *seg_any, int32_t seg_words) {
     const int32_t V = v.V;
     const int64_t W = (int64_t(V) + 31) / 32;
     const int elt = dtype == 0 ? 4 : 2;
@@ -1855,7 +1943,7 @@ cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVoc
     if (!vec) {  // any V and alignment: the two kernels one after the other
         cudaError_t e = launch_advance(t, n_nodes, v, states_in, states_out, tokens, B, err, use_trans, st);
         if (e != cudaSuccess) return e;
-        return launch_apply(logits, dtype, mask, states_out, B, V, n_nodes, num_sms, st);
+        return launch_apply(logits, dtype, mask, states_out, B, V, n_nodes, num_sms, st, seg_any, seg_words);
     }
     const AdvanceArgs aa = advance_args(t, n_nodes, v, use_trans);
     const int32_t parts = (segs + kApplyThreads / 32 - 1) / (kApplyThreads / 32);
@@ -1863,13 +1951,14 @@ cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVoc
     if (grid > INT32_MAX) return cudaErrorInvalidValue;
     if (elt == 2)
         return launch_pdl(k_advance_apply_vec<2>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
-                          states_in, tokens, states_out, err, B, W, segs, parts);
+                          states_in, tokens, states_out, err, B, W, segs, parts, seg_any, seg_words);
     return launch_pdl(k_advance_apply_vec<4>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
-                      states_in, tokens, states_out, err, B, W, segs, parts);
+                      states_in, tokens, states_out, err, B, W, segs, parts, seg_any, seg_words);
 }
 
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
-                         int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st) {
+                         int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st,
+                         const uint32_t *seg_any, int32_t seg_words) {
     const int64_t W = (int64_t(V) + 31) / 32;
     const int elt = dtype == 0 ? 4 : 2;
     const int32_t segs = int32_t((W + 31) / 32);
@@ -1880,9 +1969,9 @@ cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const in
         const int grid = grid_for(items, kApplyThreads / 32, INT32_MAX);
         if (elt == 2)
             return launch_pdl(k_apply_vec<2>, grid, kApplyThreads, st, static_cast<uint4 *>(logits), mask,
-                              states, B, V, W, n_nodes, segs);
+                              states, B, V, W, n_nodes, segs, seg_any, seg_words);
         return launch_pdl(k_apply_vec<4>, grid, kApplyThreads, st, static_cast<uint4 *>(logits), mask, states,
-                          B, V, W, n_nodes, segs);
+                          B, V, W, n_nodes, segs, seg_any, seg_words);
     }
     const int grid = grid_for(int64_t(B) * V, kApplyThreads, int64_t(num_sms) * 16);
     if (elt == 2)
@@ -2109,7 +2198,7 @@ cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bo
     e = launch_pdl_smem(k_lazy_rows, rows_grid, kLazyRowThreads, size_t(L.W) * sizeof(uint32_t), st, la, pa);
     if (e != cudaSuccess) return e;
     const int32_t n_rows = L.C + L.max_batch;
-    if (logits) return launch_apply(logits, dtype, L.rows, L.slot_of, B, L.V, n_rows, num_sms, st);
+    if (logits) return launch_apply(logits, dtype, L.rows, L.slot_of, B, L.V, n_rows, num_sms, st, nullptr, 0);
     const int grid = grid_for(int64_t(B) * L.W, kApplyThreads, int64_t(num_sms) * 8);
     return launch_pdl(k_lazy_gather, grid, kApplyThreads, st, static_cast<const uint32_t *>(L.rows),
                       static_cast<const int32_t *>(L.slot_of), B, L.W, n_rows, L.V - 1, rows_out);

@@ -246,19 +246,24 @@ struct DevTrie {
     int4 *anc = nullptr;             // [n * 4]
     ulonglong2 *trans = nullptr;     // transition table {(row << 32 | token) + 1, end node}
     uint32_t trans_mask = 0;         // slots - 1
+    uint32_t *seg_any = nullptr;     // segment summary of the dense mask (own allocation), seg_cap words
+    int64_t seg_cap = 0;
+    void *hits_base = nullptr;       // the two arrays below (allocated by the first dense compile)
     int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) pairs per node
     uint8_t *hit_count = nullptr;    // compile scratch: hits found per node
 };
 
 // Device storage of the sparse valid lists of a handle (library-owned).
 struct DevLists {
-    void *base = nullptr;           // count, off, tile_sum, total
+    void *base = nullptr;           // count, off, tile_sum, total (and a first token buffer)
+    size_t base_bytes = 0;
     int32_t *count = nullptr;       // [n] entries per row (the counting walk)
     int64_t *off = nullptr;         // [n + 1]
     int64_t *tile_sum = nullptr;    // [tiles]
     int64_t *total = nullptr;       // [1]
-    int32_t *toks = nullptr;        // [tok_cap], separate allocation
+    int32_t *toks = nullptr;        // [tok_cap]: in the block at base, or a separate allocation
     int64_t tok_cap = 0;
+    bool toks_separate = false;     // toks is an allocation of its own
     int64_t n_valid = -1;           // entries of the last build, -1 before any (read back on demand)
     bool n_valid_on_device = false; // n_valid is still only in *total
     cudaEvent_t done = nullptr;     // recorded after the last build's kernels
@@ -388,6 +393,8 @@ struct trie_s {
     std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
     int32_t mask_V = 0;
+    const uint32_t *mask_seg = nullptr;  // its segment summary (dev.seg_any), or null when not computed
+    int32_t mask_seg_words = 0;
     tmk::DevLists lists;                 // last compiled valid lists (library-owned)
     std::shared_ptr<tmk::DevVocab> trans_vocab;  // vocabulary the transition table holds
     bool trans_complete = false;         // filled by a whole compile (else partly, by lazy rows)
@@ -412,7 +419,8 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
 // Probe, fill and scatter: the mask compile with the per-node searches running
 // beside the fill (needs t.hits / t.hit_count).
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
-                                 uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st);
+                                 uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st,
+                                 uint32_t *seg_any, int32_t seg_words, bool *seg_written);
 // Fills t.first_child and t.child_bits from t.parent and t.label (which must
 // be -1 / zero on entry: the caller clears them on the same stream).
 cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
@@ -429,9 +437,10 @@ cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v,
 cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
                                  const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                                  int32_t *err, void *logits, int dtype, const uint32_t *mask, int32_t B,
-                                 int num_sms, cudaStream_t st);
+                                 int num_sms, cudaStream_t st, const uint32_t *seg_any, int32_t seg_words);
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
-                         int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st);
+                         int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st,
+                         const uint32_t *seg_any = nullptr, int32_t seg_words = 0);
 // Copies (d_k, s_k, b_k bytes), k = 0..2, in one launch; the sources are read
 // by the kernel itself (device memory, or host memory the device reads
 // coherently), so no copy engine and no host synchronisation is involved.

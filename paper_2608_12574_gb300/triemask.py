@@ -30,6 +30,7 @@ SIGNATURES = {
     "trie_build_many_device": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_num_nodes": (_I32, [_P]),
     "trie_root": (_I32, [_P, _I32]),
+    "trie_copy_roots": (ctypes.c_int, [_P, _P]),
     "trie_num_sets": (_I32, [_P]),
     "trie_num_chars": (_I64, [_P]),
     "trie_max_depth": (_I32, [_P]),
@@ -151,7 +152,9 @@ class Trie:
         return r
 
     def roots(self) -> np.ndarray:
-        return np.array([self.root(i) for i in range(self.num_sets)], np.int32)
+        out = np.empty(self.num_sets, np.int32)
+        _check(self._lib.trie_copy_roots(self.handle, _hp(out)))
+        return out
 
     def csr(self) -> dict[str, np.ndarray]:
         n = self.num_nodes
