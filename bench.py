@@ -310,6 +310,8 @@ def run_gpu(args, w, rank: int, world: int, dist):
         T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
     stream.synchronize()
     cold_compile_ms = (time.perf_counter() - t0) * 1e3
+    # the vocabulary by handle from here on (a server packs it once)
+    vh = T.trie_vocab_create(w.vocab_bytes, w.vocab_offsets, V)
     with torch.cuda.stream(stream):
         logits = [W_logits(w, s, dev) for s in range(S)]
         states0 = torch.zeros(B, dtype=torch.int32, device=dev)
@@ -354,7 +356,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
         return prev
 
     def step():
-        T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+        T.trie_compile_masks_vocab(h, vh, mask, stream)
         decode(logits)
 
     # kernel-level graphs: the compile alone; the 16 applies of a step, back to
@@ -362,7 +364,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
     adv_states = [torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(S)]
 
     def compile_only():
-        T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+        T.trie_compile_masks_vocab(h, vh, mask, stream)
 
     def apply_only():
         for t in range(S):
@@ -444,14 +446,14 @@ def run_gpu(args, w, rank: int, world: int, dist):
         # sparse valid lists: the build (CUDA events around one call; no host
         # sync inside it) and the list-driven apply over the same logits buffers
         with torch.cuda.stream(stream):
-            n_valid = T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
+            n_valid = T.trie_compile_lists_vocab(h, vh, stream)
         stream.synchronize()
         lt = []
         for _ in range(20):
             l0, l1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             with torch.cuda.stream(stream):
                 l0.record(stream)
-                T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
+                T.trie_compile_lists_vocab(h, vh, stream, count=False)
                 l1.record(stream)
             stream.synchronize()
             lt.append(l0.elapsed_time(l1))
@@ -478,7 +480,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
         n0, n1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
             n0.record(stream)
-            T.trie_compile_masks(hn, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+            T.trie_compile_masks_vocab(hn, vh, mask, stream)
             n1.record(stream)
         stream.synchronize()
         ns_dev.append(n0.elapsed_time(n1))
@@ -600,6 +602,7 @@ def run_e2e(w, n_nodes: int, logits, forced, dev, stream, steps: int, dist=None)
     sbuf = [torch.zeros(B, dtype=torch.int32, device=dev) for _ in range(2)]
     err = torch.zeros(1, dtype=torch.int32, device=dev)
     mask = torch.empty((n_nodes, T.mask_words(V)), dtype=torch.int32, device=dev)
+    vh = T.trie_vocab_create(w.vocab_bytes, w.vocab_offsets, V)  # packed and uploaded once, like a server's
     # ---- e2e: host strings -> trie_build -> compile -> decode, with the logits
     # and the step's tokens copied from pinned host memory and the states read
     # back every decode step. Steps are pipelined as a server would run them:
@@ -631,7 +634,7 @@ def run_e2e(w, n_nodes: int, logits, forced, dev, stream, steps: int, dist=None)
             for t in range(S):
                 dlogs[k][t].copy_(host_logits[t], non_blocking=True)
                 arrived[k][t].record(copy_stream)
-        T.trie_compile_masks(hh, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+        T.trie_compile_masks_vocab(hh, vh, mask, stream)
         sbuf[0].zero_()
         stream.wait_event(arrived[k][S])
         cur = 0
@@ -792,9 +795,12 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
     N = h.num_nodes
     out["N_nodes"] = N
     roots = torch.as_tensor(h.roots(), device=dev)
+    # the tokenizer's vocabulary is packed and uploaded once (a handle); the
+    # requests' sets change every batch
+    vh = T.trie_vocab_create(w.vocab_bytes, w.vocab_offsets, V)
     with torch.cuda.stream(stream):
         logits = [W.logits(w, t, device=str(dev)) for t in range(steps)]
-        T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream)
+        T.trie_compile_lists_vocab(h, vh, stream)
         states = roots.clone()
         err = torch.zeros(1, dtype=torch.int32, device=dev)
         forced = torch.zeros((steps, B), dtype=torch.int32, device=dev)
@@ -848,7 +854,7 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
             e0.record(stream)
-            T.trie_compile_lists(h, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
+            T.trie_compile_lists_vocab(h, vh, stream, count=False)
             e1.record(stream)
         stream.synchronize()
         lw.append(time.perf_counter() - t0)
@@ -894,7 +900,7 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
             with torch.cuda.stream(stream):
                 roots_host.numpy()[:] = hh.roots()
                 st[0].copy_(roots_host, non_blocking=True)
-                T.trie_compile_lists(hh, w.vocab_bytes, w.vocab_offsets, V, stream, count=False)
+                T.trie_compile_lists_vocab(hh, vh, stream, count=False)
                 T.trie_apply_lists(hh, logits[0], st[0], stream)
                 for t in range(1, steps):
                     T.trie_advance_apply_lists(hh, st[(t - 1) % 2], forced[t - 1], st[t % 2], logits[t], err,
@@ -953,9 +959,9 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
     if dense_bytes < free * 0.8:
         mask = T.alloc_mask(h, V, dev)
         with torch.cuda.stream(stream):
-            T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+            T.trie_compile_masks_vocab(h, vh, mask, stream)
             e0.record(stream)
-            T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+            T.trie_compile_masks_vocab(h, vh, mask, stream)
             e1.record(stream)
         stream.synchronize()
         ms = e0.elapsed_time(e1)
@@ -1016,8 +1022,9 @@ def run_profile(args, w) -> None:
         h = T.trie_build(w.set_bytes, w.set_offsets)
         mask = T.alloc_mask(h, w.V, dev)
         T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, w.V, mask)
+        vh = T.trie_vocab_create(w.vocab_bytes, w.vocab_offsets, w.V)
         if args.profile == "compile":
-            timed(lambda: T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, w.V, mask, stream),
+            timed(lambda: T.trie_compile_masks_vocab(h, vh, mask, stream),
                   f"{w.name} trie_compile_masks, {h.num_nodes} nodes")
         elif args.profile == "pairwise":
             timed(lambda: T.trie_compile_masks_pairwise(h, w.vocab_bytes, w.vocab_offsets, w.V, mask, stream),
@@ -1048,7 +1055,7 @@ def run_profile(args, w) -> None:
                 timed(loop, f"{w.name} lazy decode loop ({S} steps, cache {args.cache_rows} rows)")
             else:
                 def loop():
-                    T.trie_compile_masks(h, w.vocab_bytes, w.vocab_offsets, V, mask, stream)
+                    T.trie_compile_masks_vocab(h, vh, mask, stream)
                     T.trie_apply_mask(h, logits[0], s0, stream)
                     prev = s0
                     for t in range(1, S):
@@ -1063,7 +1070,8 @@ def run_profile(args, w) -> None:
         h = T.trie_build_many_device(full.set_bytes, full.set_offsets, full.set_index, stream)
     else:
         h = T.trie_build_many(full.set_bytes, full.set_offsets, full.set_index)
-    timed(lambda: T.trie_compile_lists(h, full.vocab_bytes, full.vocab_offsets, full.V, stream, count=False),
+    vh = T.trie_vocab_create(full.vocab_bytes, full.vocab_offsets, full.V)
+    timed(lambda: T.trie_compile_lists_vocab(h, vh, stream, count=False),
           f"{args.requests}-request forest trie_compile_lists, {h.num_nodes} nodes")
     print(f"{T.trie_num_valid(h)} entries")
 

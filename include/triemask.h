@@ -184,6 +184,35 @@ int trie_get_csr(trie_t h, int32_t *parent, uint8_t *label, uint8_t *terminal,
 int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets,
                        int32_t V, uint32_t *d_mask, cudaStream_t stream);
 
+/* Vocabulary handles (App. H.4 Phases 2-3: a vocabulary is packed and
+ * uploaded once). The entry points that take vocab_bytes / vocab_offsets / V
+ * find an uploaded vocabulary by comparing the caller's arrays with the
+ * cached copies, byte by byte, on every call (for a 128,000-token vocabulary
+ * about 60 us of host time before the first launch). A handle names the
+ * vocabulary instead and skips that comparison.
+ *   trie_vocab_create  packs and uploads the vocabulary (as the first
+ *                      trie_compile_masks would) on the current device, or
+ *                      takes the already uploaded copy; arguments as
+ *                      trie_compile_masks; *out receives the handle (NULL on
+ *                      error). Host-synchronous. Errors: TRIE_EINVAL,
+ *                      TRIE_ENOMEM, TRIE_ECUDA.
+ *   trie_vocab_size    V of the handle; -1 for NULL.
+ *   trie_vocab_destroy releases the handle (NULL is a no-op). The device copy
+ *                      is freed when neither the library's cache of recent
+ *                      vocabularies nor a trie handle that compiled with it
+ *                      still holds it; that cudaFree synchronises the device.
+ * The caller's arrays are not referenced after trie_vocab_create returns. */
+typedef struct trie_vocab_s *trie_vocab_t; /* opaque; owned by the caller */
+int trie_vocab_create(const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                      trie_vocab_t *out);
+int32_t trie_vocab_size(trie_vocab_t v);
+void trie_vocab_destroy(trie_vocab_t v);
+
+/* trie_compile_masks with the vocabulary of handle v (V = trie_vocab_size(v)).
+ * v must belong to the current device (else TRIE_EINVAL); the rest as
+ * trie_compile_masks. */
+int trie_compile_masks_vocab(trie_t h, trie_vocab_t v, uint32_t *d_mask, cudaStream_t stream);
+
 /* Advance B decode states in place by one token each: s' = delta*(s, bytes(t))
  * (Sec. 2, Eq. 1; the paper's stateless character walk).
  *   d_states  device int32[B], in/out
@@ -206,7 +235,11 @@ int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B
  *             the row {EOS}
  *   V         must equal the V of the last trie_compile_masks on the handle
  * Uses the mask recorded by the last trie_compile_masks (TRIE_ESTATE if
- * none). B = 0 is a no-op. */
+ * none), and the summary that compile keeps in the handle of which 1,024-token
+ * segments of each row hold an allowed token (segments without one are
+ * written without reading the mask). Both belong to the handle's last compile:
+ * work captured in a CUDA graph must not outlive a later compile of the handle
+ * with another vocabulary. B = 0 is a no-op. */
 int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states, int32_t B,
                     int32_t V, cudaStream_t stream);
 
@@ -253,7 +286,9 @@ int trie_compile_masks_pairwise(trie_t h, const uint8_t *vocab_bytes, const int6
  *   the last k edges into m is found and listed at the node k levels up
  *   (the Aho-Corasick outputs of Sec. 4.2 step 2, found per node). One walk
  *   counts every row's entries, a scan gives the offsets, a second walk
- *   writes the tokens.
+ *   writes the tokens, and beside each the node its token leads to (kept in
+ *   the handle, 8 bytes per entry in all, for trie_advance_apply_lists: the
+ *   advance is then a look-up in the state's list).
  *   Asynchronous on `stream` while the bound on the entries (a node lists at
  *   most one token string per length up to the longest token, each under
  *   every id that spells it, plus EOS) is at most 2^28 entries or fits the
@@ -266,6 +301,10 @@ int trie_compile_masks_pairwise(trie_t h, const uint8_t *vocab_bytes, const int6
  *   would exceed 2^24 - 2 nodes), TRIE_ENOMEM, TRIE_ECUDA. */
 int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
                        cudaStream_t stream);
+
+/* trie_compile_lists with the vocabulary of handle v (see trie_vocab_create);
+ * v must belong to the current device (else TRIE_EINVAL). */
+int trie_compile_lists_vocab(trie_t h, trie_vocab_t v, cudaStream_t stream);
 
 /* Number of (node, token) entries in the handle's lists; -1 before any
  * trie_compile_lists (or if reading the size back fails). The first call

@@ -668,17 +668,11 @@ static uint32_t *ensure_seg(trie_t h, int dev, cudaStream_t stream, int32_t word
     return h->dev.seg_any;
 }
 
-int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
-                       uint32_t *d_mask, cudaStream_t stream) {
-    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
-    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
-    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
-    if (!d_mask) return fail(TRIE_EINVAL, "d_mask is NULL");
-    if (reinterpret_cast<uintptr_t>(d_mask) & 3u) return fail(TRIE_EINVAL, "d_mask must be 4-byte aligned");
-    int dev, rc;
-    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
-    std::shared_ptr<tmk::DevVocab> voc;
-    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+// The mask compile with the vocabulary resolved (from the cache, or a vocabulary handle).
+static int compile_masks(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, int dev, uint32_t *d_mask,
+                         cudaStream_t stream) {
+    int rc;
+    const int32_t V = voc->V;
     if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
     if ((rc = ensure_hits(h, dev, stream)) != TRIE_OK) return rc;
     const int64_t W = (int64_t(V) + 31) / 32;
@@ -702,6 +696,44 @@ int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     h->mask_seg = seg_written ? seg : nullptr;
     h->mask_seg_words = seg_words;
     return TRIE_OK;
+}
+
+static int check_mask_arg(uint32_t *d_mask) {
+    if (!d_mask) return fail(TRIE_EINVAL, "d_mask is NULL");
+    if (reinterpret_cast<uintptr_t>(d_mask) & 3u) return fail(TRIE_EINVAL, "d_mask must be 4-byte aligned");
+    return TRIE_OK;
+}
+
+// The vocabulary of a handle, on the current device.
+static int vocab_of(trie_vocab_t v, int *dev, std::shared_ptr<tmk::DevVocab> *voc) {
+    if (!v || !v->voc) return fail(TRIE_EINVAL, "vocabulary handle is NULL");
+    int rc;
+    if ((rc = current_device(dev)) != TRIE_OK) return rc;
+    if (v->voc->device != *dev) return fail(TRIE_EINVAL, "the vocabulary handle belongs to another device");
+    *voc = v->voc;
+    return TRIE_OK;
+}
+
+int trie_compile_masks(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                       uint32_t *d_mask, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    int dev, rc;
+    if ((rc = check_mask_arg(d_mask)) != TRIE_OK) return rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    return compile_masks(h, voc, dev, d_mask, stream);
+}
+
+int trie_compile_masks_vocab(trie_t h, trie_vocab_t v, uint32_t *d_mask, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    int dev, rc;
+    if ((rc = check_mask_arg(d_mask)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = vocab_of(v, &dev, &voc)) != TRIE_OK) return rc;
+    return compile_masks(h, voc, dev, d_mask, stream);
 }
 
 int trie_advance(trie_t h, int32_t *d_states, const int32_t *d_tokens, int32_t B, int32_t *d_err,
@@ -861,14 +893,24 @@ static bool lists_built(trie_t h) {
 // The vocabulary's reversed-token trie as a device edge table (the list
 // compile's walk), built on first use: on the host, then its edges inserted
 // on the device (host-synchronous, once per vocabulary and device).
-static int ensure_rev_trie(tmk::DevVocab *voc, const uint8_t *vb, const int64_t *vo, int32_t V) {
+static int ensure_rev_trie(tmk::DevVocab *voc) {
     std::lock_guard<std::mutex> lk(voc->rt_mu);
     if (voc->rt_state == 1) return TRIE_OK;
     if (voc->rt_state < 0) return fail(TRIE_EINVAL, "the vocabulary is too large for the valid-list walk");
+    const int32_t V = voc->V;
     tmk::RevTokenTrie rt;
     std::string err;
     try {
-        err = tmk::build_reversed_token_trie(vb, vo, V, &rt);
+        // from the vocabulary's host copy: its bytes start at the caller's offsets[0]
+        const int64_t b0 = voc->src_offsets[0];
+        std::vector<int64_t> rel;
+        const int64_t *vo = voc->src_offsets.data();
+        if (b0 != 0) {
+            rel.resize(size_t(V) + 1);
+            for (size_t i = 0; i <= size_t(V); i++) rel[i] = voc->src_offsets[i] - b0;
+            vo = rel.data();
+        }
+        err = tmk::build_reversed_token_trie(voc->src_bytes.data(), vo, V, &rt);
     } catch (const std::bad_alloc &) {
         return fail(TRIE_ENOMEM, "host allocation failed while building the reversed-token trie");
     }
@@ -939,16 +981,11 @@ int trie_compile_masks_pairwise(trie_t h, const uint8_t *vocab_bytes, const int6
     return TRIE_OK;
 }
 
-int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
-                       cudaStream_t stream) {
-    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
-    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
-    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
-    int dev, rc;
-    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
-    std::shared_ptr<tmk::DevVocab> voc;
-    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
-    if ((rc = ensure_rev_trie(voc.get(), vocab_bytes, vocab_offsets, V)) != TRIE_OK) return rc;
+// The list compile with the vocabulary resolved (from the cache, or a vocabulary handle).
+static int compile_lists(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, int dev, cudaStream_t stream) {
+    int rc;
+    const int32_t V = voc->V;
+    if ((rc = ensure_rev_trie(voc.get())) != TRIE_OK) return rc;
     if ((rc = ensure_device_trie(h, dev, stream)) != TRIE_OK) return rc;
     const int32_t n = h->host.n;
     tmk::DevLists &L = h->lists;
@@ -965,7 +1002,7 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         const size_t o_off = lay.add(sizeof(int64_t) * (size_t(n) + 1));
         const size_t o_tile = lay.add(sizeof(int64_t) * (size_t(n) / 4096 + 2));
         const size_t o_tot = lay.add(sizeof(int64_t));
-        const size_t o_tok = by_bound ? lay.add(sizeof(int32_t) * size_t(std::max<int64_t>(bound, 1))) : 0;
+        const size_t o_tok = by_bound ? lay.add(2 * sizeof(int32_t) * size_t(std::max<int64_t>(bound, 1))) : 0;
         void *base = take_spare_block(dev, lay.total);
         if (!base && (rc = pool_alloc(dev, lay.total, stream, &base, "the valid lists")) != TRIE_OK) return rc;
         cudaEvent_t done = nullptr;
@@ -985,6 +1022,7 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         if (by_bound) {
             L.toks = reinterpret_cast<int32_t *>(b + o_tok);
             L.tok_cap = std::max<int64_t>(bound, 1);
+            L.ends = L.toks + L.tok_cap;
             L.toks_separate = false;
         }
     }
@@ -993,12 +1031,14 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
         if (need <= L.tok_cap) return TRIE_OK;
         if (L.toks_separate) pool_free(L.toks);  // earlier apply calls may still read it
         L.toks = nullptr;                         // (a buffer inside the block at base stays there)
+        L.ends = nullptr;
         L.tok_cap = 0;
         void *toks = nullptr;
-        int r = pool_alloc(dev, sizeof(int32_t) * size_t(std::max<int64_t>(need, 1)), stream, &toks,
-                           "the valid-list tokens");
+        need = std::max<int64_t>(need, 1);
+        int r = pool_alloc(dev, 2 * sizeof(int32_t) * size_t(need), stream, &toks, "the valid-list tokens");
         if (r != TRIE_OK) return r;
         L.toks = static_cast<int32_t *>(toks);
+        L.ends = L.toks + need;
         L.tok_cap = need;
         L.toks_separate = true;
         return TRIE_OK;
@@ -1027,6 +1067,46 @@ int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *voca
     h->vocab = voc;
     return TRIE_OK;
 }
+
+int trie_compile_lists(trie_t h, const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V,
+                       cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    return compile_lists(h, voc, dev, stream);
+}
+
+int trie_compile_lists_vocab(trie_t h, trie_vocab_t v, cudaStream_t stream) {
+    if (!h) return fail(TRIE_EINVAL, "handle is NULL");
+    int dev, rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = vocab_of(v, &dev, &voc)) != TRIE_OK) return rc;
+    return compile_lists(h, voc, dev, stream);
+}
+
+int trie_vocab_create(const uint8_t *vocab_bytes, const int64_t *vocab_offsets, int32_t V, trie_vocab_t *out) {
+    if (!out) return fail(TRIE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (!vocab_offsets) return fail(TRIE_EINVAL, "vocab_offsets is NULL");
+    if (V < 2 || V > INT32_MAX - 32) return fail(TRIE_EINVAL, "V must be in [2, 2^31-32]");
+    int dev, rc;
+    if ((rc = current_device(&dev)) != TRIE_OK) return rc;
+    std::shared_ptr<tmk::DevVocab> voc;
+    if ((rc = get_vocab(vocab_bytes, vocab_offsets, V, dev, &voc)) != TRIE_OK) return rc;
+    trie_vocab_t v = new (std::nothrow) trie_vocab_s;
+    if (!v) return fail(TRIE_ENOMEM, "host allocation failed");
+    v->voc = std::move(voc);
+    *out = v;
+    return TRIE_OK;
+}
+
+int32_t trie_vocab_size(trie_vocab_t v) { return v && v->voc ? v->voc->V : -1; }
+
+void trie_vocab_destroy(trie_vocab_t v) { delete v; }
 
 int64_t trie_num_valid(trie_t h) {
     if (!h) return -1;

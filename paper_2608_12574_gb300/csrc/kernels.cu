@@ -1170,6 +1170,7 @@ struct WalkArgs {
     int32_t *count;            // [n] entries per row (counting walk)
     unsigned long long *off;   // [n + 1]: off[i + 1] = next position of row i (writing walk)
     int32_t *toks;
+    int32_t *ends;             // [tok_cap]: the node each entry's token leads to (FINISHED for EOS)
     unsigned long long tok_cap;  // entries toks holds (a write past it is dropped)
 };
 
@@ -1220,7 +1221,7 @@ __global__ void k_rt_insert(const int32_t *__restrict__ parent, const uint8_t *_
 // the reversed trie's root for byte c.
 template <typename Tok>
 __device__ __forceinline__ void walk_node(const WalkArgs &a, const int2 *root, int32_t m, Tok tok) {
-    if (__ldg(a.terminal + m)) tok(m, a.eos);
+    if (__ldg(a.terminal + m)) tok(m, a.eos, kFinished);
     const int32_t d16 = __ldg(a.depth16 + m);
     const int32_t lim = a.lmax < d16 ? a.lmax : d16;
     if (lim <= 0) return;
@@ -1229,13 +1230,13 @@ __device__ __forceinline__ void walk_node(const WalkArgs &a, const int2 *root, i
     const int2 r0 = root[uint32_t(win.x) & 0xFFu];
     int32_t x = r0.x;
     if (x < 0) return;
-    if (r0.y >= 0) tok(__ldg(up), r0.y);
+    if (r0.y >= 0) tok(__ldg(up), r0.y, m);
     for (int32_t j = 1; j < lim; j++) {
         const uint32_t c = uint32_t((j < 8 ? win.x >> (8 * j) : win.y >> (8 * (j - 8))) & 0xFFu);
         uint4 e;
         if (!rt_step(a.edge, a.edge_mask, a.edge_shift, x, c, &e)) return;
         x = int32_t(e.y);
-        if (int32_t(e.z) >= 0) tok(__ldg(up + j), int32_t(e.z));
+        if (int32_t(e.z) >= 0) tok(__ldg(up + j), int32_t(e.z), m);
     }
     // tokens longer than the 16-label window, in a trie deeper than 16
     if (lim == 16 && a.lmax > 16) {
@@ -1246,7 +1247,7 @@ __device__ __forceinline__ void walk_node(const WalkArgs &a, const int2 *root, i
             uint4 e;
             if (!rt_step(a.edge, a.edge_mask, a.edge_shift, x, __ldg(a.label + y), &e)) return;
             x = int32_t(e.y);
-            if (int32_t(e.z) >= 0) tok(p, int32_t(e.z));
+            if (int32_t(e.z) >= 0) tok(p, int32_t(e.z), m);
             y = p;
         }
     }
@@ -1268,18 +1269,21 @@ __global__ void __launch_bounds__(kWalkThreads) k_list_walk(WalkArgs a) {
     __syncthreads();
     pdl_launch_dependents();
     pdl_wait();  // counts zeroed, or offsets scanned, by the previous kernels
-    auto emit = [&](int32_t row, int32_t t) {
+    auto emit = [&](int32_t row, int32_t t, int32_t end) {
         if (kWrite) {
             const unsigned long long p = atomicAdd(a.off + row + 1, 1ull);
-            if (p < a.tok_cap) a.toks[p] = t;
+            if (p < a.tok_cap) {
+                a.toks[p] = t;
+                a.ends[p] = end;
+            }
         } else {
             atomicAdd(a.count + row, 1);
         }
     };
-    auto tok = [&](int32_t row, int32_t t) {
-        emit(row, t);
+    auto tok = [&](int32_t row, int32_t t, int32_t end) {
+        emit(row, t, end);
         if (a.tok_next)
-            for (int32_t u = __ldg(a.tok_next + t); u >= 0; u = __ldg(a.tok_next + u)) emit(row, u);
+            for (int32_t u = __ldg(a.tok_next + t); u >= 0; u = __ldg(a.tok_next + u)) emit(row, u, end);
     };
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) walk_node(a, root, m, tok);
@@ -1298,29 +1302,46 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_lists(void *__restrict_
                                                                const int32_t *__restrict__ tokens,
                                                                int32_t *__restrict__ states_out,
                                                                int32_t *__restrict__ err, int32_t B, int32_t V,
-                                                               int32_t n_nodes, int32_t parts) {
+                                                               int32_t n_nodes, int32_t parts,
+                                                               const int32_t *__restrict__ ends) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     constexpr int kWords = 8 * 32;
     __shared__ __align__(128) uint4 tile[kVec ? kSegChunks : 1];
     __shared__ uint32_t words[kWords];
-    __shared__ int32_t state;
+    __shared__ int32_t state, moved;
     for (int i = threadIdx.x; i < kWords; i += kApplyThreads) words[i] = 0u;
+    if (threadIdx.x == 0) moved = kDead;
     if (kVec) init_ninf_tile<kElt>(tile);
     else __syncthreads();
     pdl_launch_dependents();
     pdl_wait();  // logits, states and tokens come from earlier kernels
     const int32_t b = int32_t(blockIdx.x) / parts, part = int32_t(blockIdx.x) - b * parts;
-    if (threadIdx.x == 0) {
-        const int32_t s0 = __ldg(states + b);
-        int32_t s1 = s0;
-        if (kAdvance) {
-            s1 = advance_one(aa, s0, __ldg(tokens + b));
+    const int32_t s0 = __ldg(states + b);
+    if (kAdvance) {
+        // from a node, the move is the entry of the token in the node's list
+        // (its end node, FINISHED for EOS), DEAD if the token is not there:
+        // the advance's rules, in two dependent loads instead of a byte walk
+        // (each entry's token and end are loaded together)
+        const int32_t t = __ldg(tokens + b);
+        const bool listed = ends && s0 >= 0 && s0 < n_nodes && t >= 0 && t < V;
+        if (listed) {
+            const int64_t lo = __ldg(off + s0), hi = __ldg(off + s0 + 1);
+            for (int64_t i = lo + threadIdx.x; i < hi; i += kApplyThreads) {
+                const int32_t tk = __ldg(toks + i), en = __ldg(ends + i);
+                if (tk == t) moved = en;
+            }
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int32_t s1 = listed ? moved : advance_one(aa, s0, t);
             if (part == 0) {
                 states_out[b] = s1;
                 if (s1 == kDead && s0 != kDead && err) atomicAdd(err, 1);
             }
+            state = s1;
         }
-        state = s1;
+    } else if (threadIdx.x == 0) {
+        state = s0;
     }
     __syncthreads();
     const int32_t s = state;
@@ -2053,6 +2074,7 @@ WalkArgs walk_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t
     a.count = L.count;
     a.off = reinterpret_cast<unsigned long long *>(L.off);
     a.toks = L.toks;
+    a.ends = L.ends;
     a.tok_cap = static_cast<unsigned long long>(L.tok_cap);
     return a;
 }
@@ -2101,23 +2123,23 @@ cudaError_t launch_lists(void *logits, int dtype, const DevLists &L, const Advan
     if (aa) {
         if (vec)
             return elt == 2 ? launch_pdl(k_apply_lists<2, true, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                         states, tokens, states_out, err, B, V, n_nodes, parts)
+                                         states, tokens, states_out, err, B, V, n_nodes, parts, L.ends)
                             : launch_pdl(k_apply_lists<4, true, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                         states, tokens, states_out, err, B, V, n_nodes, parts);
+                                         states, tokens, states_out, err, B, V, n_nodes, parts, L.ends);
         return elt == 2 ? launch_pdl(k_apply_lists<2, false, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                     states, tokens, states_out, err, B, V, n_nodes, parts)
+                                     states, tokens, states_out, err, B, V, n_nodes, parts, L.ends)
                         : launch_pdl(k_apply_lists<4, false, true>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                     states, tokens, states_out, err, B, V, n_nodes, parts);
+                                     states, tokens, states_out, err, B, V, n_nodes, parts, L.ends);
     }
     if (vec)
         return elt == 2 ? launch_pdl(k_apply_lists<2, true, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                     states, tokens, states_out, err, B, V, n_nodes, parts)
+                                     states, tokens, states_out, err, B, V, n_nodes, parts, L.ends)
                         : launch_pdl(k_apply_lists<4, true, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                     states, tokens, states_out, err, B, V, n_nodes, parts);
+                                     states, tokens, states_out, err, B, V, n_nodes, parts, L.ends);
     return elt == 2 ? launch_pdl(k_apply_lists<2, false, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                 states, tokens, states_out, err, B, V, n_nodes, parts)
+                                 states, tokens, states_out, err, B, V, n_nodes, parts, L.ends)
                     : launch_pdl(k_apply_lists<4, false, false>, int(grid), kApplyThreads, st, logits, of, tk, a,
-                                 states, tokens, states_out, err, B, V, n_nodes, parts);
+                                 states, tokens, states_out, err, B, V, n_nodes, parts, L.ends);
 }
 
 }  // namespace

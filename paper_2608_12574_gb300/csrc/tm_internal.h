@@ -262,8 +262,9 @@ struct DevLists {
     int64_t *tile_sum = nullptr;    // [tiles]
     int64_t *total = nullptr;       // [1]
     int32_t *toks = nullptr;        // [tok_cap]: in the block at base, or a separate allocation
+    int32_t *ends = nullptr;        // [tok_cap] after toks: the node each entry's token leads to
     int64_t tok_cap = 0;
-    bool toks_separate = false;     // toks is an allocation of its own
+    bool toks_separate = false;     // toks (with ends) is an allocation of its own
     int64_t n_valid = -1;           // entries of the last build, -1 before any (read back on demand)
     bool n_valid_on_device = false; // n_valid is still only in *total
     cudaEvent_t done = nullptr;     // recorded after the last build's kernels
@@ -382,6 +383,12 @@ struct fmt_s {
     std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
     int32_t mask_V = 0;
+};
+
+// A vocabulary handle of the C ABI: the packed, uploaded vocabulary of one
+// device, shared with the library's vocabulary cache.
+struct trie_vocab_s {
+    std::shared_ptr<tmk::DevVocab> voc;
 };
 
 // The opaque handle of the C ABI.

@@ -39,6 +39,11 @@ SIGNATURES = {
     "trie_compile_masks_pairwise": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_compile_masks_noalloc": (ctypes.c_int, [_P, _P, _P, _I32, _P, _P]),
     "trie_compile_lists": (ctypes.c_int, [_P, _P, _P, _I32, _P]),
+    "trie_vocab_create": (ctypes.c_int, [_P, _P, _I32, _P]),
+    "trie_vocab_size": (_I32, [_P]),
+    "trie_vocab_destroy": (None, [_P]),
+    "trie_compile_masks_vocab": (ctypes.c_int, [_P, _P, _P, _P]),
+    "trie_compile_lists_vocab": (ctypes.c_int, [_P, _P, _P]),
     "trie_num_valid": (_I64, [_P]),
     "trie_copy_lists": (ctypes.c_int, [_P, _P, _P, _P]),
     "trie_apply_lists": (ctypes.c_int, [_P, _P, ctypes.c_int, _P, _I32, _I32, _P]),
@@ -183,6 +188,50 @@ class Trie:
             pass
 
 
+class Vocab:
+    """Owns one vocabulary handle: the vocabulary packed and uploaded once on
+    a device, named by later compiles without comparing its arrays again."""
+
+    def __init__(self, handle: ctypes.c_void_p, device: int):
+        self._lib = load_library()
+        self.handle = handle
+        self.device = device
+
+    @property
+    def V(self) -> int:
+        return self._lib.trie_vocab_size(self.handle)
+
+    def destroy(self) -> None:
+        if self.handle:
+            self._lib.trie_vocab_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def trie_vocab_create(vocab_bytes, vocab_offsets, V: int) -> Vocab:
+    """Pack and upload the vocabulary on the current CUDA device (host-synchronous)."""
+    import torch
+    lib = load_library()
+    vb = _host(vocab_bytes, np.uint8)
+    vo = _host(vocab_offsets, np.int64)
+    if len(vo) != V + 1:
+        raise ValueError("vocab_offsets must have V+1 entries")
+    h = ctypes.c_void_p()
+    _check(lib.trie_vocab_create(_hp(vb), _hp(vo), V, ctypes.byref(h)))
+    return Vocab(h, torch.cuda.current_device())
+
+
+def _vocab_handle(v: Vocab):
+    if not isinstance(v, Vocab) or not v.handle:
+        raise ValueError("expected a live Vocab")
+    return v.handle
+
+
 def mask_words(V: int) -> int:
     return (V + 31) // 32
 
@@ -248,6 +297,16 @@ def trie_compile_masks(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stre
         raise ValueError("d_mask is smaller than num_nodes * ceil(V/32) words")
     _check(h._lib.trie_compile_masks(h.handle, _hp(vb), _hp(vo), V, p,
                                      _stream(stream, d_mask.device)))
+
+
+def trie_compile_masks_vocab(h: Trie, vocab: Vocab, d_mask, stream=None) -> None:
+    """trie_compile_masks with the vocabulary of a Vocab handle."""
+    import torch
+    vh = _vocab_handle(vocab)
+    p = _dev(d_mask, (torch.int32,), "d_mask")
+    if d_mask.numel() < h.num_nodes * mask_words(vocab.V):
+        raise ValueError("d_mask is smaller than num_nodes * ceil(V/32) words")
+    _check(h._lib.trie_compile_masks_vocab(h.handle, vh, p, _stream(stream, d_mask.device)))
 
 
 def trie_compile_masks_pairwise(h: Trie, vocab_bytes, vocab_offsets, V: int, d_mask, stream=None) -> None:
@@ -330,6 +389,13 @@ def trie_compile_lists(h: Trie, vocab_bytes, vocab_offsets, V: int, stream=None,
         raise ValueError("vocab_offsets must have V+1 entries")
     _check(h._lib.trie_compile_lists(h.handle, _hp(vb), _hp(vo), V,
                                      _stream(stream, device if device is not None else torch.cuda.current_device())))
+    return h._lib.trie_num_valid(h.handle) if count else None
+
+
+def trie_compile_lists_vocab(h: Trie, vocab: Vocab, stream=None, count: bool = True) -> int | None:
+    """trie_compile_lists with the vocabulary of a Vocab handle."""
+    vh = _vocab_handle(vocab)
+    _check(h._lib.trie_compile_lists_vocab(h.handle, vh, _stream(stream, vocab.device)))
     return h._lib.trie_num_valid(h.handle) if count else None
 
 

@@ -90,3 +90,15 @@ def test_other_wrappers_check_their_arguments(handles):
         T.trie_advance(h, _t(2, "int32"), _t(2, "int32"))
     assert T.mask_words(1) == 1 and T.mask_words(32) == 1 and T.mask_words(33) == 2
     assert np.array_equal(h.roots(), [0])
+
+
+def test_vocab_wrappers_check_their_arguments(handles):
+    h, f = handles
+    vb, vo = W.pack([b"a", b"b", b""])
+    with pytest.raises(ValueError, match="V\\+1"):
+        T.trie_vocab_create(vb, vo, 4)
+    for bad in (None, "vocab", T.Vocab(None, 0)):
+        with pytest.raises(ValueError, match="live Vocab"):
+            T.trie_compile_lists_vocab(h, bad)
+        with pytest.raises(ValueError, match="live Vocab"):
+            T.trie_compile_masks_vocab(h, bad, _t((3, 1), "int32"))

@@ -196,6 +196,30 @@ def test_null_handle_queries(lib):
     assert lib.trie_apply_mask(None, None, 0, None, 1, 10, None) == T.TRIE_EINVAL
 
 
+def test_vocab_handle_calls_checked_before_any_device_work(lib):
+    """Vocabulary handles: NULL handles and bad arguments come back before the GPU is touched."""
+    assert lib.trie_vocab_size(None) == -1
+    lib.trie_vocab_destroy(None)  # a no-op
+    out = ctypes.c_void_p(12345)
+    vo = np.array([0, 1, 1], np.int64)
+    vb = np.frombuffer(b"a", np.uint8).copy()
+    assert lib.trie_vocab_create(vb.ctypes.data, vo.ctypes.data, 2, None) == T.TRIE_EINVAL      # out NULL
+    assert lib.trie_vocab_create(vb.ctypes.data, None, 2, ctypes.byref(out)) == T.TRIE_EINVAL   # offsets NULL
+    assert out.value is None                                                                     # cleared
+    out = ctypes.c_void_p(12345)
+    assert lib.trie_vocab_create(vb.ctypes.data, vo.ctypes.data, 1, ctypes.byref(out)) == T.TRIE_EINVAL  # V < 2
+    assert out.value is None
+    sb, so = W.pack([b"ab"])
+    h = T.trie_build(sb, so)
+    assert lib.trie_compile_masks_vocab(None, None, 16, None) == T.TRIE_EINVAL        # trie handle NULL
+    assert lib.trie_compile_masks_vocab(h.handle, None, None, None) == T.TRIE_EINVAL  # d_mask NULL
+    assert lib.trie_compile_masks_vocab(h.handle, None, 2, None) == T.TRIE_EINVAL     # misaligned
+    assert lib.trie_compile_masks_vocab(h.handle, None, 16, None) == T.TRIE_EINVAL    # vocabulary NULL
+    assert lib.trie_compile_lists_vocab(None, None, None) == T.TRIE_EINVAL
+    assert lib.trie_compile_lists_vocab(h.handle, None, None) == T.TRIE_EINVAL
+    assert "vocabulary handle is NULL" in T.trie_last_error()
+
+
 def test_device_calls_checked_before_any_device_work(lib):
     """Argument errors and call-order errors come back before the GPU is touched."""
     sb, so = W.pack([b"ab"])
