@@ -56,7 +56,7 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-dynamic", action="store_true", help="skip the dynamic per-query-set measurement")
     p.add_argument("--no-graph", action="store_true", help="run the steps eagerly instead of as CUDA graphs")
-    p.add_argument("--profile", choices=["compile", "pairwise", "lists", "lazy", "step"],
+    p.add_argument("--profile", choices=["compile", "pairwise", "lists", "listdecode", "lazy", "step"],
                    help="run one part of the path alone (for profilers) and print its CUDA-event time "
                         "instead of the JSON line")
     p.add_argument("--requests", type=int, default=256, help="--profile lists: requests of the forest")
@@ -846,6 +846,7 @@ def run_dynamic(dev, stream, steps: int = 32, reps: int = 5, rank: int = 0, worl
                                    "unit": "GB/s", "frac": ab / (per_launch_us * 1e-6) / 1e9 / peak,
                                    "bytes_per_launch": ab, "us_per_launch": per_launch_us,
                                    "peak_kind": peak_kind, "kernel": "k_apply_lists",
+                                   "traffic": ncu_traffic("k_apply_lists", full.name),
                                    "timing": f"the {steps}-step decode graph (1 + {steps - 1} launches) over "
                                              f"its launches, CUDA events around {reps} replays"}
     lt, lw = [], []
@@ -1071,9 +1072,35 @@ def run_profile(args, w) -> None:
     else:
         h = T.trie_build_many(full.set_bytes, full.set_offsets, full.set_index)
     vh = T.trie_vocab_create(full.vocab_bytes, full.vocab_offsets, full.V)
-    timed(lambda: T.trie_compile_lists_vocab(h, vh, stream, count=False),
-          f"{args.requests}-request forest trie_compile_lists, {h.num_nodes} nodes")
-    print(f"{T.trie_num_valid(h)} entries")
+    if args.profile == "lists":
+        timed(lambda: T.trie_compile_lists_vocab(h, vh, stream, count=False),
+              f"{args.requests}-request forest trie_compile_lists, {h.num_nodes} nodes")
+        print(f"{T.trie_num_valid(h)} entries")
+        return
+    # listdecode: the 32-step list-driven decode of the dynamic workload
+    # (apply, then 31 fused advance + apply launches), greedy tokens replayed
+    steps, B, V = 32, full.batch, full.V
+    roots = torch.as_tensor(h.roots(), device=dev)
+    with torch.cuda.stream(stream):
+        T.trie_compile_lists_vocab(h, vh, stream)
+        logits = [W.logits(full, t, device=str(dev)) for t in range(steps)]
+        states = roots.clone()
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+        forced = torch.zeros((steps, B), dtype=torch.int32, device=dev)
+        for t in range(steps):
+            x = logits[t].clone()
+            T.trie_apply_lists(h, x, states, stream)
+            forced[t].copy_(torch.argmax(x, dim=1))
+            T.trie_advance(h, states, forced[t], err, stream)
+    sb = [torch.empty_like(roots), torch.empty_like(roots)]
+
+    def decode():
+        sb[0].copy_(roots)
+        T.trie_apply_lists(h, logits[0], sb[0], stream)
+        for t in range(1, steps):
+            T.trie_advance_apply_lists(h, sb[(t - 1) % 2], forced[t - 1], sb[t % 2], logits[t], err, stream)
+
+    timed(decode, f"{args.requests}-request list decode loop ({steps} launches, eager)")
 
 
 def launch_ranks(n: int) -> int:
