@@ -649,20 +649,29 @@ static int ensure_hits(trie_t h, int dev, cudaStream_t stream) {
 // The segment summary of the dense mask (bit g of row r set iff the row allows
 // a token of the 1,024-token segment g), which lets the apply skip reading
 // the mask words of empty segments; none when it would exceed 256 MB.
-static uint32_t *ensure_seg(trie_t h, int dev, cudaStream_t stream, int32_t words) {
+static unsigned long long *ensure_seg(trie_t h, int dev, cudaStream_t stream, int32_t words) {
     const int64_t need = int64_t(h->host.n) * words;
-    if (need * 4 > (int64_t(256) << 20)) return nullptr;
+    if (need * 8 > (int64_t(256) << 20)) return nullptr;
     std::lock_guard<std::mutex> lk(h->mu);
     if (h->dev.seg_cap < need) {
-        pool_free(h->dev.seg_any);  // an earlier apply may still read it
+        pool_free(h->dev.seg_epoch);  // an earlier apply may still read it
         h->dev.seg_any = nullptr;
+        h->dev.seg_epoch = nullptr;
         h->dev.seg_cap = 0;
         void *p = nullptr;
-        if (pool_alloc(dev, size_t(need) * 4, stream, &p, "the mask's segment summary") != TRIE_OK) {
+        const size_t bytes = 16 + size_t(need) * 8;  // the epoch word, then the summary words
+        if (pool_alloc(dev, bytes, stream, &p, "the mask's segment summary") != TRIE_OK) {
             cudaGetLastError();
             return nullptr;  // the compile and the apply work without it
         }
-        h->dev.seg_any = static_cast<uint32_t *>(p);
+        // epoch 0 is never a compile's: every word starts out empty
+        if (cudaMemsetAsync(p, 0, bytes, stream) != cudaSuccess) {
+            cudaGetLastError();
+            pool_free(p);
+            return nullptr;
+        }
+        h->dev.seg_epoch = static_cast<uint32_t *>(p);
+        h->dev.seg_any = reinterpret_cast<unsigned long long *>(static_cast<char *>(p) + 16);
         h->dev.seg_cap = need;
     }
     return h->dev.seg_any;
@@ -682,10 +691,12 @@ static int compile_masks(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, in
     bool fill_trans;
     if ((rc = prepare_trans(h, voc, sms, stream, &fill_trans)) != TRIE_OK) return rc;
     const int32_t seg_words = int32_t(((W + 31) / 32 + 31) / 32);
-    uint32_t *seg = ensure_seg(h, dev, stream, seg_words);
+    unsigned long long *seg = ensure_seg(h, dev, stream, seg_words);
+    const uint32_t epoch = h->dev.seg_epoch_next;
+    h->dev.seg_epoch_next = epoch == UINT32_MAX ? 1u : epoch + 1u;
     bool seg_written = false;
     cudaError_t e = tmk::launch_mask_compile3(h->dev, n, *voc, lmax, d_mask, W, sms, fill_trans, stream, seg,
-                                              seg_words, &seg_written);
+                                              h->dev.seg_epoch, epoch, seg_words, &seg_written);
     if (e != cudaSuccess) return fail_cuda(e, "mask compile launch");
     std::lock_guard<std::mutex> lk(h->mu);
     h->trans_vocab = voc;
@@ -693,8 +704,12 @@ static int compile_masks(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, in
     h->vocab = voc;
     h->mask = d_mask;
     h->mask_V = V;
-    h->mask_seg = seg_written ? seg : nullptr;
-    h->mask_seg_words = seg_words;
+    h->mask_seg = tmk::SegRef();
+    if (seg_written) {
+        h->mask_seg.words = seg;
+        h->mask_seg.epoch = h->dev.seg_epoch;
+        h->mask_seg.per_row = seg_words;
+    }
     return TRIE_OK;
 }
 
@@ -772,8 +787,7 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
     uint32_t *mask;
     int32_t mV;
     bool use_trans;
-    const uint32_t *seg;
-    int32_t seg_words;
+    tmk::SegRef seg;
     {
         std::lock_guard<std::mutex> lk(h->mu);
         voc = h->vocab;
@@ -781,7 +795,6 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
         mV = h->mask_V;
         use_trans = h->trans_vocab == voc;
         seg = h->mask_seg;
-        seg_words = h->mask_seg_words;
     }
     if (!mask || !voc) return fail(TRIE_ESTATE, "trie_advance_apply before trie_compile_masks on this handle");
     if (V != mV || V != voc->V) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
@@ -793,7 +806,7 @@ int trie_advance_apply(trie_t h, const int32_t *d_states_in, const int32_t *d_to
     if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
     cudaError_t e = tmk::launch_advance_apply(h->dev, h->host.n, *voc, use_trans, d_states_in, d_tokens,
                                               d_states_out, d_err, d_logits, dtype, mask, B, num_sms(dev), stream,
-                                              seg, seg_words);
+                                              seg);
     if (e != cudaSuccess) return fail_cuda(e, "advance-apply launch");
     return TRIE_OK;
 }
@@ -806,14 +819,12 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
     if (B > 0 && (!d_logits || !d_states)) return fail(TRIE_EINVAL, "d_logits / d_states is NULL");
     uint32_t *mask;
     int32_t mV;
-    const uint32_t *seg;
-    int32_t seg_words;
+    tmk::SegRef seg;
     {
         std::lock_guard<std::mutex> lk(h->mu);
         mask = h->mask;
         mV = h->mask_V;
         seg = h->mask_seg;
-        seg_words = h->mask_seg_words;
     }
     if (!mask) return fail(TRIE_ESTATE, "trie_apply_mask before trie_compile_masks on this handle");
     if (V != mV) return fail(TRIE_EINVAL, "V differs from the compiled mask's V");
@@ -823,8 +834,7 @@ int trie_apply_mask(trie_t h, void *d_logits, int dtype, const int32_t *d_states
     int dev, rc;
     if ((rc = current_device(&dev)) != TRIE_OK) return rc;
     if (dev != h->dev.device) return fail(TRIE_EINVAL, "handle belongs to another device");
-    cudaError_t e = tmk::launch_apply(d_logits, dtype, mask, d_states, B, V, h->host.n, num_sms(dev), stream, seg,
-                                      seg_words);
+    cudaError_t e = tmk::launch_apply(d_logits, dtype, mask, d_states, B, V, h->host.n, num_sms(dev), stream, seg);
     if (e != cudaSuccess) return fail_cuda(e, "apply launch");
     return TRIE_OK;
 }
@@ -1454,7 +1464,7 @@ int trie_destroy(trie_t h) {
             give_spare_block(h->dev.device, h->lists.base, h->lists.base_bytes, nullptr, 0);
         }
         pool_free(h->dev.hits_base);
-        pool_free(h->dev.seg_any);
+        pool_free(h->dev.seg_epoch);
         pool_free(h->dev.base);
         if (h->lists.done) cudaEventDestroy(h->lists.done);
     }
@@ -1532,7 +1542,7 @@ int trie_destroy_async(trie_t h, cudaStream_t stream) {
             }
         }
         free_on(h->dev.hits_base);
-        free_on(h->dev.seg_any);
+        free_on(h->dev.seg_epoch);
         free_on(h->dev.base);
         // the event may still be pending: CUDA defers its destruction
         if (h->lists.done) cudaEventDestroy(h->lists.done);

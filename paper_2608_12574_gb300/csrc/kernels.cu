@@ -125,8 +125,10 @@ struct PatchArgs {
     ulonglong2 *trans;         // transition table (row, token) -> end node, or null
     uint32_t trans_mask;       // slots - 1
     int32_t trans_fill;        // the probe inserts every transition it finds
-    uint32_t *seg_any;         // [n_nodes * seg_words]: bit g of row r = some token of segment g allowed, or null
-    int32_t seg_words;         // words per row of seg_any (segments of 1,024 tokens)
+    unsigned long long *seg_any;  // [n_nodes * seg_words] tagged summary words (see DevTrie), or null
+    uint32_t *seg_epoch;          // the device's current epoch, set to seg_tag by the probe
+    uint32_t seg_tag;             // this compile's epoch
+    int32_t seg_words;            // words per row of seg_any (segments of 1,024 tokens)
 };
 
 // Transition table: open addressing over 16-byte slots {key, end node};
@@ -569,25 +571,32 @@ __device__ __forceinline__ void set_mask_bit(const PatchArgs &a, int32_t row, in
     atomicOr(a.mask + int64_t(row) * a.W + (t >> 5), 1u << (t & 31));
 }
 
-// The bit, and the row's segment bit in the summary the apply reads first
-// (a 1,024-token segment whose bit is clear holds no allowed token).
-__device__ __forceinline__ void set_mask_bit_seg(const PatchArgs &a, int32_t row, int32_t t) {
-    set_mask_bit(a, row, t);
-    if (a.seg_any) {  // most hits of a row share a few segments: set a bit only once
-        const int32_t g = t >> 10;
-        uint32_t *w = a.seg_any + int64_t(row) * a.seg_words + (g >> 5);
-        const uint32_t bit = 1u << (g & 31);
-        if (!(*reinterpret_cast<volatile uint32_t *>(w) & bit)) atomicOr(w, bit);
+// The row's segment bit in the summary the apply reads first (a 1,024-token
+// segment whose bit is clear holds no allowed token), set by the probe while
+// the fill runs. A word that still carries an earlier compile's epoch is
+// claimed with this compile's epoch and the bit in one compare-and-swap (a
+// failed swap means another thread of this compile claimed it, so the loop
+// runs at most twice); a word of this compile gets the bit unless it has it
+// already (the rows near the root get thousands of hits in a few words).
+__device__ __forceinline__ void set_seg_bit(const PatchArgs &a, int32_t row, int32_t t) {
+    if (!a.seg_any) return;
+    const int32_t g = t >> 10;
+    unsigned long long *p = a.seg_any + int64_t(row) * a.seg_words + (g >> 5);
+    const unsigned long long bit = 1ull << (g & 31);
+    const unsigned long long tag = static_cast<unsigned long long>(a.seg_tag) << 32;
+    unsigned long long old = *reinterpret_cast<volatile unsigned long long *>(p);
+    while ((old & 0xFFFFFFFF00000000ull) != tag) {
+        const unsigned long long prev = atomicCAS(p, old, tag | bit);
+        if (prev == old) return;
+        old = prev;
     }
+    if (!(old & bit)) atomicOr(p, bit);
 }
 
-// Zeroes the segment summary (grid-stride; called by the probe, which runs
-// before the scatter that sets it).
-__device__ __forceinline__ void clear_seg_any(const PatchArgs &a) {
-    if (!a.seg_any) return;
-    const int64_t n = int64_t(a.n_nodes) * a.seg_words;
-    for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += int64_t(gridDim.x) * blockDim.x)
-        a.seg_any[i] = 0u;
+// Makes this compile's epoch the current one (the probe, before any apply of
+// this compile can read the summary).
+__device__ __forceinline__ void publish_seg_epoch(const PatchArgs &a) {
+    if (a.seg_any && blockIdx.x == 0 && threadIdx.x == 0) *a.seg_epoch = a.seg_tag;
 }
 
 // Fill-then-patch form (two kernels): climbs and probes overlap the fill,
@@ -617,7 +626,7 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
     pdl_wait();  // an earlier scatter may still read the hit buffer (an apply, the summary)
     if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
     pdl_launch_dependents();
-    clear_seg_any(a);
+    publish_seg_epoch(a);
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
         int32_t c = 0;
@@ -625,6 +634,7 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
         node_hits_window(a, m, [&](int32_t row, int32_t t) {
             if (c < kHitSlots) slot[c] = make_int2(row, t);
             c++;
+            set_seg_bit(a, row, t);
             if (a.trans_fill && t != a.eos) trans_insert(a.trans, a.trans_mask, row, t, m);
         });
         a.hit_count[m] = uint8_t(c > kHitSlots ? kHitOverflow : c);
@@ -649,7 +659,7 @@ __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs 
     if (!kOr) {
         pdl_wait();  // an earlier scatter may still read the hit buffer (an apply, the summary)
         if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
-        clear_seg_any(a);
+        publish_seg_epoch(a);
     }
     pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
@@ -701,6 +711,7 @@ __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs 
             } else {
                 if (s < kHitSlots) slot[s] = make_int2(row, tok);
                 s++;
+                set_seg_bit(a, row, tok);
             }
             if (a.trans_fill && tok != a.eos) trans_insert(a.trans, a.trans_mask, row, tok, m);
         };
@@ -718,7 +729,7 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_scatter(PatchArgs a) 
     pdl_wait();  // fill complete, and through it the probe
     const int32_t stride = gridDim.x * blockDim.x;
     for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < a.n_nodes; m += stride) {
-        auto emit = [&](int32_t row, int32_t t) { set_mask_bit_seg(a, row, t); };
+        auto emit = [&](int32_t row, int32_t t) { set_mask_bit(a, row, t); };
         const int32_t c = a.hit_count[m];
         if (c == kHitOverflow) {
             node_hits_window(a, m, emit);
@@ -881,15 +892,20 @@ __device__ __forceinline__ uint32_t row_word(const uint32_t *__restrict__ mask, 
     return (w == (eos >> 5)) ? (1u << (eos & 31)) : 0u;
 }
 
+// The current summary epoch (read once a kernel's wait for earlier work is done).
+__device__ __forceinline__ uint32_t seg_epoch_now(const SegRef &sg) { return sg.words ? __ldg(sg.epoch) : 0u; }
+
 // Mask word w of state s's row, reading the row only when the segment
-// summary (if any) says segment seg holds an allowed token.
-__device__ __forceinline__ uint32_t seg_row_word(const uint32_t *__restrict__ mask,
-                                                 const uint32_t *__restrict__ seg_any, int32_t seg_words,
+// summary (if any) says segment seg holds an allowed token: a summary word
+// that does not carry the current epoch ep says no segment of it does.
+__device__ __forceinline__ uint32_t seg_row_word(const uint32_t *__restrict__ mask, const SegRef &sg, uint32_t ep,
                                                  int32_t s, int32_t n_nodes, int64_t W, int32_t seg, int64_t w,
                                                  int32_t eos) {
-    if (seg_any && s >= 0 && s < n_nodes &&
-        !((__ldg(seg_any + int64_t(s) * seg_words + (seg >> 5)) >> (seg & 31)) & 1u))
-        return 0u;
+    if (sg.words && s >= 0 && s < n_nodes) {
+        const unsigned long long v = __ldg(sg.words + int64_t(s) * sg.per_row + (seg >> 5));
+        const uint32_t bits = uint32_t(v >> 32) == ep ? uint32_t(v) : 0u;
+        if (!((bits >> (seg & 31)) & 1u)) return 0u;
+    }
     return row_word(mask, s, n_nodes, W, w, eos);
 }
 
@@ -969,8 +985,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
                                                              const uint32_t *__restrict__ mask,
                                                              const int32_t *__restrict__ states, int32_t B,
                                                              int32_t V, int64_t W, int32_t n_nodes,
-                                                             int32_t segs, const uint32_t *__restrict__ seg_any,
-                                                             int32_t seg_words) {
+                                                             int32_t segs, SegRef sg) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     __shared__ __align__(128) uint4 tile[kSegChunks];
     init_ninf_tile<kElt>(tile);
@@ -980,7 +995,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_apply_vec(uint4 *__restrict__
     const int32_t item = int32_t(blockIdx.x) * (kApplyThreads / 32) + (threadIdx.x >> 5);
     if (item >= B * segs) return;  // uniform per warp
     const int32_t b = item / segs, seg = item - b * segs;
-    const uint32_t word = seg_row_word(mask, seg_any, seg_words, __ldg(states + b), n_nodes, W, seg,
+    const uint32_t word = seg_row_word(mask, sg, seg_epoch_now(sg), __ldg(states + b), n_nodes, W, seg,
                                        int64_t(seg) * 32 + lane, V - 1);
     const int64_t row_chunks = int64_t(V) / (16 / kElt);
     write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
@@ -1002,17 +1017,18 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
                                                                      int32_t *__restrict__ states_out,
                                                                      int32_t *__restrict__ err, int32_t B,
                                                                      int64_t W, int32_t segs, int32_t parts,
-                                                                     const uint32_t *__restrict__ seg_any,
-                                                                     int32_t seg_words) {
+                                                                     SegRef sg) {
     constexpr int kSegChunks = 1024 / (16 / kElt);
     __shared__ __align__(128) uint4 tile[kSegChunks];
     __shared__ int32_t next_state;
+    __shared__ uint32_t epoch;
     pdl_launch_dependents();
     const int32_t b = int32_t(blockIdx.x) / parts, part = int32_t(blockIdx.x) - b * parts;
     for (int i = threadIdx.x; i < kSegChunks; i += blockDim.x) tile[i] = ninf16<kElt>();
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // tile visible to the bulk copies
     if (threadIdx.x == 0) {
         pdl_wait();  // states and tokens come from earlier kernels
+        epoch = seg_epoch_now(sg);  // loaded beside the advance's chain
         const int32_t s = __ldg(states_in + b);
         const int32_t nxt = advance_one(aa, s, __ldg(tokens + b));
         next_state = nxt;
@@ -1026,7 +1042,7 @@ __global__ void __launch_bounds__(kApplyThreads) k_advance_apply_vec(AdvanceArgs
     const int lane = threadIdx.x & 31;
     const int32_t seg = part * (kApplyThreads / 32) + int32_t(threadIdx.x >> 5);
     if (seg >= segs) return;  // uniform per warp
-    const uint32_t word = seg_row_word(mask, seg_any, seg_words, next_state, aa.n_nodes, W, seg,
+    const uint32_t word = seg_row_word(mask, sg, epoch, next_state, aa.n_nodes, W, seg,
                                        int64_t(seg) * 32 + lane, aa.V - 1);
     const int64_t row_chunks = int64_t(aa.V) / (16 / kElt);
     write_segment<kElt>(logits + int64_t(b) * row_chunks, int64_t(seg) * kSegChunks, row_chunks, word, lane,
@@ -1798,6 +1814,8 @@ PatchArgs patch_args(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32
     a.trans_mask = t.trans_mask;
     a.trans_fill = 0;
     a.seg_any = nullptr;
+    a.seg_epoch = nullptr;
+    a.seg_tag = 0;
     a.seg_words = 0;
     return a;
 }
@@ -1874,7 +1892,8 @@ cudaError_t launch_vocab_pay(const DevVocab &v, uint4 *pay, int num_sms, cudaStr
 
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st,
-                                 uint32_t *seg_any, int32_t seg_words, bool *seg_written) {
+                                 unsigned long long *seg_any, uint32_t *seg_epoch, uint32_t epoch,
+                                 int32_t seg_words, bool *seg_written) {
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
     a.trans_fill = fill_trans && t.trans;
     *seg_written = false;
@@ -1893,7 +1912,9 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
         return launch_pdl(k_mask_probe_pair<true>, grid_for(2 * int64_t(n_nodes), kPatchThreads, int64_t(num_sms) * 4),
                           kPatchThreads, st, a, pf);
     }
-    a.seg_any = seg_any;  // the probe clears it, the scatter sets it
+    a.seg_any = seg_any;  // the probe sets it (with this compile's epoch)
+    a.seg_epoch = seg_epoch;
+    a.seg_tag = epoch;
     a.seg_words = seg_words;
     *seg_written = seg_any != nullptr;
     const uint64_t S = uint64_t(v.ht_mask) + 1, nn = uint64_t(n_nodes), nv = uint64_t(v.V);
@@ -1954,7 +1975,7 @@ cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v,
 cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
                                  const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                                  int32_t *err, void *logits, int dtype, const uint32_t *mask, int32_t B,
-                                 int num_sms, cudaStream_t st, const uint32_t *seg_any, int32_t seg_words) {
+                                 int num_sms, cudaStream_t st, const SegRef &seg) {
     const int32_t V = v.V;
     const int64_t W = (int64_t(V) + 31) / 32;
     const int elt = dtype == 0 ? 4 : 2;
@@ -1964,7 +1985,7 @@ cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVoc
     if (!vec) {  // any V and alignment: the two kernels one after the other
         cudaError_t e = launch_advance(t, n_nodes, v, states_in, states_out, tokens, B, err, use_trans, st);
         if (e != cudaSuccess) return e;
-        return launch_apply(logits, dtype, mask, states_out, B, V, n_nodes, num_sms, st, seg_any, seg_words);
+        return launch_apply(logits, dtype, mask, states_out, B, V, n_nodes, num_sms, st, seg);
     }
     const AdvanceArgs aa = advance_args(t, n_nodes, v, use_trans);
     const int32_t parts = (segs + kApplyThreads / 32 - 1) / (kApplyThreads / 32);
@@ -1972,14 +1993,14 @@ cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVoc
     if (grid > INT32_MAX) return cudaErrorInvalidValue;
     if (elt == 2)
         return launch_pdl(k_advance_apply_vec<2>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
-                          states_in, tokens, states_out, err, B, W, segs, parts, seg_any, seg_words);
+                          states_in, tokens, states_out, err, B, W, segs, parts, seg);
     return launch_pdl(k_advance_apply_vec<4>, grid, kApplyThreads, st, aa, static_cast<uint4 *>(logits), mask,
-                      states_in, tokens, states_out, err, B, W, segs, parts, seg_any, seg_words);
+                      states_in, tokens, states_out, err, B, W, segs, parts, seg);
 }
 
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
                          int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st,
-                         const uint32_t *seg_any, int32_t seg_words) {
+                         const SegRef &seg) {
     const int64_t W = (int64_t(V) + 31) / 32;
     const int elt = dtype == 0 ? 4 : 2;
     const int32_t segs = int32_t((W + 31) / 32);
@@ -1990,9 +2011,9 @@ cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const in
         const int grid = grid_for(items, kApplyThreads / 32, INT32_MAX);
         if (elt == 2)
             return launch_pdl(k_apply_vec<2>, grid, kApplyThreads, st, static_cast<uint4 *>(logits), mask,
-                              states, B, V, W, n_nodes, segs, seg_any, seg_words);
+                              states, B, V, W, n_nodes, segs, seg);
         return launch_pdl(k_apply_vec<4>, grid, kApplyThreads, st, static_cast<uint4 *>(logits), mask, states,
-                          B, V, W, n_nodes, segs, seg_any, seg_words);
+                          B, V, W, n_nodes, segs, seg);
     }
     const int grid = grid_for(int64_t(B) * V, kApplyThreads, int64_t(num_sms) * 16);
     if (elt == 2)
@@ -2220,7 +2241,7 @@ cudaError_t launch_lazy(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bo
     e = launch_pdl_smem(k_lazy_rows, rows_grid, kLazyRowThreads, size_t(L.W) * sizeof(uint32_t), st, la, pa);
     if (e != cudaSuccess) return e;
     const int32_t n_rows = L.C + L.max_batch;
-    if (logits) return launch_apply(logits, dtype, L.rows, L.slot_of, B, L.V, n_rows, num_sms, st, nullptr, 0);
+    if (logits) return launch_apply(logits, dtype, L.rows, L.slot_of, B, L.V, n_rows, num_sms, st);
     const int grid = grid_for(int64_t(B) * L.W, kApplyThreads, int64_t(num_sms) * 8);
     return launch_pdl(k_lazy_gather, grid, kApplyThreads, st, static_cast<const uint32_t *>(L.rows),
                       static_cast<const int32_t *>(L.slot_of), B, L.W, n_rows, L.V - 1, rows_out);

@@ -229,6 +229,14 @@ struct DevVocab {
 // searched again by the scatter).
 constexpr int kHitSlots = 16;
 
+// The segment summary an apply reads: words per row, the epoch word; words
+// null when the compile computed no summary.
+struct SegRef {
+    const unsigned long long *words = nullptr;
+    const uint32_t *epoch = nullptr;
+    int32_t per_row = 0;
+};
+
 struct DevTrie {
     int device = -1;
     void *base = nullptr;
@@ -246,7 +254,14 @@ struct DevTrie {
     int4 *anc = nullptr;             // [n * 4]
     ulonglong2 *trans = nullptr;     // transition table {(row << 32 | token) + 1, end node}
     uint32_t trans_mask = 0;         // slots - 1
-    uint32_t *seg_any = nullptr;     // segment summary of the dense mask (own allocation), seg_cap words
+    // Segment summary of the dense mask (own allocation): per row, words of 32
+    // segment bits (1,024 tokens each) tagged in their high half with the
+    // epoch of the compile that set them; a word with another tag than the
+    // device's current epoch (*seg_epoch, written by each compile's probe)
+    // holds no allowed token.
+    unsigned long long *seg_any = nullptr;  // seg_cap words
+    uint32_t *seg_epoch = nullptr;          // [1] (device), the epoch of the last compile that ran
+    uint32_t seg_epoch_next = 1;            // host: the epoch of the next compile (0 is never used)
     int64_t seg_cap = 0;
     void *hits_base = nullptr;       // the two arrays below (allocated by the first dense compile)
     int2 *hits = nullptr;            // compile scratch: kHitSlots (row, token) pairs per node
@@ -400,8 +415,7 @@ struct trie_s {
     std::shared_ptr<tmk::DevVocab> vocab; // vocabulary of the last compile
     uint32_t *mask = nullptr;            // last compiled mask (caller-owned)
     int32_t mask_V = 0;
-    const uint32_t *mask_seg = nullptr;  // its segment summary (dev.seg_any), or null when not computed
-    int32_t mask_seg_words = 0;
+    tmk::SegRef mask_seg;                // its segment summary (in dev.seg_any), words null when not computed
     tmk::DevLists lists;                 // last compiled valid lists (library-owned)
     std::shared_ptr<tmk::DevVocab> trans_vocab;  // vocabulary the transition table holds
     bool trans_complete = false;         // filled by a whole compile (else partly, by lazy rows)
@@ -427,7 +441,8 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
 // beside the fill (needs t.hits / t.hit_count).
 cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVocab &v, int32_t lmax,
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st,
-                                 uint32_t *seg_any, int32_t seg_words, bool *seg_written);
+                                 unsigned long long *seg_any, uint32_t *seg_epoch, uint32_t epoch,
+                                 int32_t seg_words, bool *seg_written);
 // Fills t.first_child and t.child_bits from t.parent and t.label (which must
 // be -1 / zero on entry: the caller clears them on the same stream).
 cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
@@ -444,10 +459,10 @@ cudaError_t launch_advance(const DevTrie &t, int32_t n_nodes, const DevVocab &v,
 cudaError_t launch_advance_apply(const DevTrie &t, int32_t n_nodes, const DevVocab &v, bool use_trans,
                                  const int32_t *states_in, const int32_t *tokens, int32_t *states_out,
                                  int32_t *err, void *logits, int dtype, const uint32_t *mask, int32_t B,
-                                 int num_sms, cudaStream_t st, const uint32_t *seg_any, int32_t seg_words);
+                                 int num_sms, cudaStream_t st, const SegRef &seg);
 cudaError_t launch_apply(void *logits, int dtype, const uint32_t *mask, const int32_t *states,
                          int32_t B, int32_t V, int32_t n_nodes, int num_sms, cudaStream_t st,
-                         const uint32_t *seg_any = nullptr, int32_t seg_words = 0);
+                         const SegRef &seg = SegRef());
 // Copies (d_k, s_k, b_k bytes), k = 0..2, in one launch; the sources are read
 // by the kernel itself (device memory, or host memory the device reads
 // coherently), so no copy engine and no host synchronisation is involved.
