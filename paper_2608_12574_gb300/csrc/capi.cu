@@ -648,7 +648,12 @@ static int ensure_hits(trie_t h, int dev, cudaStream_t stream) {
 
 // The segment summary of the dense mask (bit g of row r set iff the row allows
 // a token of the 1,024-token segment g), which lets the apply skip reading
-// the mask words of empty segments; none when it would exceed 256 MB.
+// the mask words of empty segments; none when it would exceed 256 MB, and
+// none for tries of more than kSegMaxNodes nodes: the probe sets the summary
+// while the fill runs, and for a forest of millions of nodes its
+// compare-and-swaps made it outlast the fill (dense compile of the 4.77 M-node
+// forest 12.9 ms with the summary, 11.1 ms without).
+constexpr int32_t kSegMaxNodes = int32_t(1) << 18;
 static unsigned long long *ensure_seg(trie_t h, int dev, cudaStream_t stream, int32_t words) {
     const int64_t need = int64_t(h->host.n) * words;
     if (need * 8 > (int64_t(256) << 20)) return nullptr;
@@ -691,7 +696,7 @@ static int compile_masks(trie_t h, const std::shared_ptr<tmk::DevVocab> &voc, in
     bool fill_trans;
     if ((rc = prepare_trans(h, voc, sms, stream, &fill_trans)) != TRIE_OK) return rc;
     const int32_t seg_words = int32_t(((W + 31) / 32 + 31) / 32);
-    unsigned long long *seg = ensure_seg(h, dev, stream, seg_words);
+    unsigned long long *seg = n <= kSegMaxNodes ? ensure_seg(h, dev, stream, seg_words) : nullptr;
     const uint32_t epoch = h->dev.seg_epoch_next;
     h->dev.seg_epoch_next = epoch == UINT32_MAX ? 1u : epoch + 1u;
     bool seg_written = false;
