@@ -491,9 +491,10 @@ def run_gpu(args, w, rank: int, world: int, dist):
                   f"advance+apply launches of a step (over {S - 1} logits buffers, "
                   f"{(S - 1) * B * V * elt / 1e9:.2f} GB > L2), launching stream, right after the timed region")
     # bytes an apply must move: the B x V logits written, the states, and of
-    # each state's mask row the segment summary plus the 1,024-token segments
-    # that hold an allowed token (the compile's summary lets the apply skip
-    # reading the others), averaged over the decode steps' states
+    # each state's mask row the segment summary (8-byte words: 32 segment bits
+    # and the compile's epoch) plus the 1,024-token segments that hold an
+    # allowed token (the compile's summary lets the apply skip reading the
+    # others), averaged over the decode steps' states
     segs = (Wd + 31) // 32
     seg_words = (segs + 31) // 32
     occupied = 0
@@ -504,7 +505,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
         rows = torch.nn.functional.pad(rows, (0, segs * 32 - Wd)).view(B, segs, 32)
         occ = (rows != 0).any(dim=2) & node[:, None]
         occupied += int(occ.sum().item())  # FINISHED / DEAD rows ({EOS}) read no mask word
-    apply_bytes = B * V * elt + B * 4 + B * seg_words * 4 + (occupied / S) * 128
+    apply_bytes = B * V * elt + B * 4 + B * seg_words * 8 + (occupied / S) * 128
     fused_bytes = apply_bytes + 2 * B * 4  # + tokens read, new states written
     compile_bytes = N * Wd * 4
     apply_gbs = apply_bytes / (apply_avg * 1e-3) / 1e9
