@@ -443,19 +443,19 @@ __device__ __forceinline__ int32_t anc_at(const int4 (&an)[4], int k) {
 // vocabulary where some tokens share a key, a key whose first pair is full
 // takes the sequential probe, which finds every token under it.
 // One wavefront of node_hits_window: the suffixes of lengths k0 + 1 ..
-// k0 + 8 (those within depth) of node m. h and pw hold the hash of the
+// k0 + N (those within depth) of node m (N = 8, or 4 for the quad probe). h and pw hold the hash of the
 // first k0 labels and B^k0 and are advanced over the batch; hit(i, row, t)
 // is called for every token t that is the suffix of length k0 + i + 1
 // (starting at row).
-template <typename Hit>
-__device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0, int32_t depth,
-                                           const uint32_t (&lab)[4], const int4 (&an)[4], uint64_t &h,
-                                           uint64_t &pw, Hit hit) {
+template <int N, typename Hit>
+__device__ __forceinline__ void wavefront(const PatchArgs &a, int32_t m, int k0, int32_t depth,
+                                          const uint32_t (&lab)[4], const int4 (&an)[4], uint64_t &h,
+                                          uint64_t &pw, Hit hit) {
     const ulonglong2 *pairs = reinterpret_cast<const ulonglong2 *>(a.ht_key);
-    uint64_t key[8];
-    ulonglong2 first[8];
+    uint64_t key[N];
+    ulonglong2 first[N];
 #pragma unroll
-    for (int i = 0; i < 8; i++) {
+    for (int i = 0; i < N; i++) {
         key[i] = 0ull;
         first[i] = make_ulonglong2(0ull, 0ull);
         if (k0 + i < depth) {
@@ -465,17 +465,17 @@ __device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0
             first[i] = __ldg(pairs + (uint32_t(key[i] >> 1) & a.pairs_mask));
         }
     }
-    int32_t slot[8];  // slot of the key, -1 none
+    int32_t slot[N];  // slot of the key, -1 none
     uint32_t slow = 0;  // bit i: candidate i needs the sequential probe
     if (!a.dup_keys) {
         uint32_t pending = 0;
 #pragma unroll
-        for (int i = 0; i < 8; i++)
+        for (int i = 0; i < N; i++)
             if (k0 + i < depth) pending |= 1u << i;
-        find_slots<8>(a, key, pending, first, slot);
+        find_slots<N>(a, key, pending, first, slot);
     } else {
 #pragma unroll
-        for (int i = 0; i < 8; i++) {
+        for (int i = 0; i < N; i++) {
             const bool m0 = first[i].x == key[i], m1 = first[i].y == key[i];
             const uint32_t pr = uint32_t(key[i] >> 1) & a.pairs_mask;
             slot[i] = (k0 + i < depth && (m0 || m1)) ? int32_t(2 * pr + (m0 ? 0 : 1)) : -1;
@@ -485,16 +485,16 @@ __device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0
             }
         }
     }
-    int32_t tid[8];
-    int32_t tlen[8];
-    uint32_t toff[8];
-    uint4 tb[8];
+    int32_t tid[N];
+    int32_t tlen[N];
+    uint32_t toff[N];
+    uint4 tb[N];
     if (a.ht_pay) {
         // one load per match gives the token, its length, its offset
         // and its first 8 bytes; suffixes of 9-16 bytes then read the
         // rest from the blob
 #pragma unroll
-        for (int i = 0; i < 8; i++) {
+        for (int i = 0; i < N; i++) {
             const uint4 p = slot[i] >= 0 ? __ldg(a.ht_pay + slot[i]) : make_uint4(0u, 0u, 0u, 0u);
             tid[i] = slot[i] >= 0 ? int32_t(p.x) : -1;
             tlen[i] = slot[i] >= 0 ? int32_t(p.y >> 27) : -1;
@@ -502,25 +502,25 @@ __device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0
             tb[i] = make_uint4(p.z, p.w, 0u, 0u);
         }
 #pragma unroll
-        for (int i = 0; i < 8; i++)
+        for (int i = 0; i < N; i++)
             if (k0 + i + 1 > 8 && tlen[i] == k0 + i + 1)
                 tb[i] = __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]));
     } else {
 #pragma unroll
-        for (int i = 0; i < 8; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
+        for (int i = 0; i < N; i++) tid[i] = slot[i] >= 0 ? __ldg(a.ht_val + slot[i]) : -1;
 #pragma unroll
-        for (int i = 0; i < 8; i++) {
+        for (int i = 0; i < N; i++) {
             tlen[i] = tid[i] >= 0 ? int32_t(__ldg(a.tok_len + tid[i])) : -1;
             toff[i] = tid[i] >= 0 ? __ldg(a.tok_off + tid[i]) : 0u;
         }
         // token bytes: 16-byte aligned in the blob, which has 16 bytes of tail room
 #pragma unroll
-        for (int i = 0; i < 8; i++)
+        for (int i = 0; i < N; i++)
             tb[i] = tlen[i] == k0 + i + 1 ? __ldg(reinterpret_cast<const uint4 *>(a.blob + toff[i]))
                                           : make_uint4(0u, 0u, 0u, 0u);
     }
 #pragma unroll
-    for (int i = 0; i < 8; i++) {
+    for (int i = 0; i < N; i++) {
         const int k = k0 + i + 1;  // suffix length
         if (slow & (1u << i)) {
             probe(a, key[i], k, &lab, m, [&](int32_t t) { hit(i, anc_at(an, k - 1), t); });
@@ -534,6 +534,13 @@ __device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0
             if (eq) hit(i, anc_at(an, k - 1), tid[i]);
         }
     }
+}
+
+template <typename Hit>
+__device__ __forceinline__ void wavefront8(const PatchArgs &a, int32_t m, int k0, int32_t depth,
+                                           const uint32_t (&lab)[4], const int4 (&an)[4], uint64_t &h,
+                                           uint64_t &pw, Hit hit) {
+    wavefront<8>(a, m, k0, depth, lab, an, h, pw, hit);
 }
 
 template <typename Emit>
@@ -672,21 +679,22 @@ __global__ void __launch_bounds__(kPatchThreads, 4) k_mask_probe(PatchArgs a, Pr
     }
 }
 
-// k_mask_probe with two threads per node, for tries so small that one
+// k_mask_probe with L = 2 or 4 threads per node, for tries so small that one
 // thread per node leaves most SMs idle and the probe's chain of dependent
-// loads sets the compile time: lanes 2j and 2j + 1 of a warp take node j of
-// the warp's 16, the even lane EOS and the suffixes of lengths 1-8, the odd
-// lane lengths 9-16, each as one wavefront (the same instructions on every
-// lane, k0 = 0 or 8). The pair then writes its hits in node_hits_window's
-// order (EOS, lengths 1..16) into the node's slots, so the hit buffer is
-// that of k_mask_probe. Only for vocabularies with the per-slot payload (at
-// most one token per suffix) and tokens of at most 16 bytes.
+// loads sets the compile time: lanes Lj .. Lj + L - 1 of a warp take node j
+// of the warp's 32 / L, lane q the suffixes of lengths 16q/L + 1 .. 16(q+1)/L
+// (lane 0 also EOS), each as one wavefront (the same instructions on every
+// lane). The lanes then write their hits in node_hits_window's order (EOS,
+// lengths 1..16) into the node's slots, so the hit buffer is that of
+// k_mask_probe. Only for vocabularies with the per-slot payload (at most one
+// token per suffix) and tokens of at most 16 bytes.
 //
 // kOr: the two-kernel form for small masks. The zero fill runs first; this
 // kernel searches (read-only tables) while the fill runs, waits for it, and
 // ORs its hits into the mask itself: no hit buffer, no scatter launch.
-template <bool kOr>
+template <int L, bool kOr>
 __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs a, Prefetch pf) {
+    constexpr int N = 16 / L;  // suffix lengths per lane
     if (!kOr) {
         pdl_wait();  // an earlier scatter may still read the hit buffer (an apply, the summary)
         if (threadIdx.x == 0) l2_prefetch_slice(pf, blockIdx.x, gridDim.x);
@@ -694,48 +702,54 @@ __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs 
     }
     pdl_launch_dependents();
     const int lane = threadIdx.x & 31;
-    const int half = lane & 1;
-    const int k0 = 8 * half;
+    const int q = lane & (L - 1);  // this lane's share of the node: lengths k0 + 1 .. k0 + N
+    const int k0 = N * q;
     const int64_t stride = int64_t(gridDim.x) * blockDim.x;
-    const int64_t n2 = 2 * int64_t(a.n_nodes);
+    const int64_t nl = L * int64_t(a.n_nodes);
     // every lane of a warp runs the same iterations (the shuffles below)
-    for (int64_t w0 = int64_t(blockIdx.x) * blockDim.x + (threadIdx.x & ~31); w0 < n2; w0 += stride) {
+    for (int64_t w0 = int64_t(blockIdx.x) * blockDim.x + (threadIdx.x & ~31); w0 < nl; w0 += stride) {
         const int64_t t = w0 + lane;
-        const bool valid = t < n2;
-        const int32_t m = valid ? int32_t(t >> 1) : 0;
-        int32_t found[8];
+        const bool valid = t < nl;
+        const int32_t m = valid ? int32_t(t / L) : 0;
+        int32_t found[N];
 #pragma unroll
-        for (int i = 0; i < 8; i++) found[i] = -1;
+        for (int i = 0; i < N; i++) found[i] = -1;
         int4 an[4] = {};
         bool eos = false;
         if (valid) {
             const ulonglong2 win = __ldg(a.window + m);
 #pragma unroll
-            for (int q = 0; q < 4; q++) an[q] = __ldg(a.anc + int64_t(m) * 4 + q);
+            for (int g = 0; g < 4; g++) an[g] = __ldg(a.anc + int64_t(m) * 4 + g);
             const int32_t d16 = __ldg(a.depth16 + m);
             const int32_t depth = a.lmax < d16 ? a.lmax : d16;
             const uint32_t lab[4] = {uint32_t(win.x), uint32_t(win.x >> 32), uint32_t(win.y),
                                      uint32_t(win.y >> 32)};
-            eos = half == 0 && __ldg(a.terminal + m);
+            eos = q == 0 && __ldg(a.terminal + m);
             uint64_t h = 0, pw = 1;
 #pragma unroll
-            for (int j = 0; j < 8; j++)  // the odd lane starts after the first 8 labels
-                if (half && j < depth) {
+            for (int j = 0; j < 16 - N; j++)  // the hash of the labels before this lane's first
+                if (j < k0 && j < depth) {
                     h += (uint64_t(byte_at(lab, j)) + 1ull) * pw;
                     pw *= kHashBase;
                 }
             if (k0 < depth)
-                wavefront8(a, m, k0, depth, lab, an, h, pw, [&](int i, int32_t, int32_t tok) { found[i] = tok; });
+                wavefront<N>(a, m, k0, depth, lab, an, h, pw, [&](int i, int32_t, int32_t tok) { found[i] = tok; });
         }
         int32_t c = eos ? 1 : 0;
 #pragma unroll
-        for (int i = 0; i < 8; i++) c += found[i] >= 0 ? 1 : 0;
-        const int32_t c0 = __shfl_sync(0xffffffffu, c, lane & ~1);
-        const int32_t c1 = __shfl_sync(0xffffffffu, c, lane | 1);
+        for (int i = 0; i < N; i++) c += found[i] >= 0 ? 1 : 0;
+        // hits before this lane's within the node (lanes of a node are consecutive)
+        int32_t before = 0, total = 0;
+#pragma unroll
+        for (int r = 0; r < L; r++) {
+            const int32_t cr = __shfl_sync(0xffffffffu, c, (lane & ~(L - 1)) + r);
+            before += r < q ? cr : 0;
+            total += cr;
+        }
         if (!valid) continue;
         if (kOr) pdl_wait();  // the fill of this mask (and of the transition table) is complete
         int2 *slot = a.hits + int64_t(m) * kHitSlots;
-        int32_t s = half ? c0 : 0;
+        int32_t s = before;
         auto rec = [&](int32_t row, int32_t tok) {
             if (kOr) {
                 set_mask_bit(a, row, tok);
@@ -747,20 +761,20 @@ __global__ void __launch_bounds__(kPatchThreads, 3) k_mask_probe_pair(PatchArgs 
         };
         if (eos) rec(m, a.eos);
 #pragma unroll
-        for (int i = 0; i < 8; i++)
+        for (int i = 0; i < N; i++)
             if (found[i] >= 0) rec(anc_at(an, k0 + i), found[i]);
         if (!kOr) {  // the summary bits of the lane's hits, together
-            int32_t hr[9], ht[9];
+            int32_t hr[N + 1], ht[N + 1];
 #pragma unroll
-            for (int i = 0; i < 8; i++) {
+            for (int i = 0; i < N; i++) {
                 hr[i] = anc_at(an, k0 + i);
                 ht[i] = found[i];
             }
-            hr[8] = m;
-            ht[8] = eos ? a.eos : -1;
-            set_seg_bits<9>(a, hr, ht);
+            hr[N] = m;
+            ht[N] = eos ? a.eos : -1;
+            set_seg_bits<N + 1>(a, hr, ht);
         }
-        if (!kOr && half == 0) a.hit_count[m] = uint8_t(c0 + c1 > kHitSlots ? kHitOverflow : c0 + c1);
+        if (!kOr && q == 0) a.hit_count[m] = uint8_t(total > kHitSlots ? kHitOverflow : total);
     }
 }
 
@@ -1878,11 +1892,18 @@ bool pair_probe(const PatchArgs &a, int num_sms) {
     return a.ht_pay && a.lmax <= kMaxClimb && 2 * int64_t(a.n_nodes) * 2 <= resident;
 }
 
+// Lanes per node of the small-trie probe: 4 beside the fill (K = 1,000:
+// 32.9 us per compile against 35.0 us with 2: the search under the fill's
+// write stream is the long pole there, and 4 lanes shorten each lane's
+// chain), 2 in the small-mask form (K = 100: 10.3 us against 12.3 us with 4).
+constexpr int kProbeLanesBeside = 4;
+constexpr int kProbeLanesSmall = 2;
+
 cudaError_t launch_probe(const PatchArgs &a, const Prefetch &pf, int num_sms, cudaStream_t st) {
     if (pair_probe(a, num_sms))
-        return launch_pdl(k_mask_probe_pair<false>,
-                          grid_for(2 * int64_t(a.n_nodes), kPatchThreads, int64_t(num_sms) * 4), kPatchThreads, st,
-                          a, pf);
+        return launch_pdl(k_mask_probe_pair<kProbeLanesBeside, false>,
+                          grid_for(kProbeLanesBeside * int64_t(a.n_nodes), kPatchThreads, int64_t(num_sms) * 4),
+                          kPatchThreads, st, a, pf);
     return launch_pdl(k_mask_probe, grid_for(a.n_nodes, kPatchThreads, int64_t(num_sms) * 4), kPatchThreads, st, a,
                       pf);
 }
@@ -1950,7 +1971,8 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
         // small masks: the zero fill, then the search ORing its hits itself
         cudaError_t e = launch_mask_fill(mask, n_words, num_sms, st);
         if (e != cudaSuccess) return e;
-        return launch_pdl(k_mask_probe_pair<true>, grid_for(2 * int64_t(n_nodes), kPatchThreads, int64_t(num_sms) * 4),
+        return launch_pdl(k_mask_probe_pair<kProbeLanesSmall, true>,
+                          grid_for(kProbeLanesSmall * int64_t(n_nodes), kPatchThreads, int64_t(num_sms) * 4),
                           kPatchThreads, st, a, pf);
     }
     a.seg_any = seg_any;  // the probe sets it (with this compile's epoch)
