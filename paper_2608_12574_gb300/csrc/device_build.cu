@@ -388,8 +388,9 @@ __device__ __forceinline__ int32_t set_excl_scan(int32_t v, int32_t *ws, int32_t
 }
 
 // Dynamic shared memory: the child-label sets of the current level
-// (smax rows of 8 words), the first child of each of its nodes, and a flag
-// per node of the next level that some string ends at.
+// (smax rows of 8 words), for each row the labels counted in its words before
+// each word (8 bytes), the first child of each of its nodes, and a flag per
+// node of the next level that some string ends at.
 __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restrict__ bytes,
                                                         const int64_t *__restrict__ off,
                                                         const int32_t *__restrict__ set_off, int32_t M, int32_t smax,
@@ -398,7 +399,8 @@ __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restric
                                                         unsigned long long *__restrict__ chars) {
     extern __shared__ uint4 dyn[];
     uint32_t *bits = reinterpret_cast<uint32_t *>(dyn);
-    int32_t *first = reinterpret_cast<int32_t *>(bits + int64_t(smax) * 8);
+    uint2 *cum = reinterpret_cast<uint2 *>(bits + int64_t(smax) * 8);
+    int32_t *first = reinterpret_cast<int32_t *>(cum + smax);
     uint8_t *ends = reinterpret_cast<uint8_t *>(first + smax);
     __shared__ int32_t ws[kSetThreads / 32];
     __shared__ int32_t root_term;
@@ -453,8 +455,14 @@ __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restric
             int32_t total;
             int32_t at = level_end + set_excl_scan(c, ws, &total);
             for (int32_t r = r0; r < r1; r++) {
+                const uint4 *rw = reinterpret_cast<const uint4 *>(bits + int64_t(r) * 8);
+                const uint4 lo = rw[0], hi = rw[1];
+                const uint32_t p1 = __popc(lo.x), p2 = p1 + __popc(lo.y), p3 = p2 + __popc(lo.z),
+                               p4 = p3 + __popc(lo.w), p5 = p4 + __popc(hi.x), p6 = p5 + __popc(hi.y),
+                               p7 = p6 + __popc(hi.z);
+                cum[r] = make_uint2((p1 << 8) | (p2 << 16) | (p3 << 24), p4 | (p5 << 8) | (p6 << 16) | (p7 << 24));
                 first[r] = at;
-                at += row_popc(bits, r);
+                at += int32_t(p7 + __popc(hi.w));
             }
             __syncthreads();
 #pragma unroll
@@ -462,14 +470,10 @@ __global__ void __launch_bounds__(kSetThreads) k_b_sets(const uint8_t *__restric
                 if (len[k] <= d) continue;
                 const uint32_t b = uint32_t(nb[k]);
                 const int32_t row = cur[k] - level_start;
-                const uint32_t *rw = bits + row * 8;
-                int32_t below = 0;
-#pragma unroll
-                for (int w = 0; w < 8; w++) {
-                    const int32_t lo = w * 32;
-                    if (int32_t(b) >= lo + 32) below += __popc(rw[w]);
-                    else if (int32_t(b) >= lo) below += __popc(rw[w] & ((1u << (b - lo)) - 1u));
-                }
+                const uint32_t wi = b >> 5;
+                const uint2 cm = cum[row];
+                const uint32_t before = ((wi < 4 ? cm.x : cm.y) >> (8 * (wi & 3))) & 0xFFu;
+                const int32_t below = int32_t(before + __popc(bits[row * 8 + wi] & ((1u << (b & 31)) - 1u)));
                 const int32_t ch = first[row] + below;
                 const int64_t g = ub + ch;
                 parent_ub[g] = cur[k];
@@ -523,7 +527,10 @@ __global__ void __launch_bounds__(kBThreads) k_b_set_scan(int32_t M, const int32
     if (threadIdx.x == 0) *total = carry;
 }
 
-// Every set's nodes from ub(s) + i to base(s) + i (CTA per set).
+// Every set's nodes from ub(s) + i to base(s) + i (kEmitParts CTAs per set,
+// each a share of the set's nodes: one CTA per set left each thread ~70
+// dependent copies at 256 sets of ~19,000 nodes).
+constexpr int32_t kEmitParts = 8;
 __global__ void k_b_set_emit(const int64_t *__restrict__ off, const int32_t *__restrict__ set_off, int32_t M,
                              const int32_t *__restrict__ count, const int32_t *__restrict__ roots,
                              const int32_t *__restrict__ parent_ub, const uint8_t *__restrict__ label_ub,
@@ -531,10 +538,11 @@ __global__ void k_b_set_emit(const int64_t *__restrict__ off, const int32_t *__r
                              uint8_t *__restrict__ label, uint8_t *__restrict__ terminal) {
     pdl_launch_dependents();
     pdl_wait();
-    for (int32_t s = blockIdx.x; s < M; s += gridDim.x) {
+    for (int64_t u = blockIdx.x; u < int64_t(M) * kEmitParts; u += gridDim.x) {
+        const int32_t s = int32_t(u / kEmitParts), part = int32_t(u % kEmitParts);
         const int64_t ub = off[set_off[s]] - off[0] + s;
         const int32_t base = roots[s], n = count[s];
-        for (int32_t i = threadIdx.x; i < n; i += blockDim.x) {
+        for (int32_t i = part * int32_t(blockDim.x) + threadIdx.x; i < n; i += kEmitParts * int32_t(blockDim.x)) {
             const int32_t p = parent_ub[ub + i];
             parent[base + i] = p < 0 ? -1 : base + p;
             label[base + i] = label_ub[ub + i];
@@ -738,7 +746,7 @@ cudaError_t DeviceBuild::sets(int num_sms, int32_t *n_nodes, std::vector<int32_t
     char *b = static_cast<char *>(s_->base2);
     s_->count = reinterpret_cast<int32_t *>(b + o_cnt);
     s_->total = reinterpret_cast<int32_t *>(b + o_tot);
-    const size_t smem = size_t(smax_) * (8 * sizeof(uint32_t) + sizeof(int32_t) + 1);
+    const size_t smem = size_t(smax_) * (8 * sizeof(uint32_t) + sizeof(uint2) + sizeof(int32_t) + 1);
     int per_sm = 0;
     if ((e = cudaFuncSetAttribute(k_b_sets, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem))) !=
             cudaSuccess ||
@@ -778,7 +786,8 @@ cudaError_t DeviceBuild::sets(int num_sms, int32_t *n_nodes, std::vector<int32_t
 
 cudaError_t DeviceBuild::emit(int32_t *parent, uint8_t *label, uint8_t *terminal, int num_sms) {
     if (small_)
-        return launch_pdl(k_b_set_emit, std::min<int64_t>(M_, int64_t(num_sms) * 8), kBThreads, stream_,
+        return launch_pdl(k_b_set_emit, std::min<int64_t>(int64_t(M_) * kEmitParts, int64_t(num_sms) * 16), kBThreads,
+                          stream_,
                       static_cast<const int64_t *>(s_->off), static_cast<const int32_t *>(s_->set_off), M_,
                       static_cast<const int32_t *>(s_->count), static_cast<const int32_t *>(s_->roots),
                       static_cast<const int32_t *>(s_->parent_g), static_cast<const uint8_t *>(s_->label_g),
