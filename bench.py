@@ -512,7 +512,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
     fused_gbs = fused_bytes / (fused_avg * 1e-3) / 1e9
     compile_gbs = compile_bytes / (compile_ms * 1e-3) / 1e9
 
-    e2e_s, h2d, d2h, h2d_only_s = run_e2e(w, N, logits, forced, dev, stream, args.e2e_steps, dist)
+    e2e_s, h2d, d2h, h2d_only_s, e2e_runs = run_e2e(w, N, logits, forced, dev, stream, args.e2e_steps, dist)
 
     if rank != 0:
         return
@@ -577,7 +577,10 @@ def run_gpu(args, w, rank: int, world: int, dist):
                       "apply_gbs_conventional_rw": (2 * B * V * elt + B * Wd * 4) / (apply_avg * 1e-3) / 1e9},
         "e2e": {"value": job_throughput(N * V, world, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3,
-                "h2d_only_ms": h2d_only_s * 1e3, "h2d_gbs": h2d / h2d_only_s / 1e9},
+                "h2d_only_ms": h2d_only_s * 1e3, "h2d_gbs": h2d / h2d_only_s / 1e9,
+                "runs_ms_per_step": [round(r * 1e3, 4) for r in e2e_runs],
+                "timing": f"the fastest of {len(e2e_runs)} runs of {args.e2e_steps} pipelined steps, wall clock "
+                          "around each run (the copies alone: the fastest of 5 rounds, CUDA events)"},
         "gpu_launches": args.steps * (3 + S + 1),
         "clocks": clk.summary(),
     }
@@ -653,20 +656,25 @@ def run_e2e(w, n_nodes: int, logits, forced, dev, stream, steps: int, dist=None)
         hh.destroy_async(stream)
         return nxt
 
+    # the timed loop runs three times and the fastest counts, as for the
+    # copies alone below: on these shared hosts the host link's bandwidth
+    # dropped to about half for whole runs at times (5.96 against 10.8 ms)
+    runs = []
     with torch.cuda.stream(stream):
         hh = T.trie_build(w.set_bytes, w.set_offsets)
         for i in range(2):
             hh = e2e_step(i, hh)
-        torch.cuda.synchronize()
-        if dist is not None:
-            dist.barrier()
-        t0 = time.perf_counter()
-        for i in range(steps):
-            hh = e2e_step(i, hh)
-        torch.cuda.synchronize()
-        e2e_s = (time.perf_counter() - t0) / steps
+        for _ in range(3):
+            torch.cuda.synchronize()
+            if dist is not None:
+                dist.barrier()
+            t0 = time.perf_counter()
+            for i in range(steps):
+                hh = e2e_step(i, hh)
+            torch.cuda.synchronize()
+            runs.append((time.perf_counter() - t0) / steps)
         hh.destroy()
-    e2e_s = reduce_max(e2e_s, dist, dev)
+    e2e_s = reduce_max(min(runs), dist, dev)
     # context: the step's host->device copies alone (the floor of the e2e
     # step), the fastest of a few rounds timed with events on the copy stream
     torch.cuda.synchronize()
@@ -682,7 +690,7 @@ def run_e2e(w, n_nodes: int, logits, forced, dev, stream, steps: int, dist=None)
         copy_stream.synchronize()
         rounds.append(c0.elapsed_time(c1) * 1e-3)
     h2d_only_s = min(rounds)
-    return e2e_s, h2d, d2h, h2d_only_s
+    return e2e_s, h2d, d2h, h2d_only_s, runs
 
 
 def run_lazy(w, logits, forced, dev, stream, capture, timed, reps: int) -> dict:
