@@ -76,8 +76,11 @@ def peaks() -> tuple[float, str]:
 
 
 def kernel_source_hash() -> str:
+    """Hash of kernels.cu without its // comments and blank lines: a traffic
+    record stays valid across comment edits and lapses with any code change."""
     with open(os.path.join(ROOT, "paper_2608_12574_gb300", "csrc", "kernels.cu"), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+        lines = [ln.split("//", 1)[0].rstrip() for ln in f.read().decode().splitlines()]
+    return hashlib.sha256("\n".join(ln for ln in lines if ln.strip()).encode()).hexdigest()[:16]
 
 
 def ncu_traffic(kernel: str, workload: str) -> float | None:

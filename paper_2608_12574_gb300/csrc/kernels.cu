@@ -1,30 +1,43 @@
 // sm_103a kernels of libtriemask.
 //
-//  k_mask_fill   dense part of the mask compile: writes every mask word once
-//                (zero) with 16-byte stores, 8 KB per CTA. HBM-write bound.
-//  k_mask_patch  sparse part: one thread per trie node m finds every token
-//                whose bytes spell the last k edges into m (k = 1..lmax) and
-//                sets that token's bit in the row of the node k edges above m.
-//                These are exactly the Aho-Corasick outputs of Sec. 4.2 step
-//                2 (a token whose characters end at the current node is
-//                recorded at the node |token| characters earlier, App. G.1
-//                Step 3), found by one hash lookup per suffix length instead
-//                of by failure links, so every node is independent. Cost
-//                O(N * min(depth, l)) lookups, the traversal bound of Sec. 4.2.
-//  k_advance     delta*(s, bytes(token)) per request (Sec. 2, Eq. 1).
-//  k_apply_vec   -inf into the logits of disallowed tokens (Sec. 4.2; App.
-//                H.3): one warp per 1024-token segment; a segment without an
-//                allowed token is one TMA bulk copy of a -inf tile, the rest
-//                16-byte stores, the logits read only in 16-byte chunks that
-//                hold an allowed token.
+// Mask compile (bit[n][v] for every node n and token v; Sec. 4.1-4.2):
+//  k_mask_probe        one thread per node m finds every token whose bytes
+//                      spell the last k edges into m (k = 1..lmax), to be set
+//                      in the row of the node k edges above m: the
+//                      Aho-Corasick outputs of Sec. 4.2 step 2 (a token whose
+//                      characters end at the current node is recorded at the
+//                      node |token| characters earlier), found by hashing each
+//                      suffix of the node's 16-label window instead of by
+//                      failure links, so every node is independent. It records
+//                      the hits, sets the segment summary and runs beside
+//                      k_mask_fill_beside; k_mask_probe_pair is the same with
+//                      2 or 4 threads per node for small tries.
+//  k_mask_fill_beside  writes every mask word once (zero), 16-byte evict-first
+//                      stores, 8 KB per CTA: HBM-write bound.
+//  k_mask_scatter      ORs the recorded hits into the zeroed mask.
+//  (small masks: k_mask_fill, then k_mask_probe_pair ORing its own hits;
+//  the no-allocation entry point: k_mask_fill, then k_mask_patch; the
+//  pair-by-pair form for the A/B: k_mask_pairwise.)
+// Decode (Sec. 2, Eq. 1; Sec. 4.2; App. H.3):
+//  k_advance           delta*(s, bytes(token)) per request.
+//  k_apply_vec         -inf into the logits of disallowed tokens: one warp per
+//                      1024-token segment; a segment the summary says is empty
+//                      is one TMA bulk copy of a -inf tile and reads no mask
+//                      word, the rest 16-byte stores, the logits read only in
+//                      16-byte chunks that hold an allowed token.
+//  k_advance_apply_vec the advance of one step and the apply of the next.
+// Sparse lists (valid[n] as CSR; App. H.5): k_rt_insert (per vocabulary),
+// k_list_walk (count, then write), k_scan_*, k_apply_lists.
+// Lazy rows (App. H.5): k_lazy_resolve, k_lazy_rows, k_lazy_gather.
 //
 // Every kernel is launched with programmatic stream serialization (PDL): it
 // lets the next kernel in the stream launch at once and waits for the
 // previous kernel (griddepcontrol.wait) before it touches memory that kernel
 // may write or read. That wait is the hardware grid dependency, which always
-// resolves because the previous grid never waits on this one. The patch
-// kernel does its trie climbs and hash probes (read-only data) before the
-// wait, so they overlap the fill.
+// resolves because the previous grid never waits on this one. A kernel that
+// runs beside the one before it (the fill beside the probe, the search of the
+// small-mask form beside its fill) reads only data that was complete before
+// that kernel started, and waits before it writes what the other one writes.
 #include <stdint.h>
 
 #include <algorithm>
