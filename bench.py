@@ -75,10 +75,12 @@ def peaks() -> tuple[float, str]:
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash() -> str:
-    """Hash of kernels.cu without its // comments and blank lines: a traffic
-    record stays valid across comment edits and lapses with any code change."""
-    with open(os.path.join(ROOT, "paper_2608_12574_gb300", "csrc", "kernels.cu"), "rb") as f:
+def kernel_source_hash(path: str | None = None) -> str:
+    """Hash of kernels.cu (or `path`) without its // comments and blank lines:
+    a traffic record stays valid across comment edits and lapses with any
+    code change."""
+    path = path or os.path.join(ROOT, "paper_2608_12574_gb300", "csrc", "kernels.cu")
+    with open(path, "rb") as f:
         lines = [ln.split("//", 1)[0].rstrip() for ln in f.read().decode().splitlines()]
     return hashlib.sha256("\n".join(ln for ln in lines if ln.strip()).encode()).hexdigest()[:16]
 

@@ -91,3 +91,13 @@ def test_clock_summary_parses_nvidia_smi_samples():
     assert c.summary()["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
     c.out = ""
     assert c.summary()["reasons"] == ["no samples"]
+
+
+def test_kernel_source_hash_ignores_comments_only(tmp_path):
+    import bench
+    a, b, c = tmp_path / "a.cu", tmp_path / "b.cu", tmp_path / "c.cu"
+    a.write_text("// header\nint f() { return 1; }  // one\n\n")
+    b.write_text("// another header\n\nint f() { return 1; }\n// trailing\n")
+    c.write_text("int f() { return 2; }\n")
+    assert bench.kernel_source_hash(str(a)) == bench.kernel_source_hash(str(b))
+    assert bench.kernel_source_hash(str(a)) != bench.kernel_source_hash(str(c))
