@@ -364,27 +364,35 @@ __global__ void k_trie_links(const int32_t *__restrict__ parent, const uint8_t *
 // ancestors (-1 past the root), stored as four 16-byte rows. Siblings and
 // cousins are neighbours in breadth-first order, so a warp's climbs read
 // neighbouring entries of the parent and label arrays, which stay in L2.
-// (Two alternatives measured slower on the 4.77 M-node forest: rows built by
-// doubling from the rows of the ancestors 4, 8 and 12 levels up, 230 us, whose
-// reads of the 64-byte ancestor rows come from DRAM; and two climbs per thread
-// storing each ancestor as found, 404 us, whose 4-byte stores multiply the L2
-// write traffic. This form: 114 us.)
+// Each warp stages its 32 ancestor rows (2 KB) in shared memory, a quarter
+// row as soon as its four ancestors are known, and writes them out as one
+// contiguous 2 KB run: stored straight from the climb, each 16-byte store of
+// a warp touched 32 rows 64 bytes apart (117 us on the 4.77 M-node forest
+// against 89 us staged). The 16-byte units of a row are swizzled by bits 1-2
+// of the row, so that the eight rows of a quarter-warp's stores and the two
+// rows of its loads fall on distinct banks. (Measured slower: two or four
+// climbs per thread, 97-217 us, and the labels gathered after the climb,
+// 105-240 us, both short of registers at full occupancy; rows built by
+// doubling from the rows of the ancestors 4, 8 and 12 levels up, 230 us,
+// whose reads of the 64-byte ancestor rows come from DRAM.)
 constexpr int kTableThreads = 256;
-__global__ void __launch_bounds__(kTableThreads) k_trie_tables(const int32_t *__restrict__ parent,
-                                                               const uint8_t *__restrict__ label, int32_t n,
-                                                               ulonglong2 *__restrict__ window,
-                                                               uint8_t *__restrict__ depth16,
-                                                               int4 *__restrict__ anc) {
+__global__ void __launch_bounds__(kTableThreads, 2048 / kTableThreads)
+    k_trie_tables(const int32_t *__restrict__ parent, const uint8_t *__restrict__ label, int32_t n,
+                  ulonglong2 *__restrict__ window, uint8_t *__restrict__ depth16, int4 *__restrict__ anc) {
+    __shared__ int4 stage[kTableThreads * 4];
+    const int lane = threadIdx.x & 31;
+    int4 *ws = stage + (threadIdx.x >> 5) * 128;  // this warp's 32 rows of four units
     const int32_t stride = gridDim.x * blockDim.x;
-    for (int32_t m = blockIdx.x * blockDim.x + threadIdx.x; m < n; m += stride) {
+    for (int32_t m0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); m0 < n; m0 += stride) {
+        const int32_t m = m0 + lane;
         uint64_t lo = 0, hi = 0;
-        int32_t up[kMaxClimb];
+        int32_t up[4];
         int32_t d = 0;
-        int32_t x = m;
+        int32_t x = m < n ? m : -1;
 #pragma unroll
         for (int k = 0; k < kMaxClimb; k++) {
             const int32_t p = x >= 0 ? __ldg(parent + x) : -1;
-            up[k] = p;
+            up[k & 3] = p;
             if (p >= 0) {
                 const uint64_t b = __ldg(label + x);
                 if (k < 8) lo |= b << (8 * k);
@@ -392,12 +400,20 @@ __global__ void __launch_bounds__(kTableThreads) k_trie_tables(const int32_t *__
                 d = k + 1;
             }
             x = p;
+            if ((k & 3) == 3)
+                ws[lane * 4 + ((k >> 2) ^ ((lane >> 1) & 3))] = make_int4(up[0], up[1], up[2], up[3]);
         }
-        window[m] = make_ulonglong2(lo, hi);
-        depth16[m] = uint8_t(d);
+        if (m < n) {
+            window[m] = make_ulonglong2(lo, hi);
+            depth16[m] = uint8_t(d);
+        }
+        __syncwarp();
 #pragma unroll
-        for (int q = 0; q < 4; q++)
-            anc[int64_t(m) * 4 + q] = make_int4(up[4 * q], up[4 * q + 1], up[4 * q + 2], up[4 * q + 3]);
+        for (int j = 0; j < 4; j++) {
+            const int u = j * 32 + lane, r = u >> 2, q = u & 3;  // unit u of the warp's 2 KB run
+            if (m0 + r < n) anc[int64_t(m0) * 4 + u] = ws[r * 4 + (q ^ ((r >> 1) & 3))];
+        }
+        __syncwarp();  // the rows are read before the next nodes' climbs overwrite them
     }
 }
 
