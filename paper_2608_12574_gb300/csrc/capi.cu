@@ -225,11 +225,8 @@ int alloc_device_trie(trie_t h, int dev, size_t n, cudaStream_t stream, bool wit
 // The child links and the compile's per-node tables, from the device's
 // parent / label / terminal arrays (once they are written on `stream`).
 int finish_device_trie(trie_t h, int dev, cudaStream_t stream) {
-    const size_t n = size_t(h->host.n);
     cudaError_t e;
-    if ((e = cudaMemsetAsync(h->dev.first_child, 0xFF, sizeof(int32_t) * n, stream)) == cudaSuccess &&
-        (e = cudaMemsetAsync(h->dev.child_bits, 0, sizeof(uint32_t) * 8 * n, stream)) == cudaSuccess &&
-        (e = tmk::launch_trie_links(h->dev, h->host.n, num_sms(dev), stream)) == cudaSuccess)
+    if ((e = tmk::launch_trie_links(h->dev, h->host.n, num_sms(dev), stream)) == cudaSuccess)
         e = tmk::launch_trie_tables(h->dev, h->host.n, num_sms(dev), stream);
     if (e != cudaSuccess) {
         pool_free(h->dev.base);

@@ -343,80 +343,6 @@ __global__ void k_vocab_pay(const uint64_t *__restrict__ key, const int32_t *__r
     }
 }
 
-// Child links from parent and label (thread per node c): in breadth-first
-// order the children of a node are contiguous, so c is its parent's first
-// child iff c - 1 has another parent; every child sets its label's bit in its
-// parent's 256-bit set.
-__global__ void k_trie_links(const int32_t *__restrict__ parent, const uint8_t *__restrict__ label, int32_t n,
-                             int32_t *__restrict__ first_child, uint32_t *__restrict__ child_bits) {
-    for (int32_t c = blockIdx.x * blockDim.x + threadIdx.x; c < n; c += gridDim.x * blockDim.x) {
-        const int32_t p = parent[c];
-        if (p < 0) continue;
-        if (parent[c - 1] != p) first_child[p] = c;
-        const uint32_t l = label[c];
-        atomicOr(child_bits + int64_t(p) * 8 + (l >> 5), 1u << (l & 31u));
-    }
-}
-
-// Per-node tables of the probe and of the list walk (one thread per node,
-// climbing at most 16 parents): the last 16 edge labels into m (byte i = the
-// label i levels up, 0 past the root), min(depth, 16), and the 16 nearest
-// ancestors (-1 past the root), stored as four 16-byte rows. Siblings and
-// cousins are neighbours in breadth-first order, so a warp's climbs read
-// neighbouring entries of the parent and label arrays, which stay in L2.
-// Each warp stages its 32 ancestor rows (2 KB) in shared memory, a quarter
-// row as soon as its four ancestors are known, and writes them out as one
-// contiguous 2 KB run: stored straight from the climb, each 16-byte store of
-// a warp touched 32 rows 64 bytes apart (117 us on the 4.77 M-node forest
-// against 89 us staged). The 16-byte units of a row are swizzled by bits 1-2
-// of the row, so that the eight rows of a quarter-warp's stores and the two
-// rows of its loads fall on distinct banks. (Measured slower: two or four
-// climbs per thread, 97-217 us, and the labels gathered after the climb,
-// 105-240 us, both short of registers at full occupancy; rows built by
-// doubling from the rows of the ancestors 4, 8 and 12 levels up, 230 us,
-// whose reads of the 64-byte ancestor rows come from DRAM.)
-constexpr int kTableThreads = 256;
-__global__ void __launch_bounds__(kTableThreads, 2048 / kTableThreads)
-    k_trie_tables(const int32_t *__restrict__ parent, const uint8_t *__restrict__ label, int32_t n,
-                  ulonglong2 *__restrict__ window, uint8_t *__restrict__ depth16, int4 *__restrict__ anc) {
-    __shared__ int4 stage[kTableThreads * 4];
-    const int lane = threadIdx.x & 31;
-    int4 *ws = stage + (threadIdx.x >> 5) * 128;  // this warp's 32 rows of four units
-    const int32_t stride = gridDim.x * blockDim.x;
-    for (int32_t m0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); m0 < n; m0 += stride) {
-        const int32_t m = m0 + lane;
-        uint64_t lo = 0, hi = 0;
-        int32_t up[4];
-        int32_t d = 0;
-        int32_t x = m < n ? m : -1;
-#pragma unroll
-        for (int k = 0; k < kMaxClimb; k++) {
-            const int32_t p = x >= 0 ? __ldg(parent + x) : -1;
-            up[k & 3] = p;
-            if (p >= 0) {
-                const uint64_t b = __ldg(label + x);
-                if (k < 8) lo |= b << (8 * k);
-                else hi |= b << (8 * (k - 8));
-                d = k + 1;
-            }
-            x = p;
-            if ((k & 3) == 3)
-                ws[lane * 4 + ((k >> 2) ^ ((lane >> 1) & 3))] = make_int4(up[0], up[1], up[2], up[3]);
-        }
-        if (m < n) {
-            window[m] = make_ulonglong2(lo, hi);
-            depth16[m] = uint8_t(d);
-        }
-        __syncwarp();
-#pragma unroll
-        for (int j = 0; j < 4; j++) {
-            const int u = j * 32 + lane, r = u >> 2, q = u & 3;  // unit u of the warp's 2 KB run
-            if (m0 + r < n) anc[int64_t(m0) * 4 + u] = ws[r * 4 + (q ^ ((r >> 1) & 3))];
-        }
-        __syncwarp();  // the rows are read before the next nodes' climbs overwrite them
-    }
-}
-
 // Slot of each key of a batch in the paired-slot table, -1 if absent, for
 // vocabularies in which no two tokens share a key (so a key is stored at
 // most once). f holds each key's first pair, already loaded. The keys of the
@@ -1954,20 +1880,6 @@ cudaError_t launch_mask_patch(const DevTrie &t, int32_t n_nodes, const DevVocab 
     PatchArgs a = patch_args(t, n_nodes, v, lmax, mask, W);
     const int grid = grid_for(n_nodes, kPatchThreads, int64_t(num_sms) * 32);
     return launch_pdl(k_mask_patch, grid, kPatchThreads, st, a);
-}
-
-cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st) {
-    if (n_nodes <= 0) return cudaSuccess;
-    const int grid = grid_for(n_nodes, 256, int64_t(num_sms) * 8);
-    k_trie_links<<<grid, 256, 0, st>>>(t.parent, t.label, n_nodes, t.first_child, t.child_bits);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st) {
-    if (n_nodes <= 0) return cudaSuccess;
-    const int grid = grid_for(n_nodes, kTableThreads, int64_t(num_sms) * 8);
-    k_trie_tables<<<grid, kTableThreads, 0, st>>>(t.parent, t.label, n_nodes, t.window, t.depth16, t.anc);
-    return cudaGetLastError();
 }
 
 cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st) {

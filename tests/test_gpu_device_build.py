@@ -333,3 +333,44 @@ def test_device_forest_config5(cuda):
         T.trie_lazy_init(h, w.vocab_bytes, w.vocab_offsets, w.V, cache_rows=1024, max_batch=2048)
         rows.append(_np_u32(T.trie_lazy_rows(h, torch.as_tensor(states, device=cuda), w.V)))
     assert np.array_equal(rows[0], rows[1])
+
+
+def _link_sets():
+    """Sets whose tries stress the child links: empty sets and lone terminal
+    roots next to each other, a root with all 256 children, a chain of 70
+    nodes, parents whose children run past a warp's 32 consecutive nodes
+    (100 and 256 siblings), and many one-child parents."""
+    return [[], [b""], [bytes([i]) for i in range(256)], [], [b"x" * 70],
+            [bytes([i, j]) for i in range(3) for j in range(0, 200, 2)], [b"a"], [],
+            [bytes([97 + i % 26]) * (1 + i % 9) + bytes([i]) for i in range(60)],
+            [bytes([i, 255 - i]) for i in range(256)], [b""], []]
+
+
+@pytest.mark.parametrize("builder", ["host", "device"])
+def test_child_links_walk_every_byte(cuda, builder):
+    """The child links built on the device (first child and 256-bit child-label
+    set of every node) move every (node, byte) pair to the child that the
+    parent and label arrays give, and every other pair to DEAD: trie_advance
+    by single-byte tokens walks exactly one link."""
+    import torch
+    sets = _link_sets()
+    sb, so, index = _forest(sets)
+    h = (T.trie_build_many_device(sb, so, index) if builder == "device"
+         else T.trie_build_many(sb, so, index))
+    _check_against_oracle(h, sets)
+    vb, vo = W.pack([bytes([b]) for b in range(256)] + [b""])  # token 256: EOS
+    T.trie_compile_lists(h, vb, vo, 257)
+    c = h.csr()
+    n = h.num_nodes
+    child = np.full((n, 256), T.TRIE_STATE_DEAD, np.int32)
+    for x in range(n):
+        if c["parent"][x] >= 0:
+            child[c["parent"][x], c["label"][x]] = x
+    states = torch.as_tensor(np.repeat(np.arange(n, dtype=np.int32), 256), device=cuda)
+    tokens = torch.as_tensor(np.tile(np.arange(256, dtype=np.int32), n), device=cuda)
+    err = torch.zeros(1, dtype=torch.int32, device=cuda)
+    T.trie_advance(h, states, tokens, err)
+    got = states.cpu().numpy().reshape(n, 256)
+    assert np.array_equal(got, child)
+    assert int(err.item()) == int((child == T.TRIE_STATE_DEAD).sum())
+    h.destroy()
