@@ -152,18 +152,20 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def compile_kernels(w, n_nodes: int, max_depth: int, dev) -> int:
+def compile_kernels(w, n_nodes: int, max_depth: int, num_sms: int) -> int:
     """Kernels one trie_compile_masks launches, by the library's rule: a mask
     of at most 32 MB of a trie whose search takes two threads per node (at
-    most 19,456 nodes, tokens and depth within 16 bytes; no repeated token
-    strings) is the fill and the search ORing its hits (2); otherwise the
-    search, the fill and the scatter (3)."""
+    most num_sms * 128 nodes, tokens and depth within 16 bytes, no repeated
+    token string, so that every table slot holds one token's payload) is the
+    fill and the search ORing its hits (2); otherwise the search, the fill and
+    the scatter (3). (Two distinct strings whose 64-bit keys collide also
+    take the 3-kernel form; that is not modelled.)"""
     import numpy as np
-    import torch
-    lens = np.diff(np.asarray(w.vocab_offsets))
+    vb, vo = np.asarray(w.vocab_bytes), np.asarray(w.vocab_offsets)
+    lens = np.diff(vo)[: w.V - 1]  # token V - 1 is EOS: its bytes are ignored
     lmax = min(int(lens.max()) if lens.size else 0, max_depth)
-    sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    pair = lmax <= 16 and 4 * n_nodes <= sms * 4 * 128
+    strings = [bytes(vb[vo[i]:vo[i + 1]]) for i in range(w.V - 1) if lens[i] > 0]
+    pair = lmax <= 16 and 4 * n_nodes <= num_sms * 4 * 128 and len(set(strings)) == len(strings)
     mask_bytes = n_nodes * ((w.V + 31) // 32) * 4
     return 2 if pair and mask_bytes <= (32 << 20) else 3
 
@@ -602,7 +604,7 @@ def run_gpu(args, w, rank: int, world: int, dist):
                 "runs_ms_per_step": [round(r * 1e3, 4) for r in e2e_runs],
                 "timing": f"the fastest of {len(e2e_runs)} runs of {args.e2e_steps} pipelined steps, wall clock "
                           "around each run (the copies alone: the fastest of 5 rounds, CUDA events)"},
-        "gpu_launches": args.steps * (compile_kernels(w, N, h.max_depth, dev) + S + 1),
+        "gpu_launches": args.steps * (compile_kernels(w, N, h.max_depth, torch.cuda.get_device_properties(dev).multi_processor_count) + S + 1),
         "clocks": clk.summary(),
     }
     if not args.no_dynamic:

@@ -101,3 +101,27 @@ def test_kernel_source_hash_ignores_comments_only(tmp_path):
     c.write_text("int f() { return 2; }\n")
     assert bench.kernel_source_hash(str(a)) == bench.kernel_source_hash(str(b))
     assert bench.kernel_source_hash(str(a)) != bench.kernel_source_hash(str(c))
+
+
+def test_compile_kernels_follows_the_library_rule():
+    """gpu_launches counts 2 compile kernels (fill, then the pair search ORing
+    its hits) only for masks of at most 32 MB, tries of at most 128 nodes per
+    SM, tokens and depth within 16 bytes and no repeated token string; else 3."""
+    import types
+    import bench
+    from paper_2608_12574_gb300 import workloads as W
+
+    def vocab(strings):
+        vb, vo = W.pack(list(strings) + [b""])  # the last token is EOS
+        return types.SimpleNamespace(vocab_bytes=vb, vocab_offsets=vo, V=len(strings) + 1)
+
+    small = vocab([bytes([97 + i % 26]) * (1 + i % 5) + str(i).encode() for i in range(1000)])
+    assert bench.compile_kernels(small, 1384, 20, 152) == 2
+    assert bench.compile_kernels(small, 152 * 128 + 1, 20, 152) == 3          # too many nodes for two lanes each
+    assert bench.compile_kernels(small, 152 * 128, 20, 152) == 2
+    assert bench.compile_kernels(vocab([b"x" * 17, b"a"]), 100, 20, 152) == 3  # a token longer than 16 bytes
+    assert bench.compile_kernels(vocab([b"x" * 17, b"a"]), 100, 16, 152) == 2  # ... that no path of the trie reaches
+    assert bench.compile_kernels(vocab([b"ab", b"cd", b"ab"]), 100, 20, 152) == 3  # a repeated token string
+    wide = vocab([str(i).encode() for i in range(300000)])   # V = 300,001: 9,376 words, 37,504 B per row
+    assert bench.compile_kernels(wide, 894, 20, 152) == 2     # 33,528,576 B <= 32 MB
+    assert bench.compile_kernels(wide, 895, 20, 152) == 3     # 33,566,080 B > 32 MB
