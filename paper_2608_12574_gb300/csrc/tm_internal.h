@@ -443,10 +443,10 @@ cudaError_t launch_mask_compile3(const DevTrie &t, int32_t n_nodes, const DevVoc
                                  uint32_t *mask, int64_t W, int num_sms, bool fill_trans, cudaStream_t st,
                                  unsigned long long *seg_any, uint32_t *seg_epoch, uint32_t epoch,
                                  int32_t seg_words, bool *seg_written);
-// Fills t.first_child and t.child_bits from t.parent and t.label (which must
-// be -1 / zero on entry: the caller clears them on the same stream).
+// Writes every entry of t.first_child (-1 for a leaf) and t.child_bits from
+// t.parent and t.label; nothing needs clearing first (tables.cu).
 cudaError_t launch_trie_links(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
-// Fills t.window, t.depth16 and t.anc from t.parent and t.label.
+// Fills t.window, t.depth16 and t.anc from t.parent and t.label (tables.cu).
 cudaError_t launch_trie_tables(const DevTrie &t, int32_t n_nodes, int num_sms, cudaStream_t st);
 // Zeroes the transition table (before it is filled for another vocabulary).
 cudaError_t launch_trans_clear(const DevTrie &t, int num_sms, cudaStream_t st);
