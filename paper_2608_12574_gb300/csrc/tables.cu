@@ -1,11 +1,12 @@
-// Per-node tables of a trie on the device, from its parent and label arrays
-// (Sec. 4.1; App. H.1): the child links (first child and the 256-bit set of
-// child labels, from which the byte walks find a child) and the tables of the
-// mask compile and the list walk (the last 16 edge labels, min(depth, 16),
-// the 16 nearest ancestors). They run once per trie, after its upload or its
-// build on the device, and read only parent and label: nodes in breadth-first
-// order within every set, siblings by ascending byte, the sets one after
-// another, each root first.
+// Per-node tables of a trie on the device, from its parent and label arrays:
+// the child links (first child and the 256-bit set of child labels) that the
+// character walk of the advance follows (Sec. 2, Eq. 1; Sec. 4.1), and the
+// tables that the mask compile's traversal and the list walk read in place of
+// the paper's depth-first walk with saved automaton states (App. H.4, Phase
+// 4): the last 16 edge labels, min(depth, 16), the 16 nearest ancestors. They
+// run once per trie, after its upload or its build on the device, and read
+// only parent and label: nodes in breadth-first order within every set,
+// siblings by ascending byte, the sets one after another, each root first.
 #include <stdint.h>
 
 #include <cuda_runtime.h>
